@@ -1,0 +1,40 @@
+"""fp64 CPU oracle for the EfficientEdit verification step -- TEST INFRASTRUCTURE.
+
+This package is the plain, slow, obviously-correct statement of what one
+verification step of edit-oriented speculative decoding computes (EfficientEdit,
+arXiv 2506.02780, Sec. IV-A "Reuse" and Eq. (piecewise)).  It exists to check
+the CUDA library against; it is not part of the product path.  Only the test
+suite, ``__graft_entry__.smoke()`` and ``bench.py``'s CPU-baseline / reference
+leg may import it.  It shares no code with the CUDA path and imports nothing
+from the product package.
+
+Every floating-point step runs in fp64 on exact fp64 copies of the bf16 inputs.
+Library primitives (numpy matmul, argmax) serve as single steps; nothing is
+blocked, fused or reordered beyond what each definition states.
+
+Parity status per function (what pins it, from outside this file, in
+tests/test_oracle_pins.py):
+  match_reuse      pinned: brute-force byte search, planted matches, closed forms
+  tree_prepare     pinned: walk-up brute force, chain/star closed forms
+  tree_attention   pinned: torch SDPA in fp64 over each node's linear path,
+                   single-key and equal-key closed forms, page-order invariance
+  lm_head_argmax   pinned: planted argmax targets, duplicated-row ties,
+                   pure-Python dot products on a tiny case
+  accept_path      pinned: token-by-token replay of Eq. (piecewise), brute force
+                   over all root-to-node paths, hand-worked golden cases
+  kv_compact       pinned: sequential append into a slot dictionary, canaries
+  entropy_top_tau  pinned: closed forms of Eq. (entropy) / top_tau (H=0, uniform)
+"""
+from .ee_oracle import (  # noqa: F401
+    PAGE,
+    match_reuse,
+    tree_prepare,
+    anc_to_sets,
+    tree_attention,
+    lm_head_logits,
+    lm_head_argmax,
+    accept_path,
+    kv_compact,
+    entropy_top_tau,
+    verify_step,
+)

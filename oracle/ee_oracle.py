@@ -1,0 +1,392 @@
+"""fp64 CPU oracle for the EfficientEdit verification step (test infrastructure).
+
+Only tests, ``__graft_entry__.smoke()`` and bench.py's CPU-baseline leg use this
+module.  Each function cites the passage of EfficientEdit (arXiv 2506.02780) it
+follows and states the reading taken where the paper is silent.
+
+Notation: B sequences; sequence s owns tree nodes node_off[s]..node_off[s+1]-1
+(local ids 0..T_s-1, local 0 is the root = last committed token); ctx = cached
+context length; the KV cache is paged, PAGE tokens per page, laid out
+[num_pages, n_kv, PAGE, d]; query head h reads KV head h // (n_q / n_kv).
+"""
+from __future__ import annotations
+
+import math
+
+import numpy as np
+
+PAGE = 16
+_U32 = 2.0 ** -24          # unit roundoff of fp32
+
+
+def _raw16(t):
+    """Raw 16-bit patterns of a bf16 torch tensor as a numpy uint16 array (for copies)."""
+    import torch
+    return t.detach().to("cpu").contiguous().view(torch.int16).numpy().view(np.uint16)
+
+
+def _f64(x):
+    """Exact fp64 copy of a bf16/fp32 tensor or array."""
+    if hasattr(x, "detach"):
+        return x.detach().to("cpu").double().numpy()
+    return np.asarray(x, dtype=np.float64)
+
+
+# ----------------------------------------------------------------------------
+# (1) reuse-span match -- Sec. IV-A, prefix matching to switch back to Reuse
+# ----------------------------------------------------------------------------
+
+def match_reuse(orig_tokens, orig_off, tail, cursor, max_matches):
+    """Positions p in the remaining original code where the last n generated
+    tokens occur: c[p:p+n] == tail, searched from the cursor onwards.
+
+    Sec. IV-A: when Generate switches back to Reuse, positions of the remaining
+    ``c`` that match the suffix of what was generated become new draft starts;
+    the tokens of ``c`` after such a position are the reuse draft.
+    Readings: every position p >= cursor is searched (not only p == cursor);
+    a match must leave at least one draft token, p + n < len(c); several match
+    points are returned in ascending order, up to ``max_matches``, with the
+    total count.
+
+    Returns (match_pos int32 [B, max_matches] padded with -1, n_matches int32 [B]).
+    """
+    orig_tokens = np.asarray(orig_tokens)
+    orig_off = np.asarray(orig_off)
+    tail = np.asarray(tail)
+    cursor = np.asarray(cursor)
+    B, n = tail.shape
+    if n < 1:
+        raise ValueError("n must be >= 1")
+    if max_matches < 1:
+        raise ValueError("max_matches must be >= 1")
+    match_pos = np.full((B, max_matches), -1, dtype=np.int32)
+    n_matches = np.zeros(B, dtype=np.int32)
+    for s in range(B):
+        c = orig_tokens[orig_off[s]:orig_off[s + 1]]
+        if cursor[s] < 0:
+            raise ValueError("cursor must be >= 0")
+        if len(c) < n + 1:
+            continue
+        windows = np.lib.stride_tricks.sliding_window_view(c, n)   # windows[p] = c[p:p+n]
+        hit = np.all(windows == tail[s][None, :], axis=1)
+        pos = np.nonzero(hit)[0]
+        pos = pos[(pos >= cursor[s]) & (pos + n < len(c))]
+        n_matches[s] = len(pos)
+        k = min(len(pos), max_matches)
+        match_pos[s, :k] = pos[:k]
+    return match_pos, n_matches
+
+
+# ----------------------------------------------------------------------------
+# (2) draft-tree structure
+# ----------------------------------------------------------------------------
+
+def tree_prepare(parent, node_off, max_nodes=128):
+    """depth and ancestor set of every draft-tree node.
+
+    The paper's drafts are linear (Sec. IV-A); a tree generalises them to
+    several drafts sharing a prefix (several match points, Sec. IV-A, plus
+    generated branches).  depth(root) = 0, depth(i) = depth(parent(i)) + 1;
+    anc(i) = anc(parent(i)) U {i}.  Parents precede children (parent[i] < i).
+
+    Returns (depth int32 [sum T], anc uint64 [sum T, 2]) where bit j of
+    anc[i] (word j // 64) is set when local node j is on the root-to-i path.
+    """
+    parent = np.asarray(parent)
+    node_off = np.asarray(node_off)
+    total = int(node_off[-1])
+    depth = np.zeros(total, dtype=np.int32)
+    anc = np.zeros((total, 2), dtype=np.uint64)
+    for s in range(len(node_off) - 1):
+        o, T = int(node_off[s]), int(node_off[s + 1] - node_off[s])
+        if T < 1 or T > max_nodes:
+            raise ValueError("each tree needs 1..%d nodes" % max_nodes)
+        sets = []
+        for i in range(T):
+            p = int(parent[o + i])
+            if i == 0:
+                if p != -1:
+                    raise ValueError("node 0 must be the root (parent -1)")
+                depth[o] = 0
+                sets.append({0})
+            else:
+                if not (0 <= p < i):
+                    raise ValueError("parent[i] must satisfy 0 <= parent[i] < i")
+                depth[o + i] = depth[o + p] + 1
+                sets.append(sets[p] | {i})
+            for j in sets[i]:
+                anc[o + i, j // 64] |= np.uint64(1) << np.uint64(j % 64)
+    return depth, anc
+
+
+def anc_to_sets(anc_row):
+    """Set of local node ids encoded in one [2] uint64 ancestor row."""
+    out = set()
+    for w in range(2):
+        v = int(anc_row[w])
+        for b in range(64):
+            if (v >> b) & 1:
+                out.add(64 * w + b)
+    return out
+
+
+# ----------------------------------------------------------------------------
+# (3) tree-masked attention over the paged cache -- Sec. IV-A, one target pass
+# ----------------------------------------------------------------------------
+
+def _context_kv(cache_l, block_table_row, ctx, hk):
+    """[ctx, d] fp64 rows of one KV head for cached positions 0..ctx-1."""
+    if ctx == 0:
+        return np.zeros((0, cache_l.shape[-1]))
+    npg = (ctx + PAGE - 1) // PAGE
+    pages = np.asarray(block_table_row[:npg])
+    if np.any(pages < 0) or np.any(pages >= cache_l.shape[0]):
+        raise ValueError("block table entry out of range")
+    rows = cache_l[pages, hk]                     # [npg, PAGE, d]
+    return rows.reshape(npg * PAGE, -1)[:ctx]
+
+
+def tree_attention(q, k_tree, v_tree, k_cache, v_cache, block_table, ctx_len, node_off, anc,
+                   scale=None, nodes=None, heads=None):
+    """Attention output of every draft node for ONE layer.
+
+    Sec. IV-A: one forward pass of the target over (prefix, draft) scores every
+    draft token.  With a tree, node i attends to the cached prefix (positions
+    0..ctx-1, read through the block table) and to the tree nodes on its own
+    root-to-i path (its ancestor set, i included) -- exactly what it would see
+    if its path were appended to the prefix as a linear draft.
+
+    o[i, h] = sum_j softmax_j(scale * q[i, h] . k_j) v_j, j over those keys,
+    with k_j, v_j from KV head h // (n_q / n_kv).  scale defaults to 1/sqrt(d).
+    Inputs are one layer: q [sumT, n_q, d], k_tree/v_tree [sumT, n_kv, d],
+    k_cache/v_cache [num_pages, n_kv, PAGE, d].
+
+    ``nodes`` (global node ids) and ``heads`` restrict the computation to a
+    sample; other entries of the returned fp64 [sumT, n_q, d] array are NaN.
+    """
+    q = _f64(q)
+    kt, vt = _f64(k_tree), _f64(v_tree)
+    kc, vc = _f64(k_cache), _f64(v_cache)
+    total, n_q, d = q.shape
+    n_kv = kt.shape[1]
+    if n_q % n_kv:
+        raise ValueError("n_q must be a multiple of n_kv")
+    g = n_q // n_kv
+    if scale is None:
+        scale = 1.0 / math.sqrt(d)
+    node_off = np.asarray(node_off)
+    want_nodes = set(range(total)) if nodes is None else set(int(x) for x in nodes)
+    want_heads = list(range(n_q)) if heads is None else [int(h) for h in heads]
+    out = np.full((total, n_q, d), np.nan)
+    for s in range(len(node_off) - 1):
+        o, T = int(node_off[s]), int(node_off[s + 1] - node_off[s])
+        ctx = int(ctx_len[s])
+        for hk in range(n_kv):
+            hs = [h for h in want_heads if h // g == hk]
+            if not hs:
+                continue
+            kctx = _context_kv(kc, block_table[s], ctx, hk)
+            vctx = _context_kv(vc, block_table[s], ctx, hk)
+            for i in range(T):
+                if o + i not in want_nodes:
+                    continue
+                path = sorted(anc_to_sets(anc[o + i]))
+                if any(j >= T for j in path):
+                    raise ValueError("ancestor outside the tree")
+                keys = np.concatenate([kctx, kt[[o + j for j in path], hk]], axis=0)
+                vals = np.concatenate([vctx, vt[[o + j for j in path], hk]], axis=0)
+                for h in hs:
+                    sc = scale * (keys @ q[o + i, h])
+                    p = np.exp(sc - sc.max())
+                    p /= p.sum()
+                    out[o + i, h] = p @ vals
+    return out
+
+
+# ----------------------------------------------------------------------------
+# (4) LM head, decode() = argmax, greedy acceptance -- Eq. (piecewise)
+# ----------------------------------------------------------------------------
+
+def lm_head_logits(hidden, lm_w, rows=None):
+    """logits[i, v] = hidden[i] . W[v] in fp64 (W is [V, H], vocab-major), and
+    the fp32 accumulation bound err[i, v] = 2 H 2^-24 sum_k |hidden[i,k] W[v,k]|
+    that separates honest near-ties from wrong answers.  ``rows`` restricts the
+    vocabulary to a slice (for bounded CPU timing)."""
+    x = _f64(hidden)
+    w = _f64(lm_w if rows is None else lm_w[rows])
+    logits = x @ w.T
+    err = 2.0 * x.shape[1] * _U32 * (np.abs(x) @ np.abs(w).T)
+    return logits, err
+
+
+def lm_head_argmax(hidden, lm_w):
+    """decode(p_i) of Eq. (piecewise): greedy decoding, the token of highest
+    probability, i.e. the argmax of the logits.  Ties go to the lowest token id.
+
+    Returns (argmax int32 [sumT], candidates list of int arrays, logits fp64).
+    ``candidates[i]`` holds every token whose logit is within the fp32
+    accumulation bound of the maximum -- any fp32 implementation may return one
+    of them; when it has one element the answer is unique.
+    """
+    logits, err = lm_head_logits(hidden, lm_w)
+    am = np.argmax(logits, axis=1).astype(np.int32)   # first occurrence = lowest id
+    cands = []
+    for i in range(logits.shape[0]):
+        lo = np.max(logits[i] - err[i])
+        cands.append(np.nonzero(logits[i] + err[i] >= lo)[0].astype(np.int32))
+    return am, cands, logits
+
+
+def accept_path(argmax, draft_tok, parent, node_off, max_T=None):
+    """Longest accepted draft path per sequence -- Eq. (piecewise).
+
+    In a linear draft the logits at d_{i-1} (the root for i = 1) give p_i, and
+    d_1..d_j are accepted for the largest j with decode(p_i) = d_i for all
+    i <= j.  In a tree, node u is accepted when every edge (a -> b) on its
+    root-to-u path has draft_tok[b] == argmax[a].  The accepted path is the
+    deepest accepted node's root-to-node path; among equally deep nodes the
+    lowest node id wins (this only matters when siblings carry equal tokens).
+    accept_len = that node's depth (drafts accepted, root excluded); bonus =
+    argmax at that node, the target's own next token (Sec. III-B: the token
+    sampled from the last distribution is kept as well).
+
+    Returns (accept_len int32 [B], path int32 [B, max_T] root-first local ids
+    padded with -1, bonus int32 [B]).
+    """
+    argmax = np.asarray(argmax)
+    draft_tok = np.asarray(draft_tok)
+    parent = np.asarray(parent)
+    node_off = np.asarray(node_off)
+    B = len(node_off) - 1
+    Ts = np.diff(node_off)
+    if max_T is None:
+        max_T = int(Ts.max())
+    accept_len = np.zeros(B, dtype=np.int32)
+    path = np.full((B, max_T), -1, dtype=np.int32)
+    bonus = np.zeros(B, dtype=np.int32)
+    for s in range(B):
+        o, T = int(node_off[s]), int(Ts[s])
+        accepted = [False] * T
+        depth = [0] * T
+        accepted[0] = True
+        for i in range(1, T):
+            p = int(parent[o + i])
+            depth[i] = depth[p] + 1
+            accepted[i] = accepted[p] and int(draft_tok[o + i]) == int(argmax[o + p])
+        best = 0
+        for i in range(1, T):
+            if accepted[i] and depth[i] > depth[best]:
+                best = i
+        chain = []
+        u = best
+        while u != -1:
+            chain.append(u)
+            u = int(parent[o + u]) if u != 0 else -1
+        chain.reverse()
+        accept_len[s] = depth[best]
+        path[s, :len(chain)] = chain
+        bonus[s] = int(argmax[o + best])
+    return accept_len, path, bonus
+
+
+# ----------------------------------------------------------------------------
+# (5) KV compaction of the accepted path -- Sec. IV-A, accepted tokens extend prefix
+# ----------------------------------------------------------------------------
+
+def kv_compact(k_tree, v_tree, k_cache, v_cache, block_table, ctx_len, node_off, path, accept_len):
+    """Append the accepted path's K/V to the paged cache, every layer.
+
+    Sec. IV-A: accepted draft tokens extend the prefix; their keys/values were
+    computed in the verification pass, so they become cache entries.  Path entry
+    k (k = 0..accept_len, the root first) goes to position ctx + k, i.e. slot
+    block_table[(ctx+k) // PAGE] * PAGE + (ctx+k) % PAGE.  The bonus token's K/V
+    is not computed in this pass; it becomes the next root.
+
+    k_tree/v_tree: [L, sumT, n_kv, d]; k_cache/v_cache: [L, num_pages, n_kv,
+    PAGE, d] (numpy, any dtype; copies are returned).
+    Returns (k_cache', v_cache', dst_slot int32 [B, max_T] padded with -1,
+    ctx_len' int32 [B] = ctx + accept_len + 1).
+    """
+    kc = np.array(k_cache, copy=True)
+    vc = np.array(v_cache, copy=True)
+    kt, vt = np.asarray(k_tree), np.asarray(v_tree)
+    node_off = np.asarray(node_off)
+    B = len(node_off) - 1
+    max_T = path.shape[1]
+    dst = np.full((B, max_T), -1, dtype=np.int32)
+    ctx_out = np.asarray(ctx_len, dtype=np.int32).copy()
+    for s in range(B):
+        ctx = int(ctx_len[s])
+        for k in range(int(accept_len[s]) + 1):
+            node = int(path[s, k])
+            pos = ctx + k
+            page = int(block_table[s, pos // PAGE])
+            if page < 0 or page >= kc.shape[1]:
+                raise ValueError("no page allocated for position %d" % pos)
+            off = pos % PAGE
+            dst[s, k] = page * PAGE + off
+            src = int(node_off[s]) + node
+            kc[:, page, :, off, :] = kt[:, src, :, :]
+            vc[:, page, :, off, :] = vt[:, src, :, :]
+        ctx_out[s] = ctx + int(accept_len[s]) + 1
+    return kc, vc, dst, ctx_out
+
+
+# ----------------------------------------------------------------------------
+# Entropy-aware dynamic verification -- Eq. (entropy) and the top_tau rule
+# ----------------------------------------------------------------------------
+
+def entropy_top_tau(logits, k, renormalize=False):
+    """top_tau for one position from its full-vocabulary logits.
+
+    Eq. (entropy): H_norm = -sum_{i<=k} p_i log p_i / log k over the k largest
+    probabilities of the target distribution; top_tau = ceil(k H_norm), or 1
+    when that is below 1.  Reading: p_i are the softmax probabilities over the
+    whole vocabulary, not renormalised over the top k (``renormalize`` gives the
+    other reading); top_tau counts top-k candidates, so it is at most k (H_norm
+    <= 1 for k >= 3 in exact arithmetic; the clamp only absorbs rounding of
+    H_norm = 1).  Returns (top_tau, H_norm, ranked token ids of the top k).
+    """
+    x = _f64(logits)
+    p = np.exp(x - x.max())
+    p /= p.sum()
+    order = np.lexsort((np.arange(len(p)), -p))[:k]      # descending p, ties to lowest id
+    pk = p[order]
+    if renormalize:
+        pk = pk / pk.sum()
+    nz = pk[pk > 0]
+    h = float(-(nz * np.log(nz)).sum() / math.log(k))
+    tau = min(k, max(1, math.ceil(k * h)))
+    return tau, h, order
+
+
+# ----------------------------------------------------------------------------
+# one whole step
+# ----------------------------------------------------------------------------
+
+def verify_step(w, layers=None, vocab_rows=None):
+    """The whole verification step on a workload (workloads.Workload): match,
+    tree structure, attention for the requested layers, LM head + argmax,
+    acceptance and compaction.  ``vocab_rows`` (a slice) restricts the LM head
+    to part of the vocabulary, for bounded CPU timing only."""
+    res = {}
+    res["match_pos"], res["n_matches"] = match_reuse(w.orig_tokens, w.orig_off, w.tail, w.cursor,
+                                                     w.max_matches)
+    depth, anc = tree_prepare(w.parent, w.node_off)
+    res["depth"], res["anc"] = depth, anc
+    layers = range(w.layers) if layers is None else layers
+    res["attn"] = {l: tree_attention(w.q[l], w.k_tree[l], w.v_tree[l], w.k_cache[l], w.v_cache[l],
+                                     w.block_table, w.ctx_len, w.node_off, anc) for l in layers}
+    if vocab_rows is None:
+        am, _, _ = lm_head_argmax(w.hidden_states, w.lm_w)
+    else:
+        logits, _ = lm_head_logits(w.hidden_states, w.lm_w, rows=vocab_rows)
+        am = (np.argmax(logits, axis=1) + (vocab_rows.start or 0)).astype(np.int32)
+    res["argmax"] = am
+    acc, path, bonus = accept_path(am, w.draft_tok, w.parent, w.node_off, w.max_T)
+    res["accept_len"], res["path"], res["bonus"] = acc, path, bonus
+    lay = list(layers)
+    res["k_cache"], res["v_cache"], res["dst_slot"], res["ctx_out"] = kv_compact(
+        _raw16(w.k_tree[lay]), _raw16(w.v_tree[lay]), _raw16(w.k_cache[lay]), _raw16(w.v_cache[lay]),
+        w.block_table, w.ctx_len, w.node_off, path, acc)
+    return res

@@ -1,0 +1,471 @@
+"""Pins of the fp64 oracle to facts outside itself (CPU only).
+
+Each test checks an oracle function against something it does not contain:
+hand-worked golden cases (tests/golden/, each citing its equation), a brute
+force written a different way, a library routine on a special case, a closed
+form, or an answer the input generator planted.  A plausible slip in the
+oracle -- a dropped term, a wrong sign, an off-by-one, a transposed operand, a
+wrong GQA head map -- fails at least one of them.
+"""
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+import torch
+import torch.nn.functional as F
+
+import oracle as O
+import workloads as W
+
+GOLD = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def _gold(name):
+    with open(os.path.join(GOLD, name)) as f:
+        return json.load(f)
+
+
+def _bf16_np(t):
+    return t.detach().cpu().double().numpy()
+
+
+# ----------------------------------------------------------------------------
+# match
+# ----------------------------------------------------------------------------
+
+@pytest.mark.parametrize("case", _gold("match_cases.json")["cases"], ids=lambda c: c["name"])
+def test_match_golden(case):
+    c = np.asarray(case["c"], dtype=np.int32)
+    tail = np.asarray([case["tail"]], dtype=np.int32)
+    pos, cnt = O.match_reuse(c, np.asarray([0, len(c)]), tail, np.asarray([case["cursor"]]), 4)
+    k = case["n_matches"]
+    assert cnt[0] == k
+    assert list(pos[0, :min(k, 4)]) == case["match_pos"][:4]
+    assert np.all(pos[0, min(k, 4):] == -1)
+
+
+def _bytes_find_all(c, tail, cursor):
+    """Brute force by a different route: byte-string search over 4-byte tokens."""
+    hay = np.asarray(c, dtype=">i4").tobytes()
+    needle = np.asarray(tail, dtype=">i4").tobytes()
+    out, start = [], 0
+    while True:
+        i = hay.find(needle, start)
+        if i < 0:
+            break
+        if i % 4 == 0:
+            p = i // 4
+            if p >= cursor and p + len(tail) < len(c):
+                out.append(p)
+        start = i + 1
+    return out
+
+
+@pytest.mark.parametrize("n", [2, 4, 8])
+def test_match_bruteforce_sweep(n):
+    w = W.build("sweep", B=6, layers=1, n=n, seed=77 + n)
+    pos, cnt = O.match_reuse(w.orig_tokens, w.orig_off, w.tail, w.cursor, 5)
+    for s in range(w.B):
+        ref = _bytes_find_all(w.seq_tokens(s), w.tail[s], int(w.cursor[s]))
+        assert cnt[s] == len(ref)
+        assert list(pos[s, :min(5, len(ref))]) == ref[:5]
+        if w.planted_match[s] >= 0:
+            assert w.planted_match[s] in ref or len(ref) > 5
+
+
+def test_match_closed_form_constant_code():
+    L, n = 50, 3
+    c = np.full(L, 9, dtype=np.int32)
+    for cur in [0, 5, 46, 47, 60]:
+        pos, cnt = O.match_reuse(c, np.asarray([0, L]), np.full((1, n), 9, np.int32), np.asarray([cur]), 64)
+        # every p with cur <= p <= L - n - 1 matches
+        want = list(range(cur, L - n))
+        assert cnt[0] == len(want)
+        assert list(pos[0, :len(want)]) == want
+
+
+def test_match_planted_tiny():
+    w = W.build("tiny")
+    pos, cnt = O.match_reuse(w.orig_tokens, w.orig_off, w.tail, w.cursor, w.max_matches)
+    assert pos[0, 0] == w.planted_match[0] == 296
+    # the reuse chain the generator built starts at the last matched token
+    c = w.seq_tokens(0)
+    p, n = int(pos[0, 0]), w.n
+    assert list(w.draft_tok[:12]) == list(c[p + n - 1:p + n + 11])
+
+
+def test_match_rejects_bad_args():
+    with pytest.raises(ValueError):
+        O.match_reuse(np.arange(5, dtype=np.int32), np.asarray([0, 5]), np.zeros((1, 2), np.int32),
+                      np.asarray([-1]), 2)
+
+
+# ----------------------------------------------------------------------------
+# tree structure
+# ----------------------------------------------------------------------------
+
+def _walk_up(parent, o, i):
+    path = []
+    u = i
+    while u != -1:
+        path.append(u)
+        u = int(parent[o + u])
+    return path[::-1]
+
+
+def test_tree_prepare_closed_forms():
+    chain = np.asarray([-1] + list(range(127)), dtype=np.int32)
+    star = np.asarray([-1] + [0] * 9, dtype=np.int32)
+    parent = np.concatenate([chain, star])
+    off = np.asarray([0, 128, 138])
+    depth, anc = O.tree_prepare(parent, off)
+    for i in range(128):
+        assert depth[i] == i
+        assert O.anc_to_sets(anc[i]) == set(range(i + 1))
+    for i in range(10):
+        assert depth[128 + i] == (0 if i == 0 else 1)
+        assert O.anc_to_sets(anc[128 + i]) == ({0} if i == 0 else {0, i})
+    # bit layout: node 127 of the chain sets every bit of both words
+    assert int(anc[127, 0]) == 2 ** 64 - 1 and int(anc[127, 1]) == 2 ** 64 - 1
+
+
+def test_tree_prepare_walk_up():
+    w = W.build("batched", layers=1, vocab=512, hidden=64, seed=5)
+    depth, anc = O.tree_prepare(w.parent, w.node_off)
+    for s in range(w.B):
+        o, T = int(w.node_off[s]), int(w.node_off[s + 1] - w.node_off[s])
+        for i in range(T):
+            p = _walk_up(w.parent, o, i)
+            assert depth[o + i] == len(p) - 1
+            assert O.anc_to_sets(anc[o + i]) == set(p)
+
+
+@pytest.mark.parametrize("parent", [[0, 0], [-1, 1], [-1, 0, 3, 1], [-1, -1]])
+def test_tree_prepare_rejects(parent):
+    with pytest.raises(ValueError):
+        O.tree_prepare(np.asarray(parent, np.int32), np.asarray([0, len(parent)]))
+
+
+# ----------------------------------------------------------------------------
+# attention
+# ----------------------------------------------------------------------------
+
+def _linear_kv(w, layer, s, hk, path_nodes, cache):
+    """Keys (or values) of the linear sequence context + path, gathered one position
+    at a time through the block table."""
+    kc, kt = (w.k_cache, w.k_tree) if cache == "k" else (w.v_cache, w.v_tree)
+    rows = []
+    for pos in range(int(w.ctx_len[s])):
+        page = int(w.block_table[s, pos // W.PAGE])
+        rows.append(kc[layer, page, hk, pos % W.PAGE])
+    o = int(w.node_off[s])
+    for j in path_nodes:
+        rows.append(kt[layer, o + j, hk])
+    return torch.stack(rows).double()
+
+
+def _sdpa_last(qv, keys, vals):
+    """torch SDPA (fp64, math backend) for one query vector at the end of a sequence."""
+    return F.scaled_dot_product_attention(qv[None, None, None, :], keys[None, None], vals[None, None])[0, 0, 0]
+
+
+@pytest.mark.parametrize("q_std", [1.0, 40.0])
+def test_attention_each_node_is_causal_attention_over_its_path(q_std):
+    tree = W.TreeSpec(6, [(0, 3), (3, 2)], [0, 1, 2])
+    w = W.build("tiny", ctx=37, trees=[tree, W.TreeSpec(3, [(1, 2)], [0])], q_std=q_std)
+    depth, anc = O.tree_prepare(w.parent, w.node_off)
+    out = O.tree_attention(w.q[0], w.k_tree[0], w.v_tree[0], w.k_cache[0], w.v_cache[0],
+                           w.block_table, w.ctx_len, w.node_off, anc)
+    g = w.n_q // w.n_kv
+    for s in range(w.B):
+        o, T = int(w.node_off[s]), int(w.node_off[s + 1] - w.node_off[s])
+        for i in range(T):
+            path = _walk_up(w.parent, o, i)
+            for h in range(w.n_q):
+                keys = _linear_kv(w, 0, s, h // g, path, "k")
+                vals = _linear_kv(w, 0, s, h // g, path, "v")
+                ref = _sdpa_last(w.q[0, o + i, h].double(), keys, vals).numpy()
+                np.testing.assert_allclose(out[o + i, h], ref, rtol=0, atol=1e-12)
+
+
+def test_attention_chain_equals_masked_sdpa():
+    """A chain-only tree is the paper's linear draft: causal attention over ctx + T."""
+    w = W.build("tiny", ctx=45, trees=[W.TreeSpec(9, [], [0, 1])])
+    depth, anc = O.tree_prepare(w.parent, w.node_off)
+    out = O.tree_attention(w.q[0], w.k_tree[0], w.v_tree[0], w.k_cache[0], w.v_cache[0],
+                           w.block_table, w.ctx_len, w.node_off, anc)
+    T, ctx, g = 9, 45, w.n_q // w.n_kv
+    keys = torch.stack([_linear_kv(w, 0, 0, hk, range(T), "k") for hk in range(w.n_kv)])
+    vals = torch.stack([_linear_kv(w, 0, 0, hk, range(T), "v") for hk in range(w.n_kv)])
+    keys = keys.repeat_interleave(g, dim=0)        # [n_q, ctx+T, d]
+    vals = vals.repeat_interleave(g, dim=0)
+    qq = w.q[0, :T].double().permute(1, 0, 2)      # [n_q, T, d]
+    mask = torch.arange(ctx + T)[None, :] <= (ctx + torch.arange(T))[:, None]
+    ref = F.scaled_dot_product_attention(qq[None], keys[None], vals[None], attn_mask=mask)[0]
+    np.testing.assert_allclose(out[:T], ref.permute(1, 0, 2).numpy(), rtol=0, atol=1e-12)
+
+
+def test_attention_single_key_returns_value():
+    """T = 1 and ctx = 0: softmax over one key is 1, the output is that value row."""
+    w = W.build("tiny", ctx=0, trees=[W.TreeSpec(1, [], [0])])
+    depth, anc = O.tree_prepare(w.parent, w.node_off)
+    out = O.tree_attention(w.q[0], w.k_tree[0], w.v_tree[0], w.k_cache[0], w.v_cache[0],
+                           w.block_table, w.ctx_len, w.node_off, anc)
+    g = w.n_q // w.n_kv
+    for h in range(w.n_q):
+        assert np.array_equal(out[0, h], _bf16_np(w.v_tree[0, 0, h // g]))
+
+
+def test_attention_equal_keys_average_values():
+    """All keys equal: the softmax is uniform and the output is the plain mean of the values."""
+    w = W.build("tiny", ctx=21, trees=[W.TreeSpec(4, [(1, 2)], [0])])
+    w.k_cache[:] = 0.25
+    w.k_tree[:] = 0.25
+    depth, anc = O.tree_prepare(w.parent, w.node_off)
+    out = O.tree_attention(w.q[0], w.k_tree[0], w.v_tree[0], w.k_cache[0], w.v_cache[0],
+                           w.block_table, w.ctx_len, w.node_off, anc)
+    g = w.n_q // w.n_kv
+    node = 5                              # second node of the branch hanging off node 1
+    path = _walk_up(w.parent, 0, node)
+    for h in range(w.n_q):
+        vals = _linear_kv(w, 0, 0, h // g, path, "v").numpy()
+        np.testing.assert_allclose(out[node, h], vals.mean(axis=0), rtol=0, atol=1e-14)
+
+
+def test_attention_page_order_invariance():
+    w = W.build("tiny", ctx=70)
+    depth, anc = O.tree_prepare(w.parent, w.node_off)
+    args = (w.block_table, w.ctx_len, w.node_off, anc)
+    ref = O.tree_attention(w.q[0], w.k_tree[0], w.v_tree[0], w.k_cache[0], w.v_cache[0], *args)
+    rng = np.random.default_rng(3)
+    perm = rng.permutation(w.num_pages)                 # new page p' = perm[p]
+    kc = torch.empty_like(w.k_cache[0])
+    vc = torch.empty_like(w.v_cache[0])
+    kc[torch.as_tensor(perm)] = w.k_cache[0]
+    vc[torch.as_tensor(perm)] = w.v_cache[0]
+    bt = np.where(w.block_table >= 0, perm[np.maximum(w.block_table, 0)], -1).astype(np.int32)
+    got = O.tree_attention(w.q[0], w.k_tree[0], w.v_tree[0], kc, vc, bt, w.ctx_len, w.node_off, anc)
+    np.testing.assert_allclose(got, ref, rtol=0, atol=1e-13)
+
+
+def test_attention_gqa_head_map():
+    """Query head h reads KV head h // g: perturbing KV head 1 moves heads g..2g-1 only."""
+    w = W.build("tiny", ctx=33)
+    depth, anc = O.tree_prepare(w.parent, w.node_off)
+    args = (w.block_table, w.ctx_len, w.node_off, anc)
+    ref = O.tree_attention(w.q[0], w.k_tree[0], w.v_tree[0], w.k_cache[0], w.v_cache[0], *args)
+    vc = w.v_cache[0].clone()
+    vc[:, 1] += 1.0
+    got = O.tree_attention(w.q[0], w.k_tree[0], w.v_tree[0], w.k_cache[0], vc, *args)
+    g = w.n_q // w.n_kv
+    moved = np.abs(got - ref).max(axis=(0, 2)) > 1e-6
+    assert list(np.nonzero(moved)[0]) == list(range(g, 2 * g))
+
+
+# ----------------------------------------------------------------------------
+# LM head and argmax
+# ----------------------------------------------------------------------------
+
+def test_lm_head_pure_python_dot():
+    w = W.build("tiny", vocab=37, hidden=24, trees=[W.TreeSpec(3, [], [0])])
+    logits, err = O.lm_head_logits(w.hidden_states, w.lm_w)
+    x = w.hidden_states.double().tolist()
+    wt = w.lm_w.double().tolist()
+    for i in range(len(x)):
+        for v in range(37):
+            ref = math.fsum(a * b for a, b in zip(x[i], wt[v]))
+            assert abs(logits[i, v] - ref) <= 1e-12 * (1 + abs(ref))
+            assert err[i, v] >= 0
+
+
+@pytest.mark.parametrize("name,ov", [("tiny", {}), ("7b", dict(layers=1, vocab=8192, hidden=768)),
+                                     ("batched", dict(layers=1, vocab=6000, hidden=320))])
+def test_lm_head_planted_argmax(name, ov):
+    w = W.build(name, **ov)
+    am, cands, _ = O.lm_head_argmax(w.hidden_states, w.lm_w)
+    planted = w.planted_argmax >= 0
+    assert planted.sum() > 0
+    np.testing.assert_array_equal(am[planted], w.planted_argmax[planted])
+    for i in np.nonzero(planted)[0]:
+        assert list(cands[i]) == [w.planted_argmax[i]]
+
+
+def test_lm_head_duplicate_rows_lowest_id():
+    w = W.build("tiny", dup_rows=3)
+    am, cands, logits = O.lm_head_argmax(w.hidden_states, w.lm_w)
+    planted = w.planted_argmax >= 0
+    np.testing.assert_array_equal(am[planted], w.planted_argmax[planted])
+    tied = [i for i in np.nonzero(planted)[0] if len(cands[i]) > 1]
+    assert tied, "duplicated rows must create exact ties"
+    for i in tied:
+        top = np.nonzero(logits[i] == logits[i].max())[0]
+        assert len(top) == 2 and am[i] == top.min()
+
+
+def test_lm_head_identity_closed_form():
+    """W rows = unit vectors e_v (v < H): logits are the hidden coordinates."""
+    H = 64
+    x = torch.randn(5, H, generator=torch.Generator().manual_seed(0)).to(torch.bfloat16)
+    wmat = torch.eye(H, dtype=torch.bfloat16)
+    am, cands, logits = O.lm_head_argmax(x, wmat)
+    np.testing.assert_array_equal(logits, x.double().numpy())
+    np.testing.assert_array_equal(am, np.argmax(x.double().numpy(), axis=1))
+
+
+# ----------------------------------------------------------------------------
+# acceptance
+# ----------------------------------------------------------------------------
+
+@pytest.mark.parametrize("case", _gold("accept_cases.json")["cases"], ids=lambda c: c["name"])
+def test_accept_golden(case):
+    parent = np.asarray(case["parent"], np.int32)
+    off = np.asarray([0, len(parent)])
+    acc, path, bonus = O.accept_path(np.asarray(case["argmax"]), np.asarray(case["draft_tok"]), parent, off)
+    assert acc[0] == case["accept_len"]
+    assert list(path[0, :acc[0] + 1]) == case["path"]
+    assert np.all(path[0, acc[0] + 1:] == -1)
+    assert bonus[0] == case["bonus"]
+
+
+def _replay_chain(argmax, draft):
+    """Eq. (piecewise) read literally: largest j with decode(p_i) == d_i for all i <= j."""
+    j = 0
+    while j + 1 < len(draft) and argmax[j] == draft[j + 1]:
+        j += 1
+    return j
+
+
+def _brute_longest(argmax, draft, parent):
+    """Every root-to-node path checked by replay; deepest accepted node, lowest id."""
+    best, best_len = 0, 0
+    for u in range(len(parent)):
+        path = _walk_up(parent, 0, u)
+        ok = all(draft[b] == argmax[a] for a, b in zip(path[:-1], path[1:]))
+        if ok and len(path) - 1 > best_len:
+            best, best_len = u, len(path) - 1
+    return best, best_len
+
+
+def test_accept_chain_replay_random():
+    rng = np.random.default_rng(11)
+    for _ in range(300):
+        T = int(rng.integers(1, 40))
+        draft = rng.integers(0, 3, size=T)
+        am = rng.integers(0, 3, size=T)
+        parent = np.asarray([-1] + list(range(T - 1)), np.int32)
+        acc, path, bonus = O.accept_path(am, draft, parent, np.asarray([0, T]))
+        j = _replay_chain(am, draft)
+        assert acc[0] == j and list(path[0, :j + 1]) == list(range(j + 1)) and bonus[0] == am[j]
+
+
+def test_accept_tree_bruteforce_random():
+    rng = np.random.default_rng(12)
+    for _ in range(300):
+        T = int(rng.integers(1, 30))
+        parent = np.asarray([-1] + [int(rng.integers(0, i)) for i in range(1, T)], np.int32)
+        draft = rng.integers(0, 3, size=T)          # small alphabet: equal siblings happen
+        am = rng.integers(0, 3, size=T)
+        acc, path, bonus = O.accept_path(am, draft, parent, np.asarray([0, T]))
+        u, d = _brute_longest(am, draft, parent)
+        assert acc[0] == d
+        assert list(path[0, :d + 1]) == _walk_up(parent, 0, u)
+        assert bonus[0] == am[u]
+
+
+@pytest.mark.parametrize("name", ["tiny", "7b", "batched", "33b"])
+def test_accept_planted(name):
+    w = W.build(name, layers=1, vocab=4096, hidden=256) if name != "tiny" else W.build(name)
+    am = np.where(w.planted_argmax >= 0, w.planted_argmax, -7)
+    acc, path, bonus = O.accept_path(am, w.draft_tok, w.parent, w.node_off)
+    np.testing.assert_array_equal(acc, w.planted_accept)
+    for s in range(w.B):
+        assert list(path[s, :acc[s] + 1]) == w.planted_path[s]
+
+
+# ----------------------------------------------------------------------------
+# compaction
+# ----------------------------------------------------------------------------
+
+@pytest.mark.parametrize("case", _gold("compact_cases.json")["cases"], ids=lambda c: c["name"])
+def test_compact_golden(case):
+    L, n_kv, d, T = 2, 2, 4, 8
+    npg = max(case["block_table"]) + 1
+    kt = np.arange(L * T * n_kv * d, dtype=np.float64).reshape(L, T, n_kv, d)
+    vt = -kt
+    kc = np.zeros((L, npg, n_kv, 16, d))
+    vc = np.zeros_like(kc)
+    path = np.full((1, T), -1, np.int32)
+    path[0, :len(case["path"])] = case["path"]
+    kc2, vc2, dst, ctx_out = O.kv_compact(kt, vt, kc, vc, np.asarray([case["block_table"]]),
+                                          np.asarray([case["ctx"]]), np.asarray([0, T]), path,
+                                          np.asarray([case["accept_len"]]))
+    assert list(dst[0, :len(case["dst_slot"])]) == case["dst_slot"]
+    assert ctx_out[0] == case["ctx_out"]
+    for k, slot in enumerate(case["dst_slot"]):
+        np.testing.assert_array_equal(kc2[:, slot // 16, :, slot % 16], kt[:, case["path"][k]])
+        np.testing.assert_array_equal(vc2[:, slot // 16, :, slot % 16], vt[:, case["path"][k]])
+
+
+def test_compact_sequential_append_and_canary():
+    w = W.build("sweep", B=5, layers=2, seed=9)
+    kt = w.k_tree.view(torch.int16).numpy()
+    vt = w.v_tree.view(torch.int16).numpy()
+    kc = w.k_cache.view(torch.int16).numpy()
+    vc = w.v_cache.view(torch.int16).numpy()
+    T = w.max_T
+    path = np.full((w.B, T), -1, np.int32)
+    for s in range(w.B):
+        path[s, :len(w.planted_path[s])] = w.planted_path[s]
+    kc2, vc2, dst, ctx_out = O.kv_compact(kt, vt, kc, vc, w.block_table, w.ctx_len, w.node_off, path,
+                                          w.planted_accept)
+    # independent: a dict of slots filled by appending, position by position
+    slots = {}
+    for s in range(w.B):
+        pos = int(w.ctx_len[s])
+        for node in w.planted_path[s]:
+            page = int(w.block_table[s, pos // 16])
+            slots[(page, pos % 16)] = int(w.node_off[s]) + node
+            pos += 1
+        assert ctx_out[s] == pos
+    for (page, off), src in slots.items():
+        assert np.array_equal(kc2[:, page, :, off], kt[:, src])
+        assert np.array_equal(vc2[:, page, :, off], vt[:, src])
+    # canary: every other slot keeps its bytes
+    keep = np.ones((w.num_pages, 16), bool)
+    for (page, off) in slots:
+        keep[page, off] = False
+    def by_slot(a):
+        return a.transpose(0, 1, 3, 2, 4)[:, keep]      # [L, pages, PAGE, n_kv, d] -> kept slots
+    assert np.array_equal(by_slot(kc2), by_slot(kc)) and np.array_equal(by_slot(vc2), by_slot(vc))
+
+
+# ----------------------------------------------------------------------------
+# entropy-aware verification (Eq. (entropy))
+# ----------------------------------------------------------------------------
+
+@pytest.mark.parametrize("case", _gold("entropy_cases.json")["cases"], ids=lambda c: c["name"])
+def test_entropy_golden(case):
+    p = np.asarray(case["probs"])
+    with np.errstate(divide="ignore"):
+        logits = np.where(p > 0, np.log(np.where(p > 0, p, 1.0)), -np.inf)
+    tau, h, order = O.entropy_top_tau(logits, case["k"])
+    assert tau == case["top_tau"]
+    assert abs(h - case["h_norm"]) < 1e-5
+    assert p[order[0]] == p.max()
+
+
+# ----------------------------------------------------------------------------
+# whole step on the tiny configuration
+# ----------------------------------------------------------------------------
+
+def test_verify_step_tiny_planted():
+    w = W.build("tiny")
+    r = O.verify_step(w)
+    assert r["match_pos"][0, 0] == 296
+    assert r["accept_len"][0] == w.planted_accept[0] == 7
+    assert list(r["path"][0, :8]) == list(range(8))
+    assert r["ctx_out"][0] == 512 + 8
+    assert r["bonus"][0] == w.planted_argmax[7]
+    assert not np.isnan(r["attn"][0]).any()
