@@ -1,0 +1,218 @@
+/*
+ * ee.h -- C ABI of the GB300 (sm_103a) verification-step library (libee.so).
+ *
+ * One verification step of EfficientEdit's edit-oriented speculative decoding
+ * (arXiv 2506.02780, Sec. IV-A): a draft tree -- a span of the original code
+ * reused verbatim plus short generated branches -- is scored in one target
+ * pass and the longest draft prefix on which the target's greedy choice agrees
+ * is accepted (Eq. (piecewise)).  The entry points are the steps of that pass:
+ *
+ *   ee_match_reuse       reuse-span lookup in the original code     (Sec. IV-A)
+ *   ee_tree_prepare      depth / ancestor masks of the draft tree
+ *   ee_tree_verify_attn  tree-masked attention over the paged cache (Sec. IV-A)
+ *   ee_lmhead_accept     LM head + argmax + longest accepted path   (Eq. piecewise)
+ *   ee_kv_compact        accepted path's K/V appended to the cache  (Sec. IV-A)
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ *  - Every pointer argument except `ws` in ee_read_errors' output is a DEVICE
+ *    pointer owned by the caller.  The library never allocates device memory,
+ *    never frees, never synchronises (except ee_read_errors) and enqueues all
+ *    work on `stream` (NULL = legacy default stream).
+ *  - Integer arrays are int32 unless stated; bf16 arrays are raw bf16 bit
+ *    patterns (ee_bf16), row-major, densely packed.
+ *  - Tree nodes: sequence s owns global nodes node_off[s] .. node_off[s+1]-1;
+ *    their LOCAL ids are 0..T_s-1, local 0 is the root (the last committed
+ *    token, whose K/V is computed in this pass), parent[i] holds the LOCAL
+ *    parent id, parent[0] = -1 and 0 <= parent[i] < i.  1 <= T_s <= 128.
+ *  - Paged KV cache: page = EE_PAGE tokens; one layer is laid out
+ *    [num_pages][n_kv][EE_PAGE][head_dim]; position t of sequence s lives in
+ *    page block_table[s * max_pages + t / EE_PAGE], row t % EE_PAGE.
+ *  - `ws` is a caller-owned device workspace of at least
+ *    ee_workspace_size(...) bytes, zeroed once with ee_workspace_init() before
+ *    first use.  Its first word is the device error word: kernels never trap;
+ *    on a bad index found on the device they set an EE_DEVERR_* bit there,
+ *    skip the access and continue.  ee_read_errors() reads (and clears) it.
+ *    After any error the workspace must be re-initialised.  Calls that share
+ *    one workspace must be ordered on one stream.
+ *  - Return value: EE_OK when the work was enqueued.  Host-side argument checks
+ *    run before any launch and return EE_ERR_INVALID_ARG / EE_ERR_UNSUPPORTED
+ *    without touching memory.  EE_ERR_CUDA reports a launch failure.
+ */
+#ifndef EE_H_
+#define EE_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define EE_PAGE 16
+#define EE_HEAD_DIM 128
+#define EE_MAX_TREE 128
+#define EE_MAX_NGRAM 32
+#define EE_MAX_MATCHES 1024
+#define EE_MAX_LM_NODES 2048
+
+typedef uint16_t ee_bf16;                 /* raw bfloat16 bits */
+typedef struct CUstream_st* ee_stream_t;  /* same type as cudaStream_t */
+
+typedef enum {
+  EE_OK = 0,
+  EE_ERR_INVALID_ARG = 1,   /* null pointer, bad size or alignment */
+  EE_ERR_UNSUPPORTED = 2,   /* valid but outside what the kernels support */
+  EE_ERR_CUDA = 3,          /* a CUDA call or launch failed */
+  EE_ERR_DEVICE = 4,        /* the device error word was set (ee_read_errors) */
+  EE_ERR_WORKSPACE = 5      /* ws_bytes smaller than ee_workspace_size() */
+} ee_status;
+
+/* Bits of the device error word. */
+#define EE_DEVERR_MATCH_ARGS   0x01  /* cursor < 0 or orig_off decreasing */
+#define EE_DEVERR_TREE         0x02  /* parent[] violates 0 <= parent[i] < i, or T outside 1..128 */
+#define EE_DEVERR_PAGE         0x04  /* block_table entry outside [0, num_pages) for a needed slot */
+#define EE_DEVERR_CTX          0x08  /* ctx_len < 0 or above the max_ctx passed by the host */
+#define EE_DEVERR_FP16_RANGE   0x10  /* |V| > 65504: P.V runs in fp16 and V did not fit */
+#define EE_DEVERR_TIMEOUT      0x20  /* a bounded device wait gave up */
+#define EE_DEVERR_PATH         0x40  /* path / accept_len inconsistent with the tree */
+
+const char* ee_version(void);
+const char* ee_status_string(ee_status s);
+
+/*
+ * Workspace bytes needed by every entry point for problems up to these sizes:
+ * B sequences, total_nodes tree nodes in all, n_q query heads, max_ctx cached
+ * positions in the longest sequence.  The buffer must be 256-byte aligned.
+ */
+size_t ee_workspace_size(int32_t B, int32_t total_nodes, int32_t n_q, int32_t head_dim,
+                         int32_t max_ctx);
+
+/* Zero `ws` (asynchronously, on `stream`).  Call once after allocating it. */
+ee_status ee_workspace_init(void* ws, size_t ws_bytes, ee_stream_t stream);
+
+/*
+ * Synchronise `stream`, copy the device error word to *bits (host pointer),
+ * clear it on the device.  Returns EE_ERR_DEVICE when any bit was set.
+ */
+ee_status ee_read_errors(void* ws, ee_stream_t stream, int32_t* bits);
+
+/*
+ * ee_match_reuse -- reuse-span lookup (Sec. IV-A, prefix matching that switches
+ * Generate back to Reuse).  For each sequence s, with c = orig_tokens[
+ * orig_off[s] .. orig_off[s+1]) and t = tail[s*n .. s*n+n) (the last n generated
+ * tokens), finds every position p with cursor[s] <= p and p + n < len(c) and
+ * c[p+i] == t[i] for all i < n.  The p + n < len(c) rule keeps at least one
+ * token of c after the match to serve as draft.
+ *   orig_tokens  int32 [orig_off[B]]   original code of all sequences, CSR
+ *   orig_off     int64 [B+1]           non-decreasing offsets
+ *   tail         int32 [B][n]          1 <= n <= EE_MAX_NGRAM
+ *   cursor       int32 [B]             start of the unverified remainder of c
+ *   match_pos    int32 [B][max_matches] out: matches in ascending order, -1 pad
+ *   n_matches    int32 [B]             out: total number of matches (may exceed
+ *                                      max_matches; 1 <= max_matches <= 1024)
+ * Device errors: EE_DEVERR_MATCH_ARGS (that sequence reports 0 matches).
+ */
+ee_status ee_match_reuse(const int32_t* orig_tokens, const int64_t* orig_off, int32_t B,
+                         const int32_t* tail, int32_t n, const int32_t* cursor,
+                         int32_t max_matches, int32_t* match_pos, int32_t* n_matches,
+                         void* ws, size_t ws_bytes, ee_stream_t stream);
+
+/*
+ * ee_tree_prepare -- draft-tree structure.  depth[root] = 0, depth[i] =
+ * depth[parent[i]] + 1; anc[i] = anc[parent[i]] U {i}, stored as two uint64
+ * words per node (bit j of word j/64 = local node j is on the root-to-i path).
+ *   parent    int32 [total_nodes]   local parent ids (see conventions)
+ *   node_off  int32 [B+1]
+ *   depth     int32 [total_nodes]   out
+ *   anc       uint64 [total_nodes][2] out
+ * Device errors: EE_DEVERR_TREE (that sequence's depth/anc are zeroed).
+ */
+ee_status ee_tree_prepare(const int32_t* parent, const int32_t* node_off, int32_t B,
+                          int32_t total_nodes, int32_t* depth, uint64_t* anc,
+                          void* ws, size_t ws_bytes, ee_stream_t stream);
+
+/*
+ * ee_tree_verify_attn -- tree-masked attention of every draft node, ONE layer
+ * (Sec. IV-A: one target pass over (prefix, draft)).  Node i of sequence s,
+ * query head h, attends to cached positions 0..ctx_len[s]-1 and to the tree
+ * nodes in anc[i] (its own root-to-i path):
+ *   out[i][h] = sum_j softmax_j(scale * q[i][h] . k_j) v_j,  KV head h / (n_q/n_kv).
+ *   q         bf16 [total_nodes][n_q][head_dim]   (post-RoPE)
+ *   k_tree    bf16 [total_nodes][n_kv][head_dim]  K/V of the tree nodes, this layer
+ *   v_tree    bf16 [total_nodes][n_kv][head_dim]
+ *   k_cache   bf16 [num_pages][n_kv][EE_PAGE][head_dim]  this layer's cache
+ *   v_cache   bf16 same
+ *   block_table int32 [B][max_pages]; ctx_len int32 [B], 0 <= ctx_len <= max_ctx
+ *   node_off  int32 [B+1]; anc uint64 [total_nodes][2] from ee_tree_prepare
+ *   out       fp32 [total_nodes][n_q][head_dim]   out
+ * head_dim must be 128; n_q a multiple of n_kv; max_T <= 128; all bf16 arrays
+ * 16-byte aligned.  Q.K runs on bf16 tensor cores with fp32 accumulation; P.V
+ * runs with P and V in fp16 (exact for |V| <= 65504, larger values set
+ * EE_DEVERR_FP16_RANGE); softmax and the output are fp32.
+ * Device errors: EE_DEVERR_PAGE (the key is skipped), EE_DEVERR_CTX.
+ */
+ee_status ee_tree_verify_attn(const ee_bf16* q, const ee_bf16* k_tree, const ee_bf16* v_tree,
+                              const ee_bf16* k_cache, const ee_bf16* v_cache, int32_t num_pages,
+                              const int32_t* block_table, int32_t max_pages, const int32_t* ctx_len,
+                              int32_t max_ctx, const int32_t* node_off, const uint64_t* anc,
+                              int32_t B, int32_t total_nodes, int32_t max_T, int32_t n_q,
+                              int32_t n_kv, int32_t head_dim, float scale, float* out,
+                              void* ws, size_t ws_bytes, ee_stream_t stream);
+
+/*
+ * ee_lmhead_accept -- LM head fused with greedy decode and acceptance
+ * (Eq. (piecewise)).  logits[i][v] = hidden[i] . lm_w[v] (fp32 accumulate of
+ * bf16 products, never stored unless logits_or_null is given);
+ * argmax[i] = the highest logit, lowest token id on ties.  Node i (i > 0) is
+ * accepted when every edge a -> b on its root path has draft_tok[b] ==
+ * argmax[a]; the deepest accepted node u* wins (lowest local id among equally
+ * deep ones):
+ *   accept_len[s] = depth[u*]   (draft tokens accepted, root excluded)
+ *   path[s][0..accept_len]      local ids root -> u*, rest of the row -1
+ *   bonus[s] = argmax[u*]       the target's next token after the accepted path
+ *   hidden    bf16 [total_nodes][hidden_dim]
+ *   lm_w      bf16 [vocab][hidden_dim]  (vocab-major)
+ *   draft_tok int32 [total_nodes]; parent int32 [total_nodes];
+ *   depth int32 / anc uint64[2] from ee_tree_prepare; node_off int32 [B+1]
+ *   argmax int32 [total_nodes]; accept_len/bonus int32 [B]; path int32 [B][max_T]
+ *   logits_or_null fp32 [total_nodes][vocab] or NULL
+ * hidden_dim a multiple of 8; total_nodes <= EE_MAX_LM_NODES; hidden and lm_w
+ * 16-byte aligned.  Runs as one persistent tcgen05/TMEM GEMM (vocab rows on
+ * the MMA M side) whose epilogue keeps the running argmax; the last CTA to
+ * finish runs the acceptance.
+ * Device errors: EE_DEVERR_TIMEOUT (outputs undefined).
+ */
+ee_status ee_lmhead_accept(const ee_bf16* hidden, const ee_bf16* lm_w, int32_t hidden_dim,
+                           int32_t vocab, const int32_t* draft_tok, const int32_t* parent,
+                           const int32_t* depth, const uint64_t* anc, const int32_t* node_off,
+                           int32_t B, int32_t total_nodes, int32_t max_T, int32_t* argmax,
+                           int32_t* accept_len, int32_t* path, int32_t* bonus,
+                           float* logits_or_null, void* ws, size_t ws_bytes, ee_stream_t stream);
+
+/*
+ * ee_kv_compact -- append the accepted path's K/V to the paged cache, every
+ * layer (Sec. IV-A: accepted tokens extend the prefix).  Path entry k
+ * (k = 0..accept_len[s], root first) of sequence s goes to position
+ * ctx_len_in[s] + k; ctx_len_out[s] = ctx_len_in[s] + accept_len[s] + 1.
+ *   k_tree/v_tree  bf16, layer l at + l*tree_layer_stride elements, each layer
+ *                  [total_nodes][n_kv][head_dim]
+ *   k_cache/v_cache bf16, layer l at + l*cache_layer_stride elements, each layer
+ *                  [num_pages][n_kv][EE_PAGE][head_dim]
+ *   path int32 [B][max_T], accept_len int32 [B] (from ee_lmhead_accept)
+ *   dst_slot int32 [B][max_T] out: page*EE_PAGE + row of each appended entry, -1 pad
+ *   ctx_len_out must not alias ctx_len_in.
+ * Device errors: EE_DEVERR_PAGE (entry skipped), EE_DEVERR_PATH.
+ */
+ee_status ee_kv_compact(const ee_bf16* k_tree, const ee_bf16* v_tree, int64_t tree_layer_stride,
+                        ee_bf16* k_cache, ee_bf16* v_cache, int64_t cache_layer_stride, int32_t L,
+                        int32_t num_pages, const int32_t* block_table, int32_t max_pages,
+                        const int32_t* ctx_len_in, int32_t* ctx_len_out, const int32_t* node_off,
+                        const int32_t* path, const int32_t* accept_len, int32_t B, int32_t max_T,
+                        int32_t n_kv, int32_t head_dim, int32_t* dst_slot,
+                        void* ws, size_t ws_bytes, ee_stream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* EE_H_ */

@@ -1,0 +1,109 @@
+// ee_kv_compact: append the accepted path's K/V rows to the paged cache, for
+// every layer (EfficientEdit Sec. IV-A: accepted draft tokens extend the
+// prefix, so the K/V computed for them in the verification pass become cache
+// entries).  Path entry k of sequence s lands at position ctx + k.
+//
+// Pure data movement: one warp per (layer, sequence, path entry) copies the
+// n_kv K rows and n_kv V rows (head_dim bf16 = 256 bytes each) with 16-byte
+// vector loads/stores.  HBM-bound: 2 * 2 * n_kv * 256 bytes per entry and layer.
+#include "ee_common.cuh"
+
+namespace {
+
+constexpr int kWarpsPerBlock = 8;
+
+__global__ void __launch_bounds__(32 * kWarpsPerBlock)
+kv_compact_kernel(const uint4* __restrict__ k_tree, const uint4* __restrict__ v_tree,
+                  int64_t tree_layer_stride, uint4* __restrict__ k_cache, uint4* __restrict__ v_cache,
+                  int64_t cache_layer_stride, int num_pages, const int32_t* __restrict__ block_table,
+                  int max_pages, const int32_t* __restrict__ ctx_in, int32_t* __restrict__ ctx_out,
+                  const int32_t* __restrict__ node_off, const int32_t* __restrict__ path,
+                  const int32_t* __restrict__ accept_len, int max_T, int n_kv, int total_nodes,
+                  int32_t* __restrict__ dst_slot, int32_t* err) {
+  const int lane = threadIdx.x & 31;
+  const int k = blockIdx.x * kWarpsPerBlock + (threadIdx.x >> 5);
+  const int b = blockIdx.y;
+  const int l = blockIdx.z;
+  if (k >= max_T) return;
+  const int o = node_off[b];
+  const int T = node_off[b + 1] - o;
+  const int acc = accept_len[b];
+  const int ctx = ctx_in[b];
+  const bool lead = (l == 0 && lane == 0);
+  if (acc < 0 || acc >= T || acc >= max_T || ctx < 0 || o < 0 || o + T > total_nodes) {
+    if (lead) {
+      if (k == 0) ee::flag_error(err, EE_DEVERR_PATH);
+      dst_slot[(size_t)b * max_T + k] = -1;
+    }
+    return;
+  }
+  if (k > acc) {
+    if (lead) dst_slot[(size_t)b * max_T + k] = -1;
+    return;
+  }
+  if (lead && k == 0) ctx_out[b] = ctx + acc + 1;
+  const int node = path[(size_t)b * max_T + k];
+  const int pos = ctx + k;
+  const int pg = pos / EE_PAGE;
+  const int page = pg < max_pages ? block_table[(size_t)b * max_pages + pg] : -1;
+  if (node < 0 || node >= T || page < 0 || page >= num_pages) {
+    if (lead) {
+      ee::flag_error(err, (node < 0 || node >= T) ? EE_DEVERR_PATH : EE_DEVERR_PAGE);
+      dst_slot[(size_t)b * max_T + k] = -1;
+    }
+    return;
+  }
+  const int row = pos % EE_PAGE;
+  if (lead) dst_slot[(size_t)b * max_T + k] = page * EE_PAGE + row;
+  // 16 uint4 per head row; K rows then V rows
+  constexpr int kVecPerRow = EE_HEAD_DIM * 2 / 16;
+  const int64_t tl = tree_layer_stride / 8 * l;   // strides are in bf16 elements
+  const int64_t cl = cache_layer_stride / 8 * l;
+  const int nvec = 2 * n_kv * kVecPerRow;
+  for (int v = lane; v < nvec; v += 32) {
+    const int which = v / (n_kv * kVecPerRow);  // 0 = K, 1 = V
+    const int rem = v % (n_kv * kVecPerRow);
+    const int h = rem / kVecPerRow, c = rem % kVecPerRow;
+    const int64_t src = tl + ((int64_t)(o + node) * n_kv + h) * kVecPerRow + c;
+    const int64_t dst = cl + (((int64_t)page * n_kv + h) * EE_PAGE + row) * kVecPerRow + c;
+    if (which == 0) k_cache[dst] = k_tree[src];
+    else v_cache[dst] = v_tree[src];
+  }
+}
+
+}  // namespace
+
+extern "C" ee_status ee_kv_compact(const ee_bf16* k_tree, const ee_bf16* v_tree,
+                                   int64_t tree_layer_stride, ee_bf16* k_cache, ee_bf16* v_cache,
+                                   int64_t cache_layer_stride, int32_t L, int32_t num_pages,
+                                   const int32_t* block_table, int32_t max_pages,
+                                   const int32_t* ctx_len_in, int32_t* ctx_len_out,
+                                   const int32_t* node_off, const int32_t* path,
+                                   const int32_t* accept_len, int32_t B, int32_t max_T, int32_t n_kv,
+                                   int32_t head_dim, int32_t* dst_slot, void* ws, size_t ws_bytes,
+                                   ee_stream_t stream) {
+  if (B < 0 || L < 0 || max_T < 1 || max_T > EE_MAX_TREE || n_kv < 1 || num_pages < 1 ||
+      max_pages < 1)
+    return EE_ERR_INVALID_ARG;
+  if (head_dim != EE_HEAD_DIM) return EE_ERR_UNSUPPORTED;
+  if (B == 0) return EE_OK;
+  if (!k_tree || !v_tree || !k_cache || !v_cache || !block_table || !ctx_len_in || !ctx_len_out ||
+      !node_off || !path || !accept_len || !dst_slot || !ws)
+    return EE_ERR_INVALID_ARG;
+  if (ctx_len_in == ctx_len_out) return EE_ERR_INVALID_ARG;
+  if (!ee::aligned(k_tree, 16) || !ee::aligned(v_tree, 16) || !ee::aligned(k_cache, 16) ||
+      !ee::aligned(v_cache, 16) || tree_layer_stride % 8 || cache_layer_stride % 8)
+    return EE_ERR_INVALID_ARG;
+  if (ws_bytes < ee::kAttnOff) return EE_ERR_WORKSPACE;
+  if (L == 0) return EE_OK;
+  if (tree_layer_stride % ((int64_t)n_kv * head_dim)) return EE_ERR_INVALID_ARG;
+  const int total_nodes = (int)(tree_layer_stride / ((int64_t)n_kv * head_dim));
+  dim3 grid((max_T + kWarpsPerBlock - 1) / kWarpsPerBlock, B, L);
+  kv_compact_kernel<<<grid, 32 * kWarpsPerBlock, 0, (cudaStream_t)stream>>>(
+      reinterpret_cast<const uint4*>(k_tree), reinterpret_cast<const uint4*>(v_tree),
+      tree_layer_stride, reinterpret_cast<uint4*>(k_cache), reinterpret_cast<uint4*>(v_cache),
+      cache_layer_stride, num_pages, block_table, max_pages, ctx_len_in, ctx_len_out, node_off, path,
+      accept_len, max_T, n_kv, total_nodes, dst_slot, ee::err_word(ws));
+  EE_LAUNCH_OK();
+  return EE_OK;
+}

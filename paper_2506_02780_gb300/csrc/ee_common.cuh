@@ -1,0 +1,62 @@
+// Shared device/host helpers of libee (sm_103a).  Internal header.
+#pragma once
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+#include <stdint.h>
+
+#include "../../include/ee.h"
+
+namespace ee {
+
+// ---------------------------------------------------------------------------
+// Workspace layout (bytes from the start of `ws`):
+//   [0, 4)              device error word (EE_DEVERR_* bits)
+//   [16, 20)            LM-head "CTAs finished" ticket counter
+//   [256, 256+8*EE_MAX_LM_NODES)  LM-head packed running argmax per node
+//   [kAttnOff, ...)     attention split partials (O, then (m, l) pairs)
+// ---------------------------------------------------------------------------
+constexpr size_t kErrOff = 0;
+constexpr size_t kTicketOff = 16;
+constexpr size_t kArgmaxOff = 256;
+constexpr size_t kAttnOff = 256 + 8 * (size_t)EE_MAX_LM_NODES + 256;
+constexpr int kMaxSplits = 32;
+constexpr int kAttnRows = 128;        // query rows (node x head-in-group) per attention CTA
+constexpr int kNumSMs = 152;
+
+__host__ __device__ inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+inline size_t attn_partial_bytes(int total_nodes, int n_q, int head_dim) {
+  size_t rows = (size_t)kMaxSplits * (size_t)total_nodes * (size_t)n_q;
+  return align_up(rows * (size_t)head_dim * 4, 256) + align_up(rows * 8, 256);
+}
+
+__device__ __forceinline__ void flag_error(int32_t* err, int bits) { atomicOr(err, bits); }
+
+__host__ __device__ inline int32_t* err_word(void* ws) {
+  return reinterpret_cast<int32_t*>(static_cast<char*>(ws) + kErrOff);
+}
+
+inline bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+// Number of context chunks per sequence used by the split-KV attention; the
+// split kernel and the combine kernel both derive a sequence's split count
+// from ctx and this chunk length, so they always agree.
+__host__ __device__ inline int attn_splits_for(int ctx, int chunk) {
+  int s = (ctx + chunk - 1) / chunk;
+  return s < 1 ? 1 : s;
+}
+
+}  // namespace ee
+
+#define EE_CUDA_OK(call)                                  \
+  do {                                                    \
+    cudaError_t e_ = (call);                              \
+    if (e_ != cudaSuccess) return EE_ERR_CUDA;            \
+  } while (0)
+
+#define EE_LAUNCH_OK()                                    \
+  do {                                                    \
+    cudaError_t e_ = cudaGetLastError();                  \
+    if (e_ != cudaSuccess) return EE_ERR_CUDA;            \
+  } while (0)

@@ -1,0 +1,70 @@
+// ee_tree_prepare: depth and root-path (ancestor) bitmask of every draft-tree
+// node.  The paper verifies linear drafts (EfficientEdit Sec. IV-A); several
+// match points and generated branches share a prefix, so the step scores them
+// together as a tree whose nodes each see only their own root-to-node path.
+//
+// One CTA of 128 threads per sequence; thread i walks node i up to the root
+// through the parent array staged in shared memory (at most 127 steps, each a
+// shared-memory read), after a block-wide validation that parent[i] < i.
+#include "ee_common.cuh"
+
+namespace {
+
+__global__ void __launch_bounds__(EE_MAX_TREE)
+tree_prepare_kernel(const int32_t* __restrict__ parent, const int32_t* __restrict__ node_off,
+                    int32_t* __restrict__ depth, uint64_t* __restrict__ anc, int total_nodes,
+                    int32_t* err) {
+  __shared__ int32_t s_par[EE_MAX_TREE];
+  const int b = blockIdx.x;
+  const int i = threadIdx.x;
+  const int o = node_off[b];
+  const int T = node_off[b + 1] - o;
+  if (T < 1 || T > EE_MAX_TREE || o < 0 || o + T > total_nodes) {
+    if (i == 0) ee::flag_error(err, EE_DEVERR_TREE);
+    return;
+  }
+  int p = 0;
+  bool ok = true;
+  if (i < T) {
+    p = parent[o + i];
+    ok = (i == 0) ? (p == -1) : (p >= 0 && p < i);
+    s_par[i] = p;
+  }
+  const bool all_ok = __syncthreads_and(ok);
+  if (i >= T) return;
+  if (!all_ok) {
+    if (i == 0) ee::flag_error(err, EE_DEVERR_TREE);
+    depth[o + i] = 0;
+    anc[2 * (size_t)(o + i)] = 0;
+    anc[2 * (size_t)(o + i) + 1] = 0;
+    return;
+  }
+  uint64_t a0 = 0, a1 = 0;
+  int d = 0;
+  int u = i;
+  while (u > 0) {            // terminates: parent[u] < u was checked for every node
+    if (u < 64) a0 |= 1ull << u; else a1 |= 1ull << (u - 64);
+    u = s_par[u];
+    ++d;
+  }
+  a0 |= 1ull;                // the root is on every path
+  depth[o + i] = d;
+  anc[2 * (size_t)(o + i)] = a0;
+  anc[2 * (size_t)(o + i) + 1] = a1;
+}
+
+}  // namespace
+
+extern "C" ee_status ee_tree_prepare(const int32_t* parent, const int32_t* node_off, int32_t B,
+                                     int32_t total_nodes, int32_t* depth, uint64_t* anc,
+                                     void* ws, size_t ws_bytes, ee_stream_t stream) {
+  if (B < 0 || total_nodes < 0) return EE_ERR_INVALID_ARG;
+  if (B == 0) return EE_OK;
+  if (!parent || !node_off || !depth || !anc || !ws) return EE_ERR_INVALID_ARG;
+  if (!ee::aligned(anc, 8)) return EE_ERR_INVALID_ARG;
+  if (ws_bytes < ee::kAttnOff) return EE_ERR_WORKSPACE;
+  tree_prepare_kernel<<<B, EE_MAX_TREE, 0, (cudaStream_t)stream>>>(parent, node_off, depth, anc,
+                                                                    total_nodes, ee::err_word(ws));
+  EE_LAUNCH_OK();
+  return EE_OK;
+}

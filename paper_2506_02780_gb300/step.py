@@ -1,0 +1,109 @@
+"""One whole verification step as a fixed sequence of libee calls.
+
+EfficientEdit (arXiv 2506.02780) Sec. IV-A: the target scores a draft (here a
+tree: reuse chain + generated branches) in one pass and keeps the longest
+prefix its greedy choice agrees with.  ``VerifyStep`` owns the device output
+buffers and the workspace and issues, on one stream:
+
+    ee_match_reuse -> ee_tree_prepare -> L x ee_tree_verify_attn
+        -> ee_lmhead_accept -> ee_kv_compact
+
+No arithmetic happens here; every step runs in libee's kernels.  The whole
+sequence can be captured into a CUDA graph (``capture``).
+"""
+from __future__ import annotations
+
+import math
+
+import torch
+
+from . import (EE_HEAD_DIM, ee_kv_compact, ee_lmhead_accept, ee_match_reuse, ee_tree_prepare,
+               ee_tree_verify_attn, new_workspace)
+
+
+class VerifyStep:
+    """Device-resident state for repeated verification steps of one batch.
+
+    All tensors are CUDA tensors: int32 unless noted; ``orig_off`` int64;
+    q [L, total, n_q, 128], k_tree/v_tree [L, total, n_kv, 128],
+    k_cache/v_cache [L, num_pages, n_kv, 16, 128], hidden [total, H],
+    lm_w [V, H] in bf16.  ``max_ctx`` bounds ctx_len (host-side value).
+    """
+
+    def __init__(self, *, orig_tokens, orig_off, tail, cursor, parent, node_off, draft_tok, ctx_len,
+                 block_table, q, k_tree, v_tree, k_cache, v_cache, hidden, lm_w, max_ctx, max_T,
+                 max_matches=8, scale=None, keep_layers=True):
+        self.inp = dict(orig_tokens=orig_tokens, orig_off=orig_off, tail=tail, cursor=cursor,
+                        parent=parent, node_off=node_off, draft_tok=draft_tok, ctx_len=ctx_len,
+                        block_table=block_table, q=q, k_tree=k_tree, v_tree=v_tree, k_cache=k_cache,
+                        v_cache=v_cache, hidden=hidden, lm_w=lm_w)
+        dev = q.device
+        self.L, self.total, self.n_q, d = q.shape
+        if d != EE_HEAD_DIM:
+            raise ValueError("head_dim must be 128")
+        self.B = node_off.numel() - 1
+        self.max_T = int(max_T)
+        self.max_ctx = int(max_ctx)
+        self.max_matches = int(max_matches)
+        self.scale = 1.0 / math.sqrt(d) if scale is None else float(scale)
+        i32 = dict(dtype=torch.int32, device=dev)
+        self.match_pos = torch.empty((self.B, self.max_matches), **i32)
+        self.n_matches = torch.empty(self.B, **i32)
+        self.depth = torch.empty(self.total, **i32)
+        self.anc = torch.empty((self.total, 2), dtype=torch.int64, device=dev)
+        n_out = self.L if keep_layers else 1
+        self.attn_out = torch.empty((n_out, self.total, self.n_q, d), dtype=torch.float32, device=dev)
+        self.argmax = torch.empty(self.total, **i32)
+        self.accept_len = torch.empty(self.B, **i32)
+        self.path = torch.empty((self.B, self.max_T), **i32)
+        self.bonus = torch.empty(self.B, **i32)
+        self.ctx_out = torch.empty(self.B, **i32)
+        self.dst_slot = torch.empty((self.B, self.max_T), **i32)
+        self.ws = new_workspace(self.B, self.total, self.n_q, self.max_ctx, device=dev)
+        self.graph = None
+
+    def run(self, stream=None, logits=None, layers=None):
+        """Enqueue one whole step (``layers`` restricts attention, for tests)."""
+        x = self.inp
+        ee_match_reuse(x["orig_tokens"], x["orig_off"], x["tail"], x["cursor"], self.max_matches,
+                       self.match_pos, self.n_matches, self.ws, stream)
+        ee_tree_prepare(x["parent"], x["node_off"], self.depth, self.anc, self.ws, stream)
+        for l in (range(self.L) if layers is None else layers):
+            out = self.attn_out[l if self.attn_out.shape[0] == self.L else 0]
+            ee_tree_verify_attn(x["q"][l], x["k_tree"][l], x["v_tree"][l], x["k_cache"][l],
+                                x["v_cache"][l], x["block_table"], x["ctx_len"], self.max_ctx,
+                                x["node_off"], self.anc, self.max_T, self.scale, out, self.ws, stream)
+        ee_lmhead_accept(x["hidden"], x["lm_w"], x["draft_tok"], x["parent"], self.depth, self.anc,
+                         x["node_off"], self.max_T, self.argmax, self.accept_len, self.path, self.bonus,
+                         self.ws, logits=logits, stream=stream)
+        ee_kv_compact(x["k_tree"], x["v_tree"], x["k_cache"], x["v_cache"], x["block_table"],
+                      x["ctx_len"], self.ctx_out, x["node_off"], self.path, self.accept_len,
+                      self.dst_slot, self.ws, stream)
+
+    def capture(self, stream):
+        """Capture one step into a CUDA graph on ``stream`` (a side stream)."""
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.stream(stream):
+            self.run(stream)                       # warm-up outside capture
+            stream.synchronize()
+            with torch.cuda.graph(g, stream=stream):
+                self.run(stream)
+        self.graph = g
+        return g
+
+    def launches_per_step(self) -> int:
+        """Kernels this step launches: match, prepare, 2 per attention layer, LM head, compaction."""
+        return 2 + 2 * self.L + 2
+
+
+def from_workload(w, device="cuda", keep_layers=True):
+    """VerifyStep over a workloads.Workload (its float tensors already on ``device``)."""
+    def i32(a):
+        return torch.as_tensor(a, dtype=torch.int32).to(device)
+    return VerifyStep(
+        orig_tokens=i32(w.orig_tokens), orig_off=torch.as_tensor(w.orig_off, dtype=torch.int64).to(device),
+        tail=i32(w.tail), cursor=i32(w.cursor), parent=i32(w.parent), node_off=i32(w.node_off),
+        draft_tok=i32(w.draft_tok), ctx_len=i32(w.ctx_len), block_table=i32(w.block_table),
+        q=w.q, k_tree=w.k_tree, v_tree=w.v_tree, k_cache=w.k_cache, v_cache=w.v_cache,
+        hidden=w.hidden_states, lm_w=w.lm_w, max_ctx=int(w.ctx_len.max()), max_T=w.max_T,
+        max_matches=w.max_matches, keep_layers=keep_layers)

@@ -1,0 +1,112 @@
+"""The C-ABI library builds, loads and exports every entry point include/ee.h
+declares; host-side argument checks reject bad calls before any launch
+(CPU only: nothing here touches a GPU)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def L():
+    import paper_2506_02780_gb300 as E
+    from paper_2506_02780_gb300 import build
+    if not os.path.exists(E.LIB_PATH):
+        try:
+            build.build_lib()
+        except RuntimeError as e:   # no nvcc on this machine
+            pytest.skip(str(e))
+    return E.lib()
+
+
+def declared_symbols():
+    with open(os.path.join(ROOT, "include", "ee.h")) as f:
+        text = f.read()
+    return sorted(set(re.findall(r"^\s*(?:ee_status|size_t|const char\*)\s+(ee_\w+)\(", text, re.M)))
+
+
+def test_header_declares_the_boundary():
+    syms = declared_symbols()
+    for name in ("ee_match_reuse", "ee_tree_prepare", "ee_tree_verify_attn", "ee_lmhead_accept",
+                 "ee_kv_compact", "ee_workspace_size", "ee_workspace_init", "ee_read_errors",
+                 "ee_version", "ee_status_string"):
+        assert name in syms
+
+
+def test_every_declared_symbol_is_exported(L):
+    for name in declared_symbols():
+        assert hasattr(L, name), name
+    import paper_2506_02780_gb300 as E
+    assert set(E.EXPORTS) <= set(declared_symbols())
+
+
+def test_version_and_status_strings(L):
+    assert b"sm_103a" in L.ee_version()
+    assert L.ee_status_string(0) == b"ok"
+    assert L.ee_status_string(5) == b"workspace too small"
+
+
+def test_workspace_size_grows_with_problem(L):
+    a = L.ee_workspace_size(1, 64, 28, 128, 4096)
+    b = L.ee_workspace_size(1, 128, 56, 128, 32768)
+    assert 0 < a < b
+    assert a % 256 == 0 and b % 256 == 0
+
+
+FAKE = ctypes.c_void_p(0x10000)   # never dereferenced: every call below fails validation first
+
+
+def test_match_rejects_bad_args(L):
+    f = L.ee_match_reuse
+    # n = 0, n too large, max_matches = 0
+    assert f(FAKE, FAKE, 1, FAKE, 0, FAKE, 4, FAKE, FAKE, FAKE, 1 << 20, None) == 1
+    assert f(FAKE, FAKE, 1, FAKE, 33, FAKE, 4, FAKE, FAKE, FAKE, 1 << 20, None) == 1
+    assert f(FAKE, FAKE, 1, FAKE, 4, FAKE, 0, FAKE, FAKE, FAKE, 1 << 20, None) == 1
+    assert f(FAKE, None, 1, FAKE, 4, FAKE, 4, FAKE, FAKE, FAKE, 1 << 20, None) == 1
+    assert f(FAKE, FAKE, 1, FAKE, 4, FAKE, 4, FAKE, FAKE, FAKE, 64, None) == 5      # workspace
+    assert f(None, None, 0, None, 4, None, 4, None, None, None, 0, None) == 0      # B = 0: no-op
+
+
+def test_attention_rejects_bad_args(L):
+    f = L.ee_tree_verify_attn
+    ws = 1 << 30
+    args = [FAKE] * 5 + [10, FAKE, 4, FAKE, 64, FAKE, FAKE, 1, 16, 16, 8, 2, 128,
+                         ctypes.c_float(0.088), FAKE, FAKE, ws, None]
+    bad_hd = list(args); bad_hd[17] = 64
+    assert f(*bad_hd) == 2                                   # head_dim must be 128
+    bad_g = list(args); bad_g[15] = 7                        # n_q not a multiple of n_kv
+    assert f(*bad_g) == 2
+    bad_T = list(args); bad_T[14] = 129
+    assert f(*bad_T) == 2
+    bad_ctx = list(args); bad_ctx[9] = 65                    # max_ctx > max_pages * 16
+    assert f(*bad_ctx) == 1
+    bad_scale = list(args); bad_scale[18] = ctypes.c_float(0.0)
+    assert f(*bad_scale) == 1
+    unaligned = list(args); unaligned[0] = ctypes.c_void_p(0x10002)
+    assert f(*unaligned) == 1
+    small = list(args); small[21] = 1024
+    assert f(*small) == 5
+
+
+def test_lmhead_rejects_bad_args(L):
+    f = L.ee_lmhead_accept
+    base = [FAKE, FAKE, 3584, 152064] + [FAKE] * 5 + [1, 64, 64] + [FAKE] * 4 + [None, FAKE, 1 << 20, None]
+    h7 = list(base); h7[2] = 3583
+    assert f(*h7) == 2                                       # hidden not a multiple of 8
+    many = list(base); many[10] = 4096
+    assert f(*many) == 2                                     # too many nodes for one call
+    nul = list(base); nul[4] = None
+    assert f(*nul) == 1
+
+
+def test_compact_rejects_aliasing_ctx(L):
+    f = L.ee_kv_compact
+    args = [FAKE, FAKE, 1024, FAKE, FAKE, 8192, 2, 10, FAKE, 4, FAKE, ctypes.c_void_p(0x20000), FAKE,
+            FAKE, FAKE, 1, 16, 4, 128, FAKE, FAKE, 1 << 20, None]
+    alias = list(args); alias[11] = args[10]
+    assert f(*alias) == 1
+    hd = list(args); hd[18] = 96
+    assert f(*hd) == 2

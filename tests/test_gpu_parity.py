@@ -1,0 +1,219 @@
+"""GPU parity: the CUDA verification step, called through the C ABI, against
+the fp64 oracle on the same seeded inputs (tolerances in parity_util)."""
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+import parity_util as U
+import workloads as W
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    if not torch.cuda.is_available():
+        pytest.fail("GPU tests need a CUDA device")
+    import paper_2506_02780_gb300 as E
+    from paper_2506_02780_gb300 import build
+    build.build_lib()
+    E.lib()
+
+
+def _E():
+    import paper_2506_02780_gb300 as E
+    return E
+
+
+def run_step(w, logits=True, layers=None):
+    from paper_2506_02780_gb300 import step as S
+    k0, v0 = U.raw16(w.k_cache), U.raw16(w.v_cache)
+    st = S.from_workload(w)
+    lg = torch.empty((w.total_nodes, w.vocab), dtype=torch.float32, device="cuda") if logits else None
+    st.run(logits=lg, layers=layers)
+    torch.cuda.synchronize()
+    assert _E().ee_read_errors(st.ws) == 0
+    return st, lg, k0, v0
+
+
+def full_check(w, attn_nodes=None, attn_layers=None, lm_nodes=None, logits=True):
+    st, lg, k0, v0 = run_step(w, logits=logits)
+    U.check_match(w, st)
+    anc = U.check_tree(w, st)
+    U.check_attention(w, st, range(w.layers) if attn_layers is None else attn_layers, anc,
+                      nodes=attn_nodes)
+    n_amb = U.check_argmax(w, st, nodes=lm_nodes, logits=lg)
+    acc, path = U.check_accept(w, st)
+    np.testing.assert_array_equal(acc, w.planted_accept)
+    for s in range(w.B):
+        assert list(path[s, :acc[s] + 1]) == w.planted_path[s]
+    U.check_compact(w, st, k0, v0, acc, path)
+    return st, n_amb
+
+
+# ----------------------------------------------------------------------------
+# tiny configuration and edge cases (oracle on every output)
+# ----------------------------------------------------------------------------
+
+@pytest.mark.parametrize("seed", [1234, 1, 2])
+def test_tiny(seed):
+    w = W.build("tiny", seed=seed, device="cuda")
+    st, _ = full_check(w)
+    assert st.match_pos[0, 0].item() == w.planted_match[0]
+
+
+def test_tiny_peaky_queries():
+    """Large query scale: scores of a few units, exercising the online-softmax rescale."""
+    w = W.build("tiny", seed=7, device="cuda", q_std=40.0, ctx=700)
+    full_check(w)
+
+
+def test_exact_ties_pick_lowest_token():
+    w = W.build("tiny", seed=8, device="cuda", dup_rows=4)
+    st, _ = full_check(w)
+    am_ref, cands, lg = O.lm_head_argmax(w.hidden_states, w.lm_w)
+    got = st.argmax.cpu().numpy()
+    tied = [i for i in range(w.total_nodes) if (lg[i] == lg[i].max()).sum() > 1]
+    assert tied
+    for i in tied:
+        assert got[i] == am_ref[i]           # lowest token id among exact ties
+
+
+@pytest.mark.parametrize("tree,ctx", [
+    (W.TreeSpec(1, [], [0]), 0),                                   # a plain decode step, empty cache
+    (W.TreeSpec(1, [], [0]), 16),
+    (W.TreeSpec(40, [], W.chain_path(20)), 37),                    # chain only, ragged context
+    (W.TreeSpec(1, [(0, 1)] * 15, [0, 5]), 129),                   # star: every node a child of the root
+    (W.TreeSpec(100, [(0, 14), (50, 14)], W.chain_path(60)), 1000),  # T = 128, full mask width
+    (W.TreeSpec(70, [(3, 20), (3, 20), (69, 10)], [0, 1, 2, 3, 70, 71, 72]), 63),  # path into a branch
+])
+def test_tree_edge_cases(tree, ctx):
+    w = W.build("tiny", seed=11, device="cuda", trees=[tree], ctx=ctx)
+    full_check(w)
+
+
+def test_multi_sequence_small():
+    w = W.build("batched", seed=21, device="cuda", layers=2, vocab=8192, hidden=512)
+    full_check(w)
+
+
+def test_repeat_runs_bit_identical():
+    w = W.build("tiny", seed=5, device="cuda")
+    from paper_2506_02780_gb300 import step as S
+    st = S.from_workload(w)
+    outs = []
+    for _ in range(5):
+        st.run()
+        torch.cuda.synchronize()
+        outs.append([t.clone() for t in (st.match_pos, st.argmax, st.path, st.accept_len, st.bonus,
+                                         st.dst_slot, st.attn_out)])
+    for o in outs[1:]:
+        for a, b in zip(outs[0], o):
+            assert torch.equal(a, b)
+
+
+# ----------------------------------------------------------------------------
+# device-detected bad input: error word set, access skipped, context usable
+# ----------------------------------------------------------------------------
+
+def test_device_error_word():
+    E = _E()
+    from paper_2506_02780_gb300 import step as S
+    w = W.build("tiny", seed=3, device="cuda")
+    st = S.from_workload(w)
+    st.inp["block_table"][0, 1] = w.num_pages + 5            # out-of-range page inside the context
+    st.run()
+    bits = E.ee_read_errors(st.ws)
+    assert bits & 0x04
+    st.inp["block_table"][0, 1] = int(w.block_table[0, 1])
+    st.inp["cursor"][0] = -1
+    st.run()
+    assert E.ee_read_errors(st.ws) & 0x01
+    st.inp["cursor"][0] = int(w.cursor[0])
+    bad_parent = st.inp["parent"].clone()
+    st.inp["parent"][3] = 7                                   # parent after child
+    st.run()
+    assert E.ee_read_errors(st.ws) & 0x02
+    st.inp["parent"].copy_(bad_parent)
+    E.ee_workspace_init(st.ws)
+    st.run()                                                  # a clean call afterwards works
+    torch.cuda.synchronize()
+    assert E.ee_read_errors(st.ws) == 0
+    U.check_accept(w, st)
+
+
+# ----------------------------------------------------------------------------
+# full-size configurations (sampled attention outputs, launch configuration as timed)
+# ----------------------------------------------------------------------------
+
+def _sample_nodes(w, k, seed=0):
+    rng = np.random.default_rng(seed)
+    nodes = set(rng.choice(w.total_nodes, size=min(k, w.total_nodes), replace=False).tolist())
+    for s in range(w.B):                       # first and last node of every tree
+        nodes.add(int(w.node_off[s]))
+        nodes.add(int(w.node_off[s + 1]) - 1)
+    return sorted(nodes)
+
+
+@pytest.mark.slow
+def test_7b_full_size():
+    w = W.build("7b", device="cuda")
+    full_check(w, attn_nodes=_sample_nodes(w, 10), logits=False)
+
+
+@pytest.mark.slow
+def test_batched_full_size():
+    w = W.build("batched", device="cuda")
+    lm_nodes = sorted(set(_sample_nodes(w, 40, 1)) |
+                      {int(w.node_off[s]) + u for s in range(w.B) for u in w.planted_path[s]})
+    full_check(w, attn_nodes=_sample_nodes(w, 24), attn_layers=[0, 13, 27], lm_nodes=lm_nodes,
+               logits=False)
+
+
+@pytest.mark.slow
+def test_33b_full_size():
+    w = W.build("33b", device="cuda")
+    full_check(w, attn_nodes=_sample_nodes(w, 6), attn_layers=[0, 61], logits=False)
+
+
+@pytest.mark.parametrize("n", [2, 4, 8])
+def test_sweep_match_full_size(n):
+    E = _E()
+    w = W.build("sweep", device="cuda", n=n, layers=1, seed=1238 + n)
+    dev = "cuda"
+    i32 = lambda a: torch.as_tensor(a, dtype=torch.int32, device=dev)  # noqa: E731
+    mp = torch.empty((w.B, 16), dtype=torch.int32, device=dev)
+    nm = torch.empty(w.B, dtype=torch.int32, device=dev)
+    ws = E.new_workspace(w.B, w.total_nodes, 1, 0)
+    E.ee_match_reuse(i32(w.orig_tokens), torch.as_tensor(w.orig_off, device=dev), i32(w.tail),
+                     i32(w.cursor), 16, mp, nm, ws)
+    torch.cuda.synchronize()
+    assert E.ee_read_errors(ws) == 0
+    pos, cnt = O.match_reuse(w.orig_tokens, w.orig_off, w.tail, w.cursor, 16)
+    np.testing.assert_array_equal(mp.cpu().numpy(), pos)
+    np.testing.assert_array_equal(nm.cpu().numpy(), cnt)
+    assert (cnt > 1).any()                    # repeated segments make some tails ambiguous
+
+
+def test_sweep_compaction_full_size():
+    E = _E()
+    w = W.build("sweep", device="cuda")
+    dev = "cuda"
+    i32 = lambda a: torch.as_tensor(a, dtype=torch.int32, device=dev)  # noqa: E731
+    path = np.full((w.B, w.max_T), -1, np.int32)
+    for s in range(w.B):
+        path[s, :len(w.planted_path[s])] = w.planted_path[s]
+    k0, v0 = U.raw16(w.k_cache), U.raw16(w.v_cache)
+    ctx_out = torch.empty(w.B, dtype=torch.int32, device=dev)
+    dst = torch.empty((w.B, w.max_T), dtype=torch.int32, device=dev)
+    ws = E.new_workspace(w.B, w.total_nodes, 1, 0)
+    E.ee_kv_compact(w.k_tree, w.v_tree, w.k_cache, w.v_cache, i32(w.block_table), i32(w.ctx_len),
+                    ctx_out, i32(w.node_off), i32(path), i32(w.planted_accept), dst, ws)
+    torch.cuda.synchronize()
+    assert E.ee_read_errors(ws) == 0
+    kc, vc, dref, cref = O.kv_compact(U.raw16(w.k_tree), U.raw16(w.v_tree), k0, v0, w.block_table,
+                                      w.ctx_len, w.node_off, path, w.planted_accept)
+    np.testing.assert_array_equal(dst.cpu().numpy(), dref)
+    np.testing.assert_array_equal(ctx_out.cpu().numpy(), cref)
+    assert np.array_equal(U.raw16(w.k_cache), kc) and np.array_equal(U.raw16(w.v_cache), vc)
