@@ -510,27 +510,40 @@ bool encode_2d(CUtensorMap* map, const void* base, uint64_t inner, uint64_t oute
   return r == CUDA_SUCCESS;
 }
 
-}  // namespace
-
-extern "C" ee_status ee_lmhead_accept(const ee_bf16* hidden, const ee_bf16* lm_w, int32_t hidden_dim,
-                                      int32_t vocab, const int32_t* draft_tok, const int32_t* parent,
-                                      const int32_t* depth, const uint64_t* anc,
-                                      const int32_t* node_off, int32_t B, int32_t total_nodes,
-                                      int32_t max_T, int32_t* argmax, int32_t* accept_len,
-                                      int32_t* path, int32_t* bonus, float* logits_or_null,
-                                      void* ws, size_t ws_bytes, ee_stream_t stream) {
+// Host-side argument checks shared by the LM-head entry points.  Sets *empty
+// when there is nothing to launch.
+ee_status check_lm_args(const ee_bf16* hidden, const ee_bf16* lm_w, int32_t hidden_dim,
+                        int32_t vocab, const int32_t* draft_tok, const int32_t* parent,
+                        const int32_t* depth, const uint64_t* anc, const int32_t* node_off, int32_t B,
+                        int32_t total_nodes, int32_t max_T, const int32_t* argmax,
+                        const int32_t* accept_len, const int32_t* path, const int32_t* bonus,
+                        bool* empty) {
+  *empty = false;
   if (B < 0 || total_nodes < 0 || hidden_dim < 8 || vocab < 1 || max_T < 1)
     return EE_ERR_INVALID_ARG;
   if (hidden_dim % 8 != 0 || max_T > EE_MAX_TREE || total_nodes > EE_MAX_LM_NODES)
     return EE_ERR_UNSUPPORTED;
-  if (B == 0 || total_nodes == 0) return EE_OK;
+  if (B == 0 || total_nodes == 0) {
+    *empty = true;
+    return EE_OK;
+  }
   if (!hidden || !lm_w || !draft_tok || !parent || !depth || !anc || !node_off || !argmax ||
-      !accept_len || !path || !bonus || !ws)
+      !accept_len || !path || !bonus)
     return EE_ERR_INVALID_ARG;
-  if (!ee::aligned(hidden, 16) || !ee::aligned(lm_w, 16) || !ee::aligned(ws, 256))
-    return EE_ERR_INVALID_ARG;
-  if (ws_bytes < ee::kAttnOff) return EE_ERR_WORKSPACE;
+  if (!ee::aligned(hidden, 16) || !ee::aligned(lm_w, 16)) return EE_ERR_INVALID_ARG;
+  return EE_OK;
+}
 
+// Encode the tensor maps and launch the persistent LM-head kernel; `keys`
+// (EE_MAX_LM_NODES running-argmax words, zero on entry), `ticket` (zero on
+// entry) and `err` are the kernel's scratch.
+ee_status launch_lmhead(const ee_bf16* hidden, const ee_bf16* lm_w, int32_t hidden_dim,
+                        int32_t vocab, const int32_t* draft_tok, const int32_t* parent,
+                        const int32_t* depth, const uint64_t* anc, const int32_t* node_off, int32_t B,
+                        int32_t total_nodes, int32_t max_T, int32_t* argmax, int32_t* accept_len,
+                        int32_t* path, int32_t* bonus, float* logits_or_null,
+                        unsigned long long* keys, unsigned int* ticket, int32_t* err,
+                        ee_stream_t stream) {
   LmParams p;
   p.vocab = vocab;
   p.hidden = hidden_dim;
@@ -559,10 +572,9 @@ extern "C" ee_status ee_lmhead_accept(const ee_bf16* hidden, const ee_bf16* lm_w
   p.path = path;
   p.bonus = bonus;
   p.logits = logits_or_null;
-  char* wsb = static_cast<char*>(ws);
-  p.keys = reinterpret_cast<unsigned long long*>(wsb + ee::kArgmaxOff);
-  p.ticket = reinterpret_cast<unsigned int*>(wsb + ee::kTicketOff);
-  p.err = ee::err_word(ws);
+  p.keys = keys;
+  p.ticket = ticket;
+  p.err = err;
 
   CUtensorMap tmW, tmX;
   if (!encode_2d(&tmW, lm_w, (uint64_t)hidden_dim, (uint64_t)vocab, BK, BM)) return EE_ERR_CUDA;
@@ -585,4 +597,28 @@ extern "C" ee_status ee_lmhead_accept(const ee_bf16* hidden, const ee_bf16* lm_w
   lmhead_accept_kernel<<<grid, kThreads, smem_acc, (cudaStream_t)stream>>>(tmW, tmX, p);
   EE_LAUNCH_OK();
   return EE_OK;
+}
+
+}  // namespace
+
+extern "C" ee_status ee_lmhead_accept(const ee_bf16* hidden, const ee_bf16* lm_w, int32_t hidden_dim,
+                                      int32_t vocab, const int32_t* draft_tok, const int32_t* parent,
+                                      const int32_t* depth, const uint64_t* anc,
+                                      const int32_t* node_off, int32_t B, int32_t total_nodes,
+                                      int32_t max_T, int32_t* argmax, int32_t* accept_len,
+                                      int32_t* path, int32_t* bonus, float* logits_or_null,
+                                      void* ws, size_t ws_bytes, ee_stream_t stream) {
+  bool empty = false;
+  const ee_status st = check_lm_args(hidden, lm_w, hidden_dim, vocab, draft_tok, parent, depth, anc,
+                                     node_off, B, total_nodes, max_T, argmax, accept_len, path,
+                                     bonus, &empty);
+  if (st != EE_OK || empty) return st;
+  if (!ws || !ee::aligned(ws, 256)) return EE_ERR_INVALID_ARG;
+  if (ws_bytes < ee::kAttnOff) return EE_ERR_WORKSPACE;
+  char* wsb = static_cast<char*>(ws);
+  return launch_lmhead(hidden, lm_w, hidden_dim, vocab, draft_tok, parent, depth, anc, node_off, B,
+                       total_nodes, max_T, argmax, accept_len, path, bonus, logits_or_null,
+                       reinterpret_cast<unsigned long long*>(wsb + ee::kArgmaxOff),
+                       reinterpret_cast<unsigned int*>(wsb + ee::kTicketOff), ee::err_word(ws),
+                       stream);
 }
