@@ -128,14 +128,17 @@ class Workload:
 
 def _original_code(rng, length, vocab, repeat_frac=0.0, seg=8):
     """Uniform tokens; optionally ``repeat_frac`` of them lie in copies of earlier
-    ``seg``-token segments (repeated code lines make matches ambiguous)."""
+    ``seg``-token segments (repeated code lines make matches ambiguous).
+    Returns (tokens, list of (src, dst) copy starts)."""
     c = rng.integers(0, vocab, size=length, dtype=np.int64).astype(np.int32)
     n_seg = int(repeat_frac * length) // seg
+    copies = []
     for _ in range(n_seg):
         dst = int(rng.integers(seg, length - seg + 1))
         src = int(rng.integers(0, dst - seg + 1))
         c[dst:dst + seg] = c[src:src + seg]
-    return c
+        copies.append((src, dst))
+    return c, copies
 
 
 def _prefix_with_edits(rng, c, plen, n_edits, vocab, edit_len=8, keep_tail=4):
@@ -339,12 +342,19 @@ def build(name: str, seed: int | None = None, device="cpu", *, q_std: float = 1.
     codes, tails, cursors, planted_match, chain_toks = [], [], [], [], []
     for sp in seqs:
         rep = 0.3 if name == "sweep" else 0.0
-        c = _original_code(rng, sp["len_c"], V, repeat_frac=rep)
+        c, copies = _original_code(rng, sp["len_c"], V, repeat_frac=rep)
         chain = sp["spec"].chain
         if sp["plen"] is None:
             # sweep: tail copied from a random location (90%) or random (10%)
             cur = int(rng.integers(0, len(c) // 2))
-            if rng.random() < 0.9:
+            u = rng.random()
+            late = [(a, b) for a, b in copies[-64:] if a >= cur and b + n < len(c)]
+            if u < 0.3 and late and n <= 8:
+                # tail taken from a repeated segment: it matches at least twice
+                a, b = late[int(rng.integers(0, len(late)))]
+                tail = c[b:b + n].copy()
+                pm = b
+            elif u < 0.9:
                 p = int(rng.integers(cur, len(c) - n))
                 tail = c[p:p + n].copy()
                 pm = p
