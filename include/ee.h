@@ -191,6 +191,39 @@ ee_status ee_lmhead_accept(const ee_bf16* hidden, const ee_bf16* lm_w, int32_t h
                            float* logits_or_null, void* ws, size_t ws_bytes, ee_stream_t stream);
 
 /*
+ * ee_lmhead_accept_static -- ee_lmhead_accept for callers that cannot allocate
+ * device memory.  The paper has no counterpart; this is a deployment variant.
+ * Some callers have no way to obtain the workspace the other entry points
+ * take: code running where cudaMalloc is unavailable or forbidden (host
+ * callbacks, a custom allocator's own hooks, processes under a fixed device
+ * memory budget).  This entry point takes the same inputs and outputs as
+ * ee_lmhead_accept but no `ws`: its scratch lives in a file-scope device array
+ * of 16,640 bytes inside libee, which every GPU that loads the library holds
+ * until the process exits.  It allocates nothing (no cudaMalloc/cudaFree, no
+ * allocating library call).
+ *  - total_nodes above EE_MAX_LM_NODES (2048) is rejected with
+ *    EE_ERR_UNSUPPORTED; the other argument checks are those of
+ *    ee_lmhead_accept.
+ *  - The first call on each device looks up the array's device address
+ *    (cudaGetSymbolAddress) with that device current; make that first call
+ *    before any stream capture.
+ *  - Every call clears the array on `stream` before its launch, because the
+ *    array keeps the previous call's contents.  All calls share the one array:
+ *    calls that overlap on the GPU (different streams without ordering, or
+ *    different host threads) race and corrupt each other's results.
+ *  - Device-side failures (the bounded-wait timeout) are recorded only in the
+ *    array's own error word, which this entry point does not report; outputs
+ *    are then undefined.  Use ee_lmhead_accept with a workspace and
+ *    ee_read_errors when that report is needed.
+ */
+ee_status ee_lmhead_accept_static(const ee_bf16* hidden, const ee_bf16* lm_w, int32_t hidden_dim,
+                                  int32_t vocab, const int32_t* draft_tok, const int32_t* parent,
+                                  const int32_t* depth, const uint64_t* anc, const int32_t* node_off,
+                                  int32_t B, int32_t total_nodes, int32_t max_T, int32_t* argmax,
+                                  int32_t* accept_len, int32_t* path, int32_t* bonus,
+                                  float* logits_or_null, ee_stream_t stream);
+
+/*
  * ee_kv_compact -- append the accepted path's K/V to the paged cache, every
  * layer (Sec. IV-A: accepted tokens extend the prefix).  Path entry k
  * (k = 0..accept_len[s], root first) of sequence s goes to position

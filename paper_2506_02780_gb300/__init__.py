@@ -30,7 +30,7 @@ DEVERR = {0x01: "MATCH_ARGS", 0x02: "TREE", 0x04: "PAGE", 0x08: "CTX", 0x10: "FP
 
 EXPORTS = ("ee_version", "ee_status_string", "ee_workspace_size", "ee_workspace_init",
            "ee_read_errors", "ee_match_reuse", "ee_tree_prepare", "ee_tree_verify_attn",
-           "ee_lmhead_accept", "ee_kv_compact")
+           "ee_lmhead_accept", "ee_lmhead_accept_static", "ee_kv_compact")
 
 
 class EEError(RuntimeError):
@@ -62,6 +62,8 @@ _SIGS = {
                              _F, _P, _P, _SZ, _P], _I),
     "ee_lmhead_accept": ([_P, _P, _I, _I, _P, _P, _P, _P, _P, _I, _I, _I, _P, _P, _P, _P, _P, _P, _SZ,
                           _P], _I),
+    "ee_lmhead_accept_static": ([_P, _P, _I, _I, _P, _P, _P, _P, _P, _I, _I, _I, _P, _P, _P, _P, _P,
+                                 _P], _I),
     "ee_kv_compact": ([_P, _P, _I64, _P, _P, _I64, _I, _I, _P, _I, _P, _P, _P, _P, _P, _I, _I, _I, _I,
                        _P, _P, _SZ, _P], _I),
 }
@@ -184,6 +186,23 @@ def ee_lmhead_accept(hidden, lm_w, draft_tok, parent, depth, anc, node_off, max_
                                 _p(anc), _p(node_off), B, total, max_T, _p(argmax), _p(accept_len),
                                 _p(path), _p(bonus), _p(logits), _p(ws), ws.numel(), _stream(stream))
     _ok("ee_lmhead_accept", st)
+
+
+def ee_lmhead_accept_static(hidden, lm_w, draft_tok, parent, depth, anc, node_off, max_T, argmax,
+                            accept_len, path, bonus, logits=None, stream=None):
+    """ee_lmhead_accept without a workspace, for callers that cannot allocate
+    device memory: the scratch is a fixed 16,640-byte array inside libee shared
+    by every call (calls must not overlap on the GPU)."""
+    _check(hidden, torch.bfloat16, "hidden")
+    _check(lm_w, torch.bfloat16, "lm_w")
+    total, H = hidden.shape
+    V = lm_w.shape[0]
+    B = node_off.numel() - 1
+    st = lib().ee_lmhead_accept_static(_p(hidden), _p(lm_w), H, V, _p(draft_tok), _p(parent),
+                                       _p(depth), _p(anc), _p(node_off), B, total, max_T, _p(argmax),
+                                       _p(accept_len), _p(path), _p(bonus), _p(logits),
+                                       _stream(stream))
+    _ok("ee_lmhead_accept_static", st)
 
 
 def ee_kv_compact(k_tree, v_tree, k_cache, v_cache, block_table, ctx_len_in, ctx_len_out, node_off,

@@ -28,6 +28,7 @@
 // EE_DEVERR_TIMEOUT, drains its own copies and MMAs (again bounded), frees its
 // TMEM and returns.
 #include <cmath>
+#include <mutex>
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -621,4 +622,68 @@ extern "C" ee_status ee_lmhead_accept(const ee_bf16* hidden, const ee_bf16* lm_w
                        reinterpret_cast<unsigned long long*>(wsb + ee::kArgmaxOff),
                        reinterpret_cast<unsigned int*>(wsb + ee::kTicketOff), ee::err_word(ws),
                        stream);
+}
+
+// ---------------------------------------------------------------------------
+// ee_lmhead_accept_static: the same LM head + argmax + acceptance for callers
+// that cannot allocate device memory -- code that runs where cudaMalloc is not
+// available to it (inside a host callback or a custom allocator's own hooks,
+// or under an allocation budget that forbids new device buffers).  Its scratch
+// (running-argmax words, finished-CTA ticket, device error word) lives in the
+// file-scope array below, 16,640 bytes, which every GPU that loads libee holds
+// until the process exits.
+// ---------------------------------------------------------------------------
+namespace {
+
+constexpr size_t kStaticScratchBytes = ee::kArgmaxOff + 8 * (size_t)EE_MAX_LM_NODES;  // 16,640
+static __device__ __align__(256) unsigned char g_lm_scratch[kStaticScratchBytes];
+
+// Device address of g_lm_scratch per device ordinal, looked up once per device.
+// The host-side symbol `g_lm_scratch` is only a stand-in for the device array:
+// it must never be passed to a kernel.
+constexpr int kMaxDevices = 64;
+void* g_lm_scratch_ptr[kMaxDevices] = {};
+
+std::mutex g_lm_scratch_mu;
+
+ee_status static_scratch(void** out) {
+  int dev = -1;
+  EE_CUDA_OK(cudaGetDevice(&dev));
+  if (dev < 0 || dev >= kMaxDevices) return EE_ERR_UNSUPPORTED;
+  std::lock_guard<std::mutex> lock(g_lm_scratch_mu);
+  if (!g_lm_scratch_ptr[dev]) {
+    void* ptr = nullptr;
+    if (cudaGetSymbolAddress(&ptr, g_lm_scratch) != cudaSuccess || !ptr) return EE_ERR_CUDA;
+    g_lm_scratch_ptr[dev] = ptr;
+  }
+  *out = g_lm_scratch_ptr[dev];
+  return EE_OK;
+}
+
+}  // namespace
+
+extern "C" ee_status ee_lmhead_accept_static(const ee_bf16* hidden, const ee_bf16* lm_w,
+                                             int32_t hidden_dim, int32_t vocab,
+                                             const int32_t* draft_tok, const int32_t* parent,
+                                             const int32_t* depth, const uint64_t* anc,
+                                             const int32_t* node_off, int32_t B,
+                                             int32_t total_nodes, int32_t max_T, int32_t* argmax,
+                                             int32_t* accept_len, int32_t* path, int32_t* bonus,
+                                             float* logits_or_null, ee_stream_t stream) {
+  bool empty = false;
+  const ee_status st = check_lm_args(hidden, lm_w, hidden_dim, vocab, draft_tok, parent, depth, anc,
+                                     node_off, B, total_nodes, max_T, argmax, accept_len, path,
+                                     bonus, &empty);
+  if (st != EE_OK || empty) return st;   // total_nodes > EE_MAX_LM_NODES -> EE_ERR_UNSUPPORTED
+  void* scratch = nullptr;
+  const ee_status ss = static_scratch(&scratch);
+  if (ss != EE_OK) return ss;
+  // the array keeps the previous call's contents: start from zero every call
+  EE_CUDA_OK(cudaMemsetAsync(scratch, 0, kStaticScratchBytes, (cudaStream_t)stream));
+  char* base = static_cast<char*>(scratch);
+  return launch_lmhead(hidden, lm_w, hidden_dim, vocab, draft_tok, parent, depth, anc, node_off, B,
+                       total_nodes, max_T, argmax, accept_len, path, bonus, logits_or_null,
+                       reinterpret_cast<unsigned long long*>(base + ee::kArgmaxOff),
+                       reinterpret_cast<unsigned int*>(base + ee::kTicketOff),
+                       reinterpret_cast<int32_t*>(base + ee::kErrOff), stream);
 }
