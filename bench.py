@@ -48,6 +48,8 @@ def parse_args():
     ap.add_argument("--e2e-steps", type=int, default=300)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-clocks", action="store_true")
+    ap.add_argument("--profile", action="store_true",
+                    help="run --steps eager steps and exit (for ncu captures: few launches, no timing)")
     return ap.parse_args()
 
 
@@ -196,6 +198,27 @@ def cpu_cores():
 # ----------------------------------------------------------------------------
 # our arm
 # ----------------------------------------------------------------------------
+
+def run_profile(args, local_rank):
+    """Eager steps only: every libee kernel launches --steps times, nothing else runs
+    between them, no graphs and no timing (what an ncu capture wants)."""
+    import paper_2506_02780_gb300 as E
+    from paper_2506_02780_gb300 import build as B
+    from paper_2506_02780_gb300 import step as S
+    B.build_lib()
+    dev = torch.device("cuda", local_rank)
+    torch.cuda.set_device(dev)
+    w = W.build(args.config, device=dev)
+    st = S.from_workload(w, device=dev, keep_layers=False)
+    torch.cuda.synchronize(dev)
+    for _ in range(args.steps):
+        st.run()
+    torch.cuda.synchronize(dev)
+    bits = E.ee_read_errors(st.ws)
+    print(json.dumps({"profile": args.config, "steps": args.steps, "device_errors": bits,
+                      "accept_len": st.accept_len.tolist()}), flush=True)
+    return 0 if bits == 0 else 1
+
 
 def run_ours(args, rank, world, local_rank):
     import paper_2506_02780_gb300 as E
@@ -471,6 +494,8 @@ def main():
         if out is not None:
             print(json.dumps(out), flush=True)
         return
+    if args.profile:
+        sys.exit(run_profile(args, local_rank))
     if world > 1:
         torch.cuda.set_device(local_rank)
         torch.distributed.init_process_group("nccl", device_id=torch.device("cuda", local_rank))

@@ -6,39 +6,52 @@
 // Work decomposition (split-KV):
 //   - For a (sequence, KV head) the query rows are the g = n_q / n_kv heads of
 //     the group times the T tree nodes, row r = node * g + head_in_group, so
-//     one K/V tile feeds g * T rows (GQA packing).  A CTA owns 128 rows
-//     (8 warps x 16 rows).
+//     one K/V tile feeds g * T rows (GQA packing).  A CTA owns 128 rows: the
+//     M side of a tcgen05 MMA.
 //   - The context is cut into chunks of `chunk` keys (a multiple of the 16-token
 //     page); each (row block, chunk) is one CTA.  The CTA of the last chunk
 //     also processes the tree keys, masked by the ancestor bitmask.
-//   - Each CTA streams 64-key K/V tiles into shared memory with cp.async
-//     (double buffered, 16-byte chunks, XOR-swizzled rows), computes S = Q K^T
-//     on bf16 tensor cores with fp32 accumulation, keeps an fp32 online softmax
-//     in the exp2 domain, and accumulates O += P V with P and V in fp16
-//     (V converted in shared memory; bf16 -> fp16 is exact for |v| <= 65504).
-//   - Partials (unnormalised O, running max m, running sum l) go to the
-//     workspace; a second launch merges the chunks with log-sum-exp weights and
-//     writes fp32 output.  No CTA ever waits on another.
+//   - Warp 0 streams 64-key K/V tiles with TMA (one 16-row box per page and
+//     128-byte half of the head dimension; the tree's own K/V through a 3-D map)
+//     into a 3-stage ring.  Warps 2-3 convert each landed V tile to fp16 in
+//     place.  Warp 1 issues tcgen05.mma: S = Q K^T (bf16, fp32 in TMEM, double
+//     buffered) and O += P V (fp16 P from shared memory, fp16 V read MN-major,
+//     fp32 O in TMEM).  Warps 4-7 own one query row per thread: they read S
+//     from TMEM, mask, keep the running max/sum, write P, and rescale O in TMEM
+//     only when a row's max grows by more than 2^8 (the stale max keeps every
+//     P <= 256, exact in fp16, and the final O / l is unchanged).
+//   - Partials (unnormalised O, max m, sum l per row) go to the workspace; a
+//     second launch merges the chunks with log-sum-exp weights and writes fp32
+//     output.  No CTA ever waits on another; every mbarrier wait is bounded.
 #include "ee_common.cuh"
+#include "ee_ptx.cuh"
 
 namespace {
 
-constexpr int kWarps = 8;
-constexpr int kThreads = 32 * kWarps;
-constexpr int kRows = 16 * kWarps;          // query rows per CTA
-constexpr int kKT = 64;                     // keys per tile
-constexpr int kD = EE_HEAD_DIM;             // 128
-constexpr int kTileBytes = kKT * kD * 2;    // 16 KB for K or V
-constexpr int kSmemBytes = 4 * kTileBytes;  // 2 buffers x (K, V)
+using namespace ee;
+
+constexpr int kThreads = 256;
+constexpr int kRows = 128;                       // query rows per CTA (MMA M)
+constexpr int kKT = 64;                          // keys per tile (MMA N of Q K^T)
+constexpr int kD = EE_HEAD_DIM;                  // 128
+constexpr int kNST = 3;                          // K/V ring depth
+constexpr uint32_t kQHalf = kRows * 128;         // 16 KB: one 64-dim half of Q
+constexpr uint32_t kKVHalf = kKT * 128;          // 8 KB: one 64-dim half of a K or V tile
+constexpr uint32_t kKVBytes = 2 * kKVHalf;       // 16 KB
+constexpr uint32_t kStageBytes = 2 * kKVBytes;   // K + V
+constexpr uint32_t kPBytes = kRows * kKT * 2;    // 16 KB fp16 P tile
+constexpr uint32_t kOffKV = 2 * kQHalf;
+constexpr uint32_t kOffP = kOffKV + kNST * kStageBytes;
+constexpr uint32_t kOffBar = kOffP + 2 * kPBytes;
+constexpr uint32_t kNumBars = 3 * kNST + 3 * 2 + 2;
+constexpr uint32_t kSmemBytes = 1024 + kOffBar + 8 * kNumBars + 64;
+constexpr uint32_t kTmemCols = 256;              // S0 [0,64) S1 [64,128) O [128,256)
+constexpr float kRescaleLog2 = 8.0f;
 
 static_assert(kRows == ee::kAttnRows, "row block size");
 
 struct AttnParams {
   const __nv_bfloat16* q;
-  const __nv_bfloat16* kt;
-  const __nv_bfloat16* vt;
-  const __nv_bfloat16* kc;
-  const __nv_bfloat16* vc;
   const int32_t* block_table;
   const int32_t* ctx_len;
   const int32_t* node_off;
@@ -56,129 +69,32 @@ __device__ __forceinline__ float ex2(float x) {
   return y;
 }
 
-__device__ __forceinline__ uint32_t smem_u32(const void* p) {
-  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
-
-// byte offset of 16-byte chunk `ch` (0..15) of row `row` in a 64 x 256-byte tile
-__device__ __forceinline__ uint32_t swz(int row, int ch) {
-  return (uint32_t)(row * 256 + ((ch ^ (row & 7)) << 4));
-}
-
-__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, int src_bytes) {
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(dst), "l"(src),
-               "r"(src_bytes));
-}
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::); }
-template <int N>
-__device__ __forceinline__ void cp_async_wait() {
-  asm volatile("cp.async.wait_group %0;\n" ::"n"(N));
-}
-
-__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2,
-                                        uint32_t& r3) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];\n"
-               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
-               : "r"(addr));
-}
-__device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2,
-                                          uint32_t& r3) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];\n"
-               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
-               : "r"(addr));
-}
-
-__device__ __forceinline__ void mma_bf16(float (&d)[4], const uint32_t (&a)[4], uint32_t b0,
-                                         uint32_t b1) {
-  asm volatile(
-      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, "
-      "{%8,%9}, {%0,%1,%2,%3};\n"
-      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
-      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
-}
-__device__ __forceinline__ void mma_f16(float (&d)[4], const uint32_t (&a)[4], uint32_t b0,
-                                        uint32_t b1) {
-  asm volatile(
-      "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, "
-      "{%8,%9}, {%0,%1,%2,%3};\n"
-      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
-      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
-}
-
 __device__ __forceinline__ uint32_t pack_half2(float lo, float hi) {
   __half2 h = __floats2half2_rn(lo, hi);
   return *reinterpret_cast<uint32_t*>(&h);
 }
 
-// Issue the cp.async copies of one 64-key tile (K and V) into buffer (sK, sV).
-// Context tile: keys are cache positions key0.. (< key_end); tree tile: keys are
-// local tree nodes key0.. (< T).  Missing or invalid keys are zero-filled and
-// marked invalid in s_valid.
-__device__ __forceinline__ void load_tile(const AttnParams& p, int b, int hk, int o, int T,
-                                          bool tree, int key0, int key_end, uint32_t sK,
-                                          uint32_t sV, int* s_valid) {
-#pragma unroll
-  for (int it = 0; it < (kKT * 16) / kThreads; ++it) {
-    const int idx = threadIdx.x + it * kThreads;
-    const int key = idx >> 4, ch = idx & 15;
-    const __nv_bfloat16* srck = p.kc;
-    const __nv_bfloat16* srcv = p.vc;
-    bool ok;
-    if (!tree) {
-      const int pos = key0 + key;
-      ok = pos < key_end;
-      if (ok) {
-        const int page = p.block_table[(size_t)b * p.max_pages + (pos >> 4)];
-        if (page < 0 || page >= p.num_pages) {
-          if (ch == 0) ee::flag_error(p.err, EE_DEVERR_PAGE);
-          ok = false;
-        } else {
-          const size_t row = ((size_t)page * p.n_kv + hk) * EE_PAGE + (pos & (EE_PAGE - 1));
-          srck = p.kc + row * kD + ch * 8;
-          srcv = p.vc + row * kD + ch * 8;
-        }
-      }
-    } else {
-      const int j = key0 + key;
-      ok = j < T;
-      if (ok) {
-        const size_t row = (size_t)(o + j) * p.n_kv + hk;
-        srck = p.kt + row * kD + ch * 8;
-        srcv = p.vt + row * kD + ch * 8;
-      }
-    }
-    const int nb = ok ? 16 : 0;
-    cp_async16(sK + swz(key, ch), srck, nb);
-    cp_async16(sV + swz(key, ch), srcv, nb);
-    if (ch == 0) s_valid[key] = ok ? 1 : 0;
-  }
+// Whether 16-row page block i of a context tile holds loaded keys; the producer,
+// the V converter and the softmax all derive the same answer from the inputs.
+__device__ __forceinline__ bool page_loaded(const AttnParams& p, int b, int key0, int k_end, int i,
+                                            int* page_out) {
+  const int pos = key0 + 16 * i;
+  if (pos >= k_end) return false;
+  const int page = p.block_table[(size_t)b * p.max_pages + (pos >> 4)];
+  *page_out = page;
+  return page >= 0 && page < p.num_pages;
 }
 
-// Convert this thread's own V chunks of a landed tile from bf16 to fp16 in place.
-__device__ __forceinline__ void convert_v(char* sV, int32_t* err) {
-  bool overflow = false;
-#pragma unroll
-  for (int it = 0; it < (kKT * 16) / kThreads; ++it) {
-    const int idx = threadIdx.x + it * kThreads;
-    const int key = idx >> 4, ch = idx & 15;
-    uint4* ptr = reinterpret_cast<uint4*>(sV + swz(key, ch));
-    uint4 v = *ptr;
-    uint32_t* w = reinterpret_cast<uint32_t*>(&v);
-#pragma unroll
-    for (int e = 0; e < 4; ++e) {
-      __nv_bfloat162 bb = *reinterpret_cast<__nv_bfloat162*>(&w[e]);
-      float2 f = __bfloat1622float2(bb);
-      overflow |= (fabsf(f.x) > 65504.f) || (fabsf(f.y) > 65504.f);
-      w[e] = pack_half2(f.x, f.y);
-    }
-    *ptr = v;
-  }
-  if (overflow) ee::flag_error(err, EE_DEVERR_FP16_RANGE);
-}
-
-__global__ void __launch_bounds__(kThreads, 1) attn_split_kernel(const AttnParams p) {
-  extern __shared__ __align__(1024) char smem[];
-  __shared__ int s_valid[2][kKT];
+__global__ void __launch_bounds__(kThreads, 1)
+attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__ CUtensorMap tmVc,
+               const __grid_constant__ CUtensorMap tmKt, const __grid_constant__ CUtensorMap tmVt,
+               const AttnParams p) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  __shared__ uint32_t s_tmem;
+  __shared__ volatile int s_abort;
+  __shared__ int s_issued[kNST];
 
   const int b = blockIdx.z;
   const int hk = blockIdx.y;
@@ -188,234 +104,395 @@ __global__ void __launch_bounds__(kThreads, 1) attn_split_kernel(const AttnParam
   const int T = p.node_off[b + 1] - o;
   const int R = T * p.g;
   if (T < 1 || T > EE_MAX_TREE || T > p.max_T || o < 0 || o + T > p.total_nodes) {
-    if (threadIdx.x == 0 && blockIdx.x == 0 && hk == 0) ee::flag_error(p.err, EE_DEVERR_TREE);
+    if (threadIdx.x == 0 && blockIdx.x == 0 && hk == 0) flag_error(p.err, EE_DEVERR_TREE);
     return;
   }
   if (rb * kRows >= R) return;
   int ctx = p.ctx_len[b];
   if (ctx < 0 || ctx > p.max_ctx) {
-    if (threadIdx.x == 0 && rb == 0 && split == 0 && hk == 0) ee::flag_error(p.err, EE_DEVERR_CTX);
+    if (threadIdx.x == 0 && blockIdx.x == 0 && hk == 0) flag_error(p.err, EE_DEVERR_CTX);
     ctx = ctx < 0 ? 0 : p.max_ctx;
   }
-  const int S = ee::attn_splits_for(ctx, p.chunk);
+  const int S = attn_splits_for(ctx, p.chunk);
   if (split >= S) return;
   const int k_begin = split * p.chunk;
   const int k_end = min(ctx, k_begin + p.chunk);
   const int n_ctx_tiles = k_end > k_begin ? (k_end - k_begin + kKT - 1) / kKT : 0;
-  const bool last = (split == S - 1);
-  const int n_tree_tiles = last ? (T + kKT - 1) / kKT : 0;
+  const int n_tree_tiles = (split == S - 1) ? (T + kKT - 1) / kKT : 0;
   const int n_tiles = n_ctx_tiles + n_tree_tiles;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int row_a = rb * kRows + warp * 16 + (lane >> 2);
-  const int row_b = row_a + 8;
-  const bool va = row_a < R, vb = row_b < R;
-  const int node_a = va ? row_a / p.g : 0, node_b = vb ? row_b / p.g : 0;
-  const int head_a = hk * p.g + (va ? row_a % p.g : 0);
-  const int head_b = hk * p.g + (vb ? row_b % p.g : 0);
-
-  // Q fragments (A operand, 16 rows x 128 dims per warp) straight from global memory
-  uint32_t qa[8][4];
-  {
-    const uint32_t* qra =
-        reinterpret_cast<const uint32_t*>(p.q + ((size_t)(o + node_a) * p.n_q + head_a) * kD);
-    const uint32_t* qrb =
-        reinterpret_cast<const uint32_t*>(p.q + ((size_t)(o + node_b) * p.n_q + head_b) * kD);
-    const int c = (lane & 3);
-#pragma unroll
-    for (int ks = 0; ks < 8; ++ks) {
-      qa[ks][0] = va ? __ldg(qra + ks * 8 + c) : 0u;
-      qa[ks][1] = vb ? __ldg(qrb + ks * 8 + c) : 0u;
-      qa[ks][2] = va ? __ldg(qra + ks * 8 + 4 + c) : 0u;
-      qa[ks][3] = vb ? __ldg(qrb + ks * 8 + 4 + c) : 0u;
-    }
-  }
-  const uint64_t anc_a0 = va ? p.anc[2 * (size_t)(o + node_a)] : 0ull;
-  const uint64_t anc_a1 = va ? p.anc[2 * (size_t)(o + node_a) + 1] : 0ull;
-  const uint64_t anc_b0 = vb ? p.anc[2 * (size_t)(o + node_b)] : 0ull;
-  const uint64_t anc_b1 = vb ? p.anc[2 * (size_t)(o + node_b) + 1] : 0ull;
-
-  float acc[16][4];
-#pragma unroll
-  for (int i = 0; i < 16; ++i) acc[i][0] = acc[i][1] = acc[i][2] = acc[i][3] = 0.f;
-  float m_a = -INFINITY, m_b = -INFINITY, l_a = 0.f, l_b = 0.f;
-
   const uint32_t sbase = smem_u32(smem);
-  auto tile_key0 = [&](int t) { return t < n_ctx_tiles ? k_begin + t * kKT : (t - n_ctx_tiles) * kKT; };
+  const uint32_t sQ = sbase, sKV = sbase + kOffKV, sP = sbase + kOffP;
+  const uint32_t bar0 = sbase + kOffBar;
+  const uint32_t kv_full = bar0, kv_empty = bar0 + 8 * kNST, v_ready = bar0 + 16 * kNST;
+  const uint32_t s_full = bar0 + 24 * kNST, s_free = s_full + 16, p_full = s_free + 16;
+  const uint32_t o_done = p_full + 16, drain = o_done + 8;
 
-  if (n_tiles > 0) {
-    load_tile(p, b, hk, o, T, n_ctx_tiles == 0, tile_key0(0), k_end, sbase, sbase + kTileBytes,
-              s_valid[0]);
-    cp_async_commit();
+  if (threadIdx.x == 0) {
+    s_abort = 0;
+    for (int i = 0; i < kNST; ++i) {
+      mbar_init(kv_full + 8 * i, 1);
+      mbar_init(kv_empty + 8 * i, 1);
+      mbar_init(v_ready + 8 * i, 64);
+      s_issued[i] = -1;
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(s_full + 8 * i, 1);
+      mbar_init(s_free + 8 * i, kRows);
+      mbar_init(p_full + 8 * i, kRows);
+    }
+    mbar_init(o_done, 1);
+    mbar_init(drain, 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    fence_async_smem();
   }
-  for (int t = 0; t < n_tiles; ++t) {
-    const int buf = t & 1;
-    if (t + 1 < n_tiles) {
-      const int nb = (t + 1) & 1;
-      load_tile(p, b, hk, o, T, t + 1 >= n_ctx_tiles, tile_key0(t + 1), k_end,
-                sbase + nb * 2 * kTileBytes, sbase + nb * 2 * kTileBytes + kTileBytes,
-                s_valid[nb]);
-      cp_async_commit();
-      cp_async_wait<1>();
-    } else {
-      cp_async_wait<0>();
-    }
-    convert_v(smem + buf * 2 * kTileBytes + kTileBytes, p.err);
-    __syncthreads();
-
-    const bool tree = t >= n_ctx_tiles;
-    const int key0 = tile_key0(t);
-    const uint32_t sK = sbase + buf * 2 * kTileBytes;
-    const uint32_t sV = sK + kTileBytes;
-
-    // S = Q K^T : 16 rows x 64 keys per warp
-    float s[8][4];
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     smem_u32(&s_tmem)),
+                 "r"(kTmemCols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  // Q tile: 128 rows x 128 dims, K-major with 128-byte swizzle, two 64-dim halves
+  {
+    const int row_base = rb * kRows;
 #pragma unroll
-    for (int nt = 0; nt < 8; ++nt) s[nt][0] = s[nt][1] = s[nt][2] = s[nt][3] = 0.f;
-#pragma unroll
-    for (int kk2 = 0; kk2 < 4; ++kk2) {
-#pragma unroll
-      for (int nt = 0; nt < 8; ++nt) {
-        uint32_t b0, b1, b2, b3;
-        ldsm_x4(sK + swz(nt * 8 + (lane & 7), kk2 * 4 + (lane >> 3)), b0, b1, b2, b3);
-        mma_bf16(s[nt], qa[2 * kk2], b0, b1);
-        mma_bf16(s[nt], qa[2 * kk2 + 1], b2, b3);
+    for (int it = 0; it < (kRows * 16) / kThreads; ++it) {
+      const int idx = threadIdx.x + it * kThreads;
+      const int r = idx >> 4, c = idx & 15;
+      const int rr = row_base + r;
+      uint4 v = make_uint4(0u, 0u, 0u, 0u);
+      if (rr < R) {
+        const int node = rr / p.g, j = rr - node * p.g;
+        const __nv_bfloat16* src = p.q + ((size_t)(o + node) * p.n_q + hk * p.g + j) * kD + c * 8;
+        v = __ldg(reinterpret_cast<const uint4*>(src));
       }
+      const uint32_t dst = sQ + (c >> 3) * kQHalf + r * 128 + (((c & 7) ^ (r & 7)) << 4);
+      asm volatile("st.shared.v4.b32 [%0], {%1,%2,%3,%4};" ::"r"(dst), "r"(v.x), "r"(v.y), "r"(v.z),
+                   "r"(v.w)
+                   : "memory");
     }
-    // mask + scale, row max
-    float mx_a = -INFINITY, mx_b = -INFINITY;
+    fence_async_smem();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = s_tmem;
+
+  if (warp == 0) {
+    // ---------------- TMA producer ----------------
+    if (lane == 0) {
+      for (int t = 0; t < n_tiles; ++t) {
+        const int st = t % kNST, use = t / kNST;
+        if (!mbar_wait(kv_empty + 8 * st, (uint32_t)(use & 1) ^ 1u, &s_abort)) break;
+        const uint32_t full = kv_full + 8 * st;
+        const uint32_t sK = sKV + st * kStageBytes, sV = sK + kKVBytes;
+        if (t < n_ctx_tiles) {
+          const int key0 = k_begin + t * kKT;
+          int pages[4];
+          uint32_t bytes = 0;
 #pragma unroll
-    for (int nt = 0; nt < 8; ++nt) {
+          for (int i = 0; i < 4; ++i) {
+            int pg = -1;
+            const bool ok = page_loaded(p, b, key0, k_end, i, &pg);
+            if (!ok && key0 + 16 * i < k_end) flag_error(p.err, EE_DEVERR_PAGE);
+            pages[i] = ok ? pg : -1;
+            bytes += ok ? 4u * 2048u : 0u;
+          }
+          mbar_expect_tx(full, bytes);
 #pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const int col = nt * 8 + (lane & 3) * 2 + (e & 1);
-        bool ok = s_valid[buf][col] != 0;
-        if (tree) {
-          const int j = key0 + col;
-          const uint64_t w0 = e < 2 ? anc_a0 : anc_b0;
-          const uint64_t w1 = e < 2 ? anc_a1 : anc_b1;
-          const uint64_t bit = j < 64 ? (w0 >> j) : (w1 >> (j - 64));
-          ok = ok && (bit & 1ull);
+          for (int i = 0; i < 4; ++i) {
+            if (pages[i] < 0) continue;
+            const int row0 = (pages[i] * p.n_kv + hk) * EE_PAGE;
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+              tma_load_2d(sK + h * kKVHalf + i * 2048, &tmKc, full, h * 64, row0);
+              tma_load_2d(sV + h * kKVHalf + i * 2048, &tmVc, full, h * 64, row0);
+            }
+          }
+        } else {
+          const int key0 = (t - n_ctx_tiles) * kKT;
+          mbar_expect_tx(full, 4 * kKVHalf);
+#pragma unroll
+          for (int h = 0; h < 2; ++h) {
+            tma_load_3d(sK + h * kKVHalf, &tmKt, full, h * 64, hk, o + key0);
+            tma_load_3d(sV + h * kKVHalf, &tmVt, full, h * 64, hk, o + key0);
+          }
         }
-        const float v = ok ? s[nt][e] * p.scale_log2 : -INFINITY;
-        s[nt][e] = v;
-        if (e < 2) mx_a = fmaxf(mx_a, v); else mx_b = fmaxf(mx_b, v);
+        s_issued[st] = use;
       }
     }
-    mx_a = fmaxf(mx_a, __shfl_xor_sync(0xffffffffu, mx_a, 1));
-    mx_a = fmaxf(mx_a, __shfl_xor_sync(0xffffffffu, mx_a, 2));
-    mx_b = fmaxf(mx_b, __shfl_xor_sync(0xffffffffu, mx_b, 1));
-    mx_b = fmaxf(mx_b, __shfl_xor_sync(0xffffffffu, mx_b, 2));
-    const float mn_a = fmaxf(m_a, mx_a), mn_b = fmaxf(m_b, mx_b);
-    const float mu_a = mn_a == -INFINITY ? 0.f : mn_a;
-    const float mu_b = mn_b == -INFINITY ? 0.f : mn_b;
-    const float al_a = ex2(m_a - mu_a), al_b = ex2(m_b - mu_b);
-    m_a = mn_a;
-    m_b = mn_b;
-    l_a *= al_a;
-    l_b *= al_b;
+  } else if (warp == 1) {
+    // ---------------- MMA issuer ----------------
+    if (lane == 0) {
+      const uint32_t id_qk = idesc_f16(kRows, kKT, 1, 1, 0);
+      const uint32_t id_pv = idesc_f16(kRows, kD, 0, 0, 1);
+      bool ok = true;
+      auto issue_pv = [&](int u) -> bool {
+        const int st = u % kNST, sb = u & 1;
+        if (!mbar_wait(p_full + 8 * sb, (uint32_t)((u >> 1) & 1), &s_abort)) return false;
+        if (!mbar_wait(v_ready + 8 * st, (uint32_t)((u / kNST) & 1), &s_abort)) return false;
+        tc_fence_after();
+        const uint32_t pa = sP + sb * kPBytes;
+        const uint32_t vb = sKV + st * kStageBytes + kKVBytes;
 #pragma unroll
-    for (int i = 0; i < 16; ++i) {
-      acc[i][0] *= al_a;
-      acc[i][1] *= al_a;
-      acc[i][2] *= al_b;
-      acc[i][3] *= al_b;
-    }
-    // P (fp16 A fragments) and row sums
-    uint32_t pa[4][4];
+        for (int j = 0; j < kKT / 16; ++j)
+          tc_mma(tmem + 128, smem_desc_sw128(pa + j * 32), smem_desc_sw128_mn(vb + j * 2048, kKVHalf, 1024),
+                 id_pv, (u > 0 || j > 0) ? 1u : 0u);
+        tc_commit(kv_empty + 8 * st);
+        tc_commit(o_done);
+        return true;
+      };
+      for (int t = 0; t < n_tiles && ok; ++t) {
+        const int st = t % kNST, use = t / kNST, sb = t & 1;
+        if (!mbar_wait(kv_full + 8 * st, (uint32_t)(use & 1), &s_abort)) break;
+        if (t >= 2 && !mbar_wait(s_free + 8 * sb, (uint32_t)((t >> 1) & 1) ^ 1u, &s_abort)) break;
+        tc_fence_after();
+        const uint32_t kb = sKV + st * kStageBytes;
 #pragma unroll
-    for (int nt = 0; nt < 8; ++nt) {
-      const float p0 = ex2(s[nt][0] - mu_a), p1 = ex2(s[nt][1] - mu_a);
-      const float p2 = ex2(s[nt][2] - mu_b), p3 = ex2(s[nt][3] - mu_b);
-      l_a += p0 + p1;
-      l_b += p2 + p3;
-      pa[nt >> 1][(nt & 1) * 2 + 0] = pack_half2(p0, p1);
-      pa[nt >> 1][(nt & 1) * 2 + 1] = pack_half2(p2, p3);
-    }
-    // O += P V
-#pragma unroll
-    for (int kk = 0; kk < 4; ++kk) {
-#pragma unroll
-      for (int ntp = 0; ntp < 8; ++ntp) {
-        uint32_t b0, b1, b2, b3;
-        ldsm_x4_t(sV + swz(kk * 16 + (lane & 7) + ((lane >> 3) & 1) * 8, ntp * 2 + (lane >> 4)), b0,
-                  b1, b2, b3);
-        mma_f16(acc[2 * ntp], pa[kk], b0, b1);
-        mma_f16(acc[2 * ntp + 1], pa[kk], b2, b3);
+        for (int kk = 0; kk < kD / 16; ++kk) {
+          const uint32_t off = (kk >> 2) * 0 + (kk & 3) * 32;
+          tc_mma(tmem + sb * kKT, smem_desc_sw128(sQ + (kk >> 2) * kQHalf + off),
+                 smem_desc_sw128(kb + (kk >> 2) * kKVHalf + off), id_qk, kk > 0 ? 1u : 0u);
+        }
+        tc_commit(s_full + 8 * sb);
+        if (t >= 1) ok = issue_pv(t - 1);
       }
+      if (ok && n_tiles > 0) issue_pv(n_tiles - 1);
     }
-    __syncthreads();  // buffer `buf` is refilled two tiles later
-  }
-
-  l_a += __shfl_xor_sync(0xffffffffu, l_a, 1);
-  l_a += __shfl_xor_sync(0xffffffffu, l_a, 2);
-  l_b += __shfl_xor_sync(0xffffffffu, l_b, 1);
-  l_b += __shfl_xor_sync(0xffffffffu, l_b, 2);
-
-  const size_t pra = ((size_t)split * p.total_nodes + o + node_a) * p.n_q + head_a;
-  const size_t prb = ((size_t)split * p.total_nodes + o + node_b) * p.n_q + head_b;
-  const int c0 = (lane & 3) * 2;
+  } else if (warp < 4) {
+    // ---------------- V converters: bf16 -> fp16 in place ----------------
+    const int ct = threadIdx.x - 64;
+    bool overflow = false;
+    for (int t = 0; t < n_tiles; ++t) {
+      const int st = t % kNST, use = t / kNST;
+      if (!mbar_wait(kv_full + 8 * st, (uint32_t)(use & 1), &s_abort)) break;
+      uint4* sv = reinterpret_cast<uint4*>(smem + kOffKV + st * kStageBytes + kKVBytes);
+      // rows of a context tile whose page was not loaded hold stale bytes: zero them
+      unsigned loaded = 0xFu;
+      if (t < n_ctx_tiles) {
+        const int key0 = k_begin + t * kKT;
+        loaded = 0u;
 #pragma unroll
-  for (int nt = 0; nt < 16; ++nt) {
-    if (va)
-      *reinterpret_cast<float2*>(p.part_o + pra * kD + nt * 8 + c0) = make_float2(acc[nt][0], acc[nt][1]);
-    if (vb)
-      *reinterpret_cast<float2*>(p.part_o + prb * kD + nt * 8 + c0) = make_float2(acc[nt][2], acc[nt][3]);
+        for (int i = 0; i < 4; ++i) {
+          int pg;
+          if (page_loaded(p, b, key0, k_end, i, &pg)) loaded |= 1u << i;
+        }
+      }
+#pragma unroll 4
+      for (int it = 0; it < (int)(kKVBytes / 16) / 64; ++it) {
+        const int idx = ct + it * 64;                 // 16-byte chunk; 8 per 128-byte row
+        const int row = (idx >> 3) & (kKT - 1);       // key row within the 64-dim half
+        uint4 v = sv[idx];
+        if (!((loaded >> (row >> 4)) & 1u)) {
+          v = make_uint4(0u, 0u, 0u, 0u);
+        } else {
+          uint32_t* w = reinterpret_cast<uint32_t*>(&v);
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            __nv_bfloat162 bb = *reinterpret_cast<__nv_bfloat162*>(&w[e]);
+            const float2 f = __bfloat1622float2(bb);
+            overflow |= (fabsf(f.x) > 65504.f) || (fabsf(f.y) > 65504.f);
+            w[e] = pack_half2(f.x, f.y);
+          }
+        }
+        sv[idx] = v;
+      }
+      fence_async_smem();
+      mbar_arrive(v_ready + 8 * st);
+    }
+    if (overflow) flag_error(p.err, EE_DEVERR_FP16_RANGE);
+  } else {
+    // ---------------- softmax: one query row per thread ----------------
+    const int r = threadIdx.x - 128;                  // == TMEM lane
+    const int rr = rb * kRows + r;
+    const bool vrow = rr < R;
+    const int node = vrow ? rr / p.g : 0;
+    const int head = hk * p.g + (vrow ? rr - node * p.g : 0);
+    const uint64_t a0 = vrow ? p.anc[2 * (size_t)(o + node)] : 0ull;
+    const uint64_t a1 = vrow ? p.anc[2 * (size_t)(o + node) + 1] : 0ull;
+    const uint32_t tl = tmem + ((uint32_t)((warp & 3) * 32) << 16);
+    float m_used = -INFINITY, l = 0.f;
+    bool ok = true;
+    for (int t = 0; t < n_tiles; ++t) {
+      const int sb = t & 1;
+      if (!mbar_wait(s_full + 8 * sb, (uint32_t)((t >> 1) & 1), &s_abort)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      uint32_t sr[64];
+      tc_ld32(tl + sb * kKT, *reinterpret_cast<uint32_t(*)[32]>(&sr[0]));
+      tc_ld32(tl + sb * kKT + 32, *reinterpret_cast<uint32_t(*)[32]>(&sr[32]));
+      tc_fence_before();
+      mbar_arrive(s_free + 8 * sb);
+      float tmax = -INFINITY;
+      if (t < n_ctx_tiles) {
+        const int key0 = k_begin + t * kKT;
+        unsigned loaded = 0u;
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          int pg;
+          if (page_loaded(p, b, key0, k_end, i, &pg)) loaded |= 1u << i;
+        }
+#pragma unroll
+        for (int c = 0; c < kKT; ++c) {
+          const bool v = vrow && (key0 + c < k_end) && ((loaded >> (c >> 4)) & 1u);
+          const float x = v ? __uint_as_float(sr[c]) * p.scale_log2 : -INFINITY;
+          sr[c] = __float_as_uint(x);
+          tmax = fmaxf(tmax, x);
+        }
+      } else {
+        const int key0 = (t - n_ctx_tiles) * kKT;
+        const uint64_t w = key0 == 0 ? a0 : a1;       // key0 is 0 or 64
+#pragma unroll
+        for (int c = 0; c < kKT; ++c) {
+          const bool v = vrow && (key0 + c < T) && ((w >> c) & 1ull);
+          const float x = v ? __uint_as_float(sr[c]) * p.scale_log2 : -INFINITY;
+          sr[c] = __float_as_uint(x);
+          tmax = fmaxf(tmax, x);
+        }
+      }
+      const float m_new = fmaxf(m_used, tmax);
+      if (t >= 1 && !mbar_wait(o_done, (uint32_t)((t - 1) & 1), &s_abort)) {
+        ok = false;
+        break;
+      }
+      const bool need = m_new > m_used + kRescaleLog2;
+      if (t >= 1 && __any_sync(0xffffffffu, need)) {
+        tc_fence_after();
+        const float f = need ? ex2(m_used - m_new) : 1.f;
+#pragma unroll 1
+        for (int c4 = 0; c4 < 4; ++c4) {
+          uint32_t ov[32];
+          tc_ld32(tl + 128 + 32 * c4, ov);
+#pragma unroll
+          for (int e = 0; e < 32; ++e) ov[e] = __float_as_uint(__uint_as_float(ov[e]) * f);
+          tc_st32(tl + 128 + 32 * c4, ov);
+        }
+      }
+      if (need) {
+        l *= ex2(m_used - m_new);
+        m_used = m_new;
+      }
+      const float mu = m_used == -INFINITY ? 0.f : m_used;
+      // P row (fp16) into the K-major, 128-byte-swizzled P tile
+      const uint32_t prow = sP + sb * kPBytes + r * 128;
+#pragma unroll
+      for (int ch = 0; ch < 8; ++ch) {
+        uint32_t w4[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const float p0 = ex2(__uint_as_float(sr[ch * 8 + 2 * e]) - mu);
+          const float p1 = ex2(__uint_as_float(sr[ch * 8 + 2 * e + 1]) - mu);
+          l += p0 + p1;
+          w4[e] = pack_half2(p0, p1);
+        }
+        asm volatile("st.shared.v4.b32 [%0], {%1,%2,%3,%4};" ::"r"(prow + ((ch ^ (r & 7)) << 4)),
+                     "r"(w4[0]), "r"(w4[1]), "r"(w4[2]), "r"(w4[3])
+                     : "memory");
+      }
+      fence_async_smem();
+      tc_fence_before();
+      mbar_arrive(p_full + 8 * sb);
+    }
+    if (ok && n_tiles > 0 && mbar_wait(o_done, (uint32_t)((n_tiles - 1) & 1), &s_abort)) {
+      tc_fence_after();
+      const size_t pr = ((size_t)split * p.total_nodes + o + node) * p.n_q + head;
+#pragma unroll 1
+      for (int c4 = 0; c4 < 4; ++c4) {
+        uint32_t ov[32];
+        tc_ld32(tl + 128 + 32 * c4, ov);
+        if (vrow) {
+          float4* dst = reinterpret_cast<float4*>(p.part_o + pr * kD + 32 * c4);
+#pragma unroll
+          for (int e = 0; e < 8; ++e)
+            dst[e] = make_float4(__uint_as_float(ov[4 * e]), __uint_as_float(ov[4 * e + 1]),
+                                 __uint_as_float(ov[4 * e + 2]), __uint_as_float(ov[4 * e + 3]));
+        }
+      }
+      if (vrow) p.part_ml[pr] = make_float2(m_used, l);
+    }
   }
-  if ((lane & 3) == 0) {
-    if (va) p.part_ml[pra] = make_float2(m_a, l_a);
-    if (vb) p.part_ml[prb] = make_float2(m_b, l_b);
+
+  // ---- teardown: drain on abort, free TMEM ----------------------------------
+  tc_fence_before();
+  __syncthreads();
+  const bool aborted = s_abort != 0;
+  if (aborted && threadIdx.x == 0) {
+    flag_error(p.err, EE_DEVERR_TIMEOUT);
+    for (int st = 0; st < kNST; ++st)   // TMA copies still in flight land before the CTA exits
+      if (s_issued[st] >= 0) mbar_wait_plain(kv_full + 8 * st, (uint32_t)(s_issued[st] & 1));
+  }
+  if (warp == 1) {
+    if (aborted && lane == 0) {
+      tc_commit(drain);
+      mbar_wait_plain(drain, 0);
+    }
+    __syncwarp();
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols)
+                 : "memory");
   }
 }
 
-// Merge the split partials of every (node, head) with log-sum-exp weights.
+// Merge the split partials of every (node, head) with log-sum-exp weights:
+// one warp per (node, head), lane s holds split s's (m, l), lanes own 4 dims.
 __global__ void __launch_bounds__(256)
 attn_combine_kernel(const float* __restrict__ part_o, const float2* __restrict__ part_ml,
                     const int32_t* __restrict__ ctx_len, const int32_t* __restrict__ node_off,
                     int max_ctx, int chunk, int n_q, int total_nodes, float* __restrict__ out) {
-  const int b = blockIdx.y;
+  const int b = blockIdx.z;
   const int i = blockIdx.x;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int h = blockIdx.y * 8 + warp;
   const int o = node_off[b];
   const int T = node_off[b + 1] - o;
-  if (T < 1 || T > EE_MAX_TREE || o < 0 || o + T > total_nodes || i >= T) return;
+  if (T < 1 || T > EE_MAX_TREE || o < 0 || o + T > total_nodes || i >= T || h >= n_q) return;
   int ctx = ctx_len[b];
   ctx = ctx < 0 ? 0 : (ctx > max_ctx ? max_ctx : ctx);
-  const int S = ee::attn_splits_for(ctx, chunk);
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  for (int h = warp; h < n_q; h += 8) {
-    float M = -INFINITY;
-    for (int s = 0; s < S; ++s) M = fmaxf(M, part_ml[((size_t)s * total_nodes + o + i) * n_q + h].x);
-    const float Mu = M == -INFINITY ? 0.f : M;
-    float L = 0.f;
-    float4 a = make_float4(0.f, 0.f, 0.f, 0.f);
-    for (int s = 0; s < S; ++s) {
-      const size_t r = ((size_t)s * total_nodes + o + i) * n_q + h;
-      const float2 ml = part_ml[r];
-      const float w = ex2(ml.x - Mu);
-      L += w * ml.y;
-      const float4 v = *reinterpret_cast<const float4*>(part_o + r * kD + lane * 4);
-      a.x += w * v.x;
-      a.y += w * v.y;
-      a.z += w * v.z;
-      a.w += w * v.w;
-    }
-    const float inv = L > 0.f ? 1.f / L : 0.f;
-    *reinterpret_cast<float4*>(out + ((size_t)(o + i) * n_q + h) * kD + lane * 4) =
-        make_float4(a.x * inv, a.y * inv, a.z * inv, a.w * inv);
+  const int S = attn_splits_for(ctx, chunk);
+  const size_t r0 = (size_t)(o + i) * n_q + h;
+  const size_t sstride = (size_t)total_nodes * n_q;
+  float m = -INFINITY, lsum = 0.f;
+  if (lane < S) {
+    const float2 ml = part_ml[lane * sstride + r0];
+    m = ml.x;
+    lsum = ml.y;
   }
+  float M = m;
+#pragma unroll
+  for (int d = 16; d >= 1; d >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, d));
+  const float Mu = M == -INFINITY ? 0.f : M;
+  const float w = lane < S ? ex2(m - Mu) : 0.f;
+  float L = w * lsum;
+#pragma unroll
+  for (int d = 16; d >= 1; d >>= 1) L += __shfl_xor_sync(0xffffffffu, L, d);
+  float4 a = make_float4(0.f, 0.f, 0.f, 0.f);
+  for (int s = 0; s < S; ++s) {
+    const float ws = __shfl_sync(0xffffffffu, w, s);
+    const float4 v = __ldg(reinterpret_cast<const float4*>(part_o + (s * sstride + r0) * kD) + lane);
+    a.x += ws * v.x;
+    a.y += ws * v.y;
+    a.z += ws * v.z;
+    a.w += ws * v.w;
+  }
+  const float inv = L > 0.f ? 1.f / L : 0.f;
+  reinterpret_cast<float4*>(out + r0 * kD)[lane] = make_float4(a.x * inv, a.y * inv, a.z * inv, a.w * inv);
 }
 
 // Context chunk length: the smallest number of splits whose CTA count fills
 // the 152 SMs nearly as well as the best choice does.
 int choose_chunk(int max_ctx, int per_split_ctas) {
   if (max_ctx <= 0) return EE_PAGE;
-  const int cap = std::max(1, std::min(ee::kMaxSplits, (max_ctx + 255) / 256));
+  const int cap = std::max(1, std::min(kMaxSplits, (max_ctx + 255) / 256));
   double best = 0.0;
-  double eff[ee::kMaxSplits + 1];
+  double eff[kMaxSplits + 1];
   for (int s = 1; s <= cap; ++s) {
     const long n = (long)per_split_ctas * s;
-    const long waves = (n + ee::kNumSMs - 1) / ee::kNumSMs;
-    eff[s] = (double)n / (double)(waves * ee::kNumSMs);
+    const long waves = (n + kNumSMs - 1) / kNumSMs;
+    eff[s] = (double)n / (double)(waves * kNumSMs);
     best = std::max(best, eff[s]);
   }
   int pick = cap;
@@ -450,39 +527,50 @@ extern "C" ee_status ee_tree_verify_attn(const ee_bf16* q, const ee_bf16* k_tree
   if (!q || !k_tree || !v_tree || !k_cache || !v_cache || !block_table || !ctx_len || !node_off ||
       !anc || !out || !ws)
     return EE_ERR_INVALID_ARG;
-  if (!ee::aligned(q, 16) || !ee::aligned(k_tree, 16) || !ee::aligned(v_tree, 16) ||
-      !ee::aligned(k_cache, 16) || !ee::aligned(v_cache, 16) || !ee::aligned(out, 16) ||
-      !ee::aligned(anc, 8) || !ee::aligned(ws, 256))
+  if (!aligned(q, 16) || !aligned(k_tree, 16) || !aligned(v_tree, 16) || !aligned(k_cache, 16) ||
+      !aligned(v_cache, 16) || !aligned(out, 16) || !aligned(anc, 8) || !aligned(ws, 256))
     return EE_ERR_INVALID_ARG;
-  if (ws_bytes < ee::kAttnOff + ee::attn_partial_bytes(total_nodes, n_q, head_dim))
-    return EE_ERR_WORKSPACE;
+  if (ws_bytes < kAttnOff + attn_partial_bytes(total_nodes, n_q, head_dim)) return EE_ERR_WORKSPACE;
+  if ((int64_t)num_pages * n_kv * EE_PAGE >= ((int64_t)1 << 31)) return EE_ERR_UNSUPPORTED;
 
   static bool attr_set = false;
   if (!attr_set) {
-    EE_CUDA_OK(cudaFuncSetAttribute(attn_split_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                    kSmemBytes));
+    EE_CUDA_OK(cudaFuncSetAttribute(attn_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    (int)kSmemBytes));
     attr_set = true;
+  }
+  // tensor maps: cache [pages * n_kv * 16 rows][128], tree [total][n_kv][128]
+  CUtensorMap tmKc, tmVc, tmKt, tmVt;
+  {
+    const uint64_t dims[2] = {(uint64_t)head_dim, (uint64_t)num_pages * n_kv * EE_PAGE};
+    const uint64_t strides[1] = {(uint64_t)head_dim * 2};
+    const uint32_t box[2] = {64, EE_PAGE};
+    if (!encode_bf16_tmap(&tmKc, k_cache, 2, dims, strides, box)) return EE_ERR_CUDA;
+    if (!encode_bf16_tmap(&tmVc, v_cache, 2, dims, strides, box)) return EE_ERR_CUDA;
+  }
+  {
+    const uint64_t dims[3] = {(uint64_t)head_dim, (uint64_t)n_kv, (uint64_t)total_nodes};
+    const uint64_t strides[2] = {(uint64_t)head_dim * 2, (uint64_t)n_kv * head_dim * 2};
+    const uint32_t box[3] = {64, 1, 64};
+    if (!encode_bf16_tmap(&tmKt, k_tree, 3, dims, strides, box)) return EE_ERR_CUDA;
+    if (!encode_bf16_tmap(&tmVt, v_tree, 3, dims, strides, box)) return EE_ERR_CUDA;
   }
   const int g = n_q / n_kv;
   const int nrb = (max_T * g + kRows - 1) / kRows;
   const int chunk = choose_chunk(max_ctx, nrb * n_kv * B);
-  const int S = ee::attn_splits_for(max_ctx, chunk);
+  const int S = attn_splits_for(max_ctx, chunk);
 
   char* wsb = static_cast<char*>(ws);
   AttnParams p;
   p.q = reinterpret_cast<const __nv_bfloat16*>(q);
-  p.kt = reinterpret_cast<const __nv_bfloat16*>(k_tree);
-  p.vt = reinterpret_cast<const __nv_bfloat16*>(v_tree);
-  p.kc = reinterpret_cast<const __nv_bfloat16*>(k_cache);
-  p.vc = reinterpret_cast<const __nv_bfloat16*>(v_cache);
   p.block_table = block_table;
   p.ctx_len = ctx_len;
   p.node_off = node_off;
   p.anc = anc;
-  p.part_o = reinterpret_cast<float*>(wsb + ee::kAttnOff);
-  const size_t rows = (size_t)ee::kMaxSplits * total_nodes * n_q;
-  p.part_ml = reinterpret_cast<float2*>(wsb + ee::kAttnOff + ee::align_up(rows * head_dim * 4, 256));
-  p.err = ee::err_word(ws);
+  p.part_o = reinterpret_cast<float*>(wsb + kAttnOff);
+  const size_t rows = (size_t)kMaxSplits * total_nodes * n_q;
+  p.part_ml = reinterpret_cast<float2*>(wsb + kAttnOff + align_up(rows * head_dim * 4, 256));
+  p.err = err_word(ws);
   p.num_pages = num_pages;
   p.max_pages = max_pages;
   p.max_ctx = max_ctx;
@@ -496,9 +584,9 @@ extern "C" ee_status ee_tree_verify_attn(const ee_bf16* q, const ee_bf16* k_tree
   p.scale_log2 = scale * 1.4426950408889634f;
 
   dim3 grid(nrb * S, n_kv, B);
-  attn_split_kernel<<<grid, kThreads, kSmemBytes, (cudaStream_t)stream>>>(p);
+  attn_tc_kernel<<<grid, kThreads, kSmemBytes, (cudaStream_t)stream>>>(tmKc, tmVc, tmKt, tmVt, p);
   EE_LAUNCH_OK();
-  attn_combine_kernel<<<dim3(max_T, B), 256, 0, (cudaStream_t)stream>>>(
+  attn_combine_kernel<<<dim3(max_T, (n_q + 7) / 8, B), 256, 0, (cudaStream_t)stream>>>(
       p.part_o, p.part_ml, ctx_len, node_off, max_ctx, chunk, n_q, total_nodes, out);
   EE_LAUNCH_OK();
   return EE_OK;

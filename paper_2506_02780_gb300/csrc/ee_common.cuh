@@ -1,9 +1,13 @@
 // Shared device/host helpers of libee (sm_103a).  Internal header.
 #pragma once
+#include <cuda.h>
 #include <cuda_runtime.h>
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
 #include <stdint.h>
+
+#include <algorithm>
+#include <cmath>
 
 #include "../../include/ee.h"
 
@@ -46,6 +50,12 @@ __host__ __device__ inline int attn_splits_for(int ctx, int chunk) {
   int s = (ctx + chunk - 1) / chunk;
   return s < 1 ? 1 : s;
 }
+
+// Encode a TMA tensor map over a bf16 array with 128-byte swizzle and zero
+// fill out of bounds.  dims[0] is the contiguous dimension; strides_bytes[i]
+// is the byte stride of dimension i+1.  Returns false on failure.
+bool encode_bf16_tmap(CUtensorMap* map, const void* base, int rank, const uint64_t* dims,
+                      const uint64_t* strides_bytes, const uint32_t* box);
 
 }  // namespace ee
 
