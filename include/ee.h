@@ -29,8 +29,8 @@
  *    [num_pages][n_kv][EE_PAGE][head_dim]; position t of sequence s lives in
  *    page block_table[s * max_pages + t / EE_PAGE], row t % EE_PAGE.
  *  - `ws` is a caller-owned device workspace of at least
- *    ee_workspace_size(...) bytes, zeroed once with ee_workspace_init() before
- *    first use.  Its first word is the device error word: kernels never trap;
+ *    ee_workspace_size(...) bytes (a few KB: the error word and the LM head's
+ *    running argmax), zeroed once with ee_workspace_init() before first use.  Its first word is the device error word: kernels never trap;
  *    on a bad index found on the device they set an EE_DEVERR_* bit there,
  *    skip the access and continue.  ee_read_errors() reads (and clears) it.
  *    After any error the workspace must be re-initialised.  Calls that share
@@ -73,7 +73,7 @@ typedef enum {
 #define EE_DEVERR_TREE         0x02  /* parent[] violates 0 <= parent[i] < i, or T outside 1..128 */
 #define EE_DEVERR_PAGE         0x04  /* block_table entry outside [0, num_pages) for a needed slot */
 #define EE_DEVERR_CTX          0x08  /* ctx_len < 0 or above the max_ctx passed by the host */
-#define EE_DEVERR_FP16_RANGE   0x10  /* |V| > 65504: P.V runs in fp16 and V did not fit */
+#define EE_DEVERR_FP16_RANGE   0x10  /* reserved (no current kernel sets it) */
 #define EE_DEVERR_TIMEOUT      0x20  /* a bounded device wait gave up */
 #define EE_DEVERR_PATH         0x40  /* path / accept_len inconsistent with the tree */
 
@@ -146,11 +146,15 @@ ee_status ee_tree_prepare(const int32_t* parent, const int32_t* node_off, int32_
  *   block_table int32 [B][max_pages]; ctx_len int32 [B], 0 <= ctx_len <= max_ctx
  *   node_off  int32 [B+1]; anc uint64 [total_nodes][2] from ee_tree_prepare
  *   out       fp32 [total_nodes][n_q][head_dim]   out
- * head_dim must be 128; n_q a multiple of n_kv; max_T <= 128; all bf16 arrays
- * 16-byte aligned.  Q.K runs on bf16 tensor cores with fp32 accumulation; P.V
- * runs with P and V in fp16 (exact for |V| <= 65504, larger values set
- * EE_DEVERR_FP16_RANGE); softmax and the output are fp32.
- * Device errors: EE_DEVERR_PAGE (the key is skipped), EE_DEVERR_CTX.
+ * head_dim must be 128; n_q a multiple of n_kv; max_T <= 128; max_ctx <= 262144;
+ * all bf16 arrays 16-byte aligned.  Q.K^T runs on bf16 tensor cores with fp32
+ * accumulation in TMEM; P.V runs on bf16 tensor cores with P carried as two
+ * bf16 parts (head + tail, about 2^-14 relative) and V as stored; softmax and
+ * the output are fp32.  One launch per call: a thread-block cluster of up to
+ * 8 CTAs per 128 query rows splits the context and merges its partial results
+ * in distributed shared memory.
+ * Device errors: EE_DEVERR_PAGE (the key is skipped), EE_DEVERR_CTX,
+ * EE_DEVERR_TIMEOUT (outputs undefined).
  */
 ee_status ee_tree_verify_attn(const ee_bf16* q, const ee_bf16* k_tree, const ee_bf16* v_tree,
                               const ee_bf16* k_cache, const ee_bf16* v_cache, int32_t num_pages,

@@ -21,12 +21,12 @@ extern "C" size_t ee_workspace_size(int32_t B, int32_t total_nodes, int32_t n_q,
   (void)B;
   (void)max_ctx;
   if (total_nodes < 0 || n_q < 0 || head_dim < 0) return 0;
-  return ee::kAttnOff + ee::attn_partial_bytes(total_nodes, n_q, head_dim);
+  return ee::kWorkspaceBytes;
 }
 
 extern "C" ee_status ee_workspace_init(void* ws, size_t ws_bytes, ee_stream_t stream) {
-  if (!ws || ws_bytes < ee::kAttnOff || !ee::aligned(ws, 256)) return EE_ERR_INVALID_ARG;
-  EE_CUDA_OK(cudaMemsetAsync(ws, 0, ee::kAttnOff, (cudaStream_t)stream));
+  if (!ws || ws_bytes < ee::kWorkspaceBytes || !ee::aligned(ws, 256)) return EE_ERR_INVALID_ARG;
+  EE_CUDA_OK(cudaMemsetAsync(ws, 0, ee::kWorkspaceBytes, (cudaStream_t)stream));
   return EE_OK;
 }
 

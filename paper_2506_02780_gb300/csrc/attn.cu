@@ -8,21 +8,40 @@
 //     the group times the T tree nodes, row r = node * g + head_in_group, so
 //     one K/V tile feeds g * T rows (GQA packing).  A CTA owns 128 rows: the
 //     M side of a tcgen05 MMA.
-//   - The context is cut into chunks of `chunk` keys (a multiple of the 16-token
-//     page); each (row block, chunk) is one CTA.  The CTA of the last chunk
-//     also processes the tree keys, masked by the ancestor bitmask.
-//   - Warp 0 streams 64-key K/V tiles with TMA (one 16-row box per page and
-//     128-byte half of the head dimension; the tree's own K/V through a 3-D map)
-//     into a 3-stage ring.  Warps 2-3 convert each landed V tile to fp16 in
-//     place.  Warp 1 issues tcgen05.mma: S = Q K^T (bf16, fp32 in TMEM, double
-//     buffered) and O += P V (fp16 P from shared memory, fp16 V read MN-major,
-//     fp32 O in TMEM).  Warps 4-7 own one query row per thread: they read S
-//     from TMEM, mask, keep the running max/sum, write P, and rescale O in TMEM
-//     only when a row's max grows by more than 2^8 (the stale max keeps every
-//     P <= 256, exact in fp16, and the final O / l is unchanged).
-//   - Partials (unnormalised O, max m, sum l per row) go to the workspace; a
-//     second launch merges the chunks with log-sum-exp weights and writes fp32
-//     output.  No CTA ever waits on another; every mbarrier wait is bounded.
+//   - The context is cut into S <= 8 chunks of `chunk` keys (a multiple of the
+//     16-token page, at most 2048 pages); each (row block, chunk) is one CTA.  The CTA of
+//     the last chunk also processes the tree keys (one 128-key tile), masked by
+//     the ancestor bitmask.  A CTA first stages its chunk's page ids in shared
+//     memory.
+//   - Q lives in TMEM (bf16 pairs, loaded by the softmax threads, one row each)
+//     and is the A operand of S = Q K^T, so shared memory holds only K and V.
+//   - Keys come in 128-key tiles.  Warps 0 and 2 stream K and V tiles with TMA
+//     (one 16-row box per page and 64-dim half, spread over 8 lanes; the tree's
+//     K/V through a 3-D map) into two 3-stage rings.  Warp 1 issues
+//     tcgen05.mma in a fixed order: S = Q K^T (bf16, fp32 accumulators in TMEM,
+//     double buffered), then for each tile O += P V, then the Q K^T two tiles
+//     ahead, which overwrites the TMEM columns P lived in (the in-order tensor
+//     pipe finishes reading P first).
+//   - P.V runs on bf16 operands: P is split exactly into a bf16 head (the top
+//     16 bits of the fp32 value) and a bf16 tail (the top 16 bits of the
+//     remainder), both written over S in TMEM and used as the MMA A operand;
+//     V is read straight from shared memory (MN-major).  P is carried to about
+//     2^-14 relative (fp16 would give 2^-11), V needs no conversion, and the
+//     split costs integer ops only, leaving the special-function pipe to exp2.
+//   - Warps 4-7 own one query row per thread (its TMEM lane): they read S,
+//     mask, keep the running max/sum, write P, and rescale O in TMEM only when
+//     a row's max grows by more than 2^8 (the stale max keeps every P <= 256,
+//     and the final O / l is unchanged).
+//   - The S chunk-CTAs of one row block form a thread-block cluster.  Cluster
+//     rank k owns rows k, k+S, ...: after a first cluster barrier every CTA
+//     pushes each unnormalised O row and its (max, sum) straight into the owning
+//     CTA's shared memory (distributed shared memory, remote stores); after a
+//     second barrier each CTA merges its rows locally with log-sum-exp weights
+//     and writes the fp32 output.  No partial goes through HBM and no second
+//     launch is needed.  Every CTA of a cluster, also one whose chunk is
+//     empty for a short sequence, runs the same two cluster barriers; every
+//     mbarrier wait before them is bounded, so every thread reaches them.
+// Shared-memory traffic per 128-key tile: K 64 KB + V 64 KB (TMA write, MMA read).
 #include "ee_common.cuh"
 #include "ee_ptx.cuh"
 
@@ -30,25 +49,33 @@ namespace {
 
 using namespace ee;
 
-constexpr int kThreads = 256;
+constexpr int kThreads = 256;                    // 8 warps, roles below
 constexpr int kRows = 128;                       // query rows per CTA (MMA M)
-constexpr int kKT = 64;                          // keys per tile (MMA N of Q K^T)
+constexpr int kKT = 128;                         // keys per tile (MMA N of Q K^T, K of P V)
 constexpr int kD = EE_HEAD_DIM;                  // 128
-constexpr int kNST = 3;                          // K/V ring depth
-constexpr uint32_t kQHalf = kRows * 128;         // 16 KB: one 64-dim half of Q
-constexpr uint32_t kKVHalf = kKT * 128;          // 8 KB: one 64-dim half of a K or V tile
-constexpr uint32_t kKVBytes = 2 * kKVHalf;       // 16 KB
-constexpr uint32_t kStageBytes = 2 * kKVBytes;   // K + V
-constexpr uint32_t kPBytes = kRows * kKT * 2;    // 16 KB fp16 P tile
-constexpr uint32_t kOffKV = 2 * kQHalf;
-constexpr uint32_t kOffP = kOffKV + kNST * kStageBytes;
-constexpr uint32_t kOffBar = kOffP + 2 * kPBytes;
-constexpr uint32_t kNumBars = 3 * kNST + 3 * 2 + 2;
+constexpr int kKST = 3;                          // K ring depth
+constexpr int kVST = 3;                          // V ring depth
+constexpr uint32_t kKVHalf = kKT * 128;          // 16 KB: one 64-dim half of a K or V tile
+constexpr uint32_t kKVBytes = 2 * kKVHalf;       // 32 KB
+constexpr int kMaxCtaPages = 2048;               // context pages one CTA can own (32768 keys)
+constexpr uint32_t kOffK = 0;
+constexpr uint32_t kOffV = kOffK + kKST * kKVBytes;
+constexpr uint32_t kOffPages = kOffV + kVST * kKVBytes;
+constexpr uint32_t kOffBar = kOffPages + 4 * kMaxCtaPages;
+constexpr uint32_t kNumBars = 2 * kKST + 2 * kVST + 3 * 2 + 2;
 constexpr uint32_t kSmemBytes = 1024 + kOffBar + 8 * kNumBars + 64;
-constexpr uint32_t kTmemCols = 256;              // S0 [0,64) S1 [64,128) O [128,256)
+constexpr uint32_t kTmemCols = 512;              // S0 [0,128) S1 [128,256) O [256,384) Q [384,448)
+constexpr uint32_t kColO = 256;
+constexpr uint32_t kColQ = 384;
 constexpr float kRescaleLog2 = 8.0f;
+constexpr int kMaxCluster = 8;                   // portable thread-block cluster size
+// warp roles (warp 3 is idle after set-up)
+constexpr int kWarpK = 0, kWarpMma = 1, kWarpV = 2, kWarpSoft0 = 4;
 
 static_assert(kRows == ee::kAttnRows, "row block size");
+static_assert(kThreads == 32 * (kWarpSoft0 + 4), "four softmax warps, one per TMEM lane quarter");
+static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
+static_assert(kRows * kD * 4 <= kKST * kKVBytes, "O staging fits in the idle K ring");
 
 struct AttnParams {
   const __nv_bfloat16* q;
@@ -56,10 +83,9 @@ struct AttnParams {
   const int32_t* ctx_len;
   const int32_t* node_off;
   const uint64_t* anc;
-  float* part_o;
-  float2* part_ml;
+  float* out;
   int32_t* err;
-  int num_pages, max_pages, max_ctx, n_q, n_kv, g, total_nodes, max_T, nrb, chunk;
+  int num_pages, max_pages, max_ctx, n_q, n_kv, g, total_nodes, max_T, nrb, chunk, S;
   float scale_log2;
 };
 
@@ -69,20 +95,17 @@ __device__ __forceinline__ float ex2(float x) {
   return y;
 }
 
-__device__ __forceinline__ uint32_t pack_half2(float lo, float hi) {
-  __half2 h = __floats2half2_rn(lo, hi);
-  return *reinterpret_cast<uint32_t*>(&h);
-}
-
-// Whether 16-row page block i of a context tile holds loaded keys; the producer,
-// the V converter and the softmax all derive the same answer from the inputs.
-__device__ __forceinline__ bool page_loaded(const AttnParams& p, int b, int key0, int k_end, int i,
-                                            int* page_out) {
-  const int pos = key0 + 16 * i;
-  if (pos >= k_end) return false;
-  const int page = p.block_table[(size_t)b * p.max_pages + (pos >> 4)];
-  *page_out = page;
-  return page >= 0 && page < p.num_pages;
+// Loaded-page mask of context tile t: bit i set when the tile's 16-row block i
+// holds keys below k_end in a valid page.  s_pages holds the CTA's page ids
+// (-1 for an out-of-range block-table entry).
+__device__ __forceinline__ unsigned tile_mask(const int32_t* s_pages, int t, int k_begin, int k_end) {
+  unsigned m = 0u;
+#pragma unroll
+  for (int i = 0; i < kKT / 16; ++i) {
+    const int pos = k_begin + t * kKT + 16 * i;
+    m |= (pos < k_end && s_pages[t * (kKT / 16) + i] >= 0) ? (1u << i) : 0u;
+  }
+  return m;
 }
 
 __global__ void __launch_bounds__(kThreads, 1)
@@ -94,12 +117,18 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
                                              ~static_cast<uintptr_t>(1023));
   __shared__ uint32_t s_tmem;
   __shared__ volatile int s_abort;
-  __shared__ int s_issued[kNST];
+  __shared__ int s_kissued[kKST], s_vissued[kVST];
 
+  if (threadIdx.x == 0) {
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmKc)) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmVc)) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmKt)) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmVt)) : "memory");
+  }
   const int b = blockIdx.z;
   const int hk = blockIdx.y;
-  const int rb = blockIdx.x % p.nrb;
-  const int split = blockIdx.x / p.nrb;
+  const int rb = blockIdx.x / p.S;                 // the cluster spans the S chunks of a row block
+  const int split = blockIdx.x % p.S;              // == cluster rank
   const int o = p.node_off[b];
   const int T = p.node_off[b + 1] - o;
   const int R = T * p.g;
@@ -113,397 +142,442 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
     if (threadIdx.x == 0 && blockIdx.x == 0 && hk == 0) flag_error(p.err, EE_DEVERR_CTX);
     ctx = ctx < 0 ? 0 : p.max_ctx;
   }
-  const int S = attn_splits_for(ctx, p.chunk);
-  if (split >= S) return;
+  // everything above is uniform over the cluster (same sequence, head and row
+  // block); from here on every CTA runs to the cluster barriers
+  const int S = attn_splits_for(ctx, p.chunk);     // chunks this sequence uses, <= p.S
+  const bool active = split < S;
   const int k_begin = split * p.chunk;
-  const int k_end = min(ctx, k_begin + p.chunk);
+  const int k_end = active ? min(ctx, k_begin + p.chunk) : k_begin;
   const int n_ctx_tiles = k_end > k_begin ? (k_end - k_begin + kKT - 1) / kKT : 0;
-  const int n_tree_tiles = (split == S - 1) ? (T + kKT - 1) / kKT : 0;
-  const int n_tiles = n_ctx_tiles + n_tree_tiles;
+  const int n_tiles = active ? n_ctx_tiles + ((split == S - 1) ? 1 : 0) : 0;   // + the tree tile
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  // softmax threads fetch their Q row now; it goes to TMEM once TMEM is allocated
+  uint4 qreg[16];
+  {
+    const int rr = rb * kRows + (warp & 3) * 32 + lane;
+    const bool mine = warp >= kWarpSoft0 && rr < R;
+    const int nd = mine ? rr / p.g : 0;
+    const uint4* src = reinterpret_cast<const uint4*>(
+        p.q + ((size_t)(o + nd) * p.n_q + hk * p.g + (mine ? rr - nd * p.g : 0)) * kD);
+#pragma unroll
+    for (int c = 0; c < 16; ++c) qreg[c] = mine ? __ldg(src + c) : make_uint4(0u, 0u, 0u, 0u);
+  }
   const uint32_t sbase = smem_u32(smem);
-  const uint32_t sQ = sbase, sKV = sbase + kOffKV, sP = sbase + kOffP;
+  const uint32_t sK = sbase + kOffK, sV = sbase + kOffV;
   const uint32_t bar0 = sbase + kOffBar;
-  const uint32_t kv_full = bar0, kv_empty = bar0 + 8 * kNST, v_ready = bar0 + 16 * kNST;
-  const uint32_t s_full = bar0 + 24 * kNST, s_free = s_full + 16, p_full = s_free + 16;
-  const uint32_t o_done = p_full + 16, drain = o_done + 8;
-
+  const uint32_t k_full = bar0, k_empty = k_full + 8 * kKST;
+  const uint32_t v_full = k_empty + 8 * kKST, v_empty = v_full + 8 * kVST;
+  const uint32_t s_full = v_empty + 8 * kVST, p_full = s_full + 16, o_done = p_full + 16;
+  const uint32_t drain = o_done + 16, q_ready = drain + 8;
+  int32_t* s_pages = reinterpret_cast<int32_t*>(smem + kOffPages);
+  {
+    const int npg = (k_end - k_begin + EE_PAGE - 1) / EE_PAGE;   // <= kMaxCtaPages (host caps chunk)
+    for (int i = threadIdx.x; i < npg; i += kThreads) {
+      const int pg = p.block_table[(size_t)b * p.max_pages + (k_begin >> 4) + i];
+      const bool ok = pg >= 0 && pg < p.num_pages;
+      if (!ok) flag_error(p.err, EE_DEVERR_PAGE);
+      s_pages[i] = ok ? pg : -1;
+    }
+  }
   if (threadIdx.x == 0) {
     s_abort = 0;
-    for (int i = 0; i < kNST; ++i) {
-      mbar_init(kv_full + 8 * i, 1);
-      mbar_init(kv_empty + 8 * i, 1);
-      mbar_init(v_ready + 8 * i, 64);
-      s_issued[i] = -1;
+    for (int i = 0; i < kKST; ++i) {
+      mbar_init(k_full + 8 * i, 1);
+      mbar_init(k_empty + 8 * i, 1);
+      s_kissued[i] = -1;
+    }
+    for (int i = 0; i < kVST; ++i) {
+      mbar_init(v_full + 8 * i, 1);
+      mbar_init(v_empty + 8 * i, 1);
+      s_vissued[i] = -1;
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(s_full + 8 * i, 1);
-      mbar_init(s_free + 8 * i, kRows);
       mbar_init(p_full + 8 * i, kRows);
+      mbar_init(o_done + 8 * i, 1);
     }
-    mbar_init(o_done, 1);
     mbar_init(drain, 1);
+    mbar_init(q_ready, kRows);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     fence_async_smem();
   }
-  if (warp == 1) {
+  if (warp == kWarpMma) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
                      smem_u32(&s_tmem)),
                  "r"(kTmemCols)
                  : "memory");
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
   }
-  // Q tile: 128 rows x 128 dims, K-major with 128-byte swizzle, two 64-dim halves
-  {
-    const int row_base = rb * kRows;
-#pragma unroll
-    for (int it = 0; it < (kRows * 16) / kThreads; ++it) {
-      const int idx = threadIdx.x + it * kThreads;
-      const int r = idx >> 4, c = idx & 15;
-      const int rr = row_base + r;
-      uint4 v = make_uint4(0u, 0u, 0u, 0u);
-      if (rr < R) {
-        const int node = rr / p.g, j = rr - node * p.g;
-        const __nv_bfloat16* src = p.q + ((size_t)(o + node) * p.n_q + hk * p.g + j) * kD + c * 8;
-        v = __ldg(reinterpret_cast<const uint4*>(src));
-      }
-      const uint32_t dst = sQ + (c >> 3) * kQHalf + r * 128 + (((c & 7) ^ (r & 7)) << 4);
-      asm volatile("st.shared.v4.b32 [%0], {%1,%2,%3,%4};" ::"r"(dst), "r"(v.x), "r"(v.y), "r"(v.z),
-                   "r"(v.w)
-                   : "memory");
-    }
-    fence_async_smem();
-  }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = s_tmem;
 
-  if (warp == 0) {
-    // ---------------- TMA producer ----------------
-    if (lane == 0) {
-      for (int t = 0; t < n_tiles; ++t) {
-        const int st = t % kNST, use = t / kNST;
-        if (!mbar_wait(kv_empty + 8 * st, (uint32_t)(use & 1) ^ 1u, &s_abort)) break;
-        const uint32_t full = kv_full + 8 * st;
-        const uint32_t sK = sKV + st * kStageBytes, sV = sK + kKVBytes;
-        if (t < n_ctx_tiles) {
-          const int key0 = k_begin + t * kKT;
-          int pages[4];
-          uint32_t bytes = 0;
-#pragma unroll
-          for (int i = 0; i < 4; ++i) {
-            int pg = -1;
-            const bool ok = page_loaded(p, b, key0, k_end, i, &pg);
-            if (!ok && key0 + 16 * i < k_end) flag_error(p.err, EE_DEVERR_PAGE);
-            pages[i] = ok ? pg : -1;
-            bytes += ok ? 4u * 2048u : 0u;
-          }
-          mbar_expect_tx(full, bytes);
-#pragma unroll
-          for (int i = 0; i < 4; ++i) {
-            if (pages[i] < 0) continue;
-            const int row0 = (pages[i] * p.n_kv + hk) * EE_PAGE;
-#pragma unroll
-            for (int h = 0; h < 2; ++h) {
-              tma_load_2d(sK + h * kKVHalf + i * 2048, &tmKc, full, h * 64, row0);
-              tma_load_2d(sV + h * kKVHalf + i * 2048, &tmVc, full, h * 64, row0);
-            }
-          }
-        } else {
-          const int key0 = (t - n_ctx_tiles) * kKT;
-          mbar_expect_tx(full, 4 * kKVHalf);
-#pragma unroll
-          for (int h = 0; h < 2; ++h) {
-            tma_load_3d(sK + h * kKVHalf, &tmKt, full, h * 64, hk, o + key0);
-            tma_load_3d(sV + h * kKVHalf, &tmVt, full, h * 64, hk, o + key0);
-          }
+  bool have = false;          // softmax threads: this row's partial is complete
+  float row_m = -INFINITY, row_l = 0.f;
+  if (warp == kWarpK || warp == kWarpV) {
+    // ---------------- TMA producers: warp 0 streams K, warp 2 streams V ----------------
+    // lane 0 waits for the slot and posts the byte count; lane i < 8 then issues
+    // the two boxes of the tile's 16-row block i
+    const bool isK = warp == kWarpK;
+    const int nst = isK ? kKST : kVST;
+    const uint32_t full0 = isK ? k_full : v_full, empty0 = isK ? k_empty : v_empty;
+    const uint32_t ring = isK ? sK : sV;
+    const CUtensorMap* mc = isK ? &tmKc : &tmVc;
+    const CUtensorMap* mt = isK ? &tmKt : &tmVt;
+    int* issued = isK ? s_kissued : s_vissued;
+    for (int t = 0; t < n_tiles; ++t) {
+      const int st = t % nst, use = t / nst;
+      bool go = true;
+      if (lane == 0) go = mbar_wait(empty0 + 8 * st, (uint32_t)(use & 1) ^ 1u, &s_abort);
+      if (!__shfl_sync(0xffffffffu, go, 0)) break;
+      const uint32_t full = full0 + 8 * st;
+      const uint32_t dst = ring + st * kKVBytes;
+      if (lane == 0) mbar_expect_tx(full, 2 * kKVHalf);
+      __syncwarp();
+      if (t < n_ctx_tiles) {
+        // every 16-row block is written: blocks without a loaded page are read at
+        // row -16, wholly out of range, which the TMA unit fills with zeros (a
+        // stale V row would turn 0 * P into NaN)
+        if (lane < kKT / 16) {
+          const int pos = k_begin + t * kKT + 16 * lane;
+          const int pg = pos < k_end ? s_pages[t * (kKT / 16) + lane] : -1;
+          const int row0 = pg >= 0 ? (pg * p.n_kv + hk) * EE_PAGE : -EE_PAGE;
+          tma_load_2d(dst + lane * 2048, mc, full, 0, row0);
+          tma_load_2d(dst + kKVHalf + lane * 2048, mc, full, 64, row0);
         }
-        s_issued[st] = use;
+      } else if (lane == 0) {
+        tma_load_3d(dst, mt, full, 0, hk, o);
+        tma_load_3d(dst + kKVHalf, mt, full, 64, hk, o);
       }
+      __syncwarp();
+      if (lane == 0) issued[st] = use;
     }
-  } else if (warp == 1) {
-    // ---------------- MMA issuer ----------------
+  } else if (warp == kWarpMma) {
+    // ---------------- MMA issuer: Q.K^T(0), Q.K^T(1), then P.V(t), Q.K^T(t+2) ----------------
     if (lane == 0) {
+      tc_fence_after();
       const uint32_t id_qk = idesc_f16(kRows, kKT, 1, 1, 0);
-      const uint32_t id_pv = idesc_f16(kRows, kD, 0, 0, 1);
-      bool ok = true;
-      auto issue_pv = [&](int u) -> bool {
-        const int st = u % kNST, sb = u & 1;
-        if (!mbar_wait(p_full + 8 * sb, (uint32_t)((u >> 1) & 1), &s_abort)) return false;
-        if (!mbar_wait(v_ready + 8 * st, (uint32_t)((u / kNST) & 1), &s_abort)) return false;
+      const uint32_t id_pv = idesc_f16(kRows, kD, 1, 1, 1);
+      auto issue_qk = [&](int t) -> bool {
+        if (!mbar_wait(k_full + 8 * (t % kKST), (uint32_t)((t / kKST) & 1), &s_abort)) return false;
         tc_fence_after();
-        const uint32_t pa = sP + sb * kPBytes;
-        const uint32_t vb = sKV + st * kStageBytes + kKVBytes;
-#pragma unroll
-        for (int j = 0; j < kKT / 16; ++j)
-          tc_mma(tmem + 128, smem_desc_sw128(pa + j * 32), smem_desc_sw128_mn(vb + j * 2048, kKVHalf, 1024),
-                 id_pv, (u > 0 || j > 0) ? 1u : 0u);
-        tc_commit(kv_empty + 8 * st);
-        tc_commit(o_done);
-        return true;
-      };
-      for (int t = 0; t < n_tiles && ok; ++t) {
-        const int st = t % kNST, use = t / kNST, sb = t & 1;
-        if (!mbar_wait(kv_full + 8 * st, (uint32_t)(use & 1), &s_abort)) break;
-        if (t >= 2 && !mbar_wait(s_free + 8 * sb, (uint32_t)((t >> 1) & 1) ^ 1u, &s_abort)) break;
-        tc_fence_after();
-        const uint32_t kb = sKV + st * kStageBytes;
+        const uint32_t kb = sK + (t % kKST) * kKVBytes;
 #pragma unroll
         for (int kk = 0; kk < kD / 16; ++kk) {
-          const uint32_t off = (kk >> 2) * 0 + (kk & 3) * 32;
-          tc_mma(tmem + sb * kKT, smem_desc_sw128(sQ + (kk >> 2) * kQHalf + off),
-                 smem_desc_sw128(kb + (kk >> 2) * kKVHalf + off), id_qk, kk > 0 ? 1u : 0u);
+          const uint32_t off = (kk & 3) * 32;
+          tc_mma_ts(tmem + (t & 1) * kKT, tmem + kColQ + 8 * kk,
+                    smem_desc_sw128(kb + (kk >> 2) * kKVHalf + off), id_qk, kk > 0 ? 1u : 0u);
         }
-        tc_commit(s_full + 8 * sb);
-        if (t >= 1) ok = issue_pv(t - 1);
-      }
-      if (ok && n_tiles > 0) issue_pv(n_tiles - 1);
-    }
-  } else if (warp < 4) {
-    // ---------------- V converters: bf16 -> fp16 in place ----------------
-    const int ct = threadIdx.x - 64;
-    bool overflow = false;
-    for (int t = 0; t < n_tiles; ++t) {
-      const int st = t % kNST, use = t / kNST;
-      if (!mbar_wait(kv_full + 8 * st, (uint32_t)(use & 1), &s_abort)) break;
-      uint4* sv = reinterpret_cast<uint4*>(smem + kOffKV + st * kStageBytes + kKVBytes);
-      // rows of a context tile whose page was not loaded hold stale bytes: zero them
-      unsigned loaded = 0xFu;
-      if (t < n_ctx_tiles) {
-        const int key0 = k_begin + t * kKT;
-        loaded = 0u;
+        tc_commit(k_empty + 8 * (t % kKST));
+        tc_commit(s_full + 8 * (t & 1));
+        return true;
+      };
+      bool ok = mbar_wait(q_ready, 0, &s_abort);
+      ok = ok && (n_tiles < 1 || issue_qk(0)) && (n_tiles < 2 || issue_qk(1));
+      for (int t = 0; t < n_tiles && ok; ++t) {
+        if (!mbar_wait(p_full + 8 * (t & 1), (uint32_t)((t >> 1) & 1), &s_abort) ||
+            !mbar_wait(v_full + 8 * (t % kVST), (uint32_t)((t / kVST) & 1), &s_abort))
+          break;
+        tc_fence_after();
+        const uint32_t pa = tmem + (t & 1) * kKT;          // bf16 P head: cols 0..63, tail: 64..127
+        const uint32_t vb = sV + (t % kVST) * kKVBytes;
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          int pg;
-          if (page_loaded(p, b, key0, k_end, i, &pg)) loaded |= 1u << i;
-        }
-      }
-#pragma unroll 4
-      for (int it = 0; it < (int)(kKVBytes / 16) / 64; ++it) {
-        const int idx = ct + it * 64;                 // 16-byte chunk; 8 per 128-byte row
-        const int row = (idx >> 3) & (kKT - 1);       // key row within the 64-dim half
-        uint4 v = sv[idx];
-        if (!((loaded >> (row >> 4)) & 1u)) {
-          v = make_uint4(0u, 0u, 0u, 0u);
-        } else {
-          uint32_t* w = reinterpret_cast<uint32_t*>(&v);
+        for (int part = 0; part < 2; ++part)
 #pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            __nv_bfloat162 bb = *reinterpret_cast<__nv_bfloat162*>(&w[e]);
-            const float2 f = __bfloat1622float2(bb);
-            overflow |= (fabsf(f.x) > 65504.f) || (fabsf(f.y) > 65504.f);
-            w[e] = pack_half2(f.x, f.y);
-          }
-        }
-        sv[idx] = v;
+          for (int j = 0; j < kKT / 16; ++j)
+            tc_mma_ts(tmem + kColO, pa + 64 * part + 8 * j,
+                      smem_desc_sw128_mn(vb + j * 2048, kKVHalf, 1024), id_pv,
+                      (t > 0 || part > 0 || j > 0) ? 1u : 0u);
+        tc_commit(v_empty + 8 * (t % kVST));
+        tc_commit(o_done + 8 * (t & 1));
+        if (t + 2 < n_tiles) ok = issue_qk(t + 2);
       }
-      fence_async_smem();
-      mbar_arrive(v_ready + 8 * st);
     }
-    if (overflow) flag_error(p.err, EE_DEVERR_FP16_RANGE);
-  } else {
+  } else if (warp >= kWarpSoft0) {
     // ---------------- softmax: one query row per thread ----------------
-    const int r = threadIdx.x - 128;                  // == TMEM lane
+    const int r = (warp & 3) * 32 + lane;             // == TMEM lane of this warp's quarter
     const int rr = rb * kRows + r;
     const bool vrow = rr < R;
     const int node = vrow ? rr / p.g : 0;
-    const int head = hk * p.g + (vrow ? rr - node * p.g : 0);
     const uint64_t a0 = vrow ? p.anc[2 * (size_t)(o + node)] : 0ull;
     const uint64_t a1 = vrow ? p.anc[2 * (size_t)(o + node) + 1] : 0ull;
     const uint32_t tl = tmem + ((uint32_t)((warp & 3) * 32) << 16);
+    // this row of Q into TMEM columns kColQ.. (bf16 pairs), zeros for rows past R
+    {
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        uint32_t qw[32];
+#pragma unroll
+        for (int c = 0; c < 8; ++c) {
+          const uint4 v = qreg[h * 8 + c];
+          qw[4 * c] = v.x;
+          qw[4 * c + 1] = v.y;
+          qw[4 * c + 2] = v.z;
+          qw[4 * c + 3] = v.w;
+        }
+        tc_st32(tl + kColQ + 32 * h, qw);
+      }
+      tc_fence_before();
+      mbar_arrive(q_ready);
+    }
+    // m_used is kept in raw score units (scale > 0, so the max commutes with it)
     float m_used = -INFINITY, l = 0.f;
+    const float sl2 = p.scale_log2;
     bool ok = true;
     for (int t = 0; t < n_tiles; ++t) {
       const int sb = t & 1;
-      if (!mbar_wait(s_full + 8 * sb, (uint32_t)((t >> 1) & 1), &s_abort)) {
+      // every wait outcome is made warp-uniform: the TMEM accesses that follow are
+      // warp-collective (.sync.aligned) and must be reached by all 32 lanes or none
+      if (!__all_sync(0xffffffffu, mbar_wait(s_full + 8 * sb, (uint32_t)((t >> 1) & 1), &s_abort))) {
         ok = false;
         break;
       }
       tc_fence_after();
-      uint32_t sr[64];
-      tc_ld32(tl + sb * kKT, *reinterpret_cast<uint32_t(*)[32]>(&sr[0]));
-      tc_ld32(tl + sb * kKT + 32, *reinterpret_cast<uint32_t(*)[32]>(&sr[32]));
-      tc_fence_before();
-      mbar_arrive(s_free + 8 * sb);
-      float tmax = -INFINITY;
+      uint32_t sr[kKT];
+#pragma unroll
+      for (int q4 = 0; q4 < kKT / 32; ++q4)
+        tc_ld32(tl + sb * kKT + 32 * q4, *reinterpret_cast<uint32_t(*)[32]>(&sr[32 * q4]));
+      // visibility of the tile's 128 keys, as two 64-bit words
+      uint64_t keep0, keep1;
       if (t < n_ctx_tiles) {
-        const int key0 = k_begin + t * kKT;
-        unsigned loaded = 0u;
+        const unsigned m = tile_mask(s_pages, t, k_begin, k_end);
+        const int nvalid = min(kKT, k_end - (k_begin + t * kKT));
+        uint64_t pg0 = 0ull, pg1 = 0ull;
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
-          int pg;
-          if (page_loaded(p, b, key0, k_end, i, &pg)) loaded |= 1u << i;
+          pg0 |= ((m >> i) & 1u) ? (0xFFFFull << (16 * i)) : 0ull;
+          pg1 |= ((m >> (i + 4)) & 1u) ? (0xFFFFull << (16 * i)) : 0ull;
         }
-#pragma unroll
-        for (int c = 0; c < kKT; ++c) {
-          const bool v = vrow && (key0 + c < k_end) && ((loaded >> (c >> 4)) & 1u);
-          const float x = v ? __uint_as_float(sr[c]) * p.scale_log2 : -INFINITY;
-          sr[c] = __float_as_uint(x);
-          tmax = fmaxf(tmax, x);
-        }
+        keep0 = pg0 & (nvalid >= 64 ? ~0ull : ((1ull << nvalid) - 1ull));
+        keep1 = pg1 & (nvalid >= 128 ? ~0ull : (nvalid <= 64 ? 0ull : ((1ull << (nvalid - 64)) - 1ull)));
       } else {
-        const int key0 = (t - n_ctx_tiles) * kKT;
-        const uint64_t w = key0 == 0 ? a0 : a1;       // key0 is 0 or 64
+        keep0 = a0 & (T >= 64 ? ~0ull : ((1ull << T) - 1ull));
+        keep1 = a1 & (T >= 128 ? ~0ull : (T <= 64 ? 0ull : ((1ull << (T - 64)) - 1ull)));
+      }
+      if (!vrow) keep0 = keep1 = 0ull;
+      const bool full = __all_sync(0xffffffffu, (keep0 & keep1) == ~0ull);
+      if (!full) {
 #pragma unroll
         for (int c = 0; c < kKT; ++c) {
-          const bool v = vrow && (key0 + c < T) && ((w >> c) & 1ull);
-          const float x = v ? __uint_as_float(sr[c]) * p.scale_log2 : -INFINITY;
-          sr[c] = __float_as_uint(x);
-          tmax = fmaxf(tmax, x);
+          const uint64_t kw = c < 64 ? keep0 : keep1;
+          if (!((kw >> (c & 63)) & 1ull)) sr[c] = __float_as_uint(-INFINITY);
         }
       }
+      float mx[8];
+#pragma unroll
+      for (int c = 0; c < 8; ++c) mx[c] = __uint_as_float(sr[c]);
+#pragma unroll
+      for (int c = 8; c < kKT; ++c) mx[c & 7] = fmaxf(mx[c & 7], __uint_as_float(sr[c]));
+      const float tmax = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
+                               fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
       const float m_new = fmaxf(m_used, tmax);
-      if (t >= 1 && !mbar_wait(o_done, (uint32_t)((t - 1) & 1), &s_abort)) {
-        ok = false;
-        break;
-      }
-      const bool need = m_new > m_used + kRescaleLog2;
+      const bool need = (m_new - m_used) * sl2 > kRescaleLog2;   // true when m_used = -inf < m_new
       if (t >= 1 && __any_sync(0xffffffffu, need)) {
+        // O must hold P.V(t-1) before it is rescaled
+        if (!__all_sync(0xffffffffu,
+                        mbar_wait(o_done + 8 * (sb ^ 1), (uint32_t)(((t - 1) >> 1) & 1), &s_abort))) {
+          ok = false;
+          break;
+        }
         tc_fence_after();
-        const float f = need ? ex2(m_used - m_new) : 1.f;
+        const float f = need ? ex2((m_used - m_new) * sl2) : 1.f;
 #pragma unroll 1
-        for (int c4 = 0; c4 < 4; ++c4) {
+        for (int c4 = 0; c4 < kD / 32; ++c4) {
           uint32_t ov[32];
-          tc_ld32(tl + 128 + 32 * c4, ov);
+          tc_ld32(tl + kColO + 32 * c4, ov);
 #pragma unroll
           for (int e = 0; e < 32; ++e) ov[e] = __float_as_uint(__uint_as_float(ov[e]) * f);
-          tc_st32(tl + 128 + 32 * c4, ov);
+          tc_st32(tl + kColO + 32 * c4, ov);
         }
       }
       if (need) {
-        l *= ex2(m_used - m_new);
+        l *= ex2((m_used - m_new) * sl2);
         m_used = m_new;
       }
-      const float mu = m_used == -INFINITY ? 0.f : m_used;
-      // P row (fp16) into the K-major, 128-byte-swizzled P tile
-      const uint32_t prow = sP + sb * kPBytes + r * 128;
+      const float nms = m_used == -INFINITY ? 0.f : -m_used * sl2;
+      // p = 2^(s*scale_log2 - m); P = head + tail, both bf16 (top 16 bits),
+      // head pairs over columns 0..63 of this S buffer, tail pairs over 64..127
+      float ls[8];
 #pragma unroll
-      for (int ch = 0; ch < 8; ++ch) {
-        uint32_t w4[4];
+      for (int h = 0; h < 2; ++h) {
+        uint32_t hw[32], tw[32];
 #pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const float p0 = ex2(__uint_as_float(sr[ch * 8 + 2 * e]) - mu);
-          const float p1 = ex2(__uint_as_float(sr[ch * 8 + 2 * e + 1]) - mu);
-          l += p0 + p1;
-          w4[e] = pack_half2(p0, p1);
+        for (int e = 0; e < 32; ++e) {
+          const int c = h * 64 + 2 * e;
+          const float p0 = ex2(fmaf(__uint_as_float(sr[c]), sl2, nms));
+          const float p1 = ex2(fmaf(__uint_as_float(sr[c + 1]), sl2, nms));
+          if (h == 0 && e < 8) ls[e] = p0 + p1; else ls[e & 7] += p0 + p1;
+          const uint32_t h0 = __float_as_uint(p0) & 0xFFFF0000u;
+          const uint32_t h1 = __float_as_uint(p1) & 0xFFFF0000u;
+          const uint32_t t0 = __float_as_uint(p0 - __uint_as_float(h0));
+          const uint32_t t1 = __float_as_uint(p1 - __uint_as_float(h1));
+          hw[e] = __byte_perm(h0, h1, 0x7632);
+          tw[e] = __byte_perm(t0, t1, 0x7632);
         }
-        asm volatile("st.shared.v4.b32 [%0], {%1,%2,%3,%4};" ::"r"(prow + ((ch ^ (r & 7)) << 4)),
-                     "r"(w4[0]), "r"(w4[1]), "r"(w4[2]), "r"(w4[3])
-                     : "memory");
+        tc_st32(tl + sb * kKT + 32 * h, hw);
+        tc_st32(tl + sb * kKT + 64 + 32 * h, tw);
       }
-      fence_async_smem();
+      l += ((ls[0] + ls[1]) + (ls[2] + ls[3])) + ((ls[4] + ls[5]) + (ls[6] + ls[7]));
       tc_fence_before();
       mbar_arrive(p_full + 8 * sb);
     }
-    if (ok && n_tiles > 0 && mbar_wait(o_done, (uint32_t)((n_tiles - 1) & 1), &s_abort)) {
-      tc_fence_after();
-      const size_t pr = ((size_t)split * p.total_nodes + o + node) * p.n_q + head;
-#pragma unroll 1
-      for (int c4 = 0; c4 < 4; ++c4) {
-        uint32_t ov[32];
-        tc_ld32(tl + 128 + 32 * c4, ov);
-        if (vrow) {
-          float4* dst = reinterpret_cast<float4*>(p.part_o + pr * kD + 32 * c4);
-#pragma unroll
-          for (int e = 0; e < 8; ++e)
-            dst[e] = make_float4(__uint_as_float(ov[4 * e]), __uint_as_float(ov[4 * e + 1]),
-                                 __uint_as_float(ov[4 * e + 2]), __uint_as_float(ov[4 * e + 3]));
-        }
-      }
-      if (vrow) p.part_ml[pr] = make_float2(m_used, l);
-    }
+    // wait for the last P.V; the row is pushed to its owner after the first cluster barrier
+    const bool fin =
+        ok && n_tiles > 0 &&
+        mbar_wait(o_done + 8 * ((n_tiles - 1) & 1), (uint32_t)(((n_tiles - 1) >> 1) & 1), &s_abort);
+    have = __all_sync(0xffffffffu, fin);
+    row_m = (have && vrow && m_used != -INFINITY) ? m_used * sl2 : -INFINITY;
+    row_l = (have && vrow && m_used != -INFINITY) ? l : 0.f;
   }
 
-  // ---- teardown: drain on abort, free TMEM ----------------------------------
+  // ---- CTA teardown: drain on abort ---------------------------------------------
   tc_fence_before();
   __syncthreads();
   const bool aborted = s_abort != 0;
   if (aborted && threadIdx.x == 0) {
     flag_error(p.err, EE_DEVERR_TIMEOUT);
-    for (int st = 0; st < kNST; ++st)   // TMA copies still in flight land before the CTA exits
-      if (s_issued[st] >= 0) mbar_wait_plain(kv_full + 8 * st, (uint32_t)(s_issued[st] & 1));
+    // TMA copies still in flight land before the rings are reused
+    for (int st = 0; st < kKST; ++st)
+      if (s_kissued[st] >= 0) mbar_wait_plain(k_full + 8 * st, (uint32_t)(s_kissued[st] & 1));
+    for (int st = 0; st < kVST; ++st)
+      if (s_vissued[st] >= 0) mbar_wait_plain(v_full + 8 * st, (uint32_t)(s_vissued[st] & 1));
   }
-  if (warp == 1) {
-    if (aborted && lane == 0) {
-      tc_commit(drain);
-      mbar_wait_plain(drain, 0);
+  if (warp == kWarpMma && aborted && lane == 0) {
+    tc_commit(drain);
+    mbar_wait_plain(drain, 0);
+  }
+
+  // ---- cluster merge --------------------------------------------------------------
+  // every CTA of the cluster has finished its pipeline, so every K/V ring is free
+  cluster_sync();
+  const int rpc = (kRows + p.S - 1) / p.S;          // rows each rank owns
+  const uint32_t rbuf = sbase + kOffK;              // [sender][owned row][128 fp32], the K ring
+  const uint32_t rml = sbase + kOffV;               // [sender][owned row] (m, l), the V ring
+  if (warp >= kWarpSoft0) {
+    const int r = (warp & 3) * 32 + lane;
+    const int owner = r % p.S, j = r / p.S;
+    const uint32_t slot = (uint32_t)(split * rpc + j);
+    st_cluster_f2(map_cluster(rml + slot * 8, owner), row_m, row_l);
+    // the TMEM read is warp-collective: the whole warp reads when any lane has a
+    // row to push, and each lane stores only its own valid row
+    if (__any_sync(0xffffffffu, row_l > 0.f)) {
+      tc_fence_after();
+      const uint32_t tl = tmem + ((uint32_t)((warp & 3) * 32) << 16);
+      const uint32_t dst = map_cluster(rbuf + slot * (kD * 4), owner);
+#pragma unroll 1
+      for (int c4 = 0; c4 < kD / 32; ++c4) {
+        uint32_t ov[32];
+        tc_ld32(tl + kColO + 32 * c4, ov);
+        if (row_l > 0.f) {
+#pragma unroll
+          for (int e = 0; e < 8; ++e)
+            st_cluster_u4(dst + (32 * c4 + 4 * e) * 4, ov[4 * e], ov[4 * e + 1], ov[4 * e + 2],
+                          ov[4 * e + 3]);
+        }
+      }
     }
-    __syncwarp();
+  }
+  tc_fence_before();
+  cluster_sync();   // all pushes have landed
+  if (warp == kWarpMma) {
     tc_fence_after();
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols)
                  : "memory");
   }
-}
-
-// Merge the split partials of every (node, head) with log-sum-exp weights:
-// one warp per (node, head), lane s holds split s's (m, l), lanes own 4 dims.
-__global__ void __launch_bounds__(256)
-attn_combine_kernel(const float* __restrict__ part_o, const float2* __restrict__ part_ml,
-                    const int32_t* __restrict__ ctx_len, const int32_t* __restrict__ node_off,
-                    int max_ctx, int chunk, int n_q, int total_nodes, float* __restrict__ out) {
-  const int b = blockIdx.z;
-  const int i = blockIdx.x;
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int h = blockIdx.y * 8 + warp;
-  const int o = node_off[b];
-  const int T = node_off[b + 1] - o;
-  if (T < 1 || T > EE_MAX_TREE || o < 0 || o + T > total_nodes || i >= T || h >= n_q) return;
-  int ctx = ctx_len[b];
-  ctx = ctx < 0 ? 0 : (ctx > max_ctx ? max_ctx : ctx);
-  const int S = attn_splits_for(ctx, chunk);
-  const size_t r0 = (size_t)(o + i) * n_q + h;
-  const size_t sstride = (size_t)total_nodes * n_q;
-  float m = -INFINITY, lsum = 0.f;
-  if (lane < S) {
-    const float2 ml = part_ml[lane * sstride + r0];
-    m = ml.x;
-    lsum = ml.y;
-  }
-  float M = m;
-#pragma unroll
-  for (int d = 16; d >= 1; d >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, d));
-  const float Mu = M == -INFINITY ? 0.f : M;
-  const float w = lane < S ? ex2(m - Mu) : 0.f;
-  float L = w * lsum;
-#pragma unroll
-  for (int d = 16; d >= 1; d >>= 1) L += __shfl_xor_sync(0xffffffffu, L, d);
-  float4 a = make_float4(0.f, 0.f, 0.f, 0.f);
-  for (int s = 0; s < S; ++s) {
-    const float ws = __shfl_sync(0xffffffffu, w, s);
-    const float4 v = __ldg(reinterpret_cast<const float4*>(part_o + (s * sstride + r0) * kD) + lane);
-    a.x += ws * v.x;
-    a.y += ws * v.y;
-    a.z += ws * v.z;
-    a.w += ws * v.w;
-  }
-  const float inv = L > 0.f ? 1.f / L : 0.f;
-  reinterpret_cast<float4*>(out + r0 * kD)[lane] = make_float4(a.x * inv, a.y * inv, a.z * inv, a.w * inv);
-}
-
-// Context chunk length: the smallest number of splits whose CTA count fills
-// the 152 SMs nearly as well as the best choice does.
-int choose_chunk(int max_ctx, int per_split_ctas) {
-  if (max_ctx <= 0) return EE_PAGE;
-  const int cap = std::max(1, std::min(kMaxSplits, (max_ctx + 255) / 256));
-  double best = 0.0;
-  double eff[kMaxSplits + 1];
-  for (int s = 1; s <= cap; ++s) {
-    const long n = (long)per_split_ctas * s;
-    const long waves = (n + kNumSMs - 1) / kNumSMs;
-    eff[s] = (double)n / (double)(waves * kNumSMs);
-    best = std::max(best, eff[s]);
-  }
-  int pick = cap;
-  for (int s = 1; s <= cap; ++s)
-    if (eff[s] >= 0.9 * best) {
-      pick = s;
-      break;
+  // local merge of the owned rows: one warp per row, lane = 16-byte chunk
+  for (int j = warp; j < rpc; j += kThreads / 32) {
+    const int rr0 = split + p.S * j;
+    const int rrow = rb * kRows + rr0;
+    if (rr0 >= kRows || rrow >= R) break;
+    float m = -INFINITY, lsum = 0.f;
+    if (lane < p.S) {
+      float2 ml;
+      asm volatile("ld.shared.v2.f32 {%0, %1}, [%2];"
+                   : "=f"(ml.x), "=f"(ml.y)
+                   : "r"(rml + (uint32_t)(lane * rpc + j) * 8));
+      m = ml.x;
+      lsum = ml.y;
     }
-  int chunk = (max_ctx + pick - 1) / pick;
-  chunk = (chunk + EE_PAGE - 1) / EE_PAGE * EE_PAGE;
-  return chunk;
+    float M = m;
+#pragma unroll
+    for (int d = 16; d >= 1; d >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, d));
+    const float w = (m == -INFINITY) ? 0.f : ex2(m - M);
+    float L = w * lsum;
+#pragma unroll
+    for (int d = 16; d >= 1; d >>= 1) L += __shfl_xor_sync(0xffffffffu, L, d);
+    float4 a = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+    for (int s2 = 0; s2 < kMaxCluster; ++s2) {
+      const float ws = __shfl_sync(0xffffffffu, w, s2);
+      if (s2 < p.S && ws != 0.f) {
+        float4 v;
+        asm volatile("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];"
+                     : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+                     : "r"(rbuf + (uint32_t)((s2 * rpc + j) * kD + 4 * lane) * 4));
+        a.x += ws * v.x;
+        a.y += ws * v.y;
+        a.z += ws * v.z;
+        a.w += ws * v.w;
+      }
+    }
+    const float inv = L > 0.f ? 1.f / L : 0.f;
+    const int nd = rrow / p.g;
+    const size_t orow = (size_t)(o + nd) * p.n_q + hk * p.g + (rrow - nd * p.g);
+    reinterpret_cast<float4*>(p.out + orow * kD)[lane] =
+        make_float4(a.x * inv, a.y * inv, a.z * inv, a.w * inv);
+  }
+}
+
+// Clusters of `S` CTAs that fit on the GPU at once (asked once per size).
+int active_clusters(int S) {
+  static int cache[kMaxCluster + 1] = {};
+  if (!cache[S]) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(S * 64, 1, 1);
+    cfg.blockDim = dim3(kThreads, 1, 1);
+    cfg.dynamicSmemBytes = kSmemBytes;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = S;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, attn_tc_kernel, &cfg) != cudaSuccess || n < 1) {
+      cudaGetLastError();
+      n = std::max(1, kNumSMs / S);
+    }
+    cache[S] = n;
+  }
+  return cache[S];
+}
+
+// Number of chunks (= cluster size, at most 8) and their length: minimise
+// waves x (128-key tiles of the busiest CTA + a fixed per-CTA cost of about 3).
+void choose_split(int max_ctx, int n_clusters, int* S_out, int* chunk_out) {
+  *S_out = 1;
+  *chunk_out = EE_PAGE;
+  if (max_ctx <= 0) return;
+  const int min_splits = (max_ctx + kMaxCtaPages * EE_PAGE - 1) / (kMaxCtaPages * EE_PAGE);
+  long best = -1;
+  for (int s = std::max(1, min_splits); s <= kMaxCluster; ++s) {
+    // the last chunk also carries the tree tile: size chunks over ctx + one tile
+    int chunk = (max_ctx + kKT + s - 1) / s;
+    chunk = (chunk + EE_PAGE - 1) / EE_PAGE * EE_PAGE;
+    const int used = attn_splits_for(max_ctx, chunk);
+    const int last = max_ctx - (used - 1) * chunk;
+    const int tiles = std::max((chunk + kKT - 1) / kKT, (last + kKT - 1) / kKT + 1);
+    const long waves = (n_clusters + active_clusters(used) - 1) / active_clusters(used);
+    const long cost = waves * (tiles + 3);
+    if (best < 0 || cost < best) {
+      best = cost;
+      *S_out = used;
+      *chunk_out = chunk;
+    }
+  }
 }
 
 }  // namespace
@@ -530,8 +604,10 @@ extern "C" ee_status ee_tree_verify_attn(const ee_bf16* q, const ee_bf16* k_tree
   if (!aligned(q, 16) || !aligned(k_tree, 16) || !aligned(v_tree, 16) || !aligned(k_cache, 16) ||
       !aligned(v_cache, 16) || !aligned(out, 16) || !aligned(anc, 8) || !aligned(ws, 256))
     return EE_ERR_INVALID_ARG;
-  if (ws_bytes < kAttnOff + attn_partial_bytes(total_nodes, n_q, head_dim)) return EE_ERR_WORKSPACE;
+  if (ws_bytes < kWorkspaceBytes) return EE_ERR_WORKSPACE;
   if ((int64_t)num_pages * n_kv * EE_PAGE >= ((int64_t)1 << 31)) return EE_ERR_UNSUPPORTED;
+  // a CTA stages at most kMaxCtaPages page ids, and a cluster holds at most 8 chunks
+  if ((int64_t)max_ctx > (int64_t)kMaxCluster * kMaxCtaPages * EE_PAGE) return EE_ERR_UNSUPPORTED;
 
   static bool attr_set = false;
   if (!attr_set) {
@@ -551,25 +627,22 @@ extern "C" ee_status ee_tree_verify_attn(const ee_bf16* q, const ee_bf16* k_tree
   {
     const uint64_t dims[3] = {(uint64_t)head_dim, (uint64_t)n_kv, (uint64_t)total_nodes};
     const uint64_t strides[2] = {(uint64_t)head_dim * 2, (uint64_t)n_kv * head_dim * 2};
-    const uint32_t box[3] = {64, 1, 64};
+    const uint32_t box[3] = {64, 1, (uint32_t)kKT};
     if (!encode_bf16_tmap(&tmKt, k_tree, 3, dims, strides, box)) return EE_ERR_CUDA;
     if (!encode_bf16_tmap(&tmVt, v_tree, 3, dims, strides, box)) return EE_ERR_CUDA;
   }
   const int g = n_q / n_kv;
   const int nrb = (max_T * g + kRows - 1) / kRows;
-  const int chunk = choose_chunk(max_ctx, nrb * n_kv * B);
-  const int S = attn_splits_for(max_ctx, chunk);
+  int S = 1, chunk = EE_PAGE;
+  choose_split(max_ctx, nrb * n_kv * B, &S, &chunk);
 
-  char* wsb = static_cast<char*>(ws);
   AttnParams p;
   p.q = reinterpret_cast<const __nv_bfloat16*>(q);
   p.block_table = block_table;
   p.ctx_len = ctx_len;
   p.node_off = node_off;
   p.anc = anc;
-  p.part_o = reinterpret_cast<float*>(wsb + kAttnOff);
-  const size_t rows = (size_t)kMaxSplits * total_nodes * n_q;
-  p.part_ml = reinterpret_cast<float2*>(wsb + kAttnOff + align_up(rows * head_dim * 4, 256));
+  p.out = out;
   p.err = err_word(ws);
   p.num_pages = num_pages;
   p.max_pages = max_pages;
@@ -581,13 +654,21 @@ extern "C" ee_status ee_tree_verify_attn(const ee_bf16* q, const ee_bf16* k_tree
   p.max_T = max_T;
   p.nrb = nrb;
   p.chunk = chunk;
+  p.S = S;
   p.scale_log2 = scale * 1.4426950408889634f;
 
-  dim3 grid(nrb * S, n_kv, B);
-  attn_tc_kernel<<<grid, kThreads, kSmemBytes, (cudaStream_t)stream>>>(tmKc, tmVc, tmKt, tmVt, p);
-  EE_LAUNCH_OK();
-  attn_combine_kernel<<<dim3(max_T, (n_q + 7) / 8, B), 256, 0, (cudaStream_t)stream>>>(
-      p.part_o, p.part_ml, ctx_len, node_off, max_ctx, chunk, n_q, total_nodes, out);
-  EE_LAUNCH_OK();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(nrb * S, n_kv, B);
+  cfg.blockDim = dim3(kThreads, 1, 1);
+  cfg.dynamicSmemBytes = kSmemBytes;
+  cfg.stream = (cudaStream_t)stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = S;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  EE_CUDA_OK(cudaLaunchKernelEx(&cfg, attn_tc_kernel, tmKc, tmVc, tmKt, tmVt, p));
   return EE_OK;
 }

@@ -94,7 +94,7 @@ extern "C" ee_status ee_kv_compact(const ee_bf16* k_tree, const ee_bf16* v_tree,
   if (!ee::aligned(k_tree, 16) || !ee::aligned(v_tree, 16) || !ee::aligned(k_cache, 16) ||
       !ee::aligned(v_cache, 16) || tree_layer_stride % 8 || cache_layer_stride % 8)
     return EE_ERR_INVALID_ARG;
-  if (ws_bytes < ee::kAttnOff) return EE_ERR_WORKSPACE;
+  if (ws_bytes < ee::kWorkspaceBytes) return EE_ERR_WORKSPACE;
   if (L == 0) return EE_OK;
   if (tree_layer_stride % ((int64_t)n_kv * head_dim)) return EE_ERR_INVALID_ARG;
   const int total_nodes = (int)(tree_layer_stride / ((int64_t)n_kv * head_dim));

@@ -18,22 +18,15 @@ namespace ee {
 //   [0, 4)              device error word (EE_DEVERR_* bits)
 //   [16, 20)            LM-head "CTAs finished" ticket counter
 //   [256, 256+8*EE_MAX_LM_NODES)  LM-head packed running argmax per node
-//   [kAttnOff, ...)     attention split partials (O, then (m, l) pairs)
 // ---------------------------------------------------------------------------
 constexpr size_t kErrOff = 0;
 constexpr size_t kTicketOff = 16;
 constexpr size_t kArgmaxOff = 256;
-constexpr size_t kAttnOff = 256 + 8 * (size_t)EE_MAX_LM_NODES + 256;
-constexpr int kMaxSplits = 32;
+constexpr size_t kWorkspaceBytes = 256 + 8 * (size_t)EE_MAX_LM_NODES + 256;
 constexpr int kAttnRows = 128;        // query rows (node x head-in-group) per attention CTA
 constexpr int kNumSMs = 152;
 
 __host__ __device__ inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
-
-inline size_t attn_partial_bytes(int total_nodes, int n_q, int head_dim) {
-  size_t rows = (size_t)kMaxSplits * (size_t)total_nodes * (size_t)n_q;
-  return align_up(rows * (size_t)head_dim * 4, 256) + align_up(rows * 8, 256);
-}
 
 __device__ __forceinline__ void flag_error(int32_t* err, int bits) { atomicOr(err, bits); }
 
@@ -43,9 +36,8 @@ __host__ __device__ inline int32_t* err_word(void* ws) {
 
 inline bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 
-// Number of context chunks per sequence used by the split-KV attention; the
-// split kernel and the combine kernel both derive a sequence's split count
-// from ctx and this chunk length, so they always agree.
+// Number of context chunks a sequence of `ctx` cached positions uses in the
+// split-KV attention.
 __host__ __device__ inline int attn_splits_for(int ctx, int chunk) {
   int s = (ctx + chunk - 1) / chunk;
   return s < 1 ? 1 : s;

@@ -202,7 +202,8 @@ lmhead_accept_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_const
       const int vt = t / p.n_nt, nt = t % p.n_nt;
       const int acc = lt & 1;
       const uint32_t acc_phase = (lt >> 1) & 1;
-      if (!mbar_wait(tfull0 + 8 * acc, acc_phase, &s_abort)) break;
+      // warp-uniform outcome: the tcgen05.ld below is warp-collective
+      if (!__all_sync(0xffffffffu, mbar_wait(tfull0 + 8 * acc, acc_phase, &s_abort))) break;
       tc_fence_after();
       const int row = vt * BM + q * 32 + lane;
       const bool row_ok = row < p.vocab;
@@ -489,7 +490,7 @@ extern "C" ee_status ee_lmhead_accept(const ee_bf16* hidden, const ee_bf16* lm_w
                                      bonus, &empty);
   if (st != EE_OK || empty) return st;
   if (!ws || !ee::aligned(ws, 256)) return EE_ERR_INVALID_ARG;
-  if (ws_bytes < ee::kAttnOff) return EE_ERR_WORKSPACE;
+  if (ws_bytes < ee::kWorkspaceBytes) return EE_ERR_WORKSPACE;
   char* wsb = static_cast<char*>(ws);
   return launch_lmhead(hidden, lm_w, hidden_dim, vocab, draft_tok, parent, depth, anc, node_off, B,
                        total_nodes, max_T, argmax, accept_len, path, bonus, logits_or_null,

@@ -109,7 +109,7 @@ extern "C" ee_status ee_match_reuse(const int32_t* orig_tokens, const int64_t* o
   if (B == 0) return EE_OK;
   if (!orig_tokens || !orig_off || !tail || !cursor || !match_pos || !n_matches || !ws)
     return EE_ERR_INVALID_ARG;
-  if (ws_bytes < ee::kAttnOff) return EE_ERR_WORKSPACE;
+  if (ws_bytes < ee::kWorkspaceBytes) return EE_ERR_WORKSPACE;
   match_reuse_kernel<<<B, kThreads, 0, (cudaStream_t)stream>>>(
       orig_tokens, orig_off, tail, n, cursor, max_matches, match_pos, n_matches,
       ee::err_word(ws));

@@ -62,7 +62,7 @@ extern "C" ee_status ee_tree_prepare(const int32_t* parent, const int32_t* node_
   if (B == 0) return EE_OK;
   if (!parent || !node_off || !depth || !anc || !ws) return EE_ERR_INVALID_ARG;
   if (!ee::aligned(anc, 8)) return EE_ERR_INVALID_ARG;
-  if (ws_bytes < ee::kAttnOff) return EE_ERR_WORKSPACE;
+  if (ws_bytes < ee::kWorkspaceBytes) return EE_ERR_WORKSPACE;
   tree_prepare_kernel<<<B, EE_MAX_TREE, 0, (cudaStream_t)stream>>>(parent, node_off, depth, anc,
                                                                     total_nodes, ee::err_word(ws));
   EE_LAUNCH_OK();
