@@ -53,6 +53,22 @@ def parse_args():
     return ap.parse_args()
 
 
+def rank_seed(config, rank):
+    """Seed of the synthetic batch a rank verifies: every rank owns an independent
+    batch of sequences (the path partitions by sequence, so ranks never exchange
+    data; only the timing scalar is reduced)."""
+    return W.BASE_SEED + W.CONFIG_NAMES.index(config) + 1000 * rank
+
+
+def reduce_max(value, world, device=None):
+    """Max of a float over all ranks (identity when world == 1)."""
+    if world <= 1:
+        return float(value)
+    t = torch.tensor([float(value)], dtype=torch.float64, device=device)
+    torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    return float(t.item())
+
+
 def load_peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(p):
@@ -227,8 +243,7 @@ def run_ours(args, rank, world, local_rank):
     B.build_lib()
     dev = torch.device("cuda", local_rank)
     torch.cuda.set_device(dev)
-    seed = W.BASE_SEED + W.CONFIG_NAMES.index(args.config) + 1000 * rank
-    w = W.build(args.config, seed=seed, device=dev)
+    w = W.build(args.config, seed=rank_seed(args.config, rank), device=dev)
     alg = algorithmic(w)
     st = S.from_workload(w, device=dev, keep_layers=False)
     stream = torch.cuda.Stream(device=dev)
@@ -310,10 +325,7 @@ def run_ours(args, rank, world, local_rank):
     torch.cuda.synchronize(dev)
     ms_step = timed(plain, args.steps)
     torch.cuda.synchronize(dev)
-    if world > 1:
-        tt = torch.tensor([ms_step], device=dev, dtype=torch.float64)
-        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
-        ms_step = float(tt.item())
+    ms_step = reduce_max(ms_step, world, dev)
     ms_step_instr = timed(graphs, max(1, args.steps // 2), harvest) if phase_events else None
     torch.cuda.synchronize(dev)
     if world > 1:
@@ -439,11 +451,7 @@ def run_e2e(st, graph, stream, steps, dev, world):
     t0 = time.perf_counter()
     for _ in range(steps):
         one()
-    dt = time.perf_counter() - t0
-    if world > 1:
-        tt = torch.tensor([dt], device=dev, dtype=torch.float64)
-        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
-        dt = float(tt.item())
+    dt = reduce_max(time.perf_counter() - t0, world, dev)
     return {"value": round(world * steps / dt, 2), "unit": UNIT, "h2d_bytes_per_step": int(h2d),
             "d2h_bytes_per_step": int(d2h), "ms_per_step": round(1e3 * dt / steps, 4)}
 
