@@ -20,6 +20,8 @@ kv_compact_kernel(const uint4* __restrict__ k_tree, const uint4* __restrict__ v_
                   const int32_t* __restrict__ node_off, const int32_t* __restrict__ path,
                   const int32_t* __restrict__ accept_len, int max_T, int n_kv, int total_nodes,
                   int32_t* __restrict__ dst_slot, int32_t* err) {
+  ee::pdl_allow_next();
+  ee::pdl_wait();   // no global access before the previous kernel's writes are visible
   const int lane = threadIdx.x & 31;
   const int k = blockIdx.x * kWarpsPerBlock + (threadIdx.x >> 5);
   const int b = blockIdx.y;
@@ -99,11 +101,11 @@ extern "C" ee_status ee_kv_compact(const ee_bf16* k_tree, const ee_bf16* v_tree,
   if (tree_layer_stride % ((int64_t)n_kv * head_dim)) return EE_ERR_INVALID_ARG;
   const int total_nodes = (int)(tree_layer_stride / ((int64_t)n_kv * head_dim));
   dim3 grid((max_T + kWarpsPerBlock - 1) / kWarpsPerBlock, B, L);
-  kv_compact_kernel<<<grid, 32 * kWarpsPerBlock, 0, (cudaStream_t)stream>>>(
+  EE_CUDA_OK(ee::launch_pdl(
+      kv_compact_kernel, grid, dim3(32 * kWarpsPerBlock), 0, (cudaStream_t)stream, 1,
       reinterpret_cast<const uint4*>(k_tree), reinterpret_cast<const uint4*>(v_tree),
       tree_layer_stride, reinterpret_cast<uint4*>(k_cache), reinterpret_cast<uint4*>(v_cache),
       cache_layer_stride, num_pages, block_table, max_pages, ctx_len_in, ctx_len_out, node_off, path,
-      accept_len, max_T, n_kv, total_nodes, dst_slot, ee::err_word(ws));
-  EE_LAUNCH_OK();
+      accept_len, max_T, n_kv, total_nodes, dst_slot, ee::err_word(ws)));
   return EE_OK;
 }

@@ -84,6 +84,8 @@ lmhead_accept_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_const
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
+  ee::pdl_allow_next();
+  ee::pdl_wait();   // no global access before the previous kernel's writes are visible
   const int S = p.stages, BN = p.BN;
   const uint32_t bBytes = (uint32_t)BN * BK * 2;
   uint8_t* sA = smem;
@@ -419,7 +421,7 @@ ee_status launch_lmhead(const ee_bf16* hidden, const ee_bf16* lm_w, int32_t hidd
                         int32_t total_nodes, int32_t max_T, int32_t* argmax, int32_t* accept_len,
                         int32_t* path, int32_t* bonus, float* logits_or_null,
                         unsigned long long* keys, unsigned int* ticket, int32_t* err,
-                        ee_stream_t stream) {
+                        ee_stream_t stream, bool pdl) {
   LmParams p;
   p.vocab = vocab;
   p.hidden = hidden_dim;
@@ -470,8 +472,13 @@ ee_status launch_lmhead(const ee_bf16* hidden, const ee_bf16* lm_w, int32_t hidd
   int grid = (ee::kNumSMs / p.n_nt) * p.n_nt;   // multiple of n_nt: each CTA keeps one node tile
   if (grid > num_tiles) grid = num_tiles;
   if (grid < 1) grid = 1;
-  lmhead_accept_kernel<<<grid, kThreads, smem_acc, (cudaStream_t)stream>>>(tmW, tmX, p);
-  EE_LAUNCH_OK();
+  if (pdl) {
+    EE_CUDA_OK(ee::launch_pdl(lmhead_accept_kernel, dim3(grid), dim3(kThreads), smem_acc,
+                              (cudaStream_t)stream, 1, tmW, tmX, p));
+  } else {
+    lmhead_accept_kernel<<<grid, kThreads, smem_acc, (cudaStream_t)stream>>>(tmW, tmX, p);
+    EE_LAUNCH_OK();
+  }
   return EE_OK;
 }
 
@@ -496,7 +503,7 @@ extern "C" ee_status ee_lmhead_accept(const ee_bf16* hidden, const ee_bf16* lm_w
                        total_nodes, max_T, argmax, accept_len, path, bonus, logits_or_null,
                        reinterpret_cast<unsigned long long*>(wsb + ee::kArgmaxOff),
                        reinterpret_cast<unsigned int*>(wsb + ee::kTicketOff), ee::err_word(ws),
-                       stream);
+                       stream, true);
 }
 
 // ---------------------------------------------------------------------------
@@ -560,5 +567,5 @@ extern "C" ee_status ee_lmhead_accept_static(const ee_bf16* hidden, const ee_bf1
                        total_nodes, max_T, argmax, accept_len, path, bonus, logits_or_null,
                        reinterpret_cast<unsigned long long*>(base + ee::kArgmaxOff),
                        reinterpret_cast<unsigned int*>(base + ee::kTicketOff),
-                       reinterpret_cast<int32_t*>(base + ee::kErrOff), stream);
+                       reinterpret_cast<int32_t*>(base + ee::kErrOff), stream, false);
 }

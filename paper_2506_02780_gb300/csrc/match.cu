@@ -27,6 +27,8 @@ match_reuse_kernel(const int32_t* __restrict__ tok, const int64_t* __restrict__ 
   __shared__ int32_t s_wtot[kWarps];
   __shared__ int32_t s_wexcl[kWarps];
   __shared__ int32_t s_tile_total;
+  ee::pdl_allow_next();
+  ee::pdl_wait();   // no global access before the previous kernel's writes are visible
   const int b = blockIdx.x;
   const int tid = threadIdx.x;
   const int lane = tid & 31, warp = tid >> 5;
@@ -110,9 +112,8 @@ extern "C" ee_status ee_match_reuse(const int32_t* orig_tokens, const int64_t* o
   if (!orig_tokens || !orig_off || !tail || !cursor || !match_pos || !n_matches || !ws)
     return EE_ERR_INVALID_ARG;
   if (ws_bytes < ee::kWorkspaceBytes) return EE_ERR_WORKSPACE;
-  match_reuse_kernel<<<B, kThreads, 0, (cudaStream_t)stream>>>(
-      orig_tokens, orig_off, tail, n, cursor, max_matches, match_pos, n_matches,
-      ee::err_word(ws));
-  EE_LAUNCH_OK();
+  EE_CUDA_OK(ee::launch_pdl(match_reuse_kernel, dim3(B), dim3(kThreads), 0, (cudaStream_t)stream, 1,
+                             orig_tokens, orig_off, tail, n, cursor, max_matches, match_pos,
+                             n_matches, ee::err_word(ws)));
   return EE_OK;
 }

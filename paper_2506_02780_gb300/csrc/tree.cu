@@ -15,6 +15,8 @@ tree_prepare_kernel(const int32_t* __restrict__ parent, const int32_t* __restric
                     int32_t* __restrict__ depth, uint64_t* __restrict__ anc, int total_nodes,
                     int32_t* err) {
   __shared__ int32_t s_par[EE_MAX_TREE];
+  ee::pdl_allow_next();
+  ee::pdl_wait();   // no global access before the previous kernel's writes are visible
   const int b = blockIdx.x;
   const int i = threadIdx.x;
   const int o = node_off[b];
@@ -63,8 +65,7 @@ extern "C" ee_status ee_tree_prepare(const int32_t* parent, const int32_t* node_
   if (!parent || !node_off || !depth || !anc || !ws) return EE_ERR_INVALID_ARG;
   if (!ee::aligned(anc, 8)) return EE_ERR_INVALID_ARG;
   if (ws_bytes < ee::kWorkspaceBytes) return EE_ERR_WORKSPACE;
-  tree_prepare_kernel<<<B, EE_MAX_TREE, 0, (cudaStream_t)stream>>>(parent, node_off, depth, anc,
-                                                                    total_nodes, ee::err_word(ws));
-  EE_LAUNCH_OK();
+  EE_CUDA_OK(ee::launch_pdl(tree_prepare_kernel, dim3(B), dim3(EE_MAX_TREE), 0, (cudaStream_t)stream,
+                             1, parent, node_off, depth, anc, total_nodes, ee::err_word(ws)));
   return EE_OK;
 }

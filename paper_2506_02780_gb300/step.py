@@ -92,8 +92,8 @@ class VerifyStep:
         return g
 
     def launches_per_step(self) -> int:
-        """Kernels this step launches: match, prepare, 2 per attention layer, LM head, compaction."""
-        return 2 + 2 * self.L + 2
+        """Kernels this step launches: match, prepare, 1 per attention layer, LM head, compaction."""
+        return 2 + self.L + 2
 
 
 def from_workload(w, device="cuda", keep_layers=True):
