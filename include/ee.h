@@ -29,8 +29,11 @@
  *    [num_pages][n_kv][EE_PAGE][head_dim]; position t of sequence s lives in
  *    page block_table[s * max_pages + t / EE_PAGE], row t % EE_PAGE.
  *  - `ws` is a caller-owned device workspace of at least
- *    ee_workspace_size(...) bytes (a few KB: the error word and the LM head's
- *    running argmax), zeroed once with ee_workspace_init() before first use.  Its first word is the device error word: kernels never trap;
+ *    ee_workspace_size(...) bytes: a zeroed head of about 16.5 KB (the error
+ *    word and the LM head's running argmax), zeroed once with
+ *    ee_workspace_init() before first use, then the attention's per-CTA
+ *    partial results (65 KB per CTA, B x n_q x 8 CTAs at most, never zeroed).
+ *    Its first word is the device error word: kernels never trap;
  *    on a bad index found on the device they set an EE_DEVERR_* bit there,
  *    skip the access and continue.  ee_read_errors() reads (and clears) it.
  *    After any error the workspace must be re-initialised.  Calls that share
@@ -84,6 +87,9 @@ const char* ee_status_string(ee_status s);
  * Workspace bytes needed by every entry point for problems up to these sizes:
  * B sequences, total_nodes tree nodes in all, n_q query heads, max_ctx cached
  * positions in the longest sequence.  The buffer must be 256-byte aligned.
+ * 16,896 bytes when max_ctx is 0, else 16,896 + B * n_q * 8 * 66,560 (the
+ * attention's partial slots; about 15 MB for one sequence with 28 heads).
+ * Returns 0 for negative arguments.
  */
 size_t ee_workspace_size(int32_t B, int32_t total_nodes, int32_t n_q, int32_t head_dim,
                          int32_t max_ctx);
@@ -151,8 +157,10 @@ ee_status ee_tree_prepare(const int32_t* parent, const int32_t* node_off, int32_
  * accumulation in TMEM; P.V runs on bf16 tensor cores with P carried as two
  * bf16 parts (head + tail, about 2^-14 relative) and V as stored; softmax and
  * the output are fp32.  One launch per call: a thread-block cluster of up to
- * 8 CTAs per 128 query rows splits the context and merges its partial results
- * in distributed shared memory.
+ * 8 CTAs per 128 query rows splits the context; each CTA writes its partial
+ * result to its slot in `ws` (L2-resident) and, after one cluster barrier,
+ * each CTA merges a share of the rows.  EE_ERR_WORKSPACE when ws_bytes is
+ * below ee_workspace_size(B, total_nodes, n_q, head_dim, max_ctx).
  * Device errors: EE_DEVERR_PAGE (the key is skipped), EE_DEVERR_CTX,
  * EE_DEVERR_TIMEOUT (outputs undefined).
  */

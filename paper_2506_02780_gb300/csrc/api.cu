@@ -18,15 +18,16 @@ extern "C" const char* ee_status_string(ee_status s) {
 
 extern "C" size_t ee_workspace_size(int32_t B, int32_t total_nodes, int32_t n_q, int32_t head_dim,
                                     int32_t max_ctx) {
-  (void)B;
-  (void)max_ctx;
-  if (total_nodes < 0 || n_q < 0 || head_dim < 0) return 0;
-  return ee::kWorkspaceBytes;
+  if (B < 0 || total_nodes < 0 || n_q < 0 || head_dim < 0 || max_ctx < 0) return 0;
+  if (max_ctx == 0) return ee::kWorkspaceBytes;   // one chunk per row block: no partials
+  // attention CTAs of a split launch: B x n_kv x ceil(max_T * g / 128) row
+  // blocks (<= B x n_q, as max_T <= 128) x at most 16 chunks
+  return ee::kWorkspaceBytes + (size_t)B * n_q * ee::kAttnMaxSplits * ee::kAttnPartBytes;
 }
 
 extern "C" ee_status ee_workspace_init(void* ws, size_t ws_bytes, ee_stream_t stream) {
   if (!ws || ws_bytes < ee::kWorkspaceBytes || !ee::aligned(ws, 256)) return EE_ERR_INVALID_ARG;
-  EE_CUDA_OK(cudaMemsetAsync(ws, 0, ee::kWorkspaceBytes, (cudaStream_t)stream));
+  EE_CUDA_OK(cudaMemsetAsync(ws, 0, ws_bytes, (cudaStream_t)stream));
   return EE_OK;
 }
 

@@ -32,15 +32,27 @@
 //     mask, keep the running max/sum, write P, and rescale O in TMEM only when
 //     a row's max grows by more than 2^8 (the stale max keeps every P <= 256,
 //     and the final O / l is unchanged).
-//   - The S chunk-CTAs of one row block form a thread-block cluster.  Cluster
-//     rank k owns rows k, k+S, ...: after a first cluster barrier every CTA
-//     pushes each unnormalised O row and its (max, sum) straight into the owning
-//     CTA's shared memory (distributed shared memory, remote stores); after a
-//     second barrier each CTA merges its rows locally with log-sum-exp weights
-//     and writes the fp32 output.  No partial goes through HBM and no second
-//     launch is needed.  Every CTA of a cluster, also one whose chunk is
-//     empty for a short sequence, runs the same two cluster barriers; every
-//     mbarrier wait before them is bounded, so every thread reaches them.
+//   - Every chunk-CTA writes its unnormalised O rows and (max, sum) from TMEM
+//     to its own slot of the workspace (fp32, column-chunk major so that a
+//     warp's stores are contiguous; the slots stay in L2).  Once all S slots of
+//     a row block are written, chunk k merges the contiguous rows
+//     [k * ceil(128 / S), ...) of all S slots with log-sum-exp weights and
+//     writes the fp32 output: one launch, no second pass, and L2 moves the
+//     partials several times faster than distributed shared memory does.
+//     With S = 1 the CTA writes O / l directly.  The S CTAs of a row block
+//     learn that all slots are written in one of two ways, chosen by the host:
+//       cluster: they form a thread-block cluster and meet at one cluster
+//         barrier (release / acquire at cluster scope);
+//       cooperative: the launch is cooperative (every CTA resident at once),
+//         each CTA adds 1 to the row block's counter (release) and waits for
+//         it to reach S (acquire); the last CTA to finish merging returns the
+//         counters to zero.  No GPC packing constraint: S can be any value up
+//         to 16, so the grid can cover every SM.
+//     Every CTA, also one whose chunk is empty for a short sequence, arrives:
+//     every wait before the arrival is bounded.
+//   - The next kernel in the stream may launch (programmatic dependent launch)
+//     once every CTA has drained its pipeline; triggering earlier lets its
+//     CTAs hold SMs that a later wave of this grid still needs.
 // Shared-memory traffic per 128-key tile: K 64 KB + V 64 KB (TMA write, MMA read).
 #include "ee_common.cuh"
 #include "ee_ptx.cuh"
@@ -69,13 +81,15 @@ constexpr uint32_t kColO = 256;
 constexpr uint32_t kColQ = 384;
 constexpr float kRescaleLog2 = 8.0f;
 constexpr int kMaxCluster = 8;                   // portable thread-block cluster size
+constexpr int kMaxSplits = ee::kAttnMaxSplits;   // chunks per row block (cooperative launch)
 // warp roles (warp 3 is idle after set-up)
 constexpr int kWarpK = 0, kWarpMma = 1, kWarpV = 2, kWarpSoft0 = 4;
 
 static_assert(kRows == ee::kAttnRows, "row block size");
 static_assert(kThreads == 32 * (kWarpSoft0 + 4), "four softmax warps, one per TMEM lane quarter");
 static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
-static_assert(kRows * kD * 4 <= kKST * kKVBytes, "O staging fits in the idle K ring");
+static_assert(kMaxCtaPages % kThreads == 0, "page ids per thread");
+static_assert(ee::kAttnMlOff == kRows * kD * 4, "partial slot: O rows, then (m, l), then counters");
 
 struct AttnParams {
   const __nv_bfloat16* q;
@@ -84,8 +98,10 @@ struct AttnParams {
   const int32_t* node_off;
   const uint64_t* anc;
   float* out;
+  uint8_t* part;               // per-CTA partial slots (ee::kAttnPartBytes each), S > 1 only
   int32_t* err;
   int num_pages, max_pages, max_ctx, n_q, n_kv, g, total_nodes, max_T, nrb, chunk, S;
+  int coop;                    // 1: cooperative launch, counters; 0: cluster barrier
   float scale_log2;
 };
 
@@ -108,6 +124,67 @@ __device__ __forceinline__ unsigned tile_mask(const int32_t* s_pages, int t, int
   return m;
 }
 
+// Merge rows [r0, r0 + nown) of a row block (query rows row0, ...) from its S
+// partial slots with log-sum-exp weights (Sec. IV-A: the scores of one row
+// are normalised over all keys it sees) and write the fp32 output.  Thread t
+// takes row t % nown and the 16-byte column chunks t / nown + k * tpr, where
+// tpr = 256 / nown threads share a row: the loads of a warp for one chunk are
+// contiguous, and every load is issued before the first one is used.  Rows
+// without keys have (m, l) = (-inf, 0) and weight 0; their O words, never
+// written, are not used.
+template <int S>
+__device__ __forceinline__ void merge_rows(const AttnParams& p, const uint8_t* slot0, int row0, int r0,
+                                           int nown, int o, int hk) {
+  constexpr int kRpc = (kRows + S - 1) / S;
+  constexpr int kTprMin = kThreads / kRpc;
+  constexpr int kCh = (kD / 4 + kTprMin - 1) / kTprMin;   // chunks per thread, at most
+  const int tpr = kThreads / nown;                        // >= kTprMin, as nown <= kRpc
+  const int j = threadIdx.x % nown, cg = threadIdx.x / nown;
+  if (cg >= tpr) return;
+  float2 ml[S];
+#pragma unroll
+  for (int s = 0; s < S; ++s)
+    ml[s] = __ldcg(reinterpret_cast<const float2*>(slot0 + (size_t)s * kAttnPartBytes + kAttnMlOff) + r0 + j);
+  float4 v[kCh][S];
+#pragma unroll
+  for (int k = 0; k < kCh; ++k) {
+    const int c = cg + k * tpr;
+#pragma unroll
+    for (int s = 0; s < S; ++s)
+      v[k][s] = c < kD / 4 ? __ldcg(reinterpret_cast<const float4*>(slot0 + (size_t)s * kAttnPartBytes) +
+                                    (size_t)c * kRows + r0 + j)
+                           : make_float4(0.f, 0.f, 0.f, 0.f);
+  }
+  float M = -INFINITY;
+#pragma unroll
+  for (int s = 0; s < S; ++s) M = fmaxf(M, ml[s].x);
+  float w[S], L = 0.f;
+#pragma unroll
+  for (int s = 0; s < S; ++s) {
+    w[s] = ml[s].x == -INFINITY ? 0.f : ex2(ml[s].x - M);
+    L += w[s] * ml[s].y;
+  }
+  const float il = L > 0.f ? 1.f / L : 0.f;
+  const int rrow = row0 + j;
+  const int nd = rrow / p.g;
+  float4* dst = reinterpret_cast<float4*>(p.out + ((size_t)(o + nd) * p.n_q + hk * p.g + (rrow - nd * p.g)) * kD);
+#pragma unroll
+  for (int k = 0; k < kCh; ++k) {
+    const int c = cg + k * tpr;
+    if (c >= kD / 4) break;
+    float4 a = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+    for (int s = 0; s < S; ++s) {
+      if (w[s] == 0.f) continue;
+      a.x = fmaf(w[s], v[k][s].x, a.x);
+      a.y = fmaf(w[s], v[k][s].y, a.y);
+      a.z = fmaf(w[s], v[k][s].z, a.z);
+      a.w = fmaf(w[s], v[k][s].w, a.w);
+    }
+    dst[c] = make_float4(a.x * il, a.y * il, a.z * il, a.w * il);
+  }
+}
+
 __global__ void __launch_bounds__(kThreads, 1)
 attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__ CUtensorMap tmVc,
                const __grid_constant__ CUtensorMap tmKt, const __grid_constant__ CUtensorMap tmVt,
@@ -125,10 +202,22 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmKt)) : "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmVt)) : "memory");
   }
+  pdl_wait();   // no global access before the previous kernel's writes are visible
   const int b = blockIdx.z;
   const int hk = blockIdx.y;
   const int rb = blockIdx.x / p.S;                 // the cluster spans the S chunks of a row block
   const int split = blockIdx.x % p.S;              // == cluster rank
+  // this chunk's page ids, fetched now beside the sequence's node range and
+  // context length so that the two round trips overlap (validated below)
+  constexpr int kPgPerThread = kMaxCtaPages / kThreads;
+  const int pg_first = split * (p.chunk / EE_PAGE);
+  const int npg_cap = max(0, min(p.chunk / EE_PAGE, p.max_pages - pg_first));
+  int32_t pgr[kPgPerThread];
+#pragma unroll
+  for (int k = 0; k < kPgPerThread; ++k) {
+    const int i = threadIdx.x + k * kThreads;
+    pgr[k] = i < npg_cap ? __ldg(p.block_table + (size_t)b * p.max_pages + pg_first + i) : -1;
+  }
   const int o = p.node_off[b];
   const int T = p.node_off[b + 1] - o;
   const int R = T * p.g;
@@ -172,12 +261,17 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
   const uint32_t drain = o_done + 16, q_ready = drain + 8;
   int32_t* s_pages = reinterpret_cast<int32_t*>(smem + kOffPages);
   {
-    const int npg = (k_end - k_begin + EE_PAGE - 1) / EE_PAGE;   // <= kMaxCtaPages (host caps chunk)
-    for (int i = threadIdx.x; i < npg; i += kThreads) {
-      const int pg = p.block_table[(size_t)b * p.max_pages + (k_begin >> 4) + i];
-      const bool ok = pg >= 0 && pg < p.num_pages;
-      if (!ok) flag_error(p.err, EE_DEVERR_PAGE);
-      s_pages[i] = ok ? pg : -1;
+    // pages that hold keys of this chunk: <= npg_cap (k_end <= ctx <= max_pages * 16)
+    const int npg = (k_end - k_begin + EE_PAGE - 1) / EE_PAGE;
+#pragma unroll
+    for (int k = 0; k < kPgPerThread; ++k) {
+      const int i = threadIdx.x + k * kThreads;
+      if (i < npg) {
+        const int pg = pgr[k];
+        const bool ok = pg >= 0 && pg < p.num_pages;
+        if (!ok) flag_error(p.err, EE_DEVERR_PAGE);
+        s_pages[i] = ok ? pg : -1;
+      }
     }
   }
   if (threadIdx.x == 0) {
@@ -423,18 +517,58 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
       tc_fence_before();
       mbar_arrive(p_full + 8 * sb);
     }
-    // wait for the last P.V; the row is pushed to its owner after the first cluster barrier
+    // wait for the last P.V, then write this row out: O / l itself when the
+    // CTA is alone, else the partial (O, m, l) to this CTA's slot
     const bool fin =
         ok && n_tiles > 0 &&
         mbar_wait(o_done + 8 * ((n_tiles - 1) & 1), (uint32_t)(((n_tiles - 1) >> 1) & 1), &s_abort);
     have = __all_sync(0xffffffffu, fin);
     row_m = (have && vrow && m_used != -INFINITY) ? m_used * sl2 : -INFINITY;
     row_l = (have && vrow && m_used != -INFINITY) ? l : 0.f;
+    const bool alone = p.S == 1;
+    const size_t cta = ((size_t)blockIdx.z * gridDim.y + blockIdx.y) * gridDim.x + blockIdx.x;
+    float4* dst;
+    size_t dstride;                                   // float4 between column chunks
+    float inv = 1.f;
+    if (alone) {
+      const size_t orow = (size_t)(o + node) * p.n_q + hk * p.g + (rr - node * p.g);
+      dst = reinterpret_cast<float4*>(p.out + orow * kD);
+      dstride = 1;
+      inv = row_l > 0.f ? 1.f / row_l : 0.f;
+    } else {
+      dst = reinterpret_cast<float4*>(p.part + cta * kAttnPartBytes) + r;
+      dstride = kRows;
+    }
+    const bool store = alone ? vrow : row_l > 0.f;
+    // the TMEM read is warp-collective: the whole warp reads when any lane stores
+    if (__any_sync(0xffffffffu, store)) {
+      tc_fence_after();
+#pragma unroll 1
+      for (int c4 = 0; c4 < kD / 32; ++c4) {
+        uint32_t ov[32];
+        tc_ld32(tl + kColO + 32 * c4, ov);
+        if (store) {
+#pragma unroll
+          for (int e = 0; e < 8; ++e) {
+            const float4 v = make_float4(__uint_as_float(ov[4 * e]) * inv, __uint_as_float(ov[4 * e + 1]) * inv,
+                                         __uint_as_float(ov[4 * e + 2]) * inv,
+                                         __uint_as_float(ov[4 * e + 3]) * inv);
+            __stcg(dst + (size_t)(8 * c4 + e) * dstride, v);
+          }
+        }
+      }
+    }
+    if (!alone) {
+      __stcg(reinterpret_cast<float2*>(p.part + cta * kAttnPartBytes + kAttnMlOff) + r,
+             make_float2(row_m, row_l));
+      __threadfence();
+    }
   }
 
-  // ---- CTA teardown: drain on abort ---------------------------------------------
+  // ---- CTA teardown: drain on abort, free TMEM --------------------------------
   tc_fence_before();
   __syncthreads();
+  pdl_allow_next();   // this grid's pipeline is done: the next kernel may take SMs as they free
   const bool aborted = s_abort != 0;
   if (aborted && threadIdx.x == 0) {
     flag_error(p.err, EE_DEVERR_TIMEOUT);
@@ -444,89 +578,70 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
     for (int st = 0; st < kVST; ++st)
       if (s_vissued[st] >= 0) mbar_wait_plain(v_full + 8 * st, (uint32_t)(s_vissued[st] & 1));
   }
-  if (warp == kWarpMma && aborted && lane == 0) {
-    tc_commit(drain);
-    mbar_wait_plain(drain, 0);
-  }
-
-  // ---- cluster merge --------------------------------------------------------------
-  // every CTA of the cluster has finished its pipeline, so every K/V ring is free
-  cluster_sync();
-  const int rpc = (kRows + p.S - 1) / p.S;          // rows each rank owns
-  const uint32_t rbuf = sbase + kOffK;              // [sender][owned row][128 fp32], the K ring
-  const uint32_t rml = sbase + kOffV;               // [sender][owned row] (m, l), the V ring
-  if (warp >= kWarpSoft0) {
-    const int r = (warp & 3) * 32 + lane;
-    const int owner = r % p.S, j = r / p.S;
-    const uint32_t slot = (uint32_t)(split * rpc + j);
-    st_cluster_f2(map_cluster(rml + slot * 8, owner), row_m, row_l);
-    // the TMEM read is warp-collective: the whole warp reads when any lane has a
-    // row to push, and each lane stores only its own valid row
-    if (__any_sync(0xffffffffu, row_l > 0.f)) {
-      tc_fence_after();
-      const uint32_t tl = tmem + ((uint32_t)((warp & 3) * 32) << 16);
-      const uint32_t dst = map_cluster(rbuf + slot * (kD * 4), owner);
-#pragma unroll 1
-      for (int c4 = 0; c4 < kD / 32; ++c4) {
-        uint32_t ov[32];
-        tc_ld32(tl + kColO + 32 * c4, ov);
-        if (row_l > 0.f) {
-#pragma unroll
-          for (int e = 0; e < 8; ++e)
-            st_cluster_u4(dst + (32 * c4 + 4 * e) * 4, ov[4 * e], ov[4 * e + 1], ov[4 * e + 2],
-                          ov[4 * e + 3]);
-        }
-      }
-    }
-  }
-  tc_fence_before();
-  cluster_sync();   // all pushes have landed
   if (warp == kWarpMma) {
+    if (aborted && lane == 0) {
+      tc_commit(drain);
+      mbar_wait_plain(drain, 0);
+    }
+    __syncwarp();
     tc_fence_after();
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols)
                  : "memory");
   }
-  // local merge of the owned rows: one warp per row, lane = 16-byte chunk
-  for (int j = warp; j < rpc; j += kThreads / 32) {
-    const int rr0 = split + p.S * j;
-    const int rrow = rb * kRows + rr0;
-    if (rr0 >= kRows || rrow >= R) break;
-    float m = -INFINITY, lsum = 0.f;
-    if (lane < p.S) {
-      float2 ml;
-      asm volatile("ld.shared.v2.f32 {%0, %1}, [%2];"
-                   : "=f"(ml.x), "=f"(ml.y)
-                   : "r"(rml + (uint32_t)(lane * rpc + j) * 8));
-      m = ml.x;
-      lsum = ml.y;
+  if (p.S == 1) return;
+
+  // ---- merge ----------------------------------------------------------------------------
+  // once every slot of the row block is complete and visible, chunk `split`
+  // merges rows [r0, r0 + nown) of the row block
+  const size_t cta0 = ((size_t)blockIdx.z * gridDim.y + blockIdx.y) * gridDim.x + (size_t)rb * p.S;
+  const uint8_t* slot0 = p.part + cta0 * kAttnPartBytes;
+  uint32_t* cnt = reinterpret_cast<uint32_t*>(p.part + cta0 * kAttnPartBytes + kAttnCntOff);
+  __shared__ int s_ready;
+  if (p.coop) {
+    if (threadIdx.x == 0) {
+      red_add_release(cnt, 1u);     // this CTA's slot (ordered before by the fences and barrier)
+      const uint64_t t0 = globaltimer();
+      bool ready = true;
+      while (ld_acquire(cnt) < (uint32_t)p.S)
+        if (globaltimer() - t0 > kWaitLimitNs) {
+          ready = false;
+          break;
+        }
+      if (!ready) flag_error(p.err, EE_DEVERR_TIMEOUT);
+      s_ready = ready;
     }
-    float M = m;
-#pragma unroll
-    for (int d = 16; d >= 1; d >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, d));
-    const float w = (m == -INFINITY) ? 0.f : ex2(m - M);
-    float L = w * lsum;
-#pragma unroll
-    for (int d = 16; d >= 1; d >>= 1) L += __shfl_xor_sync(0xffffffffu, L, d);
-    float4 a = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll
-    for (int s2 = 0; s2 < kMaxCluster; ++s2) {
-      const float ws = __shfl_sync(0xffffffffu, w, s2);
-      if (s2 < p.S && ws != 0.f) {
-        float4 v;
-        asm volatile("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];"
-                     : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
-                     : "r"(rbuf + (uint32_t)((s2 * rpc + j) * kD + 4 * lane) * 4));
-        a.x += ws * v.x;
-        a.y += ws * v.y;
-        a.z += ws * v.z;
-        a.w += ws * v.w;
-      }
+    __syncthreads();
+  } else {
+    cluster_sync();
+    if (threadIdx.x == 0) s_ready = 1;
+    __syncthreads();
+  }
+  const int rpc = (kRows + p.S - 1) / p.S;
+  const int r0 = split * rpc;
+  const int nown = s_ready ? max(0, min(rpc, min(kRows, R - rb * kRows) - r0)) : 0;
+  if (nown > 0) {
+    const int row0 = rb * kRows + r0;
+    switch (p.S) {
+#define EE_MERGE_CASE(n) \
+  case n:                \
+    merge_rows<n>(p, slot0, row0, r0, nown, o, hk); \
+    break;
+      EE_MERGE_CASE(2) EE_MERGE_CASE(3) EE_MERGE_CASE(4) EE_MERGE_CASE(5) EE_MERGE_CASE(6)
+      EE_MERGE_CASE(7) EE_MERGE_CASE(8) EE_MERGE_CASE(9) EE_MERGE_CASE(10) EE_MERGE_CASE(11)
+      EE_MERGE_CASE(12) EE_MERGE_CASE(13) EE_MERGE_CASE(14) EE_MERGE_CASE(15) EE_MERGE_CASE(16)
+#undef EE_MERGE_CASE
+      default:
+        break;
     }
-    const float inv = L > 0.f ? 1.f / L : 0.f;
-    const int nd = rrow / p.g;
-    const size_t orow = (size_t)(o + nd) * p.n_q + hk * p.g + (rrow - nd * p.g);
-    reinterpret_cast<float4*>(p.out + orow * kD)[lane] =
-        make_float4(a.x * inv, a.y * inv, a.z * inv, a.w * inv);
+  }
+  if (p.coop) {
+    // every CTA of the row block has passed its wait once all have counted
+    // themselves here: the last returns both counters to zero
+    __syncthreads();
+    if (threadIdx.x == 0 && s_ready && atomicAdd(cnt + 1, 1u) == (uint32_t)p.S - 1) {
+      cnt[0] = 0u;
+      cnt[1] = 0u;
+    }
   }
 }
 
@@ -555,29 +670,79 @@ int active_clusters(int S) {
   return cache[S];
 }
 
-// Number of chunks (= cluster size, at most 8) and their length: minimise
-// waves x (128-key tiles of the busiest CTA + a fixed per-CTA cost of about 3).
-void choose_split(int max_ctx, int n_clusters, int* S_out, int* chunk_out) {
-  *S_out = 1;
-  *chunk_out = EE_PAGE;
-  if (max_ctx <= 0) return;
-  const int min_splits = (max_ctx + kMaxCtaPages * EE_PAGE - 1) / (kMaxCtaPages * EE_PAGE);
-  long best = -1;
-  for (int s = std::max(1, min_splits); s <= kMaxCluster; ++s) {
-    // the last chunk also carries the tree tile: size chunks over ctx + one tile
-    int chunk = (max_ctx + kKT + s - 1) / s;
-    chunk = (chunk + EE_PAGE - 1) / EE_PAGE * EE_PAGE;
-    const int used = attn_splits_for(max_ctx, chunk);
-    const int last = max_ctx - (used - 1) * chunk;
-    const int tiles = std::max((chunk + kKT - 1) / kKT, (last + kKT - 1) / kKT + 1);
-    const long waves = (n_clusters + active_clusters(used) - 1) / active_clusters(used);
-    const long cost = waves * (tiles + 3);
-    if (best < 0 || cost < best) {
-      best = cost;
-      *S_out = used;
-      *chunk_out = chunk;
+// CTAs of this kernel the GPU holds at once (asked once; -1 if unknown).
+int resident_ctas() {
+  static int cap = 0;
+  if (!cap) {
+    int dev = 0, sms = 0, per = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
+        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per, attn_tc_kernel, kThreads, kSmemBytes) !=
+            cudaSuccess ||
+        per < 1) {
+      cudaGetLastError();
+      cap = -1;
+    } else {
+      cap = sms * per;
     }
   }
+  return cap;
+}
+
+// Chunk length for s chunks (the last one also carries the tree tile), the
+// chunks actually used and the 128-key tiles of the busiest CTA.
+void chunk_for(int max_ctx, int s, int* chunk, int* used, int* tiles) {
+  int c = (max_ctx + kKT + s - 1) / s;
+  c = (c + EE_PAGE - 1) / EE_PAGE * EE_PAGE;
+  c = std::min(c, kMaxCtaPages * EE_PAGE);          // a CTA stages at most kMaxCtaPages page ids
+  *chunk = c;
+  *used = attn_splits_for(max_ctx, c);
+  const int last = max_ctx - (*used - 1) * c;
+  *tiles = std::max((c + kKT - 1) / kKT, (last + kKT - 1) / kKT + 1);
+}
+
+struct Split {
+  int S = 1, chunk = EE_PAGE;
+  bool coop = false;
+};
+
+// Number of chunks per row block, their length and the synchronisation mode.
+// Cost = waves x (tiles of the busiest CTA + a fixed per-CTA cost of about 3):
+//   cluster mode: S <= 8, waves from the clusters the GPU holds at once;
+//   cooperative mode: one wave by construction, S up to 16 with n_rb x S
+//   CTAs no more than the GPU holds.  Ties go to the cooperative mode.
+Split choose_split(int max_ctx, int n_rb) {
+  Split best;
+  if (max_ctx <= 0) return best;
+  const int min_splits = (max_ctx + kMaxCtaPages * EE_PAGE - 1) / (kMaxCtaPages * EE_PAGE);
+  long best_cost = -1;
+  for (int s = std::max(1, min_splits); s <= kMaxCluster; ++s) {
+    int chunk, used, tiles;
+    chunk_for(max_ctx, s, &chunk, &used, &tiles);
+    const long waves = (n_rb + active_clusters(used) - 1) / active_clusters(used);
+    const long cost = waves * (tiles + 3);
+    if (best_cost < 0 || cost < best_cost) {
+      best_cost = cost;
+      best.S = used;
+      best.chunk = chunk;
+    }
+  }
+  const int cap = resident_ctas();
+  if (cap > 0) {
+    for (int s = std::max(2, min_splits); s <= kMaxSplits && (long)s * n_rb <= cap; ++s) {
+      int chunk, used, tiles;
+      chunk_for(max_ctx, s, &chunk, &used, &tiles);
+      if (used < 2) continue;
+      const long cost = tiles + 3;
+      if (cost <= best_cost) {
+        best_cost = cost;
+        best.S = used;
+        best.chunk = chunk;
+        best.coop = true;
+      }
+    }
+  }
+  return best;
 }
 
 }  // namespace
@@ -633,8 +798,11 @@ extern "C" ee_status ee_tree_verify_attn(const ee_bf16* q, const ee_bf16* k_tree
   }
   const int g = n_q / n_kv;
   const int nrb = (max_T * g + kRows - 1) / kRows;
-  int S = 1, chunk = EE_PAGE;
-  choose_split(max_ctx, nrb * n_kv * B, &S, &chunk);
+  const Split sp = choose_split(max_ctx, nrb * n_kv * B);
+  const int S = sp.S, chunk = sp.chunk;
+  // a split launch writes one partial slot per CTA after the zeroed part
+  if (S > 1 && ws_bytes < kWorkspaceBytes + (size_t)nrb * S * n_kv * B * kAttnPartBytes)
+    return EE_ERR_WORKSPACE;
 
   AttnParams p;
   p.q = reinterpret_cast<const __nv_bfloat16*>(q);
@@ -643,6 +811,7 @@ extern "C" ee_status ee_tree_verify_attn(const ee_bf16* q, const ee_bf16* k_tree
   p.node_off = node_off;
   p.anc = anc;
   p.out = out;
+  p.part = static_cast<uint8_t*>(ws) + kWorkspaceBytes;
   p.err = err_word(ws);
   p.num_pages = num_pages;
   p.max_pages = max_pages;
@@ -655,20 +824,30 @@ extern "C" ee_status ee_tree_verify_attn(const ee_bf16* q, const ee_bf16* k_tree
   p.nrb = nrb;
   p.chunk = chunk;
   p.S = S;
+  p.coop = (S > 1 && sp.coop) ? 1 : 0;
   p.scale_log2 = scale * 1.4426950408889634f;
 
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(nrb * S, n_kv, B);
-  cfg.blockDim = dim3(kThreads, 1, 1);
+  cfg.blockDim = dim3(kThreads);
   cfg.dynamicSmemBytes = kSmemBytes;
   cfg.stream = (cudaStream_t)stream;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = S;
-  attr[0].val.clusterDim.y = 1;
-  attr[0].val.clusterDim.z = 1;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
+  if (p.coop) {
+    attr[1].id = cudaLaunchAttributeCooperative;
+    attr[1].val.cooperative = 1;
+    cfg.numAttrs = 2;
+  } else if (S > 1) {
+    attr[1].id = cudaLaunchAttributeClusterDimension;
+    attr[1].val.clusterDim.x = S;
+    attr[1].val.clusterDim.y = 1;
+    attr[1].val.clusterDim.z = 1;
+    cfg.numAttrs = 2;
+  }
   EE_CUDA_OK(cudaLaunchKernelEx(&cfg, attn_tc_kernel, tmKc, tmVc, tmKt, tmVt, p));
   return EE_OK;
 }

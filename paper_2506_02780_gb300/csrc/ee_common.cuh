@@ -19,12 +19,22 @@ namespace ee {
 //   [0, 4)              device error word (EE_DEVERR_* bits)
 //   [16, 20)            LM-head "CTAs finished" ticket counter
 //   [256, 256+8*EE_MAX_LM_NODES)  LM-head packed running argmax per node
+//   [kWorkspaceBytes, ...)        attention partial slots, kAttnPartBytes per
+//                                 CTA of a split launch; the trailer of a row
+//                                 block's first slot holds its arrival counters
 // ---------------------------------------------------------------------------
 constexpr size_t kErrOff = 0;
 constexpr size_t kTicketOff = 16;
 constexpr size_t kArgmaxOff = 256;
-constexpr size_t kWorkspaceBytes = 256 + 8 * (size_t)EE_MAX_LM_NODES + 256;
+constexpr size_t kWorkspaceBytes = 256 + 8 * (size_t)EE_MAX_LM_NODES + 256;   // the zeroed part
 constexpr int kAttnRows = 128;        // query rows (node x head-in-group) per attention CTA
+constexpr int kAttnMaxSplits = 16;    // context chunks per row block
+// one CTA's partial: 128 rows x 128 fp32 of O (column-chunk major), then
+// 128 x (m, l), then a 256-byte trailer (two uint32 counters, zeroed by
+// ee_workspace_init and returned to zero by every launch that uses them)
+constexpr size_t kAttnMlOff = (size_t)kAttnRows * 128 * 4;
+constexpr size_t kAttnCntOff = kAttnMlOff + (size_t)kAttnRows * 8;
+constexpr size_t kAttnPartBytes = kAttnCntOff + 256;
 constexpr int kNumSMs = 152;
 
 __host__ __device__ inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }

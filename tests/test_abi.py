@@ -49,14 +49,22 @@ def test_version_and_status_strings(L):
     assert L.ee_status_string(5) == b"workspace too small"
 
 
-def test_workspace_size_is_small_and_fixed(L):
-    """The workspace holds the error word, the LM head's ticket and its running
-    argmax words (8 bytes per node, up to EE_MAX_LM_NODES); attention keeps its
-    split partials in on-chip memory, so the size does not grow with the problem."""
-    a = L.ee_workspace_size(1, 64, 28, 128, 4096)
-    b = L.ee_workspace_size(8, 2048, 56, 128, 262144)
-    assert a == b
-    assert a % 256 == 0 and 8 * 2048 < a <= 32 * 1024
+def test_workspace_size(L):
+    """A zeroed head (error word, LM-head ticket, running argmax words: 8 bytes
+    per node up to EE_MAX_LM_NODES) plus, when the context is split, one
+    attention partial slot per CTA: 128 rows x 128 fp32 + 128 x (m, l) + a
+    256-byte counter trailer, for at most B x n_q row blocks x 16 chunks.
+    Independent of the node count."""
+    head = L.ee_workspace_size(1, 64, 28, 128, 0)
+    assert head == L.ee_workspace_size(8, 2048, 56, 128, 0)
+    assert head % 256 == 0 and 8 * 2048 < head <= 32 * 1024
+    slot = 128 * 128 * 4 + 128 * 8 + 256
+    assert slot % 256 == 0
+    for B, n_q, ctx in ((1, 28, 4096), (8, 56, 262144), (3, 8, 16)):
+        assert L.ee_workspace_size(B, 64, n_q, 128, ctx) == head + B * n_q * 16 * slot
+        assert L.ee_workspace_size(B, 2048, n_q, 128, ctx) == head + B * n_q * 16 * slot
+    assert L.ee_workspace_size(-1, 64, 28, 128, 16) == 0
+    assert L.ee_workspace_size(1, 64, 28, 128, -1) == 0
 
 
 FAKE = ctypes.c_void_p(0x10000)   # never dereferenced: every call below fails validation first

@@ -143,6 +143,26 @@ def test_device_error_word():
     U.check_accept(w, st)
 
 
+def test_attention_rejects_small_workspace():
+    """A split launch needs one partial slot per CTA: a workspace sized for an
+    empty context is refused before anything is launched."""
+    E = _E()
+    from paper_2506_02780_gb300 import step as S
+    w = W.build("tiny", seed=4, device="cuda")
+    st = S.from_workload(w)
+    small = E.new_workspace(w.B, w.total_nodes, w.n_q, 0)
+    assert small.numel() < st.ws.numel()
+    x = st.inp
+    out = torch.full_like(st.attn_out[0], 7.0)
+    with pytest.raises(E.EEError) as ei:
+        E.ee_tree_verify_attn(x["q"][0], x["k_tree"][0], x["v_tree"][0], x["k_cache"][0],
+                              x["v_cache"][0], x["block_table"], x["ctx_len"], st.max_ctx,
+                              x["node_off"], st.anc, st.max_T, st.scale, out, small)
+    assert ei.value.status == 5
+    torch.cuda.synchronize()
+    assert bool((out == 7.0).all())
+
+
 # ----------------------------------------------------------------------------
 # full-size configurations (sampled attention outputs, launch configuration as timed)
 # ----------------------------------------------------------------------------
