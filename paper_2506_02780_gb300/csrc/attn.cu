@@ -196,62 +196,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
   __shared__ volatile int s_abort;
   __shared__ int s_kissued[kKST], s_vissued[kVST];
 
-  if (threadIdx.x == 0) {
-    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmKc)) : "memory");
-    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmVc)) : "memory");
-    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmKt)) : "memory");
-    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmVt)) : "memory");
-  }
-  pdl_wait();   // no global access before the previous kernel's writes are visible
-  const int b = blockIdx.z;
-  const int hk = blockIdx.y;
-  const int rb = blockIdx.x / p.S;                 // the cluster spans the S chunks of a row block
-  const int split = blockIdx.x % p.S;              // == cluster rank
-  // this chunk's page ids, fetched now beside the sequence's node range and
-  // context length so that the two round trips overlap (validated below)
-  constexpr int kPgPerThread = kMaxCtaPages / kThreads;
-  const int pg_first = split * (p.chunk / EE_PAGE);
-  const int npg_cap = max(0, min(p.chunk / EE_PAGE, p.max_pages - pg_first));
-  int32_t pgr[kPgPerThread];
-#pragma unroll
-  for (int k = 0; k < kPgPerThread; ++k) {
-    const int i = threadIdx.x + k * kThreads;
-    pgr[k] = i < npg_cap ? __ldg(p.block_table + (size_t)b * p.max_pages + pg_first + i) : -1;
-  }
-  const int o = p.node_off[b];
-  const int T = p.node_off[b + 1] - o;
-  const int R = T * p.g;
-  if (T < 1 || T > EE_MAX_TREE || T > p.max_T || o < 0 || o + T > p.total_nodes) {
-    if (threadIdx.x == 0 && blockIdx.x == 0 && hk == 0) flag_error(p.err, EE_DEVERR_TREE);
-    return;
-  }
-  if (rb * kRows >= R) return;
-  int ctx = p.ctx_len[b];
-  if (ctx < 0 || ctx > p.max_ctx) {
-    if (threadIdx.x == 0 && blockIdx.x == 0 && hk == 0) flag_error(p.err, EE_DEVERR_CTX);
-    ctx = ctx < 0 ? 0 : p.max_ctx;
-  }
-  // everything above is uniform over the cluster (same sequence, head and row
-  // block); from here on every CTA runs to the cluster barriers
-  const int S = attn_splits_for(ctx, p.chunk);     // chunks this sequence uses, <= p.S
-  const bool active = split < S;
-  const int k_begin = split * p.chunk;
-  const int k_end = active ? min(ctx, k_begin + p.chunk) : k_begin;
-  const int n_ctx_tiles = k_end > k_begin ? (k_end - k_begin + kKT - 1) / kKT : 0;
-  const int n_tiles = active ? n_ctx_tiles + ((split == S - 1) ? 1 : 0) : 0;   // + the tree tile
-
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  // softmax threads fetch their Q row now; it goes to TMEM once TMEM is allocated
-  uint4 qreg[16];
-  {
-    const int rr = rb * kRows + (warp & 3) * 32 + lane;
-    const bool mine = warp >= kWarpSoft0 && rr < R;
-    const int nd = mine ? rr / p.g : 0;
-    const uint4* src = reinterpret_cast<const uint4*>(
-        p.q + ((size_t)(o + nd) * p.n_q + hk * p.g + (mine ? rr - nd * p.g : 0)) * kD);
-#pragma unroll
-    for (int c = 0; c < 16; ++c) qreg[c] = mine ? __ldg(src + c) : make_uint4(0u, 0u, 0u, 0u);
-  }
   const uint32_t sbase = smem_u32(smem);
   const uint32_t sK = sbase + kOffK, sV = sbase + kOffV;
   const uint32_t bar0 = sbase + kOffBar;
@@ -259,22 +204,14 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
   const uint32_t v_full = k_empty + 8 * kKST, v_empty = v_full + 8 * kVST;
   const uint32_t s_full = v_empty + 8 * kVST, p_full = s_full + 16, o_done = p_full + 16;
   const uint32_t drain = o_done + 16, q_ready = drain + 8;
-  int32_t* s_pages = reinterpret_cast<int32_t*>(smem + kOffPages);
-  {
-    // pages that hold keys of this chunk: <= npg_cap (k_end <= ctx <= max_pages * 16)
-    const int npg = (k_end - k_begin + EE_PAGE - 1) / EE_PAGE;
-#pragma unroll
-    for (int k = 0; k < kPgPerThread; ++k) {
-      const int i = threadIdx.x + k * kThreads;
-      if (i < npg) {
-        const int pg = pgr[k];
-        const bool ok = pg >= 0 && pg < p.num_pages;
-        if (!ok) flag_error(p.err, EE_DEVERR_PAGE);
-        s_pages[i] = ok ? pg : -1;
-      }
-    }
-  }
+
+  // on-chip set-up first: it touches no global memory, so it overlaps the end
+  // of the previous kernel in the stream
   if (threadIdx.x == 0) {
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmKc)) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmVc)) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmKt)) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmVt)) : "memory");
     s_abort = 0;
     for (int i = 0; i < kKST; ++i) {
       mbar_init(k_full + 8 * i, 1);
@@ -303,6 +240,84 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
                  : "memory");
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
   }
+
+  pdl_wait();   // no global access before the previous kernel's writes are visible
+  const int b = blockIdx.z;
+  const int hk = blockIdx.y;
+  const int rb = blockIdx.x / p.S;                 // the S chunks of a row block are consecutive
+  const int split = blockIdx.x % p.S;              // == cluster rank in the cluster mode
+  // this chunk's page ids, issued now beside the sequence's node range and
+  // context length so that the round trips overlap (validated below)
+  constexpr int kPgPerThread = kMaxCtaPages / kThreads;
+  const int pg_first = split * (p.chunk / EE_PAGE);
+  const int npg_cap = max(0, min(p.chunk / EE_PAGE, p.max_pages - pg_first));
+  int32_t pgr[kPgPerThread];
+#pragma unroll
+  for (int k = 0; k < kPgPerThread; ++k) {
+    const int i = threadIdx.x + k * kThreads;
+    pgr[k] = i < npg_cap ? ld_nc_pinned(p.block_table + (size_t)b * p.max_pages + pg_first + i) : -1;
+  }
+  const int o = p.node_off[b];
+  const int T = p.node_off[b + 1] - o;
+  int ctx = p.ctx_len[b];
+  const int R = T * p.g;
+  const bool bad_tree = T < 1 || T > EE_MAX_TREE || T > p.max_T || o < 0 || o + T > p.total_nodes;
+  if (bad_tree && threadIdx.x == 0 && blockIdx.x == 0 && hk == 0) flag_error(p.err, EE_DEVERR_TREE);
+  if (bad_tree || rb * kRows >= R) {                // uniform over the CTA (and the row block)
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == kWarpMma)
+      asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(s_tmem),
+                   "r"(kTmemCols)
+                   : "memory");
+    return;
+  }
+  if (ctx < 0 || ctx > p.max_ctx) {
+    if (threadIdx.x == 0 && blockIdx.x == 0 && hk == 0) flag_error(p.err, EE_DEVERR_CTX);
+    ctx = ctx < 0 ? 0 : p.max_ctx;
+  }
+  // everything above is uniform over the row block's CTAs; from here on every
+  // CTA reaches the merge synchronisation
+  const int S = attn_splits_for(ctx, p.chunk);     // chunks this sequence uses, <= p.S
+  const bool active = split < S;
+  const int k_begin = split * p.chunk;
+  const int k_end = active ? min(ctx, k_begin + p.chunk) : k_begin;
+  const int n_ctx_tiles = k_end > k_begin ? (k_end - k_begin + kKT - 1) / kKT : 0;
+  const int n_tiles = active ? n_ctx_tiles + ((split == S - 1) ? 1 : 0) : 0;   // + the tree tile
+
+  // softmax threads issue the coalesced loads of the block's Q rows now (a
+  // half-warp reads one 256-byte row; rows past R read row R - 1 and are
+  // zeroed later) so that they leave before the K/V stream starts; the values
+  // are consumed after the barrier below
+  const int qhalf = lane >> 4, qc = lane & 15;
+  uint4 qv[kRows / 8];
+  if (warp >= kWarpSoft0) {
+#pragma unroll
+    for (int k = 0; k < kRows / 8; ++k) {
+      const int rq = 2 * ((warp - kWarpSoft0) + 4 * k) + qhalf;   // 0..127
+      const int rrq = min(rb * kRows + rq, R - 1);
+      const int nq = rrq / p.g;
+      qv[k] = __ldg(reinterpret_cast<const uint4*>(
+                        p.q + ((size_t)(o + nq) * p.n_q + hk * p.g + (rrq - nq * p.g)) * kD) +
+                    qc);
+    }
+  }
+  int32_t* s_pages = reinterpret_cast<int32_t*>(smem + kOffPages);
+  {
+    // pages that hold keys of this chunk: <= npg_cap (k_end <= ctx <= max_pages * 16)
+    const int npg = (k_end - k_begin + EE_PAGE - 1) / EE_PAGE;
+#pragma unroll
+    for (int k = 0; k < kPgPerThread; ++k) {
+      const int i = threadIdx.x + k * kThreads;
+      if (i < npg) {
+        const int pg = pgr[k];
+        const bool ok = pg >= 0 && pg < p.num_pages;
+        if (!ok) flag_error(p.err, EE_DEVERR_PAGE);
+        s_pages[i] = ok ? pg : -1;
+      }
+    }
+  }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -325,6 +340,8 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
       const int st = t % nst, use = t / nst;
       bool go = true;
       if (lane == 0) go = mbar_wait(empty0 + 8 * st, (uint32_t)(use & 1) ^ 1u, &s_abort);
+      // the last V stage holds the staged Q rows until they are in TMEM
+      if (!isK && st == kVST - 1 && use == 0 && lane == 0) go = go && mbar_wait(q_ready, 0, &s_abort);
       if (!__shfl_sync(0xffffffffu, go, 0)) break;
       const uint32_t full = full0 + 8 * st;
       const uint32_t dst = ring + st * kKVBytes;
@@ -398,8 +415,24 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
     const uint64_t a0 = vrow ? p.anc[2 * (size_t)(o + node)] : 0ull;
     const uint64_t a1 = vrow ? p.anc[2 * (size_t)(o + node) + 1] : 0ull;
     const uint32_t tl = tmem + ((uint32_t)((warp & 3) * 32) << 16);
-    // this row of Q into TMEM columns kColQ.. (bf16 pairs), zeros for rows past R
+    // this row of Q into TMEM columns kColQ.. (bf16 pairs), zeros for rows past
+    // R.  The block's rows, loaded before the barrier, go through the last V
+    // stage (which the V producer fills only after q_ready): chunk c of row r
+    // sits at 16 * (c ^ (r & 15)), so that each thread then reads its own row
+    // without bank conflicts.
     {
+      uint8_t* qs = smem + kOffV + (kVST - 1) * kKVBytes;
+#pragma unroll
+      for (int k = 0; k < kRows / 8; ++k) {
+        const int rq = 2 * ((warp - kWarpSoft0) + 4 * k) + qhalf;
+        *reinterpret_cast<uint4*>(qs + rq * 256 + 16 * (qc ^ (rq & 15))) =
+            rb * kRows + rq < R ? qv[k] : make_uint4(0u, 0u, 0u, 0u);
+      }
+      asm volatile("bar.sync 1, 128;" ::: "memory");   // the four softmax warps
+      uint4 qreg[16];
+#pragma unroll
+      for (int c2 = 0; c2 < 16; ++c2)
+        qreg[c2] = *reinterpret_cast<const uint4*>(qs + r * 256 + 16 * (c2 ^ (r & 15)));
 #pragma unroll
       for (int h = 0; h < 2; ++h) {
         uint32_t qw[32];

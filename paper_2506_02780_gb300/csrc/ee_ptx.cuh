@@ -173,6 +173,13 @@ __device__ __forceinline__ void cluster_sync() {
       "barrier.cluster.arrive.release.aligned;\n"
       "barrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
+// Read-only global load that the compiler issues where it is written (volatile:
+// not sunk past branches), so that independent round trips overlap.
+__device__ __forceinline__ int32_t ld_nc_pinned(const int32_t* a) {
+  int32_t v;
+  asm volatile("ld.global.nc.s32 %0, [%1];" : "=r"(v) : "l"(a));
+  return v;
+}
 // gpu-scope release add / acquire load on a global counter
 __device__ __forceinline__ void red_add_release(uint32_t* a, uint32_t v) {
   asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(a), "r"(v) : "memory");
