@@ -385,7 +385,9 @@ def run_ours(args, rank, world, local_rank):
         "config": dict(W.describe(w), workload=args.config + ": " + _config_text(args.config),
                        l2="inputs larger than L2 (%.2f GB touched per step)" %
                           ((alg["lm_bytes"] + w.layers * alg["attn_bytes"]) / 1e9),
-                       parallelism=f"replicas x{world}"),
+                       parallelism=f"replicas x{world}",
+                       attention_launch=E.ee_attn_plan(w.B, w.max_T, w.n_q, w.n_kv,
+                                                       int(w.ctx_len.max()))),
         "draft_tokens_per_s": round(steps_per_s * alg["draft_nodes"], 1),
         "roofline": roofline, "roofline_kernels": rl, "kernels": kernels,
         "e2e": e2e, "gpu_launches": st.launches_per_step() * args.steps, "clocks": clk,

@@ -173,6 +173,18 @@ ee_status ee_tree_verify_attn(const ee_bf16* q, const ee_bf16* k_tree, const ee_
                               void* ws, size_t ws_bytes, ee_stream_t stream);
 
 /*
+ * ee_attn_plan -- the launch plan ee_tree_verify_attn uses for these sizes
+ * (introspection only; the paper has no counterpart).  *splits = context
+ * chunks per 128 query rows (1..16), *chunk = keys per chunk, *mode = 0
+ * (one chunk, no merge), 1 (chunks of a row block form a thread-block
+ * cluster) or 2 (cooperative launch, merge counters in the workspace),
+ * *ctas = CTAs launched.  Needs the device (occupancy queries): EE_ERR_CUDA
+ * without one; EE_ERR_INVALID_ARG for sizes ee_tree_verify_attn rejects.
+ */
+ee_status ee_attn_plan(int32_t B, int32_t max_T, int32_t n_q, int32_t n_kv, int32_t max_ctx,
+                       int32_t* splits, int32_t* chunk, int32_t* mode, int32_t* ctas);
+
+/*
  * ee_lmhead_accept -- LM head fused with greedy decode and acceptance
  * (Eq. (piecewise)).  logits[i][v] = hidden[i] . lm_w[v] (fp32 accumulate of
  * bf16 products, never stored unless logits_or_null is given);

@@ -29,7 +29,7 @@ DEVERR = {0x01: "MATCH_ARGS", 0x02: "TREE", 0x04: "PAGE", 0x08: "CTX", 0x10: "FP
           0x20: "TIMEOUT", 0x40: "PATH"}
 
 EXPORTS = ("ee_version", "ee_status_string", "ee_workspace_size", "ee_workspace_init",
-           "ee_read_errors", "ee_match_reuse", "ee_tree_prepare", "ee_tree_verify_attn",
+           "ee_read_errors", "ee_match_reuse", "ee_tree_prepare", "ee_tree_verify_attn", "ee_attn_plan",
            "ee_lmhead_accept", "ee_lmhead_accept_static", "ee_kv_compact")
 
 
@@ -60,6 +60,8 @@ _SIGS = {
     "ee_tree_prepare": ([_P, _P, _I, _I, _P, _P, _P, _SZ, _P], _I),
     "ee_tree_verify_attn": ([_P, _P, _P, _P, _P, _I, _P, _I, _P, _I, _P, _P, _I, _I, _I, _I, _I, _I,
                              _F, _P, _P, _SZ, _P], _I),
+    "ee_attn_plan": ([_I, _I, _I, _I, _I, ctypes.POINTER(_I), ctypes.POINTER(_I), ctypes.POINTER(_I),
+                      ctypes.POINTER(_I)], _I),
     "ee_lmhead_accept": ([_P, _P, _I, _I, _P, _P, _P, _P, _P, _I, _I, _I, _P, _P, _P, _P, _P, _P, _SZ,
                           _P], _I),
     "ee_lmhead_accept_static": ([_P, _P, _I, _I, _P, _P, _P, _P, _P, _I, _I, _I, _P, _P, _P, _P, _P,
@@ -173,6 +175,15 @@ def ee_tree_verify_attn(q, k_tree, v_tree, k_cache, v_cache, block_table, ctx_le
                                    _p(anc), B, total, max_T, n_q, n_kv, d, float(scale), _p(out),
                                    _p(ws), ws.numel(), _stream(stream))
     _ok("ee_tree_verify_attn", st)
+
+
+def ee_attn_plan(B, max_T, n_q, n_kv, max_ctx) -> dict:
+    """The launch plan ee_tree_verify_attn uses for these sizes."""
+    v = [_I(0) for _ in range(4)]
+    st = lib().ee_attn_plan(B, max_T, n_q, n_kv, max_ctx, *[ctypes.byref(x) for x in v])
+    _ok("ee_attn_plan", st)
+    return {"splits": v[0].value, "chunk": v[1].value,
+            "mode": ("single", "cluster", "cooperative")[v[2].value], "ctas": v[3].value}
 
 
 def ee_lmhead_accept(hidden, lm_w, draft_tok, parent, depth, anc, node_off, max_T, argmax, accept_len,

@@ -61,7 +61,7 @@ namespace {
 
 using namespace ee;
 
-constexpr int kThreads = 256;                    // 8 warps, roles below
+constexpr int kThreads = 384;                    // 12 warps, roles below
 constexpr int kRows = 128;                       // query rows per CTA (MMA M)
 constexpr int kKT = 128;                         // keys per tile (MMA N of Q K^T, K of P V)
 constexpr int kD = EE_HEAD_DIM;                  // 128
@@ -82,13 +82,14 @@ constexpr uint32_t kColQ = 384;
 constexpr float kRescaleLog2 = 8.0f;
 constexpr int kMaxCluster = 8;                   // portable thread-block cluster size
 constexpr int kMaxSplits = ee::kAttnMaxSplits;   // chunks per row block (cooperative launch)
-// warp roles (warp 3 is idle after set-up)
+// warp roles (warp 3 is idle after set-up); softmax warps 4..11, two per TMEM
+// lane quarter
 constexpr int kWarpK = 0, kWarpMma = 1, kWarpV = 2, kWarpSoft0 = 4;
+constexpr int kSoftThreads = 8 * 32;
 
 static_assert(kRows == ee::kAttnRows, "row block size");
-static_assert(kThreads == 32 * (kWarpSoft0 + 4), "four softmax warps, one per TMEM lane quarter");
+static_assert(kThreads == 32 * kWarpSoft0 + kSoftThreads, "eight softmax warps, two per TMEM lane quarter");
 static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
-static_assert(kMaxCtaPages % kThreads == 0, "page ids per thread");
 static_assert(ee::kAttnMlOff == kRows * kD * 4, "partial slot: O rows, then (m, l), then counters");
 
 struct AttnParams {
@@ -195,6 +196,8 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
   __shared__ uint32_t s_tmem;
   __shared__ volatile int s_abort;
   __shared__ int s_kissued[kKST], s_vissued[kVST];
+  __shared__ float s_xmax[2][2][kRows];             // [tile parity][half][row]: softmax pair exchange
+  __shared__ float s_xl[2][kRows];                  // [half][row]: final row sums
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t sbase = smem_u32(smem);
@@ -225,11 +228,11 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(s_full + 8 * i, 1);
-      mbar_init(p_full + 8 * i, kRows);
+      mbar_init(p_full + 8 * i, 2 * kRows);
       mbar_init(o_done + 8 * i, 1);
     }
     mbar_init(drain, 1);
-    mbar_init(q_ready, kRows);
+    mbar_init(q_ready, 2 * kRows);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     fence_async_smem();
   }
@@ -248,7 +251,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
   const int split = blockIdx.x % p.S;              // == cluster rank in the cluster mode
   // this chunk's page ids, issued now beside the sequence's node range and
   // context length so that the round trips overlap (validated below)
-  constexpr int kPgPerThread = kMaxCtaPages / kThreads;
+  constexpr int kPgPerThread = (kMaxCtaPages + kThreads - 1) / kThreads;
   const int pg_first = split * (p.chunk / EE_PAGE);
   const int npg_cap = max(0, min(p.chunk / EE_PAGE, p.max_pages - pg_first));
   int32_t pgr[kPgPerThread];
@@ -291,11 +294,11 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
   // zeroed later) so that they leave before the K/V stream starts; the values
   // are consumed after the barrier below
   const int qhalf = lane >> 4, qc = lane & 15;
-  uint4 qv[kRows / 8];
+  uint4 qv[kRows / 16];
   if (warp >= kWarpSoft0) {
 #pragma unroll
-    for (int k = 0; k < kRows / 8; ++k) {
-      const int rq = 2 * ((warp - kWarpSoft0) + 4 * k) + qhalf;   // 0..127
+    for (int k = 0; k < kRows / 16; ++k) {
+      const int rq = 2 * ((warp - kWarpSoft0) + 8 * k) + qhalf;   // 0..127
       const int rrq = min(rb * kRows + rq, R - 1);
       const int nq = rrq / p.g;
       qv[k] = __ldg(reinterpret_cast<const uint4*>(
@@ -407,116 +410,127 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
       }
     }
   } else if (warp >= kWarpSoft0) {
-    // ---------------- softmax: one query row per thread ----------------
-    const int r = (warp & 3) * 32 + lane;             // == TMEM lane of this warp's quarter
+    // ---------------- softmax: one query row and half of every tile per thread ----------------
+    // Warps w and w + 4 share TMEM lane quarter w & 3 (32 query rows); half hf
+    // of the pair takes keys [64 hf, 64 hf + 64) of every tile and O columns
+    // [64 hf, 64 hf + 64).  The pair agrees on each tile's row maximum through
+    // shared memory at a 64-thread named barrier, so both halves take the same
+    // rescale decisions; each keeps the sum over its own keys, and the two sums
+    // are added (half 0 first) at the end.  Two warps per sub-partition hide
+    // each other's latencies.  Every exit from the tile loop happens right
+    // after the pair barrier and on a decision both warps share.
+    const int qd = warp & 3;
+    const int hf = (warp - kWarpSoft0) >> 2;
+    const uint32_t pair_bar = 2 + qd;
+    const int r = qd * 32 + lane;                     // == TMEM lane of this quarter
     const int rr = rb * kRows + r;
     const bool vrow = rr < R;
     const int node = vrow ? rr / p.g : 0;
-    const uint64_t a0 = vrow ? p.anc[2 * (size_t)(o + node)] : 0ull;
-    const uint64_t a1 = vrow ? p.anc[2 * (size_t)(o + node) + 1] : 0ull;
-    const uint32_t tl = tmem + ((uint32_t)((warp & 3) * 32) << 16);
-    // this row of Q into TMEM columns kColQ.. (bf16 pairs), zeros for rows past
-    // R.  The block's rows, loaded before the barrier, go through the last V
-    // stage (which the V producer fills only after q_ready): chunk c of row r
-    // sits at 16 * (c ^ (r & 15)), so that each thread then reads its own row
-    // without bank conflicts.
+    const uint64_t ancw = vrow ? p.anc[2 * (size_t)(o + node) + hf] : 0ull;   // this half's tree keys
+    const uint32_t tl = tmem + ((uint32_t)(qd * 32) << 16);
+    // this row of Q into TMEM columns kColQ + 32 hf.. (bf16 pairs of this half's
+    // 64 dims), zeros for rows past R.  The block's rows, loaded before the
+    // barrier, go through the last V stage (which the V producer fills only
+    // after q_ready): chunk c of row r sits at 16 * (c ^ (r & 15)), so that each
+    // thread then reads its own row without bank conflicts.
     {
       uint8_t* qs = smem + kOffV + (kVST - 1) * kKVBytes;
 #pragma unroll
-      for (int k = 0; k < kRows / 8; ++k) {
-        const int rq = 2 * ((warp - kWarpSoft0) + 4 * k) + qhalf;
+      for (int k = 0; k < kRows / 16; ++k) {
+        const int rq = 2 * ((warp - kWarpSoft0) + 8 * k) + qhalf;
         *reinterpret_cast<uint4*>(qs + rq * 256 + 16 * (qc ^ (rq & 15))) =
             rb * kRows + rq < R ? qv[k] : make_uint4(0u, 0u, 0u, 0u);
       }
-      asm volatile("bar.sync 1, 128;" ::: "memory");   // the four softmax warps
-      uint4 qreg[16];
+      asm volatile("bar.sync 1, %0;" ::"n"(kSoftThreads) : "memory");   // the eight softmax warps
+      uint32_t qw[32];
 #pragma unroll
-      for (int c2 = 0; c2 < 16; ++c2)
-        qreg[c2] = *reinterpret_cast<const uint4*>(qs + r * 256 + 16 * (c2 ^ (r & 15)));
-#pragma unroll
-      for (int h = 0; h < 2; ++h) {
-        uint32_t qw[32];
-#pragma unroll
-        for (int c = 0; c < 8; ++c) {
-          const uint4 v = qreg[h * 8 + c];
-          qw[4 * c] = v.x;
-          qw[4 * c + 1] = v.y;
-          qw[4 * c + 2] = v.z;
-          qw[4 * c + 3] = v.w;
-        }
-        tc_st32(tl + kColQ + 32 * h, qw);
+      for (int c = 0; c < 8; ++c) {
+        const int ch = 8 * hf + c;
+        const uint4 v = *reinterpret_cast<const uint4*>(qs + r * 256 + 16 * (ch ^ (r & 15)));
+        qw[4 * c] = v.x;
+        qw[4 * c + 1] = v.y;
+        qw[4 * c + 2] = v.z;
+        qw[4 * c + 3] = v.w;
       }
+      tc_st32(tl + kColQ + 32 * hf, qw);
       tc_fence_before();
       mbar_arrive(q_ready);
     }
     // m_used is kept in raw score units (scale > 0, so the max commutes with it)
     float m_used = -INFINITY, l = 0.f;
     const float sl2 = p.scale_log2;
+    const float kFail = __int_as_float(0x7fffffff);   // NaN: "this half's wait failed"
     bool ok = true;
     for (int t = 0; t < n_tiles; ++t) {
       const int sb = t & 1;
-      // every wait outcome is made warp-uniform: the TMEM accesses that follow are
-      // warp-collective (.sync.aligned) and must be reached by all 32 lanes or none
-      if (!__all_sync(0xffffffffu, mbar_wait(s_full + 8 * sb, (uint32_t)((t >> 1) & 1), &s_abort))) {
+      // wait outcomes are warp-uniform: the TMEM accesses that follow are
+      // warp-collective (.sync.aligned)
+      const bool got =
+          __all_sync(0xffffffffu, mbar_wait(s_full + 8 * sb, (uint32_t)((t >> 1) & 1), &s_abort));
+      uint32_t sr[64];
+      float tmax = -INFINITY;
+      if (got) {
+        tc_fence_after();
+        tc_ld32(tl + sb * kKT + 64 * hf, *reinterpret_cast<uint32_t(*)[32]>(&sr[0]));
+        tc_ld32(tl + sb * kKT + 64 * hf + 32, *reinterpret_cast<uint32_t(*)[32]>(&sr[32]));
+        // visibility of this half's 64 keys as one 64-bit word
+        uint64_t kw;
+        if (t < n_ctx_tiles) {
+          const unsigned m = tile_mask(s_pages, t, k_begin, k_end);
+          const int nv = min(max(k_end - (k_begin + t * kKT) - 64 * hf, 0), 64);
+          uint64_t pgw = 0ull;
+#pragma unroll
+          for (int i = 0; i < 4; ++i) pgw |= ((m >> (4 * hf + i)) & 1u) ? (0xFFFFull << (16 * i)) : 0ull;
+          kw = pgw & (nv >= 64 ? ~0ull : ((1ull << nv) - 1ull));
+        } else {
+          const int th = min(max(T - 64 * hf, 0), 64);
+          kw = ancw & (th >= 64 ? ~0ull : ((1ull << th) - 1ull));
+        }
+        if (!vrow) kw = 0ull;
+        if (!__all_sync(0xffffffffu, kw == ~0ull)) {
+#pragma unroll
+          for (int c = 0; c < 64; ++c)
+            if (!((kw >> c) & 1ull)) sr[c] = __float_as_uint(-INFINITY);
+        }
+        float mx[8];
+#pragma unroll
+        for (int c = 0; c < 8; ++c) mx[c] = __uint_as_float(sr[c]);
+#pragma unroll
+        for (int c = 8; c < 64; ++c) mx[c & 7] = fmaxf(mx[c & 7], __uint_as_float(sr[c]));
+        tmax = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
+                     fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
+      }
+      // the pair swaps its halves' maxima; both S halves are in registers before
+      // either warp overwrites S with P
+      s_xmax[sb][hf][r] = got ? tmax : kFail;
+      tc_fence_before();
+      asm volatile("bar.sync %0, 64;" ::"r"(pair_bar) : "memory");
+      tc_fence_after();
+      const float other = s_xmax[sb][hf ^ 1][r];
+      if (!__all_sync(0xffffffffu, got && other == other)) {
         ok = false;
         break;
       }
-      tc_fence_after();
-      uint32_t sr[kKT];
-#pragma unroll
-      for (int q4 = 0; q4 < kKT / 32; ++q4)
-        tc_ld32(tl + sb * kKT + 32 * q4, *reinterpret_cast<uint32_t(*)[32]>(&sr[32 * q4]));
-      // visibility of the tile's 128 keys, as two 64-bit words
-      uint64_t keep0, keep1;
-      if (t < n_ctx_tiles) {
-        const unsigned m = tile_mask(s_pages, t, k_begin, k_end);
-        const int nvalid = min(kKT, k_end - (k_begin + t * kKT));
-        uint64_t pg0 = 0ull, pg1 = 0ull;
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          pg0 |= ((m >> i) & 1u) ? (0xFFFFull << (16 * i)) : 0ull;
-          pg1 |= ((m >> (i + 4)) & 1u) ? (0xFFFFull << (16 * i)) : 0ull;
-        }
-        keep0 = pg0 & (nvalid >= 64 ? ~0ull : ((1ull << nvalid) - 1ull));
-        keep1 = pg1 & (nvalid >= 128 ? ~0ull : (nvalid <= 64 ? 0ull : ((1ull << (nvalid - 64)) - 1ull)));
-      } else {
-        keep0 = a0 & (T >= 64 ? ~0ull : ((1ull << T) - 1ull));
-        keep1 = a1 & (T >= 128 ? ~0ull : (T <= 64 ? 0ull : ((1ull << (T - 64)) - 1ull)));
-      }
-      if (!vrow) keep0 = keep1 = 0ull;
-      const bool full = __all_sync(0xffffffffu, (keep0 & keep1) == ~0ull);
-      if (!full) {
-#pragma unroll
-        for (int c = 0; c < kKT; ++c) {
-          const uint64_t kw = c < 64 ? keep0 : keep1;
-          if (!((kw >> (c & 63)) & 1ull)) sr[c] = __float_as_uint(-INFINITY);
-        }
-      }
-      float mx[8];
-#pragma unroll
-      for (int c = 0; c < 8; ++c) mx[c] = __uint_as_float(sr[c]);
-#pragma unroll
-      for (int c = 8; c < kKT; ++c) mx[c & 7] = fmaxf(mx[c & 7], __uint_as_float(sr[c]));
-      const float tmax = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
-                               fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
+      tmax = fmaxf(tmax, other);
       const float m_new = fmaxf(m_used, tmax);
       const bool need = (m_new - m_used) * sl2 > kRescaleLog2;   // true when m_used = -inf < m_new
       if (t >= 1 && __any_sync(0xffffffffu, need)) {
-        // O must hold P.V(t-1) before it is rescaled
-        if (!__all_sync(0xffffffffu,
-                        mbar_wait(o_done + 8 * (sb ^ 1), (uint32_t)(((t - 1) >> 1) & 1), &s_abort))) {
-          ok = false;
-          break;
-        }
-        tc_fence_after();
-        const float f = need ? ex2((m_used - m_new) * sl2) : 1.f;
+        // O must hold P.V(t-1) before this half's columns are rescaled; a failed
+        // wait sets the abort flag, and the pair stops at the next barrier
+        if (__all_sync(0xffffffffu,
+                       mbar_wait(o_done + 8 * (sb ^ 1), (uint32_t)(((t - 1) >> 1) & 1), &s_abort))) {
+          tc_fence_after();
+          const float f = need ? ex2((m_used - m_new) * sl2) : 1.f;
 #pragma unroll 1
-        for (int c4 = 0; c4 < kD / 32; ++c4) {
-          uint32_t ov[32];
-          tc_ld32(tl + kColO + 32 * c4, ov);
+          for (int c4 = 0; c4 < 2; ++c4) {
+            uint32_t ov[32];
+            tc_ld32(tl + kColO + 64 * hf + 32 * c4, ov);
 #pragma unroll
-          for (int e = 0; e < 32; ++e) ov[e] = __float_as_uint(__uint_as_float(ov[e]) * f);
-          tc_st32(tl + kColO + 32 * c4, ov);
+            for (int e = 0; e < 32; ++e) ov[e] = __float_as_uint(__uint_as_float(ov[e]) * f);
+            tc_st32(tl + kColO + 64 * hf + 32 * c4, ov);
+          }
+        } else {
+          ok = false;
         }
       }
       if (need) {
@@ -524,40 +538,42 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
         m_used = m_new;
       }
       const float nms = m_used == -INFINITY ? 0.f : -m_used * sl2;
-      // p = 2^(s*scale_log2 - m); P = head + tail, both bf16 (top 16 bits),
-      // head pairs over columns 0..63 of this S buffer, tail pairs over 64..127
+      // p = 2^(s*scale_log2 - m); P = head + tail, both bf16 (top 16 bits): this
+      // half's head pairs go to columns 32 hf.. of the S buffer, its tail pairs
+      // to 64 + 32 hf..
       float ls[8];
+      uint32_t hw[32], tw[32];
 #pragma unroll
-      for (int h = 0; h < 2; ++h) {
-        uint32_t hw[32], tw[32];
-#pragma unroll
-        for (int e = 0; e < 32; ++e) {
-          const int c = h * 64 + 2 * e;
-          const float p0 = ex2(fmaf(__uint_as_float(sr[c]), sl2, nms));
-          const float p1 = ex2(fmaf(__uint_as_float(sr[c + 1]), sl2, nms));
-          if (h == 0 && e < 8) ls[e] = p0 + p1; else ls[e & 7] += p0 + p1;
-          const uint32_t h0 = __float_as_uint(p0) & 0xFFFF0000u;
-          const uint32_t h1 = __float_as_uint(p1) & 0xFFFF0000u;
-          const uint32_t t0 = __float_as_uint(p0 - __uint_as_float(h0));
-          const uint32_t t1 = __float_as_uint(p1 - __uint_as_float(h1));
-          hw[e] = __byte_perm(h0, h1, 0x7632);
-          tw[e] = __byte_perm(t0, t1, 0x7632);
-        }
-        tc_st32(tl + sb * kKT + 32 * h, hw);
-        tc_st32(tl + sb * kKT + 64 + 32 * h, tw);
+      for (int e = 0; e < 32; ++e) {
+        const float p0 = ex2(fmaf(__uint_as_float(sr[2 * e]), sl2, nms));
+        const float p1 = ex2(fmaf(__uint_as_float(sr[2 * e + 1]), sl2, nms));
+        if (e < 8) ls[e] = p0 + p1; else ls[e & 7] += p0 + p1;
+        const uint32_t h0 = __float_as_uint(p0) & 0xFFFF0000u;
+        const uint32_t h1 = __float_as_uint(p1) & 0xFFFF0000u;
+        const uint32_t t0 = __float_as_uint(p0 - __uint_as_float(h0));
+        const uint32_t t1 = __float_as_uint(p1 - __uint_as_float(h1));
+        hw[e] = __byte_perm(h0, h1, 0x7632);
+        tw[e] = __byte_perm(t0, t1, 0x7632);
       }
+      tc_st32(tl + sb * kKT + 32 * hf, hw);
+      tc_st32(tl + sb * kKT + 64 + 32 * hf, tw);
       l += ((ls[0] + ls[1]) + (ls[2] + ls[3])) + ((ls[4] + ls[5]) + (ls[6] + ls[7]));
       tc_fence_before();
       mbar_arrive(p_full + 8 * sb);
     }
-    // wait for the last P.V, then write this row out: O / l itself when the
-    // CTA is alone, else the partial (O, m, l) to this CTA's slot
+    // wait for the last P.V; the pair adds its two sums, then each half writes
+    // its 64 columns out: O / l itself when the CTA is alone, else the partial
+    // (O, m, l) to this CTA's slot
     const bool fin =
         ok && n_tiles > 0 &&
         mbar_wait(o_done + 8 * ((n_tiles - 1) & 1), (uint32_t)(((n_tiles - 1) >> 1) & 1), &s_abort);
     have = __all_sync(0xffffffffu, fin);
-    row_m = (have && vrow && m_used != -INFINITY) ? m_used * sl2 : -INFINITY;
-    row_l = (have && vrow && m_used != -INFINITY) ? l : 0.f;
+    s_xl[hf][r] = have ? l : kFail;
+    asm volatile("bar.sync %0, 64;" ::"r"(pair_bar) : "memory");
+    const float l_sum = s_xl[0][r] + s_xl[1][r];     // NaN when either half failed
+    const bool both = have && l_sum == l_sum;
+    row_m = (both && vrow && m_used != -INFINITY) ? m_used * sl2 : -INFINITY;
+    row_l = (both && vrow && m_used != -INFINITY) ? l_sum : 0.f;
     const bool alone = p.S == 1;
     const size_t cta = ((size_t)blockIdx.z * gridDim.y + blockIdx.y) * gridDim.x + blockIdx.x;
     float4* dst;
@@ -577,23 +593,24 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
     if (__any_sync(0xffffffffu, store)) {
       tc_fence_after();
 #pragma unroll 1
-      for (int c4 = 0; c4 < kD / 32; ++c4) {
+      for (int c4 = 0; c4 < 2; ++c4) {
         uint32_t ov[32];
-        tc_ld32(tl + kColO + 32 * c4, ov);
+        tc_ld32(tl + kColO + 64 * hf + 32 * c4, ov);
         if (store) {
 #pragma unroll
           for (int e = 0; e < 8; ++e) {
             const float4 v = make_float4(__uint_as_float(ov[4 * e]) * inv, __uint_as_float(ov[4 * e + 1]) * inv,
                                          __uint_as_float(ov[4 * e + 2]) * inv,
                                          __uint_as_float(ov[4 * e + 3]) * inv);
-            __stcg(dst + (size_t)(8 * c4 + e) * dstride, v);
+            __stcg(dst + (size_t)(16 * hf + 8 * c4 + e) * dstride, v);
           }
         }
       }
     }
     if (!alone) {
-      __stcg(reinterpret_cast<float2*>(p.part + cta * kAttnPartBytes + kAttnMlOff) + r,
-             make_float2(row_m, row_l));
+      if (hf == 0)
+        __stcg(reinterpret_cast<float2*>(p.part + cta * kAttnPartBytes + kAttnMlOff) + r,
+               make_float2(row_m, row_l));
       __threadfence();
     }
   }
@@ -633,10 +650,10 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
   if (p.coop) {
     if (threadIdx.x == 0) {
       red_add_release(cnt, 1u);     // this CTA's slot (ordered before by the fences and barrier)
-      const uint64_t t0 = globaltimer();
+      const long long t0 = cycles();
       bool ready = true;
       while (ld_acquire(cnt) < (uint32_t)p.S)
-        if (globaltimer() - t0 > kWaitLimitNs) {
+        if (cycles() - t0 > kWaitLimitCycles) {
           ready = false;
           break;
         }
@@ -741,7 +758,8 @@ struct Split {
 
 // Number of chunks per row block, their length and the synchronisation mode.
 // Cost = waves x (tiles of the busiest CTA + a fixed per-CTA cost of about 3):
-//   cluster mode: S <= 8, waves from the clusters the GPU holds at once;
+//   cluster mode: S <= 8, waves from the clusters the GPU holds at once (one
+//   slot fewer per wave once a second wave is needed);
 //   cooperative mode: one wave by construction, S up to 16 with n_rb x S
 //   CTAs no more than the GPU holds.  Ties go to the cooperative mode.
 Split choose_split(int max_ctx, int n_rb) {
@@ -752,7 +770,12 @@ Split choose_split(int max_ctx, int n_rb) {
   for (int s = std::max(1, min_splits); s <= kMaxCluster; ++s) {
     int chunk, used, tiles;
     chunk_for(max_ctx, s, &chunk, &used, &tiles);
-    const long waves = (n_rb + active_clusters(used) - 1) / active_clusters(used);
+    // from the second wave on, clusters start as earlier ones finish, and free
+    // SMs scattered over the GPCs can leave a slot unusable: plan such launches
+    // with one cluster slot fewer
+    const long act = active_clusters(used);
+    long waves = (n_rb + act - 1) / act;
+    if (waves >= 2 && act > 1) waves = (n_rb + act - 2) / (act - 1);
     const long cost = waves * (tiles + 3);
     if (best_cost < 0 || cost < best_cost) {
       best_cost = cost;
@@ -779,6 +802,27 @@ Split choose_split(int max_ctx, int n_rb) {
 }
 
 }  // namespace
+
+extern "C" ee_status ee_attn_plan(int32_t B, int32_t max_T, int32_t n_q, int32_t n_kv,
+                                  int32_t max_ctx, int32_t* splits, int32_t* chunk, int32_t* mode,
+                                  int32_t* ctas) {
+  if (B < 1 || max_T < 1 || max_T > EE_MAX_TREE || n_q < 1 || n_kv < 1 || n_q % n_kv != 0 ||
+      max_ctx < 0 || !splits || !chunk || !mode || !ctas)
+    return EE_ERR_INVALID_ARG;
+  static bool attr_set = false;
+  if (!attr_set) {
+    EE_CUDA_OK(cudaFuncSetAttribute(attn_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    (int)kSmemBytes));
+    attr_set = true;
+  }
+  const int nrb = (max_T * (n_q / n_kv) + kRows - 1) / kRows;
+  const Split sp = choose_split(max_ctx, nrb * n_kv * B);
+  *splits = sp.S;
+  *chunk = sp.chunk;
+  *mode = sp.S == 1 ? 0 : (sp.coop ? 2 : 1);
+  *ctas = nrb * sp.S * n_kv * B;
+  return EE_OK;
+}
 
 extern "C" ee_status ee_tree_verify_attn(const ee_bf16* q, const ee_bf16* k_tree,
                                          const ee_bf16* v_tree, const ee_bf16* k_cache,

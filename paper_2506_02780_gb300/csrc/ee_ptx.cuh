@@ -7,16 +7,16 @@
 
 namespace ee {
 
-constexpr uint64_t kWaitLimitNs = 1000000000ull;   // every device wait gives up after 1 s
+// Every device wait gives up after 2e9 SM clock cycles (about 1 s at the
+// 2.07 GHz boost clock, at most a few seconds at any lower clock).  The bound
+// is counted with the SM's own cycle counter, which is cheap to read inside a
+// spin loop.
+constexpr long long kWaitLimitCycles = 2000000000ll;
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }
-__device__ __forceinline__ uint64_t globaltimer() {
-  uint64_t t;
-  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
-  return t;
-}
+__device__ __forceinline__ long long cycles() { return clock64(); }
 __device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
   asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
 }
@@ -51,12 +51,12 @@ __device__ __forceinline__ bool mbar_test(uint32_t bar, uint32_t parity) {
 // Bounded wait: false when the CTA was told to abort or the time limit passed.
 __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag) {
   if (mbar_try(bar, parity)) return true;
-  const uint64_t t0 = globaltimer();
+  const long long t0 = cycles();
   for (uint32_t i = 1;; ++i) {
     if (mbar_try(bar, parity)) return true;
     if ((i & 63) == 0) {
       if (*abort_flag) return false;
-      if (globaltimer() - t0 > kWaitLimitNs) {
+      if (cycles() - t0 > kWaitLimitCycles) {
         *abort_flag = 1;
         return false;
       }
@@ -64,9 +64,9 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatil
   }
 }
 __device__ __forceinline__ bool mbar_wait_plain(uint32_t bar, uint32_t parity) {
-  const uint64_t t0 = globaltimer();
+  const long long t0 = cycles();
   while (!mbar_try(bar, parity))
-    if (globaltimer() - t0 > kWaitLimitNs) return false;
+    if (cycles() - t0 > kWaitLimitCycles) return false;
   return true;
 }
 __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, uint32_t bar,

@@ -24,7 +24,7 @@
 //     workspace state for the next call.
 //   - The kernel is bound by streaming W from HBM when the node count is below
 //     the ridge point (~250), by the tensor pipe above it.
-// Every mbarrier wait is bounded (1 s of globaltimer); on expiry the CTA sets
+// Every mbarrier wait is bounded (2e9 SM cycles, about 1 s); on expiry the CTA sets
 // EE_DEVERR_TIMEOUT, drains its own copies and MMAs (again bounded), frees its
 // TMEM and returns.
 #include <cmath>

@@ -70,6 +70,17 @@ def test_workspace_size(L):
 FAKE = ctypes.c_void_p(0x10000)   # never dereferenced: every call below fails validation first
 
 
+def test_attn_plan_rejects_bad_args(L):
+    out = [ctypes.c_int32(0) for _ in range(4)]
+    ptrs = [ctypes.byref(x) for x in out]
+    f = L.ee_attn_plan
+    assert f(0, 64, 28, 4, 4096, *ptrs) == 1          # no sequence
+    assert f(1, 129, 28, 4, 4096, *ptrs) == 1         # tree larger than 128 nodes
+    assert f(1, 64, 28, 5, 4096, *ptrs) == 1          # n_q not a multiple of n_kv
+    assert f(1, 64, 28, 4, -1, *ptrs) == 1            # negative context
+    assert f(1, 64, 28, 4, 4096, None, *ptrs[1:]) == 1
+
+
 def test_match_rejects_bad_args(L):
     f = L.ee_match_reuse
     # n = 0, n too large, max_matches = 0
