@@ -50,7 +50,18 @@ def parse_args():
     ap.add_argument("--no-clocks", action="store_true")
     ap.add_argument("--profile", action="store_true",
                     help="run --steps eager steps and exit (for ncu captures: few launches, no timing)")
+    ap.add_argument("--layers", type=int, default=None,
+                    help="--profile only: build the workload with this many layers (small captures)")
     return ap.parse_args()
+
+
+# DRAM bytes (read + write) per launch from one ncu capture of the kernel as it
+# now stands (profiles/ names the capture); a kernel changed since has no entry.
+TRAFFIC = {
+    ("tree_verify_attn", "7b"): 9061632,          # profiles/attn_tc_7b.md
+    ("tree_verify_attn", "33b"): 139859968,       # profiles/attn_tc_33b.md
+    ("lmhead_accept", "7b"): 1095463424,          # profiles/lmhead_accept_7b.md
+}
 
 
 def rank_seed(config, rank):
@@ -224,7 +235,8 @@ def run_profile(args, local_rank):
     B.build_lib()
     dev = torch.device("cuda", local_rank)
     torch.cuda.set_device(dev)
-    w = W.build(args.config, device=dev)
+    over = {} if args.layers is None else {"layers": args.layers}
+    w = W.build(args.config, device=dev, **over)
     st = S.from_workload(w, device=dev, keep_layers=False)
     torch.cuda.synchronize(dev)
     for _ in range(args.steps):
@@ -372,7 +384,7 @@ def run_ours(args, rank, world, local_rank):
             rl[name].update({"hbm_frac": round(gbs / hbm, 4), "us_per_launch": round(1e3 * c["ms"], 2),
                              "share_of_step": round(c["ms"] * c["launches"] / ms_step_instr, 4),
                              "peak_source": f"{peak_src} ({'copy' if rl[name]['unit'] == 'GB/s' else 'sustained'})",
-                             "traffic": None})
+                             "traffic": TRAFFIC.get((name, args.config))})
         dom = max(cand, key=lambda n: cand[n]["ms"] * cand[n]["launches"])
         roofline = dict(rl[dom], kernel=dom)
 
