@@ -1,5 +1,5 @@
 #!/usr/bin/env python3
-"""Benchmark of one EfficientEdit verification step (arXiv 2506.02780, Sec. IV-A)
+"""Benchmark of one EfficientEdit verification step (arXiv 2506.02780, Sec. III-A)
 on GB300: reuse-span match, tree prepare, L layers of tree-masked paged
 attention, LM head + argmax + acceptance, KV compaction -- all in libee's
 sm_103a kernels, captured as one CUDA graph per step.

@@ -2,16 +2,16 @@
  * ee.h -- C ABI of the GB300 (sm_103a) verification-step library (libee.so).
  *
  * One verification step of EfficientEdit's edit-oriented speculative decoding
- * (arXiv 2506.02780, Sec. IV-A): a draft tree -- a span of the original code
+ * (arXiv 2506.02780, Sec. III-A): a draft tree -- a span of the original code
  * reused verbatim plus short generated branches -- is scored in one target
  * pass and the longest draft prefix on which the target's greedy choice agrees
  * is accepted (Eq. (piecewise)).  The entry points are the steps of that pass:
  *
- *   ee_match_reuse       reuse-span lookup in the original code     (Sec. IV-A)
+ *   ee_match_reuse       reuse-span lookup in the original code     (Sec. III-A)
  *   ee_tree_prepare      depth / ancestor masks of the draft tree
- *   ee_tree_verify_attn  tree-masked attention over the paged cache (Sec. IV-A)
+ *   ee_tree_verify_attn  tree-masked attention over the paged cache (Sec. III-A)
  *   ee_lmhead_accept     LM head + argmax + longest accepted path   (Eq. piecewise)
- *   ee_kv_compact        accepted path's K/V appended to the cache  (Sec. IV-A)
+ *   ee_kv_compact        accepted path's K/V appended to the cache  (Sec. III-A)
  *
  * Conventions shared by every entry point
  * ---------------------------------------
@@ -104,7 +104,7 @@ ee_status ee_workspace_init(void* ws, size_t ws_bytes, ee_stream_t stream);
 ee_status ee_read_errors(void* ws, ee_stream_t stream, int32_t* bits);
 
 /*
- * ee_match_reuse -- reuse-span lookup (Sec. IV-A, prefix matching that switches
+ * ee_match_reuse -- reuse-span lookup (Sec. III-A, prefix matching that switches
  * Generate back to Reuse).  For each sequence s, with c = orig_tokens[
  * orig_off[s] .. orig_off[s+1]) and t = tail[s*n .. s*n+n) (the last n generated
  * tokens), finds every position p with cursor[s] <= p and p + n < len(c) and
@@ -140,7 +140,7 @@ ee_status ee_tree_prepare(const int32_t* parent, const int32_t* node_off, int32_
 
 /*
  * ee_tree_verify_attn -- tree-masked attention of every draft node, ONE layer
- * (Sec. IV-A: one target pass over (prefix, draft)).  Node i of sequence s,
+ * (Sec. III-A: one target pass over (prefix, draft)).  Node i of sequence s,
  * query head h, attends to cached positions 0..ctx_len[s]-1 and to the tree
  * nodes in anc[i] (its own root-to-i path):
  *   out[i][h] = sum_j softmax_j(scale * q[i][h] . k_j) v_j,  KV head h / (n_q/n_kv).
@@ -249,7 +249,7 @@ ee_status ee_lmhead_accept_static(const ee_bf16* hidden, const ee_bf16* lm_w, in
 
 /*
  * ee_kv_compact -- append the accepted path's K/V to the paged cache, every
- * layer (Sec. IV-A: accepted tokens extend the prefix).  Path entry k
+ * layer (Sec. III-A: accepted tokens extend the prefix).  Path entry k
  * (k = 0..accept_len[s], root first) of sequence s goes to position
  * ctx_len_in[s] + k; ctx_len_out[s] = ctx_len_in[s] + accept_len[s] + 1.
  *   k_tree/v_tree  bf16, layer l at + l*tree_layer_stride elements, each layer

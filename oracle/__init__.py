@@ -2,7 +2,7 @@
 
 This package is the plain, slow, obviously-correct statement of what one
 verification step of edit-oriented speculative decoding computes (EfficientEdit,
-arXiv 2506.02780, Sec. IV-A "Reuse" and Eq. (piecewise)).  It exists to check
+arXiv 2506.02780, Sec. III-A "Reuse" and Eq. (piecewise)).  It exists to check
 the CUDA library against; it is not part of the product path.  Only the test
 suite, ``__graft_entry__.smoke()`` and ``bench.py``'s CPU-baseline / reference
 leg may import it.  It shares no code with the CUDA path and imports nothing

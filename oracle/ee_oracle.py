@@ -33,14 +33,14 @@ def _f64(x):
 
 
 # ----------------------------------------------------------------------------
-# (1) reuse-span match -- Sec. IV-A, prefix matching to switch back to Reuse
+# (1) reuse-span match -- Sec. III-A, prefix matching to switch back to Reuse
 # ----------------------------------------------------------------------------
 
 def match_reuse(orig_tokens, orig_off, tail, cursor, max_matches):
     """Positions p in the remaining original code where the last n generated
     tokens occur: c[p:p+n] == tail, searched from the cursor onwards.
 
-    Sec. IV-A: when Generate switches back to Reuse, positions of the remaining
+    Sec. III-A: when Generate switches back to Reuse, positions of the remaining
     ``c`` that match the suffix of what was generated become new draft starts;
     the tokens of ``c`` after such a position are the reuse draft.
     Readings: every position p >= cursor is searched (not only p == cursor);
@@ -84,8 +84,8 @@ def match_reuse(orig_tokens, orig_off, tail, cursor, max_matches):
 def tree_prepare(parent, node_off, max_nodes=128):
     """depth and ancestor set of every draft-tree node.
 
-    The paper's drafts are linear (Sec. IV-A); a tree generalises them to
-    several drafts sharing a prefix (several match points, Sec. IV-A, plus
+    The paper's drafts are linear (Sec. III-A); a tree generalises them to
+    several drafts sharing a prefix (several match points, Sec. III-A, plus
     generated branches).  depth(root) = 0, depth(i) = depth(parent(i)) + 1;
     anc(i) = anc(parent(i)) U {i}.  Parents precede children (parent[i] < i).
 
@@ -131,7 +131,7 @@ def anc_to_sets(anc_row):
 
 
 # ----------------------------------------------------------------------------
-# (3) tree-masked attention over the paged cache -- Sec. IV-A, one target pass
+# (3) tree-masked attention over the paged cache -- Sec. III-A, one target pass
 # ----------------------------------------------------------------------------
 
 def _context_kv(cache_l, block_table_row, ctx, hk):
@@ -150,7 +150,7 @@ def tree_attention(q, k_tree, v_tree, k_cache, v_cache, block_table, ctx_len, no
                    scale=None, nodes=None, heads=None):
     """Attention output of every draft node for ONE layer.
 
-    Sec. IV-A: one forward pass of the target over (prefix, draft) scores every
+    Sec. III-A: one forward pass of the target over (prefix, draft) scores every
     draft token.  With a tree, node i attends to the cached prefix (positions
     0..ctx-1, read through the block table) and to the tree nodes on its own
     root-to-i path (its ancestor set, i included) -- exactly what it would see
@@ -247,7 +247,7 @@ def accept_path(argmax, draft_tok, parent, node_off, max_T=None):
     deepest accepted node's root-to-node path; among equally deep nodes the
     lowest node id wins (this only matters when siblings carry equal tokens).
     accept_len = that node's depth (drafts accepted, root excluded); bonus =
-    argmax at that node, the target's own next token (Sec. III-B: the token
+    argmax at that node, the target's own next token (Sec. II-B: the token
     sampled from the last distribution is kept as well).
 
     Returns (accept_len int32 [B], path int32 [B, max_T] root-first local ids
@@ -290,13 +290,13 @@ def accept_path(argmax, draft_tok, parent, node_off, max_T=None):
 
 
 # ----------------------------------------------------------------------------
-# (5) KV compaction of the accepted path -- Sec. IV-A, accepted tokens extend prefix
+# (5) KV compaction of the accepted path -- Sec. III-A, accepted tokens extend prefix
 # ----------------------------------------------------------------------------
 
 def kv_compact(k_tree, v_tree, k_cache, v_cache, block_table, ctx_len, node_off, path, accept_len):
     """Append the accepted path's K/V to the paged cache, every layer.
 
-    Sec. IV-A: accepted draft tokens extend the prefix; their keys/values were
+    Sec. III-A: accepted draft tokens extend the prefix; their keys/values were
     computed in the verification pass, so they become cache entries.  Path entry
     k (k = 0..accept_len, the root first) goes to position ctx + k, i.e. slot
     block_table[(ctx+k) // PAGE] * PAGE + (ctx+k) % PAGE.  The bonus token's K/V

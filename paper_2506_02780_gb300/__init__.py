@@ -1,5 +1,5 @@
 """Python binding of libee, the sm_103a library for one EfficientEdit
-verification step (arXiv 2506.02780, Sec. IV-A).
+verification step (arXiv 2506.02780, Sec. III-A).
 
 Every function here has the name of the C entry point it wraps (include/ee.h)
 and only marshals arguments: torch CUDA tensors become raw device pointers,

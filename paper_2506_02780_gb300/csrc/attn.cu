@@ -1,6 +1,6 @@
 // ee_tree_verify_attn: tree-masked attention of every draft node over the
 // paged KV cache plus the tree's own K/V, one layer per call (EfficientEdit
-// Sec. IV-A: a single target forward pass over (prefix, draft) scores every
+// Sec. III-A: a single target forward pass over (prefix, draft) scores every
 // draft token; with a tree, each node sees the prefix and its own root path).
 //
 // Work decomposition (split-KV):
@@ -126,7 +126,7 @@ __device__ __forceinline__ unsigned tile_mask(const int32_t* s_pages, int t, int
 }
 
 // Merge rows [r0, r0 + nown) of a row block (query rows row0, ...) from its S
-// partial slots with log-sum-exp weights (Sec. IV-A: the scores of one row
+// partial slots with log-sum-exp weights (Sec. III-A: the scores of one row
 // are normalised over all keys it sees) and write the fp32 output.  Thread t
 // takes row t % nown and the 16-byte column chunks t / nown + k * tpr, where
 // tpr = 256 / nown threads share a row: the loads of a warp for one chunk are

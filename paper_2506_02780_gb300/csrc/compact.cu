@@ -1,5 +1,5 @@
 // ee_kv_compact: append the accepted path's K/V rows to the paged cache, for
-// every layer (EfficientEdit Sec. IV-A: accepted draft tokens extend the
+// every layer (EfficientEdit Sec. III-A: accepted draft tokens extend the
 // prefix, so the K/V computed for them in the verification pass become cache
 // entries).  Path entry k of sequence s lands at position ctx + k.
 //

@@ -1,5 +1,5 @@
 // ee_lmhead_accept: LM head fused with greedy decode and path acceptance
-// (EfficientEdit Sec. IV-A, Eq. (piecewise): a draft token is accepted while the
+// (EfficientEdit Sec. III-A, Eq. (piecewise): a draft token is accepted while the
 // target's greedy choice at the previous position equals it).
 //
 // Design (sm_103a, one persistent CTA per SM):

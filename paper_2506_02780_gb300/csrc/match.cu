@@ -1,5 +1,5 @@
 // ee_match_reuse: reuse-span lookup of the last n generated tokens in the
-// original code (EfficientEdit Sec. IV-A, prefix matching that switches the
+// original code (EfficientEdit Sec. III-A, prefix matching that switches the
 // Generate phase back to Reuse).
 //
 // One CTA per sequence scans the positions p >= cursor in tiles of

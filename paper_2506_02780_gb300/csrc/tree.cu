@@ -1,5 +1,5 @@
 // ee_tree_prepare: depth and root-path (ancestor) bitmask of every draft-tree
-// node.  The paper verifies linear drafts (EfficientEdit Sec. IV-A); several
+// node.  The paper verifies linear drafts (EfficientEdit Sec. III-A); several
 // match points and generated branches share a prefix, so the step scores them
 // together as a tree whose nodes each see only their own root-to-node path.
 //

@@ -1,6 +1,6 @@
 """One whole verification step as a fixed sequence of libee calls.
 
-EfficientEdit (arXiv 2506.02780) Sec. IV-A: the target scores a draft (here a
+EfficientEdit (arXiv 2506.02780) Sec. III-A: the target scores a draft (here a
 tree: reuse chain + generated branches) in one pass and keeps the longest
 prefix its greedy choice agrees with.  ``VerifyStep`` owns the device output
 buffers and the workspace and issues, on one stream:

@@ -4,9 +4,9 @@ EfficientEdit (arXiv 2506.02780) measures on CanItEdit and CodeIF-Bench with
 Qwen2.5-Coder and DeepSeek-Coder models (Sec. V-A, V-D).  Neither the datasets
 nor the weights are used here: these generators stand in for them with random
 arrays of the same shapes and reuse structure -- original code ``c`` as a token
-array, a generated prefix that copies ``c`` with a few planted edits (Sec. IV-A),
+array, a generated prefix that copies ``c`` with a few planted edits (Sec. III-A),
 a draft tree made of a reuse chain taken from ``c`` plus short generated
-branches (gamma = 7-ish, Sec. V-D), a paged bf16 KV cache, query/hidden states
+branches (gamma = 7-ish, Sec. IV-E), a paged bf16 KV cache, query/hidden states
 and LM-head weights.
 
 This module draws random numbers and lays out structure only.  It holds none of
