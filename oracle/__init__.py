@@ -24,6 +24,9 @@ tests/test_oracle_pins.py):
                    over all root-to-node paths, hand-worked golden cases
   kv_compact       pinned: sequential append into a slot dictionary, canaries
   entropy_top_tau  pinned: closed forms of Eq. (entropy) / top_tau (H=0, uniform)
+  verify_accept    pinned: reduces to accept_path (greedy; top-1; all-reuse trees),
+                   top-V = direct, brute force over root-to-node paths, H = 0 and
+                   uniform top-k distributions
 """
 from .ee_oracle import (  # noqa: F401
     PAGE,
@@ -36,5 +39,8 @@ from .ee_oracle import (  # noqa: F401
     accept_path,
     kv_compact,
     entropy_top_tau,
+    VERIFY_MODES,
+    node_ranking,
+    verify_accept,
     verify_step,
 )

@@ -360,6 +360,104 @@ def entropy_top_tau(logits, k, renormalize=False):
     return tau, h, order
 
 
+VERIFY_MODES = ("greedy", "direct", "topk", "entropy")
+
+
+def node_ranking(logits, K):
+    """The K most probable tokens of one target distribution, most probable
+    first; among equal probabilities (equal logits) the lower token id ranks
+    first (the tie rule of decode(), reading A6)."""
+    x = _f64(logits)
+    return np.lexsort((np.arange(len(x)), -x))[:K]
+
+
+def verify_accept(logits, draft_tok, parent, node_off, mode, k=1, gen_mask=None, max_T=None,
+                  tau_override=None):
+    """Longest accepted draft path under one of the verification rules the
+    paper compares (Sec. V-C, RQ3), applied along every root-to-node path of
+    the tree as in accept_path.
+
+    The edge a -> b (b drafted after a) is judged on the target distribution at
+    a (the logits of node a).  Edit content -- the nodes with gen_mask[b] = 1,
+    every node when gen_mask is None -- is judged by ``mode``; reused code stays
+    greedy (Sec. IV-E: only the edit content of EfficientEdit uses the
+    entropy-aware rule, the Reuse phase verifies greedily):
+      greedy   draft_tok[b] is the target's most probable token (rank 0);
+      direct   accepted without verification;
+      topk     draft_tok[b] ranks within the target's k most probable tokens;
+      entropy  draft_tok[b] ranks within the first top_tau of them, top_tau
+               from Eq. (entropy) at a (entropy_top_tau, Sec. III-B).
+    Ranks order tokens by probability, lower id first among equal ones.  The
+    accepted path is the deepest accepted node's root path (lowest node id
+    among equally deep ones, reading A9); bonus = the target's most probable
+    token at that node (Sec. II-B).
+
+    ``tau_override`` (int array [sum T]) replaces the computed top_tau of the
+    entropy rule node by node -- for checking a kernel's acceptance given its
+    own top_tau where k * H_norm sits at an integer.
+
+    Returns (accept_len int32 [B], path int32 [B, max_T], bonus int32 [B],
+    tau int32 [sum T]) where tau[a] is the number of leading ranks an
+    edit-content child of a may hold (greedy 1, topk k, entropy top_tau,
+    direct 0 = any).
+    """
+    if mode not in VERIFY_MODES:
+        raise ValueError(mode)
+    x = _f64(logits)
+    draft_tok = np.asarray(draft_tok)
+    parent = np.asarray(parent)
+    node_off = np.asarray(node_off)
+    total = len(draft_tok)
+    gen = np.ones(total, dtype=bool) if gen_mask is None else np.asarray(gen_mask).astype(bool)
+    B = len(node_off) - 1
+    Ts = np.diff(node_off)
+    if max_T is None:
+        max_T = int(Ts.max())
+    kk = max(1, int(k))
+    ranked = [node_ranking(x[a], max(kk, 1)) for a in range(total)]
+    tau = np.zeros(total, dtype=np.int32)
+    for a in range(total):
+        if mode == "greedy":
+            tau[a] = 1
+        elif mode == "topk":
+            tau[a] = kk
+        elif mode == "entropy":
+            tau[a] = entropy_top_tau(x[a], kk)[0] if tau_override is None else int(tau_override[a])
+    accept_len = np.zeros(B, dtype=np.int32)
+    path = np.full((B, max_T), -1, dtype=np.int32)
+    bonus = np.zeros(B, dtype=np.int32)
+    for s in range(B):
+        o, T = int(node_off[s]), int(Ts[s])
+        accepted = [False] * T
+        depth = [0] * T
+        accepted[0] = True
+        for i in range(1, T):
+            p = int(parent[o + i])
+            depth[i] = depth[p] + 1
+            a, tok = o + p, int(draft_tok[o + i])
+            if not gen[o + i]:
+                ok = tok == int(ranked[a][0])                      # reused code: greedy
+            elif mode == "direct":
+                ok = True
+            else:
+                ok = tok in [int(t) for t in ranked[a][:int(tau[a])]]
+            accepted[i] = accepted[p] and ok
+        best = 0
+        for i in range(1, T):
+            if accepted[i] and depth[i] > depth[best]:
+                best = i
+        chain = []
+        u = best
+        while u != -1:
+            chain.append(u)
+            u = int(parent[o + u]) if u != 0 else -1
+        chain.reverse()
+        accept_len[s] = depth[best]
+        path[s, :len(chain)] = chain
+        bonus[s] = int(ranked[o + best][0])
+    return accept_len, path, bonus, tau
+
+
 # ----------------------------------------------------------------------------
 # one whole step
 # ----------------------------------------------------------------------------

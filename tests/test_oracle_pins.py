@@ -457,6 +457,120 @@ def test_entropy_golden(case):
 
 
 # ----------------------------------------------------------------------------
+# verification rules (Sec. V-C: Greedy / Direct / Top-k / Entropy)
+# ----------------------------------------------------------------------------
+
+def _rank(x, tok):
+    """Rank of token tok in one distribution, counted: tokens with a higher logit,
+    plus tokens with an equal logit and a lower id."""
+    return sum(1 for v in range(len(x)) if x[v] > x[tok] or (x[v] == x[tok] and v < tok))
+
+
+def _random_case(rng, T, V, levels=4):
+    parent = np.asarray([-1] + [int(rng.integers(0, i)) for i in range(1, T)], np.int32)
+    logits = rng.integers(0, levels, size=(T, V)).astype(np.float64)   # few levels: ties happen
+    draft = rng.integers(0, V, size=T)
+    gen = rng.integers(0, 2, size=T)
+    return parent, logits, draft, gen
+
+
+def test_verify_greedy_is_accept_path():
+    rng = np.random.default_rng(21)
+    for _ in range(200):
+        T = int(rng.integers(1, 25))
+        parent, x, draft, gen = _random_case(rng, T, 5)
+        off = np.asarray([0, T])
+        am = np.argmax(x, axis=1)                              # first maximum = lowest id
+        ref = O.accept_path(am, draft, parent, off)
+        for g in (None, gen):
+            got = O.verify_accept(x, draft, parent, off, "greedy", gen_mask=g)
+            for r, q in zip(ref, got[:3]):
+                np.testing.assert_array_equal(r, q)
+
+
+def test_verify_top1_is_greedy_and_reuse_only_is_greedy():
+    rng = np.random.default_rng(22)
+    for _ in range(200):
+        T = int(rng.integers(1, 25))
+        parent, x, draft, gen = _random_case(rng, T, 6)
+        off = np.asarray([0, T])
+        greedy = O.verify_accept(x, draft, parent, off, "greedy", gen_mask=gen)[:3]
+        top1 = O.verify_accept(x, draft, parent, off, "topk", k=1, gen_mask=gen)[:3]
+        for r, q in zip(greedy, top1):
+            np.testing.assert_array_equal(r, q)
+        zero = np.zeros(T, int)
+        ref = O.accept_path(np.argmax(x, axis=1), draft, parent, off)     # all reused: greedy
+        for mode, k in (("direct", 1), ("topk", 3), ("entropy", 3)):
+            got = O.verify_accept(x, draft, parent, off, mode, k=k, gen_mask=zero)[:3]
+            for r, q in zip(ref, got):
+                np.testing.assert_array_equal(r, q)
+
+
+def test_verify_top_vocab_is_direct():
+    rng = np.random.default_rng(23)
+    V = 6
+    for _ in range(200):
+        T = int(rng.integers(1, 25))
+        parent, x, draft, gen = _random_case(rng, T, V)
+        off = np.asarray([0, T])
+        a = O.verify_accept(x, draft, parent, off, "topk", k=V, gen_mask=gen)[:3]
+        b = O.verify_accept(x, draft, parent, off, "direct", gen_mask=gen)[:3]
+        for r, q in zip(a, b):
+            np.testing.assert_array_equal(r, q)
+
+
+@pytest.mark.parametrize("mode,k", [("topk", 2), ("topk", 3), ("entropy", 3), ("entropy", 5),
+                                    ("direct", 1), ("greedy", 1)])
+def test_verify_bruteforce_random(mode, k):
+    """Every root-to-node path checked edge by edge with counted ranks; the
+    entropy rule's top_tau comes from its own (separately pinned) function."""
+    rng = np.random.default_rng(24 + k)
+    for _ in range(150):
+        T = int(rng.integers(1, 20))
+        V = int(rng.integers(2, 9))
+        parent, x, draft, gen = _random_case(rng, T, V)
+        off = np.asarray([0, T])
+        acc, path, bonus, tau = O.verify_accept(x, draft, parent, off, mode, k=k, gen_mask=gen)
+        def edge_ok(a, b):
+            if not gen[b]:
+                return _rank(x[a], draft[b]) == 0
+            if mode == "direct":
+                return True
+            lim = {"greedy": 1, "topk": k}.get(mode)
+            if lim is None:
+                lim = O.entropy_top_tau(x[a], k)[0]
+            return _rank(x[a], draft[b]) < lim
+        best, best_len = 0, 0
+        for u in range(T):
+            pth = _walk_up(parent, 0, u)
+            if all(edge_ok(a, b) for a, b in zip(pth[:-1], pth[1:])) and len(pth) - 1 > best_len:
+                best, best_len = u, len(pth) - 1
+        assert acc[0] == best_len
+        assert list(path[0, :best_len + 1]) == _walk_up(parent, 0, best)
+        assert bonus[0] == int(np.argmax(x[best]))
+
+
+def test_verify_entropy_closed_forms():
+    """H_norm = 0 (one dominant token) gives top_tau = 1, the greedy rule; k equal
+    probabilities and nothing else give H_norm = 1, top_tau = k, the top-k rule."""
+    V, k = 12, 4
+    T = 6
+    parent = np.asarray([-1, 0, 1, 2, 3, 4], np.int32)
+    off = np.asarray([0, T])
+    draft = np.asarray([0, 3, 2, 1, 0, 2])            # ranks 3, 2, 1, 0, 2 of the uniform top-4
+    uniform = np.full((T, V), -np.inf)
+    uniform[:, :k] = 0.0                               # p = 1/k on tokens 0..k-1
+    onehot = np.full((T, V), -np.inf)
+    onehot[:, 0] = 0.0
+    acc_u, _, _, tau_u = O.verify_accept(uniform, draft, parent, off, "entropy", k=k)
+    acc_t = O.verify_accept(uniform, draft, parent, off, "topk", k=k)[0]
+    assert list(tau_u) == [k] * T and acc_u[0] == acc_t[0] == T - 1
+    acc_o, _, _, tau_o = O.verify_accept(onehot, draft, parent, off, "entropy", k=k)
+    acc_g = O.verify_accept(onehot, draft, parent, off, "greedy")[0]
+    assert list(tau_o) == [1] * T and acc_o[0] == acc_g[0] == 0
+
+
+# ----------------------------------------------------------------------------
 # whole step on the tiny configuration
 # ----------------------------------------------------------------------------
 
