@@ -48,6 +48,8 @@ def parse_args():
     ap.add_argument("--e2e-steps", type=int, default=300)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-clocks", action="store_true")
+    ap.add_argument("--no-variants", action="store_true",
+                    help="skip the verification-rule variants (entropy k=3, k=5)")
     ap.add_argument("--profile", action="store_true",
                     help="run --steps eager steps and exit (for ncu captures: few launches, no timing)")
     ap.add_argument("--layers", type=int, default=None,
@@ -343,6 +345,32 @@ def run_ours(args, rank, world, local_rank):
     if world > 1:
         torch.distributed.barrier()
     clk = None if args.no_clocks else clocks.stop()
+
+    # the same step under the entropy-aware rule (Sec. III-B) for the generated
+    # branches, with the paper's two settings of k (Sec. IV-E: 3 and 5)
+    variants = {}
+    if not args.no_variants and w.lm_w is not None:
+        for k in (3, 5):
+            sv = S.from_workload(w, device=dev, keep_layers=False, verify=("entropy", k))
+            pool = []
+            with torch.cuda.stream(stream):
+                sv.run(stream)
+                stream.synchronize()
+                for _ in range(2):
+                    g = torch.cuda.CUDAGraph()
+                    with torch.cuda.graph(g, stream=stream):
+                        sv.run(stream)
+                    pool.append(g)
+            for i in range(max(3, args.warmup // 4)):
+                pool[i % 2].replay()
+            stream.synchronize()
+            ms_v = timed(pool, max(8, args.steps // 4))
+            assert E.ee_read_errors(sv.ws, stream) == 0
+            variants[f"entropy_k{k}"] = {
+                "value": round(world * 1e3 / ms_v, 2), "ms_per_step": round(ms_v, 5),
+                "accept_len": [int(a) for a in sv.accept_len.cpu().tolist()[:8]],
+                "greedy_accept_len": [int(a) for a in st.accept_len.cpu().tolist()[:8]]}
+            del pool, sv
     assert E.ee_read_errors(st.ws, stream) == 0
 
     # ---- end to end: host inputs -> device -> step -> host results ---------
@@ -403,6 +431,7 @@ def run_ours(args, rank, world, local_rank):
         "draft_tokens_per_s": round(steps_per_s * alg["draft_nodes"], 1),
         "roofline": roofline, "roofline_kernels": rl, "kernels": kernels,
         "e2e": e2e, "gpu_launches": st.launches_per_step() * args.steps, "clocks": clk,
+        "verify_variants": variants,
         "planted_accept": [int(a) for a in w.planted_accept[:8]],
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:

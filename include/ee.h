@@ -29,10 +29,10 @@
  *    [num_pages][n_kv][EE_PAGE][head_dim]; position t of sequence s lives in
  *    page block_table[s * max_pages + t / EE_PAGE], row t % EE_PAGE.
  *  - `ws` is a caller-owned device workspace of at least
- *    ee_workspace_size(...) bytes: a zeroed head of about 16.5 KB (the error
- *    word and the LM head's running argmax), zeroed once with
- *    ee_workspace_init() before first use, then the attention's per-CTA
- *    partial results (65 KB per CTA, B x n_q x 8 CTAs at most, never zeroed).
+ *    ee_workspace_size(...) bytes, zeroed once with ee_workspace_init() before
+ *    first use: a 16.5 KB head (the error word and the LM head's running
+ *    argmax), 2.7 MB of LM-head verification partials and thresholds, then the attention's
+ *    per-CTA partial results (65 KB per CTA, B x n_q x 16 CTAs at most).
  *    Its first word is the device error word: kernels never trap;
  *    on a bad index found on the device they set an EE_DEVERR_* bit there,
  *    skip the access and continue.  ee_read_errors() reads (and clears) it.
@@ -87,8 +87,8 @@ const char* ee_status_string(ee_status s);
  * Workspace bytes needed by every entry point for problems up to these sizes:
  * B sequences, total_nodes tree nodes in all, n_q query heads, max_ctx cached
  * positions in the longest sequence.  The buffer must be 256-byte aligned.
- * 16,896 bytes when max_ctx is 0, else 16,896 + B * n_q * 8 * 66,560 (the
- * attention's partial slots; about 15 MB for one sequence with 28 heads).
+ * 2,908,672 bytes when max_ctx is 0, else 2,908,672 + B * n_q * 16 * 66,816
+ * (the attention's partial slots; about 30 MB for one sequence with 28 heads).
  * Returns 0 for negative arguments.
  */
 size_t ee_workspace_size(int32_t B, int32_t total_nodes, int32_t n_q, int32_t head_dim,
@@ -171,6 +171,51 @@ ee_status ee_tree_verify_attn(const ee_bf16* q, const ee_bf16* k_tree, const ee_
                               int32_t B, int32_t total_nodes, int32_t max_T, int32_t n_q,
                               int32_t n_kv, int32_t head_dim, float scale, float* out,
                               void* ws, size_t ws_bytes, ee_stream_t stream);
+
+/*
+ * ee_lmhead_verify -- the LM head with the verification rules the paper
+ * compares (Sec. V-C, RQ3), including its entropy-aware dynamic verification
+ * (Sec. III-B, Eq. (entropy) and the top_tau rule).  Same inputs, argmax,
+ * path, accept_len and bonus as ee_lmhead_accept; what differs is how the edge
+ * a -> b (b drafted after a) of edit content is judged on the target
+ * distribution at a:
+ *   EE_VERIFY_GREEDY   draft_tok[b] is the target's most probable token;
+ *   EE_VERIFY_DIRECT   accepted without verification;
+ *   EE_VERIFY_TOPK     draft_tok[b] is among the target's k most probable;
+ *   EE_VERIFY_ENTROPY  draft_tok[b] is among the first top_tau of them, where
+ *                      H_norm = -sum_{i<=k} p_i ln p_i / ln k over the k
+ *                      largest probabilities p_i of the full-vocabulary
+ *                      softmax (not renormalised) and top_tau =
+ *                      max(1, ceil(k * H_norm)), at most k.
+ * Probabilities rank by logit, lower token id first among equal logits.
+ * gen_mask_or_null uint8 [total_nodes]: 1 = edit content (the mode's rule),
+ * 0 = reused code (always greedy, as the paper verifies the Reuse phase);
+ * NULL = every node is edit content.  k: 1..8 (2..8 for ENTROPY; unused by
+ * GREEDY and DIRECT except as the length of topk_ids).
+ * Optional outputs (NULL to skip): topk_ids int32 [total_nodes][k] ranked
+ * token ids; top_tau int32 [total_nodes] the number of leading ranks an edit
+ * child may hold (greedy 1, top-k k, entropy top_tau, direct 0 = any);
+ * h_norm fp32 [total_nodes] (0 when k = 1).  Logits, the log-sum-exp and
+ * H_norm are fp32.  The workspace must hold ee_workspace_size(...) bytes
+ * (per-CTA partials of the top-k lists live there).  EE_ERR_INVALID_ARG for a
+ * bad mode or k; otherwise as ee_lmhead_accept.
+ */
+typedef enum {
+  EE_VERIFY_GREEDY = 0,
+  EE_VERIFY_DIRECT = 1,
+  EE_VERIFY_TOPK = 2,
+  EE_VERIFY_ENTROPY = 3
+} ee_verify_mode;
+
+ee_status ee_lmhead_verify(const ee_bf16* hidden, const ee_bf16* lm_w, int32_t hidden_dim,
+                           int32_t vocab, const int32_t* draft_tok, const int32_t* parent,
+                           const int32_t* depth, const uint64_t* anc, const int32_t* node_off,
+                           const uint8_t* gen_mask_or_null, int32_t B, int32_t total_nodes,
+                           int32_t max_T, int32_t mode, int32_t k, int32_t* argmax,
+                           int32_t* topk_ids_or_null, int32_t* top_tau_or_null,
+                           float* h_norm_or_null, int32_t* accept_len, int32_t* path,
+                           int32_t* bonus, float* logits_or_null, void* ws, size_t ws_bytes,
+                           ee_stream_t stream);
 
 /*
  * ee_attn_plan -- the launch plan ee_tree_verify_attn uses for these sizes

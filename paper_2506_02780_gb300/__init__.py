@@ -30,7 +30,9 @@ DEVERR = {0x01: "MATCH_ARGS", 0x02: "TREE", 0x04: "PAGE", 0x08: "CTX", 0x10: "FP
 
 EXPORTS = ("ee_version", "ee_status_string", "ee_workspace_size", "ee_workspace_init",
            "ee_read_errors", "ee_match_reuse", "ee_tree_prepare", "ee_tree_verify_attn", "ee_attn_plan",
-           "ee_lmhead_accept", "ee_lmhead_accept_static", "ee_kv_compact")
+           "ee_lmhead_accept", "ee_lmhead_verify", "ee_lmhead_accept_static", "ee_kv_compact")
+
+VERIFY_MODES = {"greedy": 0, "direct": 1, "topk": 2, "entropy": 3}
 
 
 class EEError(RuntimeError):
@@ -64,6 +66,8 @@ _SIGS = {
                       ctypes.POINTER(_I)], _I),
     "ee_lmhead_accept": ([_P, _P, _I, _I, _P, _P, _P, _P, _P, _I, _I, _I, _P, _P, _P, _P, _P, _P, _SZ,
                           _P], _I),
+    "ee_lmhead_verify": ([_P, _P, _I, _I, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _P, _P, _P, _P, _P,
+                          _P, _P, _P, _P, _SZ, _P], _I),
     "ee_lmhead_accept_static": ([_P, _P, _I, _I, _P, _P, _P, _P, _P, _I, _I, _I, _P, _P, _P, _P, _P,
                                  _P], _I),
     "ee_kv_compact": ([_P, _P, _I64, _P, _P, _I64, _I, _I, _P, _I, _P, _P, _P, _P, _P, _I, _I, _I, _I,
@@ -197,6 +201,27 @@ def ee_lmhead_accept(hidden, lm_w, draft_tok, parent, depth, anc, node_off, max_
                                 _p(anc), _p(node_off), B, total, max_T, _p(argmax), _p(accept_len),
                                 _p(path), _p(bonus), _p(logits), _p(ws), ws.numel(), _stream(stream))
     _ok("ee_lmhead_accept", st)
+
+
+def ee_lmhead_verify(hidden, lm_w, draft_tok, parent, depth, anc, node_off, max_T, mode, k, argmax,
+                     accept_len, path, bonus, ws, gen_mask=None, topk_ids=None, top_tau=None,
+                     h_norm=None, logits=None, stream=None):
+    """LM head + argmax + acceptance under a verification rule: ``mode`` is one of
+    "greedy", "direct", "topk", "entropy" (or its EE_VERIFY_* number);
+    ``gen_mask`` uint8 marks edit content (None: every node)."""
+    _check(hidden, torch.bfloat16, "hidden")
+    _check(lm_w, torch.bfloat16, "lm_w")
+    if gen_mask is not None:
+        _check(gen_mask, torch.uint8, "gen_mask")
+    total, H = hidden.shape
+    V = lm_w.shape[0]
+    B = node_off.numel() - 1
+    m = VERIFY_MODES[mode] if isinstance(mode, str) else int(mode)
+    st = lib().ee_lmhead_verify(_p(hidden), _p(lm_w), H, V, _p(draft_tok), _p(parent), _p(depth),
+                                _p(anc), _p(node_off), _p(gen_mask), B, total, max_T, m, k,
+                                _p(argmax), _p(topk_ids), _p(top_tau), _p(h_norm), _p(accept_len),
+                                _p(path), _p(bonus), _p(logits), _p(ws), ws.numel(), _stream(stream))
+    _ok("ee_lmhead_verify", st)
 
 
 def ee_lmhead_accept_static(hidden, lm_w, draft_tok, parent, depth, anc, node_off, max_T, argmax,

@@ -19,10 +19,10 @@ extern "C" const char* ee_status_string(ee_status s) {
 extern "C" size_t ee_workspace_size(int32_t B, int32_t total_nodes, int32_t n_q, int32_t head_dim,
                                     int32_t max_ctx) {
   if (B < 0 || total_nodes < 0 || n_q < 0 || head_dim < 0 || max_ctx < 0) return 0;
-  if (max_ctx == 0) return ee::kWorkspaceBytes;   // one chunk per row block: no partials
+  if (max_ctx == 0) return ee::kAttnPartOff;      // one chunk per row block: no attention slots
   // attention CTAs of a split launch: B x n_kv x ceil(max_T * g / 128) row
   // blocks (<= B x n_q, as max_T <= 128) x at most 16 chunks
-  return ee::kWorkspaceBytes + (size_t)B * n_q * ee::kAttnMaxSplits * ee::kAttnPartBytes;
+  return ee::kAttnPartOff + (size_t)B * n_q * ee::kAttnMaxSplits * ee::kAttnPartBytes;
 }
 
 extern "C" ee_status ee_workspace_init(void* ws, size_t ws_bytes, ee_stream_t stream) {

@@ -878,7 +878,7 @@ extern "C" ee_status ee_tree_verify_attn(const ee_bf16* q, const ee_bf16* k_tree
   const Split sp = choose_split(max_ctx, nrb * n_kv * B);
   const int S = sp.S, chunk = sp.chunk;
   // a split launch writes one partial slot per CTA after the zeroed part
-  if (S > 1 && ws_bytes < kWorkspaceBytes + (size_t)nrb * S * n_kv * B * kAttnPartBytes)
+  if (S > 1 && ws_bytes < kAttnPartOff + (size_t)nrb * S * n_kv * B * kAttnPartBytes)
     return EE_ERR_WORKSPACE;
 
   AttnParams p;
@@ -888,7 +888,7 @@ extern "C" ee_status ee_tree_verify_attn(const ee_bf16* q, const ee_bf16* k_tree
   p.node_off = node_off;
   p.anc = anc;
   p.out = out;
-  p.part = static_cast<uint8_t*>(ws) + kWorkspaceBytes;
+  p.part = static_cast<uint8_t*>(ws) + kAttnPartOff;
   p.err = err_word(ws);
   p.num_pages = num_pages;
   p.max_pages = max_pages;

@@ -18,15 +18,33 @@ namespace ee {
 // Workspace layout (bytes from the start of `ws`):
 //   [0, 4)              device error word (EE_DEVERR_* bits)
 //   [16, 20)            LM-head "CTAs finished" ticket counter
+//   [24, 28)            verification finalize "CTAs finished" ticket counter
 //   [256, 256+8*EE_MAX_LM_NODES)  LM-head packed running argmax per node
-//   [kWorkspaceBytes, ...)        attention partial slots, kAttnPartBytes per
+//   [kLmVerifyOff, +kLmVerifyBytes) LM-head verification partials
+//   [kAttnPartOff, ...)           attention partial slots, kAttnPartBytes per
 //                                 CTA of a split launch; the trailer of a row
 //                                 block's first slot holds its arrival counters
 // ---------------------------------------------------------------------------
 constexpr size_t kErrOff = 0;
 constexpr size_t kTicketOff = 16;
 constexpr size_t kArgmaxOff = 256;
-constexpr size_t kWorkspaceBytes = 256 + 8 * (size_t)EE_MAX_LM_NODES + 256;   // the zeroed part
+constexpr size_t kWorkspaceBytes = 256 + 8 * (size_t)EE_MAX_LM_NODES + 256;   // the fixed head
+constexpr int kNumSMsMax = 152;       // LM-head grid bound (one persistent CTA per SM)
+// LM-head verification partials (ee_lmhead_verify): per CTA and node of its
+// node tile, the CTA's top-k (value, id) list and its (max, sum) of 2^logit;
+// then the per-node global pruning threshold
+constexpr int kLmMaxK = 8;
+constexpr int kLmMaxBN = 256;
+constexpr size_t kLmVerifyOff = kWorkspaceBytes;
+constexpr size_t kLmPartBytes = (size_t)kNumSMsMax * kLmMaxBN * (8 * kLmMaxK + 8);
+// then one u64 per node: the best K-th key any CTA has published (zero between
+// calls); then the finalize step's ranked ids [node][K] and top_tau [node]
+constexpr size_t kLmGthrOff = kLmPartBytes;
+constexpr size_t kLmTkOff = kLmGthrOff + 8 * (size_t)EE_MAX_LM_NODES;
+constexpr size_t kLmTauOff = kLmTkOff + 4 * (size_t)EE_MAX_LM_NODES * kLmMaxK;
+constexpr size_t kLmVerifyBytes = kLmTauOff + 4 * (size_t)EE_MAX_LM_NODES;
+constexpr size_t kFinTicketOff = 24;   // in the head: finalize CTAs finished
+constexpr size_t kAttnPartOff = kLmVerifyOff + kLmVerifyBytes;   // attention partial slots
 constexpr int kAttnRows = 128;        // query rows (node x head-in-group) per attention CTA
 constexpr int kAttnMaxSplits = 16;    // context chunks per row block
 // one CTA's partial: 128 rows x 128 fp32 of O (column-chunk major), then

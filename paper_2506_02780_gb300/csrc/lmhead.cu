@@ -40,7 +40,9 @@ using namespace ee;
 
 constexpr int BM = 128;           // vocab rows per tile (MMA M)
 constexpr int BK = 64;            // bf16 per 128-byte swizzle row
-constexpr int kThreads = 192;     // warp 0 TMA, warp 1 MMA, warps 2..5 epilogue
+constexpr int kThreads = 320;     // warp 0 TMA, warp 1 MMA, warps 2..9 epilogue
+constexpr int kEpiWarps = 8;      // two per TMEM lane quarter, alternate 16-column chunks
+constexpr int kEpiThreads = 32 * kEpiWarps;
 constexpr int kABytes = BM * BK * 2;
 
 struct LmParams {
@@ -59,7 +61,39 @@ struct LmParams {
   unsigned long long* keys;   // [EE_MAX_LM_NODES] running argmax keys (workspace)
   unsigned int* ticket;       // CTAs finished (workspace)
   int32_t* err;
+  // verification rules (ee_lmhead_verify only)
+  int mode, K;                // EE_VERIFY_*, list length k
+  const uint8_t* gen_mask;    // 1 = edit content (the mode's rule), 0 = reused (greedy); NULL = all 1
+  int32_t* topk_ids;          // [total][K] or NULL
+  int32_t* tau_out;           // [total] or NULL
+  float* h_out;               // [total] or NULL
+  uint8_t* part;              // per-CTA partials (workspace), BN * (8 K + 8) bytes per CTA
+  unsigned long long* gthr;   // [EE_MAX_LM_NODES] best K-th key published by any CTA (workspace)
 };
+
+constexpr float kLog2e = 1.4426950408889634f;
+
+__device__ __forceinline__ float ex2f(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+// (m1, s1) + (m2, s2): sums of 2^((l - m) log2 e) kept against a running max
+__device__ __forceinline__ void lse_add(float& m, float& sm, float m2, float s2) {
+  if (m2 == -INFINITY) return;
+  if (m == -INFINITY) {
+    m = m2;
+    sm = s2;
+    return;
+  }
+  const float mm = fmaxf(m, m2);
+  sm = sm * ex2f((m - mm) * kLog2e) + s2 * ex2f((m2 - mm) * kLog2e);
+  m = mm;
+}
+// lane that owns column c after the 16-column reduce-scatter below
+__device__ __forceinline__ int lane_of_col(int c) {
+  return (((c >> 3) & 1) << 4) | (((c >> 2) & 1) << 3) | (((c >> 1) & 1) << 2) | ((c & 1) << 1);
+}
 
 __device__ __forceinline__ uint32_t ordered(float f) {
   const uint32_t u = __float_as_uint(f);
@@ -72,12 +106,129 @@ __device__ __forceinline__ bool better(float v, int i, float w, int j) {
   return v > w || (v == w && i < j);
 }
 
+__device__ __forceinline__ float unordered(uint32_t k) {
+  return __uint_as_float((k & 0x80000000u) ? (k & 0x7FFFFFFFu) : ~k);
+}
+// One round of a warp-wide selection over one (value, id) per lane: the best
+// value (order-preserving 32-bit key, one warp reduction), the lowest id among
+// lanes holding exactly that value.  Returns the winner in (*wv, *wi).
+__device__ __forceinline__ void warp_best(float v, int id, float* wv, int* wi) {
+  const uint32_t key = ordered(v);
+  const uint32_t mx = __reduce_max_sync(0xffffffffu, key);
+  const uint32_t mid = __reduce_min_sync(0xffffffffu, key == mx ? (uint32_t)id : 0xFFFFFFFFu);
+  *wv = unordered(mx);
+  *wi = (int)mid;
+}
 struct BestPair {
   float v;
   int i;
 };
 
 // ---------------------------------------------------------------------------
+// Acceptance for every sequence (one warp each): node i is accepted when every
+// edge on its root path is accepted -- a 128-bit "edge rejected" ballot mask
+// ANDed with each node's ancestor mask -- and the deepest accepted node (lowest
+// local id among equally deep ones) gives the path, accept_len and bonus.
+// An edge a -> b of reused code is accepted when draft_tok[b] = argmax[a];
+// with kVerify, edit content follows the mode's rule on the ranked ids tk and
+// top_tau of a.  kGlobal: am / tk / tau live in global memory (read through L2).
+struct AcceptArgs {
+  int B, max_T, total, mode, K;
+  const int32_t* node_off;
+  const int32_t* parent;
+  const int32_t* draft_tok;
+  const int32_t* depth;
+  const uint64_t* anc;
+  const uint8_t* gen_mask;
+  int32_t* accept_len;
+  int32_t* path;
+  int32_t* bonus;
+  int32_t* err;
+};
+
+template <bool kVerify>
+__device__ void accept_sequences(const AcceptArgs& a, const int32_t* am, const int32_t* tk,
+                                 const int32_t* tau, int warp, int lane, int nwarps) {
+  auto ld_i = [](const int32_t* q) -> int {
+    if constexpr (kVerify)
+      return __ldcg(q);
+    else
+      return *q;
+  };
+  for (int s = warp; s < a.B; s += nwarps) {
+    const int o = a.node_off[s];
+    const int T = a.node_off[s + 1] - o;
+    if (T < 1 || T > EE_MAX_TREE || T > a.max_T || o < 0 || o + T > a.total) {
+      if (lane == 0) ee::flag_error(a.err, EE_DEVERR_TREE);
+      continue;
+    }
+    // notok bit i: node i's edge from its parent is rejected
+    uint32_t notok[4];
+    uint64_t a0[4], a1[4];
+    int key_best = -1;
+#pragma unroll
+    for (int c = 0; c < 4; ++c) {
+      const int i = c * 32 + lane;
+      bool bad = false;
+      if (i < T && i > 0) {
+        const int par = a.parent[o + i];
+        if (par < 0 || par >= i) {
+          bad = true;
+        } else {
+          const int tok = a.draft_tok[o + i];
+          if (!kVerify || (a.gen_mask && !a.gen_mask[o + i])) {
+            bad = tok != ld_i(am + o + par);               // reused code: greedy
+          } else if (a.mode == EE_VERIFY_DIRECT) {
+            bad = false;
+          } else {
+            const int lim = a.mode == EE_VERIFY_GREEDY ? 1
+                          : (a.mode == EE_VERIFY_TOPK ? a.K : ld_i(tau + o + par));
+            bad = true;
+            for (int rr = 0; rr < lim; ++rr)
+              if (ld_i(tk + (size_t)(o + par) * a.K + rr) == tok) bad = false;
+          }
+        }
+      }
+      notok[c] = __ballot_sync(0xffffffffu, bad);
+      a0[c] = i < T ? a.anc[2 * (size_t)(o + i)] : 0ull;
+      a1[c] = i < T ? a.anc[2 * (size_t)(o + i) + 1] : 0ull;
+    }
+    const uint64_t nz0 = (uint64_t)notok[0] | ((uint64_t)notok[1] << 32);
+    const uint64_t nz1 = (uint64_t)notok[2] | ((uint64_t)notok[3] << 32);
+#pragma unroll
+    for (int c = 0; c < 4; ++c) {
+      const int i = c * 32 + lane;
+      if (i < T && (a0[c] & nz0) == 0 && (a1[c] & nz1) == 0) {
+        const int k = (a.depth[o + i] << 8) | (255 - i);
+        key_best = max(key_best, k);
+      }
+    }
+#pragma unroll
+    for (int d = 16; d >= 1; d >>= 1) key_best = max(key_best, __shfl_xor_sync(0xffffffffu, key_best, d));
+    const int u = 255 - (key_best & 255);
+    const int du = key_best >> 8;
+    const uint64_t w0 = a.anc[2 * (size_t)(o + u)], w1 = a.anc[2 * (size_t)(o + u) + 1];
+    for (int j = lane; j < a.max_T; j += 32) a.path[(size_t)s * a.max_T + j] = -1;
+    __syncwarp();
+#pragma unroll
+    for (int c = 0; c < 4; ++c) {
+      const int j = c * 32 + lane;
+      const bool on = j < 64 ? ((w0 >> j) & 1ull) : ((w1 >> (j - 64)) & 1ull);
+      if (j < T && on) {
+        const int pos = j < 64 ? __popcll(w0 & ((1ull << j) - 1ull))
+                               : __popcll(w0) + __popcll(w1 & ((1ull << (j - 64)) - 1ull));
+        if (pos < a.max_T) a.path[(size_t)s * a.max_T + pos] = j;
+      }
+    }
+    if (lane == 0) {
+      a.accept_len[s] = du;
+      a.bonus[s] = ld_i(am + o + u);
+    }
+  }
+}
+
+
+template <bool kVerify>
 __global__ void __launch_bounds__(kThreads, 1)
 lmhead_accept_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmX,
                      const LmParams p) {
@@ -94,6 +245,15 @@ lmhead_accept_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_const
   uint64_t* bars = reinterpret_cast<uint64_t*>(tail);   // full[S], empty[S], tfull[2], tempty[2], drain
   BestPair* s_best = reinterpret_cast<BestPair*>(tail + 8 * (2 * S + 5) + 8);  // [4][BN]
   uint32_t* s_tmem = reinterpret_cast<uint32_t*>(tail + 8 * (2 * S + 5));
+  // verification state per epilogue warp and node: top-K list, (max, sum) of 2^logit
+  const int K = kVerify ? p.K : 1;
+  float* s_lv = reinterpret_cast<float*>(s_best + 4 * BN);          // [4][BN][K]
+  int* s_li = reinterpret_cast<int*>(s_lv + 4 * BN * K);            // [4][BN][K]
+  float2* s_lse = reinterpret_cast<float2*>(s_li + 4 * BN * K);     // [4][BN]
+  // per node, the best K-th entry over the 4 warps' lists (an order-preserving
+  // key): a row below it cannot be among the CTA's K best
+  unsigned long long* s_thr = reinterpret_cast<unsigned long long*>(s_lse + 4 * BN);   // [BN]
+  unsigned long long* s_pub = s_thr + BN;   // [BN] the key this CTA last published
   __shared__ volatile int s_abort;
   __shared__ int s_last;
   __shared__ int s_issued, s_consumed;
@@ -112,7 +272,7 @@ lmhead_accept_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_const
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(tfull0 + 8 * a, 1);
-      mbar_init(tempty0 + 8 * a, 4);
+      mbar_init(tempty0 + 8 * a, kEpiWarps);
     }
     mbar_init(drain, 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -126,6 +286,17 @@ lmhead_accept_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_const
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
   }
   for (int i = threadIdx.x; i < 4 * BN; i += kThreads) s_best[i] = BestPair{-INFINITY, 0x7fffffff};
+  if (kVerify) {
+    for (int i = threadIdx.x; i < 4 * BN * K; i += kThreads) {
+      s_lv[i] = -INFINITY;
+      s_li[i] = 0x7fffffff;
+    }
+    for (int i = threadIdx.x; i < 4 * BN; i += kThreads) s_lse[i] = make_float2(-INFINITY, 0.f);
+    for (int i = threadIdx.x; i < BN; i += kThreads) {
+      s_thr[i] = 0ull;
+      s_pub[i] = 0ull;
+    }
+  }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -196,8 +367,9 @@ lmhead_accept_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_const
     }
   } else {
     // epilogue warps 2..5: TMEM lane quarter = warp % 4
-    const int q = warp & 3;
-    const int ew = warp - 2;
+    const int q = warp & 3;                 // TMEM lane quarter
+    const int ew = q;                       // per-quarter state index
+    const int half = (warp - 2) >> 2;       // which 16-column chunks: c0 / 16 = half mod 2
     BestPair* mybest = s_best + ew * BN;
     int lt = 0;
     for (int t = blockIdx.x; t < num_tiles; t += gridDim.x, ++lt) {
@@ -207,16 +379,24 @@ lmhead_accept_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_const
       // warp-uniform outcome: the tcgen05.ld below is warp-collective
       if (!__all_sync(0xffffffffu, mbar_wait(tfull0 + 8 * acc, acc_phase, &s_abort))) break;
       tc_fence_after();
+      if (kVerify) {
+        // fold the other CTAs' published K-th keys into the shared threshold (a
+        // stale value only lets more rows through)
+        for (int c = threadIdx.x - 64; c < BN; c += kEpiThreads)
+          if (nt * BN + c < p.total_nodes) atomicMax(&s_thr[c], __ldcg(p.gthr + nt * BN + c));
+      }
       const int row = vt * BM + q * 32 + lane;
       const bool row_ok = row < p.vocab;
-      for (int c0 = 0; c0 < BN; c0 += 16) {
+      for (int c0 = 16 * half; c0 < BN; c0 += 32) {
         uint32_t r[16];
         tc_ld16(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN + c0), r);
         float v[16];
         int id[16];
+        float v0[16];   // this row's logits, kept for the verification state
 #pragma unroll
         for (int j = 0; j < 16; ++j) {
           v[j] = row_ok ? __uint_as_float(r[j]) : -INFINITY;
+          v0[j] = v[j];
           id[j] = row;
         }
         if (p.logits != nullptr && row_ok) {
@@ -257,16 +437,118 @@ lmhead_accept_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_const
           BestPair cur = mybest[c0 + col];
           if (better(v[0], id[0], cur.v, cur.i)) mybest[c0 + col] = BestPair{v[0], id[0]};
         }
+        if (kVerify) {
+          // (1) log-sum-exp: each column's sum over this warp's rows of
+          //     2^((l - colmax) log2 e), reduce-scattered like the maximum, then
+          //     folded into the warp's running (max, sum) of the node
+          float e[16];
+#pragma unroll
+          for (int j = 0; j < 16; ++j) {
+            const float cm = __shfl_sync(0xffffffffu, v[0], lane_of_col(j));
+            e[j] = cm == -INFINITY ? 0.f : ex2f((v0[j] - cm) * kLog2e);
+          }
+#pragma unroll
+          for (int half = 8, bit = 16; half >= 1; half >>= 1, bit >>= 1) {
+            const bool upper = (lane & bit) != 0;
+#pragma unroll
+            for (int j = 0; j < half; ++j) {
+              const float keep = upper ? e[j + half] : e[j];
+              const float give = upper ? e[j] : e[j + half];
+              e[j] = keep + __shfl_xor_sync(0xffffffffu, give, bit);
+            }
+          }
+          e[0] += __shfl_xor_sync(0xffffffffu, e[0], 1);
+          if ((lane & 1) == 0) {
+            float2 cur = s_lse[ew * BN + c0 + col];
+            lse_add(cur.x, cur.y, v[0], e[0]);
+            s_lse[ew * BN + c0 + col] = cur;
+          }
+          __syncwarp();
+          // (2) top-K per node column: a row is a candidate when its key beats the
+          //     CTA's shared threshold; up to four candidates are inserted into
+          //     the warp's sorted list by lane 0, more re-select the K best of
+          //     list + candidates with K rounds of a warp argmax
+          const int row0 = vt * BM + q * 32;
+#pragma unroll
+          for (int j = 0; j < 16; ++j) {
+            float* lv = s_lv + (size_t)(ew * BN + c0 + j) * K;
+            int* li = s_li + (size_t)(ew * BN + c0 + j) * K;
+            const bool cand = row_ok && make_key(v0[j], row) > s_thr[c0 + j];
+            unsigned mask = __ballot_sync(0xffffffffu, cand);
+            if (mask == 0u) continue;
+            if (__popc(mask) <= 4) {
+              while (mask) {
+                const int src = __ffs(mask) - 1;
+                mask &= mask - 1;
+                const float cv = __shfl_sync(0xffffffffu, v0[j], src);
+                const int ci = row0 + src;
+                if (lane == 0 && better(cv, ci, lv[K - 1], li[K - 1])) {
+                  int pos = K - 1;
+                  while (pos > 0 && better(cv, ci, lv[pos - 1], li[pos - 1])) {
+                    lv[pos] = lv[pos - 1];
+                    li[pos] = li[pos - 1];
+                    --pos;
+                  }
+                  lv[pos] = cv;
+                  li[pos] = ci;
+                }
+                __syncwarp();
+              }
+            } else {
+              float av = lane < K ? lv[lane] : -INFINITY;
+              int ai = lane < K ? li[lane] : 0x7fffffff;
+              float bv = cand ? v0[j] : -INFINITY;
+              int bi = cand ? row : 0x7fffffff;
+              __syncwarp();
+              for (int rr = 0; rr < K; ++rr) {
+                const bool useA = better(av, ai, bv, bi);
+                const float mv = useA ? av : bv;
+                const int mi = useA ? ai : bi;
+                float xv;
+                int xi;
+                warp_best(mv, mi, &xv, &xi);
+                if (mi == xi && mv == xv) {   // (value, id) pairs are unique: this lane held it
+                  if (useA) {
+                    av = -INFINITY;
+                    ai = 0x7fffffff;
+                  } else {
+                    bv = -INFINITY;
+                    bi = 0x7fffffff;
+                  }
+                }
+                if (lane == 0) {
+                  lv[rr] = xv;
+                  li[rr] = xi;
+                }
+              }
+              __syncwarp();
+            }
+            if (lane == 0 && li[K - 1] != 0x7fffffff)
+              atomicMax(&s_thr[c0 + j], make_key(lv[K - 1], li[K - 1]));
+            __syncwarp();
+          }
+        }
       }
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(tempty0 + 8 * acc);
+      if (kVerify) {
+        // publish this CTA's K-th keys: no row below another CTA's K-th entry
+        // can be among the K best of the whole vocabulary
+        for (int c = threadIdx.x - 64; c < BN; c += kEpiThreads) {
+          const unsigned long long key = s_thr[c];
+          if (key > s_pub[c] && nt * BN + c < p.total_nodes) {   // only when it improved
+            atomicMax(p.gthr + nt * BN + c, key);
+            s_pub[c] = key;
+          }
+        }
+      }
     }
     // publish this CTA's best per node (every tile of a CTA has the same node tile)
-    asm volatile("bar.sync 1, 128;" ::: "memory");
+    asm volatile("bar.sync 1, %0;" ::"n"(kEpiThreads) : "memory");
     if (blockIdx.x < num_tiles) {
       const int nt = blockIdx.x % p.n_nt;
-      for (int c = threadIdx.x - 64; c < BN; c += 128) {
+      for (int c = threadIdx.x - 64; c < BN; c += kEpiThreads) {
         BestPair b = s_best[c];
         for (int w = 1; w < 4; ++w) {
           const BestPair o = s_best[w * BN + c];
@@ -274,6 +556,43 @@ lmhead_accept_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_const
         }
         const int node = nt * BN + c;
         if (node < p.total_nodes && b.i != 0x7fffffff) atomicMax(&p.keys[node], make_key(b.v, b.i));
+        if (kVerify) {
+          // this CTA's partial for the node: the 4 warps' lists merged, their sums added
+          float* pv = reinterpret_cast<float*>(p.part + (size_t)blockIdx.x * BN * (8 * K + 8)) +
+                      (size_t)c * K;
+          int* pi = reinterpret_cast<int*>(p.part + (size_t)blockIdx.x * BN * (8 * K + 8) +
+                                           (size_t)BN * K * 4) + (size_t)c * K;
+          float2* pl = reinterpret_cast<float2*>(p.part + (size_t)blockIdx.x * BN * (8 * K + 8) +
+                                                 (size_t)BN * K * 8) + c;
+          int hs[4] = {0, 0, 0, 0};   // next entry of each warp's sorted list
+          for (int rr = 0; rr < K; ++rr) {
+            int wb = -1;
+            float bv = -INFINITY;
+            int bi = 0x7fffffff;
+#pragma unroll
+            for (int w = 0; w < 4; ++w) {
+              if (hs[w] >= K) continue;   // exhausted
+              const float ov = s_lv[(size_t)(w * BN + c) * K + hs[w]];
+              const int oi = s_li[(size_t)(w * BN + c) * K + hs[w]];
+              if (wb < 0 || better(ov, oi, bv, bi)) {
+                bv = ov;
+                bi = oi;
+                wb = w;
+              }
+            }
+            pv[rr] = bv;
+            pi[rr] = bi;
+#pragma unroll
+            for (int w = 0; w < 4; ++w) hs[w] += wb == w;
+          }
+          float m = -INFINITY, sm = 0.f;
+#pragma unroll
+          for (int w = 0; w < 4; ++w) {
+            const float2 x = s_lse[w * BN + c];
+            lse_add(m, sm, x.x, x.y);
+          }
+          *pl = make_float2(m, sm);
+        }
       }
     }
     __threadfence();
@@ -304,7 +623,7 @@ lmhead_accept_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_const
   }
   if (aborted) return;
 
-  // ---- last CTA: argmax decode + acceptance ---------------------------------
+  // ---- last CTA: argmax decode (+ greedy acceptance) -------------------------
   if (threadIdx.x == 0) {
     __threadfence();
     const unsigned int ticket = atomicAdd(p.ticket, 1u);
@@ -321,62 +640,212 @@ lmhead_accept_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_const
     p.argmax[i] = a;
   }
   if (threadIdx.x == 0) *p.ticket = 0u;
+  if (kVerify) return;   // the finalize kernel ranks, decides top_tau and accepts
   __syncthreads();
-  for (int s = warp; s < p.B; s += kThreads / 32) {
-    const int o = p.node_off[s];
-    const int T = p.node_off[s + 1] - o;
-    if (T < 1 || T > EE_MAX_TREE || T > p.max_T || o < 0 || o + T > p.total_nodes) {
-      if (lane == 0) ee::flag_error(p.err, EE_DEVERR_TREE);
-      continue;
-    }
-    // notok bit i: node i's edge from its parent is rejected
-    uint32_t notok[4];
-    uint64_t a0[4], a1[4];
-    int key_best = -1;
+  AcceptArgs aa{p.B, p.max_T, p.total_nodes, EE_VERIFY_GREEDY, 1, p.node_off, p.parent, p.draft_tok,
+                p.depth, p.anc, nullptr, p.accept_len, p.path, p.bonus, p.err};
+  accept_sequences<false>(aa, s_am, nullptr, nullptr, warp, lane, kThreads / 32);
+}
+
+
+// ---------------------------------------------------------------------------
+// Verification finalize (second launch of ee_lmhead_verify): one warp per node
+// merges the per-CTA partials of the LM head -- its K best (logit, id) over the
+// whole vocabulary and the log-sum-exp -- computes H_norm of Eq. (entropy) and
+// top_tau, writes the ranked ids and top_tau to the workspace; the last CTA to
+// finish runs the acceptance and zeroes the pruning thresholds.
+// ---------------------------------------------------------------------------
+constexpr int kFinWarps = 8;
+constexpr int kSurv = 256;   // per warp: entries that can still be among a node's K best
+
+struct FinParams {
+  int total, B, max_T, BN, n_nt, n_src, K, mode;
+  const uint8_t* part;
+  unsigned long long* gthr;
+  int32_t* tk;                // [total][K] (workspace)
+  int32_t* tau;               // [total] (workspace)
+  int32_t* topk_ids;          // user outputs or NULL
+  int32_t* tau_out;
+  float* h_out;
+  const int32_t* argmax;      // written by the LM head
+  unsigned int* ticket;
+  AcceptArgs acc;
+};
+
+__global__ void __launch_bounds__(32 * kFinWarps, 1) lm_verify_finalize_kernel(const FinParams p) {
+  ee::pdl_allow_next();
+  ee::pdl_wait();   // the LM head's partials, thresholds and argmax are complete
+  __shared__ float s_sv[kFinWarps][kSurv];
+  __shared__ int s_svi[kFinWarps][kSurv];
+  __shared__ int s_svn[kFinWarps];
+  __shared__ int s_last;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int K = p.K, BN = p.BN;
+  const int node = blockIdx.x * kFinWarps + warp;
+  if (node < p.total) {
+    const int nt = node / BN, c = node - nt * BN;
+    const size_t pstride = (size_t)BN * (8 * K + 8);
+    // the best K-th key any CTA published: at most the node's true K-th best,
+    // so only entries reaching it can be among the K best
+    const unsigned long long g = __ldcg(p.gthr + node);
+    constexpr int kMaxU = (kNumSMsMax + 31) / 32;
+    float cv[kMaxU][kLmMaxK];
+    int ci[kMaxU][kLmMaxK];
+    float2 xs[kMaxU];
+    // every partial of the node: lane l takes source CTAs l, l + 32, ...;
+    // unconditional loads from always-valid addresses (source 0 and entry K - 1
+    // stand in for absent ones), masked afterwards, so that all are in flight
 #pragma unroll
-    for (int c = 0; c < 4; ++c) {
-      const int i = c * 32 + lane;
-      bool bad = false;
-      if (i < T && i > 0) {
-        const int par = p.parent[o + i];
-        bad = (par < 0 || par >= i) ? true : (p.draft_tok[o + i] != s_am[o + par]);
+    for (int u = 0; u < kMaxU; ++u) {
+      const int q2 = lane + 32 * u;
+      const uint8_t* pc = p.part + (size_t)(q2 < p.n_src ? q2 * p.n_nt + nt : nt) * pstride;
+      xs[u] = __ldcg(reinterpret_cast<const float2*>(pc + (size_t)BN * K * 8) + c);
+      const float* pv = reinterpret_cast<const float*>(pc) + (size_t)c * K;
+      const int* pi = reinterpret_cast<const int*>(pc + (size_t)BN * K * 4) + (size_t)c * K;
+#pragma unroll
+      for (int rr = 0; rr < kLmMaxK; ++rr) {
+        cv[u][rr] = __ldcg(pv + min(rr, K - 1));
+        ci[u][rr] = __ldcg(pi + min(rr, K - 1));
       }
-      notok[c] = __ballot_sync(0xffffffffu, bad);
-      a0[c] = i < T ? p.anc[2 * (size_t)(o + i)] : 0ull;
-      a1[c] = i < T ? p.anc[2 * (size_t)(o + i) + 1] : 0ull;
     }
-    const uint64_t nz0 = (uint64_t)notok[0] | ((uint64_t)notok[1] << 32);
-    const uint64_t nz1 = (uint64_t)notok[2] | ((uint64_t)notok[3] << 32);
+    float m = -INFINITY, sm = 0.f;
 #pragma unroll
-    for (int c = 0; c < 4; ++c) {
-      const int i = c * 32 + lane;
-      if (i < T && (a0[c] & nz0) == 0 && (a1[c] & nz1) == 0) {
-        const int k = (p.depth[o + i] << 8) | (255 - i);
-        key_best = max(key_best, k);
-      }
+    for (int u = 0; u < kMaxU; ++u) {
+      const bool valid = lane + 32 * u < p.n_src;
+      if (valid) lse_add(m, sm, xs[u].x, xs[u].y);
+#pragma unroll
+      for (int rr = 0; rr < kLmMaxK; ++rr)
+        if (!valid || rr >= K) {
+          cv[u][rr] = -INFINITY;
+          ci[u][rr] = 0x7fffffff;
+        }
     }
 #pragma unroll
-    for (int d = 16; d >= 1; d >>= 1) key_best = max(key_best, __shfl_xor_sync(0xffffffffu, key_best, d));
-    const int u = 255 - (key_best & 255);
-    const int du = key_best >> 8;
-    const uint64_t w0 = p.anc[2 * (size_t)(o + u)], w1 = p.anc[2 * (size_t)(o + u) + 1];
-    for (int j = lane; j < p.max_T; j += 32) p.path[(size_t)s * p.max_T + j] = -1;
+    for (int d = 16; d >= 1; d >>= 1) {
+      const float mo = __shfl_xor_sync(0xffffffffu, m, d);
+      const float so = __shfl_xor_sync(0xffffffffu, sm, d);
+      lse_add(m, sm, mo, so);
+    }
+    const float lse = m + logf(sm);
+    // survivors into the warp's buffer
+    float* sv = s_sv[warp];
+    int* svi = s_svi[warp];
+    if (lane == 0) s_svn[warp] = 0;
     __syncwarp();
 #pragma unroll
-    for (int c = 0; c < 4; ++c) {
-      const int j = c * 32 + lane;
-      const bool on = j < 64 ? ((w0 >> j) & 1ull) : ((w1 >> (j - 64)) & 1ull);
-      if (j < T && on) {
-        const int pos = j < 64 ? __popcll(w0 & ((1ull << j) - 1ull))
-                               : __popcll(w0) + __popcll(w1 & ((1ull << (j - 64)) - 1ull));
-        if (pos < p.max_T) p.path[(size_t)s * p.max_T + pos] = j;
+    for (int u = 0; u < kMaxU; ++u)
+#pragma unroll
+      for (int rr = 0; rr < kLmMaxK; ++rr)
+        if (ci[u][rr] != 0x7fffffff && make_key(cv[u][rr], ci[u][rr]) >= g) {
+          const int pos = atomicAdd(&s_svn[warp], 1);
+          if (pos < kSurv) {
+            sv[pos] = cv[u][rr];
+            svi[pos] = ci[u][rr];
+          }
+        }
+    __syncwarp();
+    const int n_sv = s_svn[warp];
+    const bool few = n_sv <= kSurv;
+    // overflow (not seen with a published threshold): each lane merges its own
+    // sorted source lists, then the warp takes the K best of the lane heads
+    float lv[kLmMaxK];
+    int li[kLmMaxK];
+#pragma unroll
+    for (int t = 0; t < kLmMaxK; ++t) {
+      lv[t] = -INFINITY;
+      li[t] = 0x7fffffff;
+    }
+    if (!few) {
+#pragma unroll
+      for (int rr = 0; rr < kLmMaxK; ++rr) {
+        if (rr >= K) break;
+        int wu = 0;
+        float bv = cv[0][0];
+        int bi = ci[0][0];
+#pragma unroll
+        for (int u = 1; u < kMaxU; ++u)
+          if (better(cv[u][0], ci[u][0], bv, bi)) {
+            wu = u;
+            bv = cv[u][0];
+            bi = ci[u][0];
+          }
+        lv[rr] = bv;
+        li[rr] = bi;
+#pragma unroll
+        for (int u = 0; u < kMaxU; ++u) {
+          if (u != wu) continue;
+#pragma unroll
+          for (int t = 0; t < kLmMaxK - 1; ++t) {
+            cv[u][t] = cv[u][t + 1];
+            ci[u][t] = ci[u][t + 1];
+          }
+          cv[u][kLmMaxK - 1] = -INFINITY;
+          ci[u][kLmMaxK - 1] = 0x7fffffff;
+        }
+      }
+    }
+    float hsum = 0.f;   // -sum p ln p over the K best, with ln p = logit - lse
+    for (int rr = 0; rr < K; ++rr) {
+      float xv;
+      int xi;
+      if (few) {
+        float bv = -INFINITY;
+        int bi = 0x7fffffff, bpos = -1;
+        for (int pos = lane; pos < n_sv; pos += 32)
+          if (better(sv[pos], svi[pos], bv, bi)) {
+            bv = sv[pos];
+            bi = svi[pos];
+            bpos = pos;
+          }
+        warp_best(bv, bi, &xv, &xi);
+        if (bpos >= 0 && bi == xi && bv == xv) {
+          sv[bpos] = -INFINITY;
+          svi[bpos] = 0x7fffffff;
+        }
+        __syncwarp();
+      } else {
+        warp_best(lv[0], li[0], &xv, &xi);
+        if (xi != 0x7fffffff && li[0] == xi && lv[0] == xv) {   // this lane held it: next one up
+#pragma unroll
+          for (int t = 0; t < kLmMaxK - 1; ++t) {
+            lv[t] = lv[t + 1];
+            li[t] = li[t + 1];
+          }
+          lv[kLmMaxK - 1] = -INFINITY;
+          li[kLmMaxK - 1] = 0x7fffffff;
+        }
+      }
+      const float pr = ex2f((xv - lse) * kLog2e);
+      if (pr > 0.f) hsum += pr * (lse - xv);
+      if (lane == 0) {
+        p.tk[(size_t)node * K + rr] = xi;
+        if (p.topk_ids) p.topk_ids[(size_t)node * K + rr] = xi;
       }
     }
     if (lane == 0) {
-      p.accept_len[s] = du;
-      p.bonus[s] = s_am[o + u];
+      int tau = 1;
+      float h = 0.f;
+      if (K >= 2) h = hsum / logf((float)K);
+      if (p.mode == EE_VERIFY_ENTROPY) tau = min(K, max(1, (int)ceilf((float)K * h)));
+      else if (p.mode == EE_VERIFY_TOPK) tau = K;
+      else if (p.mode == EE_VERIFY_DIRECT) tau = 0;
+      p.tau[node] = tau;
+      if (p.tau_out) p.tau_out[node] = tau;
+      if (p.h_out) p.h_out[node] = h;
     }
   }
+  // the last CTA to finish: acceptance, then zero the thresholds for the next call
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    __threadfence();
+    s_last = atomicAdd(p.ticket, 1u) == gridDim.x - 1 ? 1 : 0;
+  }
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();
+  for (int i = threadIdx.x; i < p.total; i += blockDim.x) p.gthr[i] = 0ull;
+  if (threadIdx.x == 0) *p.ticket = 0u;
+  accept_sequences<true>(p.acc, p.argmax, p.tk, p.tau, warp, lane, kFinWarps);
 }
 
 // ---------------------------------------------------------------------------
@@ -412,16 +881,28 @@ ee_status check_lm_args(const ee_bf16* hidden, const ee_bf16* lm_w, int32_t hidd
   return EE_OK;
 }
 
+// Arguments of the verification rules (ee_lmhead_verify).
+struct VerifyArgs {
+  int mode, k;
+  const uint8_t* gen_mask;
+  int32_t* topk_ids;
+  int32_t* tau;
+  float* h_norm;
+  uint8_t* part;               // the workspace's verification region (kLmVerifyOff)
+  unsigned int* fin_ticket;
+};
+
 // Encode the tensor maps and launch the persistent LM-head kernel; `keys`
 // (EE_MAX_LM_NODES running-argmax words, zero on entry), `ticket` (zero on
-// entry) and `err` are the kernel's scratch.
+// entry) and `err` are the kernel's scratch.  `va` selects the verification
+// variant (NULL: greedy acceptance).
 ee_status launch_lmhead(const ee_bf16* hidden, const ee_bf16* lm_w, int32_t hidden_dim,
                         int32_t vocab, const int32_t* draft_tok, const int32_t* parent,
                         const int32_t* depth, const uint64_t* anc, const int32_t* node_off, int32_t B,
                         int32_t total_nodes, int32_t max_T, int32_t* argmax, int32_t* accept_len,
                         int32_t* path, int32_t* bonus, float* logits_or_null,
                         unsigned long long* keys, unsigned int* ticket, int32_t* err,
-                        ee_stream_t stream, bool pdl) {
+                        ee_stream_t stream, bool pdl, const VerifyArgs* va = nullptr) {
   LmParams p;
   p.vocab = vocab;
   p.hidden = hidden_dim;
@@ -433,7 +914,11 @@ ee_status launch_lmhead(const ee_bf16* hidden, const ee_bf16* lm_w, int32_t hidd
   p.n_vt = (vocab + BM - 1) / BM;
   p.nkb = (hidden_dim + BK - 1) / BK;
   const size_t stage_bytes = (size_t)kABytes + (size_t)p.BN * BK * 2;
-  const size_t fixed = 1024 /*align slack*/ + 8 * (2 * 8 + 5) + 8 + 4 * (size_t)p.BN * sizeof(BestPair);
+  const int K = va ? va->k : 1;
+  // epilogue state: running best per warp and node (+ top-K lists and sums)
+  const size_t epi = 4 * (size_t)p.BN * sizeof(BestPair) +
+                     (va ? 4 * (size_t)p.BN * (8 * K + 8) + 16 * (size_t)p.BN : 0);
+  const size_t fixed = 1024 /*align slack*/ + 8 * (2 * 8 + 5) + 8 + epi;
   const size_t budget = 227 * 1024 - fixed - 64;
   p.stages = (int)std::min<size_t>(8, budget / stage_bytes);
   if (p.stages < 2) return EE_ERR_UNSUPPORTED;
@@ -453,30 +938,70 @@ ee_status launch_lmhead(const ee_bf16* hidden, const ee_bf16* lm_w, int32_t hidd
   p.keys = keys;
   p.ticket = ticket;
   p.err = err;
+  p.mode = va ? va->mode : EE_VERIFY_GREEDY;
+  p.K = K;
+  p.gen_mask = va ? va->gen_mask : nullptr;
+  p.topk_ids = va ? va->topk_ids : nullptr;
+  p.tau_out = va ? va->tau : nullptr;
+  p.h_out = va ? va->h_norm : nullptr;
+  p.part = va ? va->part : nullptr;
+  p.gthr = va ? reinterpret_cast<unsigned long long*>(va->part + ee::kLmGthrOff) : nullptr;
 
   CUtensorMap tmW, tmX;
   if (!encode_2d(&tmW, lm_w, (uint64_t)hidden_dim, (uint64_t)vocab, BK, BM)) return EE_ERR_CUDA;
   if (!encode_2d(&tmX, hidden, (uint64_t)hidden_dim, (uint64_t)total_nodes, BK, p.BN))
     return EE_ERR_CUDA;
 
-  const size_t smem = 1024 + (size_t)p.stages * stage_bytes + 8 * (2 * p.stages + 5) + 8 +
-                      4 * (size_t)p.BN * sizeof(BestPair);
-  const size_t smem_acc = std::max(smem, (size_t)1024 + (size_t)EE_MAX_LM_NODES * 4);
-  static size_t attr_bytes = 0;
-  if (attr_bytes < smem_acc) {
-    EE_CUDA_OK(cudaFuncSetAttribute(lmhead_accept_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                    (int)smem_acc));
-    attr_bytes = smem_acc;
+  const size_t smem = 1024 + (size_t)p.stages * stage_bytes + 8 * (2 * p.stages + 5) + 8 + epi;
+  // the last CTA reuses the pipeline buffers: argmax (+ ranked ids and top_tau) per node
+  const size_t last = 1024 + (size_t)(EE_MAX_LM_NODES + 4) * 4;   // the last CTA: argmax per node
+  const size_t smem_acc = std::max(smem, last);
+  if (smem_acc > 227 * 1024) return EE_ERR_UNSUPPORTED;
+  static size_t attr_bytes[2] = {0, 0};
+  if (attr_bytes[va ? 1 : 0] < smem_acc) {
+    if (va)
+      EE_CUDA_OK(cudaFuncSetAttribute(lmhead_accept_kernel<true>,
+                                      cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_acc));
+    else
+      EE_CUDA_OK(cudaFuncSetAttribute(lmhead_accept_kernel<false>,
+                                      cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_acc));
+    attr_bytes[va ? 1 : 0] = smem_acc;
   }
   const int num_tiles = p.n_vt * p.n_nt;
   int grid = (ee::kNumSMs / p.n_nt) * p.n_nt;   // multiple of n_nt: each CTA keeps one node tile
   if (grid > num_tiles) grid = num_tiles;
   if (grid < 1) grid = 1;
-  if (pdl) {
-    EE_CUDA_OK(ee::launch_pdl(lmhead_accept_kernel, dim3(grid), dim3(kThreads), smem_acc,
+  if (va && (size_t)grid * p.BN * (8 * K + 8) > ee::kLmPartBytes) return EE_ERR_UNSUPPORTED;
+  if (va) {
+    EE_CUDA_OK(ee::launch_pdl(lmhead_accept_kernel<true>, dim3(grid), dim3(kThreads), smem_acc,
+                              (cudaStream_t)stream, 1, tmW, tmX, p));
+    FinParams fp;
+    fp.total = total_nodes;
+    fp.B = B;
+    fp.max_T = max_T;
+    fp.BN = p.BN;
+    fp.n_nt = p.n_nt;
+    fp.n_src = grid / p.n_nt;
+    fp.K = K;
+    fp.mode = va->mode;
+    fp.part = va->part;
+    fp.gthr = p.gthr;
+    fp.tk = reinterpret_cast<int32_t*>(va->part + ee::kLmTkOff);
+    fp.tau = reinterpret_cast<int32_t*>(va->part + ee::kLmTauOff);
+    fp.topk_ids = va->topk_ids;
+    fp.tau_out = va->tau;
+    fp.h_out = va->h_norm;
+    fp.argmax = argmax;
+    fp.ticket = va->fin_ticket;
+    fp.acc = AcceptArgs{B, max_T, total_nodes, va->mode, K, node_off, parent, draft_tok, depth, anc,
+                        va->gen_mask, accept_len, path, bonus, err};
+    EE_CUDA_OK(ee::launch_pdl(lm_verify_finalize_kernel, dim3((total_nodes + kFinWarps - 1) / kFinWarps),
+                              dim3(32 * kFinWarps), 0, (cudaStream_t)stream, 1, fp));
+  } else if (pdl) {
+    EE_CUDA_OK(ee::launch_pdl(lmhead_accept_kernel<false>, dim3(grid), dim3(kThreads), smem_acc,
                               (cudaStream_t)stream, 1, tmW, tmX, p));
   } else {
-    lmhead_accept_kernel<<<grid, kThreads, smem_acc, (cudaStream_t)stream>>>(tmW, tmX, p);
+    lmhead_accept_kernel<false><<<grid, kThreads, smem_acc, (cudaStream_t)stream>>>(tmW, tmX, p);
     EE_LAUNCH_OK();
   }
   return EE_OK;
@@ -504,6 +1029,37 @@ extern "C" ee_status ee_lmhead_accept(const ee_bf16* hidden, const ee_bf16* lm_w
                        reinterpret_cast<unsigned long long*>(wsb + ee::kArgmaxOff),
                        reinterpret_cast<unsigned int*>(wsb + ee::kTicketOff), ee::err_word(ws),
                        stream, true);
+}
+
+extern "C" ee_status ee_lmhead_verify(const ee_bf16* hidden, const ee_bf16* lm_w, int32_t hidden_dim,
+                                      int32_t vocab, const int32_t* draft_tok, const int32_t* parent,
+                                      const int32_t* depth, const uint64_t* anc,
+                                      const int32_t* node_off, const uint8_t* gen_mask_or_null,
+                                      int32_t B, int32_t total_nodes, int32_t max_T, int32_t mode,
+                                      int32_t k, int32_t* argmax, int32_t* topk_ids_or_null,
+                                      int32_t* top_tau_or_null, float* h_norm_or_null,
+                                      int32_t* accept_len, int32_t* path, int32_t* bonus,
+                                      float* logits_or_null, void* ws, size_t ws_bytes,
+                                      ee_stream_t stream) {
+  if (mode < EE_VERIFY_GREEDY || mode > EE_VERIFY_ENTROPY || k < 1 || k > ee::kLmMaxK ||
+      (mode == EE_VERIFY_ENTROPY && k < 2))
+    return EE_ERR_INVALID_ARG;
+  bool empty = false;
+  const ee_status st = check_lm_args(hidden, lm_w, hidden_dim, vocab, draft_tok, parent, depth, anc,
+                                     node_off, B, total_nodes, max_T, argmax, accept_len, path,
+                                     bonus, &empty);
+  if (st != EE_OK || empty) return st;
+  if (!ws || !ee::aligned(ws, 256)) return EE_ERR_INVALID_ARG;
+  if (ws_bytes < ee::kLmVerifyOff + ee::kLmVerifyBytes) return EE_ERR_WORKSPACE;
+  char* wsb = static_cast<char*>(ws);
+  VerifyArgs va{mode, k, gen_mask_or_null, topk_ids_or_null, top_tau_or_null, h_norm_or_null,
+                reinterpret_cast<uint8_t*>(wsb + ee::kLmVerifyOff),
+                reinterpret_cast<unsigned int*>(wsb + ee::kFinTicketOff)};
+  return launch_lmhead(hidden, lm_w, hidden_dim, vocab, draft_tok, parent, depth, anc, node_off, B,
+                       total_nodes, max_T, argmax, accept_len, path, bonus, logits_or_null,
+                       reinterpret_cast<unsigned long long*>(wsb + ee::kArgmaxOff),
+                       reinterpret_cast<unsigned int*>(wsb + ee::kTicketOff), ee::err_word(ws),
+                       stream, true, &va);
 }
 
 // ---------------------------------------------------------------------------

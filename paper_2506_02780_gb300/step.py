@@ -17,8 +17,8 @@ import math
 
 import torch
 
-from . import (EE_HEAD_DIM, ee_kv_compact, ee_lmhead_accept, ee_match_reuse, ee_tree_prepare,
-               ee_tree_verify_attn, new_workspace)
+from . import (EE_HEAD_DIM, ee_kv_compact, ee_lmhead_accept, ee_lmhead_verify, ee_match_reuse,
+               ee_tree_prepare, ee_tree_verify_attn, new_workspace)
 
 
 class VerifyStep:
@@ -28,11 +28,14 @@ class VerifyStep:
     q [L, total, n_q, 128], k_tree/v_tree [L, total, n_kv, 128],
     k_cache/v_cache [L, num_pages, n_kv, 16, 128], hidden [total, H],
     lm_w [V, H] in bf16.  ``max_ctx`` bounds ctx_len (host-side value).
+    ``verify`` = (mode, k) switches the LM head to ee_lmhead_verify with that
+    rule for the edit content marked by ``gen_mask`` (uint8 [total]); None
+    keeps the greedy ee_lmhead_accept.
     """
 
     def __init__(self, *, orig_tokens, orig_off, tail, cursor, parent, node_off, draft_tok, ctx_len,
                  block_table, q, k_tree, v_tree, k_cache, v_cache, hidden, lm_w, max_ctx, max_T,
-                 max_matches=8, scale=None, keep_layers=True):
+                 max_matches=8, scale=None, keep_layers=True, verify=None, gen_mask=None):
         self.inp = dict(orig_tokens=orig_tokens, orig_off=orig_off, tail=tail, cursor=cursor,
                         parent=parent, node_off=node_off, draft_tok=draft_tok, ctx_len=ctx_len,
                         block_table=block_table, q=q, k_tree=k_tree, v_tree=v_tree, k_cache=k_cache,
@@ -60,6 +63,13 @@ class VerifyStep:
         self.ctx_out = torch.empty(self.B, **i32)
         self.dst_slot = torch.empty((self.B, self.max_T), **i32)
         self.ws = new_workspace(self.B, self.total, self.n_q, self.max_ctx, device=dev)
+        self.verify = None if verify is None else (verify[0], int(verify[1]))
+        self.gen_mask = gen_mask
+        if self.verify is not None:
+            k = self.verify[1]
+            self.topk_ids = torch.empty((self.total, k), **i32)
+            self.top_tau = torch.empty(self.total, **i32)
+            self.h_norm = torch.empty(self.total, dtype=torch.float32, device=dev)
         self.graph = None
 
     def run(self, stream=None, logits=None, layers=None):
@@ -73,9 +83,16 @@ class VerifyStep:
             ee_tree_verify_attn(x["q"][l], x["k_tree"][l], x["v_tree"][l], x["k_cache"][l],
                                 x["v_cache"][l], x["block_table"], x["ctx_len"], self.max_ctx,
                                 x["node_off"], self.anc, self.max_T, self.scale, out, self.ws, stream)
-        ee_lmhead_accept(x["hidden"], x["lm_w"], x["draft_tok"], x["parent"], self.depth, self.anc,
-                         x["node_off"], self.max_T, self.argmax, self.accept_len, self.path, self.bonus,
-                         self.ws, logits=logits, stream=stream)
+        if self.verify is None:
+            ee_lmhead_accept(x["hidden"], x["lm_w"], x["draft_tok"], x["parent"], self.depth, self.anc,
+                             x["node_off"], self.max_T, self.argmax, self.accept_len, self.path,
+                             self.bonus, self.ws, logits=logits, stream=stream)
+        else:
+            ee_lmhead_verify(x["hidden"], x["lm_w"], x["draft_tok"], x["parent"], self.depth, self.anc,
+                             x["node_off"], self.max_T, self.verify[0], self.verify[1], self.argmax,
+                             self.accept_len, self.path, self.bonus, self.ws, gen_mask=self.gen_mask,
+                             topk_ids=self.topk_ids, top_tau=self.top_tau, h_norm=self.h_norm,
+                             logits=logits, stream=stream)
         ee_kv_compact(x["k_tree"], x["v_tree"], x["k_cache"], x["v_cache"], x["block_table"],
                       x["ctx_len"], self.ctx_out, x["node_off"], self.path, self.accept_len,
                       self.dst_slot, self.ws, stream)
@@ -92,12 +109,14 @@ class VerifyStep:
         return g
 
     def launches_per_step(self) -> int:
-        """Kernels this step launches: match, prepare, 1 per attention layer, LM head, compaction."""
-        return 2 + self.L + 2
+        """Kernels this step launches: match, prepare, 1 per attention layer, LM head (+ the
+        verification finalize), compaction."""
+        return 2 + self.L + 2 + (0 if self.verify is None else 1)
 
 
-def from_workload(w, device="cuda", keep_layers=True):
-    """VerifyStep over a workloads.Workload (its float tensors already on ``device``)."""
+def from_workload(w, device="cuda", keep_layers=True, verify=None):
+    """VerifyStep over a workloads.Workload (its float tensors already on ``device``);
+    ``verify`` = (mode, k) uses that rule on the workload's generated branches."""
     def i32(a):
         return torch.as_tensor(a, dtype=torch.int32).to(device)
     return VerifyStep(
@@ -106,4 +125,5 @@ def from_workload(w, device="cuda", keep_layers=True):
         draft_tok=i32(w.draft_tok), ctx_len=i32(w.ctx_len), block_table=i32(w.block_table),
         q=w.q, k_tree=w.k_tree, v_tree=w.v_tree, k_cache=w.k_cache, v_cache=w.v_cache,
         hidden=w.hidden_states, lm_w=w.lm_w, max_ctx=int(w.ctx_len.max()), max_T=w.max_T,
-        max_matches=w.max_matches, keep_layers=keep_layers)
+        max_matches=w.max_matches, keep_layers=keep_layers, verify=verify,
+        gen_mask=torch.as_tensor(w.gen_mask).to(device) if verify is not None else None)

@@ -50,14 +50,18 @@ def test_version_and_status_strings(L):
 
 
 def test_workspace_size(L):
-    """A zeroed head (error word, LM-head ticket, running argmax words: 8 bytes
-    per node up to EE_MAX_LM_NODES) plus, when the context is split, one
-    attention partial slot per CTA: 128 rows x 128 fp32 + 128 x (m, l) + a
-    256-byte counter trailer, for at most B x n_q row blocks x 16 chunks.
-    Independent of the node count."""
+    """A fixed head (error word, LM-head ticket, running argmax words: 8 bytes
+    per node up to EE_MAX_LM_NODES), the LM-head verification partials (152
+    CTAs x 256 nodes x (8 top-k values + 8 ids + max + sum), then one 8-byte
+    pruning threshold per node, the finalize step's 8 ranked ids and top_tau
+    per node), and, when the
+    context is split, one attention partial slot per CTA: 128 rows x 128 fp32
+    + 128 x (m, l) + a 256-byte counter trailer, for at most B x n_q row blocks
+    x 16 chunks.  Independent of the node count."""
     head = L.ee_workspace_size(1, 64, 28, 128, 0)
     assert head == L.ee_workspace_size(8, 2048, 56, 128, 0)
-    assert head % 256 == 0 and 8 * 2048 < head <= 32 * 1024
+    assert head % 256 == 0
+    assert head == 16896 + 152 * 256 * (8 * 8 + 8) + 8 * 2048 + 4 * 2048 * 8 + 4 * 2048
     slot = 128 * 128 * 4 + 128 * 8 + 256
     assert slot % 256 == 0
     for B, n_q, ctx in ((1, 28, 4096), (8, 56, 262144), (3, 8, 16)):
@@ -68,6 +72,16 @@ def test_workspace_size(L):
 
 
 FAKE = ctypes.c_void_p(0x10000)   # never dereferenced: every call below fails validation first
+
+
+def test_lmhead_verify_rejects_bad_mode_or_k(L):
+    f = L.ee_lmhead_verify
+    def call(mode, k):
+        return f(FAKE, FAKE, 64, 100, FAKE, FAKE, FAKE, FAKE, FAKE, None, 1, 4, 4, mode, k,
+                 FAKE, None, None, None, FAKE, FAKE, FAKE, None, FAKE, 1 << 30, None)
+    assert call(4, 3) == 1 and call(-1, 3) == 1          # no such mode
+    assert call(2, 0) == 1 and call(2, 9) == 1           # k out of 1..8
+    assert call(3, 1) == 1                               # entropy needs k >= 2 (ln k > 0)
 
 
 def test_attn_plan_rejects_bad_args(L):

@@ -105,6 +105,8 @@ class Workload:
     v_cache: torch.Tensor        # [L, num_pages, n_kv, PAGE, d]
     hidden_states: torch.Tensor  # [sum T, H]
     lm_w: torch.Tensor           # [V, H]
+    # edit content: 1 for generated-branch nodes, 0 for the reuse chain (host numpy uint8 [sum T])
+    gen_mask: np.ndarray = None
 
     @property
     def total_nodes(self) -> int:
@@ -289,10 +291,15 @@ def _randn_bf16(gen, shape, std, device, chunk_rows=None):
     return out
 
 
-def _lm_inputs(gen, rng, V, H, total, planted_argmax, draft_tok, dup_rows, plant_scale, device):
+def _lm_inputs(gen, rng, V, H, total, planted_argmax, draft_tok, dup_rows, plant_scale, device,
+               extra=None):
     """LM-head weight W ~ N(0, 0.02^2) and hidden states.  A planted node's hidden
     state is plant_scale * (unit vector along W[target]) + N(0, 1) noise, so its
-    target wins by a wide logit margin; other nodes get pure noise."""
+    target wins by a wide logit margin; other nodes get pure noise.  ``extra``
+    maps a node to (tokens, logits): its hidden state is then replaced by the
+    least-squares vector h = W_P^T (W_P W_P^T)^-1 L that gives exactly those
+    logits to those tokens (W_P their rows), plus N(0, 0.05^2) noise -- ranked
+    planting with controlled gaps."""
     lm_w = _randn_bf16(gen, (V, H), 0.02, device, chunk_rows=16384)
     if dup_rows:
         # exact ties: a planted target row is copied to a higher, unused token id
@@ -314,12 +321,18 @@ def _lm_inputs(gen, rng, V, H, total, planted_argmax, draft_tok, dup_rows, plant
         unit = rows / rows.norm(dim=1, keepdim=True)
         sel = torch.as_tensor(idx, device=device, dtype=torch.long)
         hidden[sel] = hidden[sel] + plant_scale * unit
+    for node, (toks, lgts) in sorted((extra or {}).items()):
+        wp = lm_w[torch.as_tensor(toks, device=device, dtype=torch.long)].double()
+        lv = torch.as_tensor(lgts, device=device, dtype=torch.float64)
+        h = wp.T @ torch.linalg.solve(wp @ wp.T, lv)
+        hidden[node] = h.float() + 0.05 * torch.randn(H, generator=gen, device=device)
     return lm_w, hidden.to(torch.bfloat16)
 
 
 def build(name: str, seed: int | None = None, device="cpu", *, q_std: float = 1.0,
           plant_scale: float = 12.0, noise_frac: float = 0.1, max_matches: int = 8,
-          dup_rows: int = 0, lm_head: bool | None = None, **overrides) -> Workload:
+          dup_rows: int = 0, lm_head: bool | None = None, verify_plant: bool = False,
+          **overrides) -> Workload:
     """Draw one workload.
 
     ``name`` is one of CONFIG_NAMES; ``seed`` defaults to 1234 + the config's
@@ -329,7 +342,13 @@ def build(name: str, seed: int | None = None, device="cpu", *, q_std: float = 1.
     the softmax peaky).  ``dup_rows`` > 0 copies that many planted target rows of
     the LM-head weight to a higher token id, creating exact logit ties.
     ``lm_head`` (default: every configuration but the sweep) draws the LM-head
-    weight and hidden states; without it both are None.
+    weight and hidden states; without it both are None.  ``verify_plant`` puts
+    the draft token of every generated node on a planted path at rank 0, 1 or 2
+    of its parent's distribution, between decoy tokens: exact logits top, top -
+    gap, top - 2 gap, ... with top = ln(V) + 8 and gap 0.1, 0.6 or 3.0 (so the
+    entropy-aware rule meets near-uniform, medium and peaked positions);
+    planted_accept / planted_path then describe the greedy rule only up to the
+    first edge planted below rank 0.
     """
     if seed is None:
         seed = BASE_SEED + CONFIG_NAMES.index(name)
@@ -397,6 +416,32 @@ def build(name: str, seed: int | None = None, device="cpu", *, q_std: float = 1.
     planted_argmax = np.concatenate(tgts).astype(np.int32)
     planted_accept = np.asarray([len(p) - 1 for p in paths], dtype=np.int32)
     total = int(node_off[-1])
+    gen_mask = np.concatenate([(np.arange(sp["spec"].T) >= sp["spec"].chain) for sp in seqs]
+                              ).astype(np.uint8)
+    extra = {}
+    if verify_plant:
+        # ranked planting on generated edges of the planted paths: the draft token
+        # gets rank r; decoys fill the other ranks down to r + 2, scales falling by
+        # `gap` per rank
+        for s_i, (sp, pth) in enumerate(zip(seqs, paths)):
+            o = int(node_off[s_i])
+            for a, b in zip(pth[:-1], pth[1:]):
+                if not gen_mask[o + b]:
+                    continue
+                r = int(rng.integers(0, 3))
+                gap = float(rng.choice([0.1, 0.6, 3.0]))
+                avoid = {int(draft_tok[o + b])} | {int(x) for x in draft_tok[o:o + sp["spec"].T]}
+                ranked = []
+                for j in range(r + 3):
+                    if j == r:
+                        ranked.append(int(draft_tok[o + b]))
+                    else:
+                        t = _distinct_token(rng, V, avoid)
+                        avoid.add(t)
+                        ranked.append(t)
+                planted_argmax[o + a] = ranked[0]
+                top = math.log(V) + 8.0
+                extra[o + a] = (ranked, [top - gap * j for j in range(len(ranked))])
 
     # --- paged KV layout: ctx + T slots per sequence, random page order -----
     ctx_len = np.asarray([sp["ctx"] for sp in seqs], dtype=np.int32)
@@ -427,7 +472,7 @@ def build(name: str, seed: int | None = None, device="cpu", *, q_std: float = 1.
     lm_w = hidden_states = None
     if lm_head:
         lm_w, hidden_states = _lm_inputs(gen, rng, V, H, total, planted_argmax, draft_tok,
-                                         dup_rows, plant_scale, device)
+                                         dup_rows, plant_scale, device, extra)
 
     return Workload(
 
@@ -439,7 +484,7 @@ def build(name: str, seed: int | None = None, device="cpu", *, q_std: float = 1.
         planted_argmax=planted_argmax, planted_accept=planted_accept, planted_path=paths,
         ctx_len=ctx_len, block_table=block_table, num_pages=num_pages,
         q=q, k_tree=k_tree, v_tree=v_tree, k_cache=k_cache, v_cache=v_cache,
-        hidden_states=hidden_states, lm_w=lm_w,
+        hidden_states=hidden_states, lm_w=lm_w, gen_mask=gen_mask,
     )
 
 
