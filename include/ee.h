@@ -31,7 +31,7 @@
  *  - `ws` is a caller-owned device workspace of at least
  *    ee_workspace_size(...) bytes, zeroed once with ee_workspace_init() before
  *    first use: a 16.5 KB head (the error word and the LM head's running
- *    argmax), 2.7 MB of LM-head verification partials and thresholds, then the attention's
+ *    argmax), 3.1 MB of LM-head verification partials and thresholds, then the attention's
  *    per-CTA partial results (65 KB per CTA, B x n_q x 16 CTAs at most).
  *    Its first word is the device error word: kernels never trap;
  *    on a bad index found on the device they set an EE_DEVERR_* bit there,
@@ -87,7 +87,7 @@ const char* ee_status_string(ee_status s);
  * Workspace bytes needed by every entry point for problems up to these sizes:
  * B sequences, total_nodes tree nodes in all, n_q query heads, max_ctx cached
  * positions in the longest sequence.  The buffer must be 256-byte aligned.
- * 2,908,672 bytes when max_ctx is 0, else 2,908,672 + B * n_q * 16 * 66,816
+ * 3,219,968 bytes when max_ctx is 0, else 3,219,968 + B * n_q * 16 * 66,816
  * (the attention's partial slots; about 30 MB for one sequence with 28 heads).
  * Returns 0 for negative arguments.
  */

@@ -36,7 +36,9 @@ constexpr int kNumSMsMax = 152;       // LM-head grid bound (one persistent CTA 
 constexpr int kLmMaxK = 8;
 constexpr int kLmMaxBN = 256;
 constexpr size_t kLmVerifyOff = kWorkspaceBytes;
-constexpr size_t kLmPartBytes = (size_t)kNumSMsMax * kLmMaxBN * (8 * kLmMaxK + 8);
+// one (CTA, node) record: K values, K ids, (max, sum), padded to 16 bytes
+__host__ __device__ constexpr int lm_rec_bytes(int K) { return (8 * K + 8 + 15) / 16 * 16; }
+constexpr size_t kLmPartBytes = (size_t)kNumSMsMax * kLmMaxBN * lm_rec_bytes(kLmMaxK);
 // then one u64 per node: the best K-th key any CTA has published (zero between
 // calls); then the finalize step's ranked ids [node][K] and top_tau [node]
 constexpr size_t kLmGthrOff = kLmPartBytes;

@@ -558,12 +558,10 @@ lmhead_accept_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_const
         if (node < p.total_nodes && b.i != 0x7fffffff) atomicMax(&p.keys[node], make_key(b.v, b.i));
         if (kVerify) {
           // this CTA's partial for the node: the 4 warps' lists merged, their sums added
-          float* pv = reinterpret_cast<float*>(p.part + (size_t)blockIdx.x * BN * (8 * K + 8)) +
-                      (size_t)c * K;
-          int* pi = reinterpret_cast<int*>(p.part + (size_t)blockIdx.x * BN * (8 * K + 8) +
-                                           (size_t)BN * K * 4) + (size_t)c * K;
-          float2* pl = reinterpret_cast<float2*>(p.part + (size_t)blockIdx.x * BN * (8 * K + 8) +
-                                                 (size_t)BN * K * 8) + c;
+          uint8_t* rec = p.part + ((size_t)blockIdx.x * BN + c) * lm_rec_bytes(K);
+          float* pv = reinterpret_cast<float*>(rec);
+          int* pi = reinterpret_cast<int*>(rec + 4 * K);
+          float2* pl = reinterpret_cast<float2*>(rec + 8 * K);
           int hs[4] = {0, 0, 0, 0};   // next entry of each warp's sorted list
           for (int rr = 0; rr < K; ++rr) {
             int wb = -1;
@@ -672,6 +670,7 @@ struct FinParams {
   AcceptArgs acc;
 };
 
+template <int K>
 __global__ void __launch_bounds__(32 * kFinWarps, 1) lm_verify_finalize_kernel(const FinParams p) {
   ee::pdl_allow_next();
   ee::pdl_wait();   // the LM head's partials, thresholds and argmax are complete
@@ -680,33 +679,39 @@ __global__ void __launch_bounds__(32 * kFinWarps, 1) lm_verify_finalize_kernel(c
   __shared__ int s_svn[kFinWarps];
   __shared__ int s_last;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int K = p.K, BN = p.BN;
+  const int BN = p.BN;
   const int node = blockIdx.x * kFinWarps + warp;
   if (node < p.total) {
     const int nt = node / BN, c = node - nt * BN;
-    const size_t pstride = (size_t)BN * (8 * K + 8);
+    constexpr int kRec = lm_rec_bytes(K) / 16;   // 16-byte words per (CTA, node) record
     // the best K-th key any CTA published: at most the node's true K-th best,
     // so only entries reaching it can be among the K best
     const unsigned long long g = __ldcg(p.gthr + node);
     constexpr int kMaxU = (kNumSMsMax + 31) / 32;
-    float cv[kMaxU][kLmMaxK];
-    int ci[kMaxU][kLmMaxK];
+    float cv[kMaxU][K];
+    int ci[kMaxU][K];
     float2 xs[kMaxU];
-    // every partial of the node: lane l takes source CTAs l, l + 32, ...;
-    // unconditional loads from always-valid addresses (source 0 and entry K - 1
-    // stand in for absent ones), masked afterwards, so that all are in flight
+    // every record of the node: lane l takes source CTAs l, l + 32, ...; all
+    // loads are unconditional (source 0 stands in for absent ones) and in flight
+    // together, the absent ones masked afterwards
+    uint4 w[kMaxU][kRec];
 #pragma unroll
     for (int u = 0; u < kMaxU; ++u) {
       const int q2 = lane + 32 * u;
-      const uint8_t* pc = p.part + (size_t)(q2 < p.n_src ? q2 * p.n_nt + nt : nt) * pstride;
-      xs[u] = __ldcg(reinterpret_cast<const float2*>(pc + (size_t)BN * K * 8) + c);
-      const float* pv = reinterpret_cast<const float*>(pc) + (size_t)c * K;
-      const int* pi = reinterpret_cast<const int*>(pc + (size_t)BN * K * 4) + (size_t)c * K;
+      const uint4* rec = reinterpret_cast<const uint4*>(
+          p.part + ((size_t)(q2 < p.n_src ? q2 * p.n_nt + nt : nt) * BN + c) * lm_rec_bytes(K));
 #pragma unroll
-      for (int rr = 0; rr < kLmMaxK; ++rr) {
-        cv[u][rr] = __ldcg(pv + min(rr, K - 1));
-        ci[u][rr] = __ldcg(pi + min(rr, K - 1));
+      for (int t = 0; t < kRec; ++t) w[u][t] = __ldcg(rec + t);
+    }
+#pragma unroll
+    for (int u = 0; u < kMaxU; ++u) {
+      const uint32_t* ww = reinterpret_cast<const uint32_t*>(w[u]);
+#pragma unroll
+      for (int rr = 0; rr < K; ++rr) {
+        cv[u][rr] = __uint_as_float(ww[rr]);
+        ci[u][rr] = (int)ww[K + rr];
       }
+      xs[u] = make_float2(__uint_as_float(ww[2 * K]), __uint_as_float(ww[2 * K + 1]));
     }
     float m = -INFINITY, sm = 0.f;
 #pragma unroll
@@ -714,8 +719,8 @@ __global__ void __launch_bounds__(32 * kFinWarps, 1) lm_verify_finalize_kernel(c
       const bool valid = lane + 32 * u < p.n_src;
       if (valid) lse_add(m, sm, xs[u].x, xs[u].y);
 #pragma unroll
-      for (int rr = 0; rr < kLmMaxK; ++rr)
-        if (!valid || rr >= K) {
+      for (int rr = 0; rr < K; ++rr)
+        if (!valid) {
           cv[u][rr] = -INFINITY;
           ci[u][rr] = 0x7fffffff;
         }
@@ -735,7 +740,7 @@ __global__ void __launch_bounds__(32 * kFinWarps, 1) lm_verify_finalize_kernel(c
 #pragma unroll
     for (int u = 0; u < kMaxU; ++u)
 #pragma unroll
-      for (int rr = 0; rr < kLmMaxK; ++rr)
+      for (int rr = 0; rr < K; ++rr)
         if (ci[u][rr] != 0x7fffffff && make_key(cv[u][rr], ci[u][rr]) >= g) {
           const int pos = atomicAdd(&s_svn[warp], 1);
           if (pos < kSurv) {
@@ -748,17 +753,16 @@ __global__ void __launch_bounds__(32 * kFinWarps, 1) lm_verify_finalize_kernel(c
     const bool few = n_sv <= kSurv;
     // overflow (not seen with a published threshold): each lane merges its own
     // sorted source lists, then the warp takes the K best of the lane heads
-    float lv[kLmMaxK];
-    int li[kLmMaxK];
+    float lv[K];
+    int li[K];
 #pragma unroll
-    for (int t = 0; t < kLmMaxK; ++t) {
+    for (int t = 0; t < K; ++t) {
       lv[t] = -INFINITY;
       li[t] = 0x7fffffff;
     }
     if (!few) {
 #pragma unroll
-      for (int rr = 0; rr < kLmMaxK; ++rr) {
-        if (rr >= K) break;
+      for (int rr = 0; rr < K; ++rr) {
         int wu = 0;
         float bv = cv[0][0];
         int bi = ci[0][0];
@@ -775,12 +779,12 @@ __global__ void __launch_bounds__(32 * kFinWarps, 1) lm_verify_finalize_kernel(c
         for (int u = 0; u < kMaxU; ++u) {
           if (u != wu) continue;
 #pragma unroll
-          for (int t = 0; t < kLmMaxK - 1; ++t) {
+          for (int t = 0; t < K - 1; ++t) {
             cv[u][t] = cv[u][t + 1];
             ci[u][t] = ci[u][t + 1];
           }
-          cv[u][kLmMaxK - 1] = -INFINITY;
-          ci[u][kLmMaxK - 1] = 0x7fffffff;
+          cv[u][K - 1] = -INFINITY;
+          ci[u][K - 1] = 0x7fffffff;
         }
       }
     }
@@ -807,12 +811,12 @@ __global__ void __launch_bounds__(32 * kFinWarps, 1) lm_verify_finalize_kernel(c
         warp_best(lv[0], li[0], &xv, &xi);
         if (xi != 0x7fffffff && li[0] == xi && lv[0] == xv) {   // this lane held it: next one up
 #pragma unroll
-          for (int t = 0; t < kLmMaxK - 1; ++t) {
+          for (int t = 0; t < K - 1; ++t) {
             lv[t] = lv[t + 1];
             li[t] = li[t + 1];
           }
-          lv[kLmMaxK - 1] = -INFINITY;
-          li[kLmMaxK - 1] = 0x7fffffff;
+          lv[K - 1] = -INFINITY;
+          li[K - 1] = 0x7fffffff;
         }
       }
       const float pr = ex2f((xv - lse) * kLog2e);
@@ -971,7 +975,7 @@ ee_status launch_lmhead(const ee_bf16* hidden, const ee_bf16* lm_w, int32_t hidd
   int grid = (ee::kNumSMs / p.n_nt) * p.n_nt;   // multiple of n_nt: each CTA keeps one node tile
   if (grid > num_tiles) grid = num_tiles;
   if (grid < 1) grid = 1;
-  if (va && (size_t)grid * p.BN * (8 * K + 8) > ee::kLmPartBytes) return EE_ERR_UNSUPPORTED;
+  if (va && (size_t)grid * p.BN * ee::lm_rec_bytes(K) > ee::kLmPartBytes) return EE_ERR_UNSUPPORTED;
   if (va) {
     EE_CUDA_OK(ee::launch_pdl(lmhead_accept_kernel<true>, dim3(grid), dim3(kThreads), smem_acc,
                               (cudaStream_t)stream, 1, tmW, tmX, p));
@@ -995,8 +999,20 @@ ee_status launch_lmhead(const ee_bf16* hidden, const ee_bf16* lm_w, int32_t hidd
     fp.ticket = va->fin_ticket;
     fp.acc = AcceptArgs{B, max_T, total_nodes, va->mode, K, node_off, parent, draft_tok, depth, anc,
                         va->gen_mask, accept_len, path, bonus, err};
-    EE_CUDA_OK(ee::launch_pdl(lm_verify_finalize_kernel, dim3((total_nodes + kFinWarps - 1) / kFinWarps),
-                              dim3(32 * kFinWarps), 0, (cudaStream_t)stream, 1, fp));
+    const dim3 fg((total_nodes + kFinWarps - 1) / kFinWarps), fb(32 * kFinWarps);
+    cudaError_t fe = cudaErrorInvalidValue;
+    switch (K) {
+#define EE_FIN_CASE(n) \
+  case n:              \
+    fe = ee::launch_pdl(lm_verify_finalize_kernel<n>, fg, fb, 0, (cudaStream_t)stream, 1, fp); \
+    break;
+      EE_FIN_CASE(1) EE_FIN_CASE(2) EE_FIN_CASE(3) EE_FIN_CASE(4)
+      EE_FIN_CASE(5) EE_FIN_CASE(6) EE_FIN_CASE(7) EE_FIN_CASE(8)
+#undef EE_FIN_CASE
+      default:
+        break;
+    }
+    EE_CUDA_OK(fe);
   } else if (pdl) {
     EE_CUDA_OK(ee::launch_pdl(lmhead_accept_kernel<false>, dim3(grid), dim3(kThreads), smem_acc,
                               (cudaStream_t)stream, 1, tmW, tmX, p));
