@@ -13,15 +13,19 @@
 //     the last chunk also processes the tree keys (one 128-key tile), masked by
 //     the ancestor bitmask.  A CTA first stages its chunk's page ids in shared
 //     memory.
-//   - Q lives in TMEM (bf16 pairs, loaded by the softmax threads, one row each)
-//     and is the A operand of S = Q K^T, so shared memory holds only K and V.
+//   - Q lives in shared memory (the softmax threads load the block's rows
+//     coalesced and store them in the 128-byte-swizzled K-major layout TMA
+//     gives the K tiles) and is the A operand of S = Q K^T; TMEM holds three S
+//     buffers and O (4 x 128 fp32 columns).
 //   - Keys come in 128-key tiles.  Warps 0 and 2 stream K and V tiles with TMA
 //     (one 16-row box per page and 64-dim half, spread over 8 lanes; the tree's
-//     K/V through a 3-D map) into two 3-stage rings.  Warp 1 issues
-//     tcgen05.mma in a fixed order: S = Q K^T (bf16, fp32 accumulators in TMEM,
-//     double buffered), then for each tile O += P V, then the Q K^T two tiles
-//     ahead, which overwrites the TMEM columns P lived in (the in-order tensor
-//     pipe finishes reading P first).
+//     K/V through a 3-D map) into a 3-stage K ring and a 2-stage V ring.  Warp
+//     1 issues tcgen05.mma in a fixed order: S = Q K^T for the first three
+//     tiles (bf16, fp32 accumulators in TMEM), then for each tile O += P V
+//     followed by the Q K^T three tiles ahead, which overwrites the TMEM
+//     columns P lived in (the in-order tensor pipe finishes reading P first).
+//     With three S buffers the hand-off chain P(t) -> P.V(t) -> Q.K^T(t+3) ->
+//     softmax(t+3) spans three tiles, so it no longer sets the tile period.
 //   - P.V runs on bf16 operands: P is split exactly into a bf16 head (the top
 //     16 bits of the fp32 value) and a bf16 tail (the top 16 bits of the
 //     remainder), both written over S in TMEM and used as the MMA A operand;
@@ -53,7 +57,8 @@
 //   - The next kernel in the stream may launch (programmatic dependent launch)
 //     once every CTA has drained its pipeline; triggering earlier lets its
 //     CTAs hold SMs that a later wave of this grid still needs.
-// Shared-memory traffic per 128-key tile: K 64 KB + V 64 KB (TMA write, MMA read).
+// Shared-memory traffic per 128-key tile: K 64 KB + V 64 KB (TMA write, MMA
+// read) + Q 32 KB (MMA read).
 #include "ee_common.cuh"
 #include "ee_ptx.cuh"
 
@@ -66,19 +71,20 @@ constexpr int kRows = 128;                       // query rows per CTA (MMA M)
 constexpr int kKT = 128;                         // keys per tile (MMA N of Q K^T, K of P V)
 constexpr int kD = EE_HEAD_DIM;                  // 128
 constexpr int kKST = 3;                          // K ring depth
-constexpr int kVST = 3;                          // V ring depth
+constexpr int kVST = 2;                          // V ring depth
+constexpr int kSB = 3;                           // S buffers in TMEM (Q.K^T runs kSB tiles ahead)
 constexpr uint32_t kKVHalf = kKT * 128;          // 16 KB: one 64-dim half of a K or V tile
 constexpr uint32_t kKVBytes = 2 * kKVHalf;       // 32 KB
 constexpr int kMaxCtaPages = 2048;               // context pages one CTA can own (32768 keys)
 constexpr uint32_t kOffK = 0;
 constexpr uint32_t kOffV = kOffK + kKST * kKVBytes;
-constexpr uint32_t kOffPages = kOffV + kVST * kKVBytes;
+constexpr uint32_t kOffQ = kOffV + kVST * kKVBytes;  // Q block, 128 rows x 128 bf16, SW128 K-major
+constexpr uint32_t kOffPages = kOffQ + kKVBytes;
 constexpr uint32_t kOffBar = kOffPages + 4 * kMaxCtaPages;
-constexpr uint32_t kNumBars = 2 * kKST + 2 * kVST + 3 * 2 + 2;
+constexpr uint32_t kNumBars = 2 * kKST + 2 * kVST + 2 * kSB + 2 + 2;
 constexpr uint32_t kSmemBytes = 1024 + kOffBar + 8 * kNumBars + 64;
-constexpr uint32_t kTmemCols = 512;              // S0 [0,128) S1 [128,256) O [256,384) Q [384,448)
-constexpr uint32_t kColO = 256;
-constexpr uint32_t kColQ = 384;
+constexpr uint32_t kTmemCols = 512;              // S0 [0,128) S1 [128,256) S2 [256,384) O [384,512)
+constexpr uint32_t kColO = 384;
 constexpr float kRescaleLog2 = 8.0f;
 constexpr int kMaxCluster = 8;                   // portable thread-block cluster size
 constexpr int kMaxSplits = ee::kAttnMaxSplits;   // chunks per row block (cooperative launch)
@@ -205,7 +211,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
   const uint32_t bar0 = sbase + kOffBar;
   const uint32_t k_full = bar0, k_empty = k_full + 8 * kKST;
   const uint32_t v_full = k_empty + 8 * kKST, v_empty = v_full + 8 * kVST;
-  const uint32_t s_full = v_empty + 8 * kVST, p_full = s_full + 16, o_done = p_full + 16;
+  const uint32_t s_full = v_empty + 8 * kVST, p_full = s_full + 8 * kSB, o_done = p_full + 8 * kSB;
   const uint32_t drain = o_done + 16, q_ready = drain + 8;
 
   // on-chip set-up first: it touches no global memory, so it overlaps the end
@@ -226,11 +232,11 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
       mbar_init(v_empty + 8 * i, 1);
       s_vissued[i] = -1;
     }
-    for (int i = 0; i < 2; ++i) {
+    for (int i = 0; i < kSB; ++i) {
       mbar_init(s_full + 8 * i, 1);
       mbar_init(p_full + 8 * i, 2 * kRows);
-      mbar_init(o_done + 8 * i, 1);
     }
+    for (int i = 0; i < 2; ++i) mbar_init(o_done + 8 * i, 1);
     mbar_init(drain, 1);
     mbar_init(q_ready, 2 * kRows);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -344,7 +350,6 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
       bool go = true;
       if (lane == 0) go = mbar_wait(empty0 + 8 * st, (uint32_t)(use & 1) ^ 1u, &s_abort);
       // the last V stage holds the staged Q rows until they are in TMEM
-      if (!isK && st == kVST - 1 && use == 0 && lane == 0) go = go && mbar_wait(q_ready, 0, &s_abort);
       if (!__shfl_sync(0xffffffffu, go, 0)) break;
       const uint32_t full = full0 + 8 * st;
       const uint32_t dst = ring + st * kKVBytes;
@@ -369,10 +374,11 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
       if (lane == 0) issued[st] = use;
     }
   } else if (warp == kWarpMma) {
-    // ---------------- MMA issuer: Q.K^T(0), Q.K^T(1), then P.V(t), Q.K^T(t+2) ----------------
+    // ---------- MMA issuer: Q.K^T(0..kSB-1), then P.V(t), Q.K^T(t+kSB) ----------
     if (lane == 0) {
       tc_fence_after();
       const uint32_t id_qk = idesc_f16(kRows, kKT, 1, 1, 0);
+      const uint32_t sQ = sbase + kOffQ;
       const uint32_t id_pv = idesc_f16(kRows, kD, 1, 1, 1);
       auto issue_qk = [&](int t) -> bool {
         if (!mbar_wait(k_full + 8 * (t % kKST), (uint32_t)((t / kKST) & 1), &s_abort)) return false;
@@ -381,21 +387,21 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
 #pragma unroll
         for (int kk = 0; kk < kD / 16; ++kk) {
           const uint32_t off = (kk & 3) * 32;
-          tc_mma_ts(tmem + (t & 1) * kKT, tmem + kColQ + 8 * kk,
-                    smem_desc_sw128(kb + (kk >> 2) * kKVHalf + off), id_qk, kk > 0 ? 1u : 0u);
+          tc_mma(tmem + (t % kSB) * kKT, smem_desc_sw128(sQ + (kk >> 2) * kKVHalf + off),
+                 smem_desc_sw128(kb + (kk >> 2) * kKVHalf + off), id_qk, kk > 0 ? 1u : 0u);
         }
         tc_commit(k_empty + 8 * (t % kKST));
-        tc_commit(s_full + 8 * (t & 1));
+        tc_commit(s_full + 8 * (t % kSB));
         return true;
       };
       bool ok = mbar_wait(q_ready, 0, &s_abort);
-      ok = ok && (n_tiles < 1 || issue_qk(0)) && (n_tiles < 2 || issue_qk(1));
+      for (int t = 0; t < kSB && t < n_tiles && ok; ++t) ok = issue_qk(t);
       for (int t = 0; t < n_tiles && ok; ++t) {
-        if (!mbar_wait(p_full + 8 * (t & 1), (uint32_t)((t >> 1) & 1), &s_abort) ||
+        if (!mbar_wait(p_full + 8 * (t % kSB), (uint32_t)((t / kSB) & 1), &s_abort) ||
             !mbar_wait(v_full + 8 * (t % kVST), (uint32_t)((t / kVST) & 1), &s_abort))
           break;
         tc_fence_after();
-        const uint32_t pa = tmem + (t & 1) * kKT;          // bf16 P head: cols 0..63, tail: 64..127
+        const uint32_t pa = tmem + (t % kSB) * kKT;        // bf16 P head: cols 0..63, tail: 64..127
         const uint32_t vb = sV + (t % kVST) * kKVBytes;
 #pragma unroll
         for (int part = 0; part < 2; ++part)
@@ -406,7 +412,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
                       (t > 0 || part > 0 || j > 0) ? 1u : 0u);
         tc_commit(v_empty + 8 * (t % kVST));
         tc_commit(o_done + 8 * (t & 1));
-        if (t + 2 < n_tiles) ok = issue_qk(t + 2);
+        if (t + kSB < n_tiles) ok = issue_qk(t + kSB);
       }
     }
   } else if (warp >= kWarpSoft0) {
@@ -428,32 +434,22 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
     const int node = vrow ? rr / p.g : 0;
     const uint64_t ancw = vrow ? p.anc[2 * (size_t)(o + node) + hf] : 0ull;   // this half's tree keys
     const uint32_t tl = tmem + ((uint32_t)(qd * 32) << 16);
-    // this row of Q into TMEM columns kColQ + 32 hf.. (bf16 pairs of this half's
-    // 64 dims), zeros for rows past R.  The block's rows, loaded before the
-    // barrier, go through the last V stage (which the V producer fills only
-    // after q_ready): chunk c of row r sits at 16 * (c ^ (r & 15)), so that each
-    // thread then reads its own row without bank conflicts.
+    // the block's Q rows into shared memory as the A operand of Q.K^T: 128 rows
+    // x 128 bf16 in two 64-column slabs, 128-byte swizzled K-major (the layout
+    // TMA gives the K tiles): 16-byte chunk j of row r at slab (j / 8),
+    // (r / 8) * 1024 + (r % 8) * 128 + ((j % 8) ^ (r % 8)) * 16; rows past R are
+    // zero.  The rows were loaded (coalesced) before the set-up barrier.
     {
-      uint8_t* qs = smem + kOffV + (kVST - 1) * kKVBytes;
+      uint8_t* qs = smem + kOffQ;
 #pragma unroll
       for (int k = 0; k < kRows / 16; ++k) {
         const int rq = 2 * ((warp - kWarpSoft0) + 8 * k) + qhalf;
-        *reinterpret_cast<uint4*>(qs + rq * 256 + 16 * (qc ^ (rq & 15))) =
+        const int j = qc & 7;
+        *reinterpret_cast<uint4*>(qs + (qc >> 3) * kKVHalf + (rq >> 3) * 1024 + (rq & 7) * 128 +
+                                  ((j ^ (rq & 7)) << 4)) =
             rb * kRows + rq < R ? qv[k] : make_uint4(0u, 0u, 0u, 0u);
       }
-      asm volatile("bar.sync 1, %0;" ::"n"(kSoftThreads) : "memory");   // the eight softmax warps
-      uint32_t qw[32];
-#pragma unroll
-      for (int c = 0; c < 8; ++c) {
-        const int ch = 8 * hf + c;
-        const uint4 v = *reinterpret_cast<const uint4*>(qs + r * 256 + 16 * (ch ^ (r & 15)));
-        qw[4 * c] = v.x;
-        qw[4 * c + 1] = v.y;
-        qw[4 * c + 2] = v.z;
-        qw[4 * c + 3] = v.w;
-      }
-      tc_st32(tl + kColQ + 32 * hf, qw);
-      tc_fence_before();
+      fence_async_smem();   // generic-proxy writes, read by the tensor core
       mbar_arrive(q_ready);
     }
     // m_used is kept in raw score units (scale > 0, so the max commutes with it)
@@ -462,11 +458,12 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
     const float kFail = __int_as_float(0x7fffffff);   // NaN: "this half's wait failed"
     bool ok = true;
     for (int t = 0; t < n_tiles; ++t) {
-      const int sb = t & 1;
+      const int sb = t % kSB;     // S buffer of this tile
+      const int xb = t & 1;       // pair-exchange slot
       // wait outcomes are warp-uniform: the TMEM accesses that follow are
       // warp-collective (.sync.aligned)
       const bool got =
-          __all_sync(0xffffffffu, mbar_wait(s_full + 8 * sb, (uint32_t)((t >> 1) & 1), &s_abort));
+          __all_sync(0xffffffffu, mbar_wait(s_full + 8 * sb, (uint32_t)((t / kSB) & 1), &s_abort));
       uint32_t sr[64];
       float tmax = -INFINITY;
       if (got) {
@@ -502,11 +499,11 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
       }
       // the pair swaps its halves' maxima; both S halves are in registers before
       // either warp overwrites S with P
-      s_xmax[sb][hf][r] = got ? tmax : kFail;
+      s_xmax[xb][hf][r] = got ? tmax : kFail;
       tc_fence_before();
       asm volatile("bar.sync %0, 64;" ::"r"(pair_bar) : "memory");
       tc_fence_after();
-      const float other = s_xmax[sb][hf ^ 1][r];
+      const float other = s_xmax[xb][hf ^ 1][r];
       if (!__all_sync(0xffffffffu, got && other == other)) {
         ok = false;
         break;
@@ -518,7 +515,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
         // O must hold P.V(t-1) before this half's columns are rescaled; a failed
         // wait sets the abort flag, and the pair stops at the next barrier
         if (__all_sync(0xffffffffu,
-                       mbar_wait(o_done + 8 * (sb ^ 1), (uint32_t)(((t - 1) >> 1) & 1), &s_abort))) {
+                       mbar_wait(o_done + 8 * ((t - 1) & 1), (uint32_t)(((t - 1) >> 1) & 1), &s_abort))) {
           tc_fence_after();
           const float f = need ? ex2((m_used - m_new) * sl2) : 1.f;
 #pragma unroll 1
