@@ -538,23 +538,38 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
       // p = 2^(s*scale_log2 - m); P = head + tail, both bf16 (top 16 bits): this
       // half's head pairs go to columns 32 hf.. of the S buffer, its tail pairs
       // to 64 + 32 hf..
-      float ls[8];
+      // (pairs of columns run on packed fp32x2 arithmetic: the scale-and-shift,
+      // the running sums and the tail subtraction take one instruction per pair)
+      const uint64_t sl2x2 = f2_pack(__float_as_uint(sl2), __float_as_uint(sl2));
+      const uint64_t nmsx2 = f2_pack(__float_as_uint(nms), __float_as_uint(nms));
+      uint64_t ls2[4];
       uint32_t hw[32], tw[32];
 #pragma unroll
       for (int e = 0; e < 32; ++e) {
-        const float p0 = ex2(fmaf(__uint_as_float(sr[2 * e]), sl2, nms));
-        const float p1 = ex2(fmaf(__uint_as_float(sr[2 * e + 1]), sl2, nms));
-        if (e < 8) ls[e] = p0 + p1; else ls[e & 7] += p0 + p1;
-        const uint32_t h0 = __float_as_uint(p0) & 0xFFFF0000u;
-        const uint32_t h1 = __float_as_uint(p1) & 0xFFFF0000u;
-        const uint32_t t0 = __float_as_uint(p0 - __uint_as_float(h0));
-        const uint32_t t1 = __float_as_uint(p1 - __uint_as_float(h1));
+        uint32_t y0, y1;
+        f2_unpack(f2_fma(f2_pack(sr[2 * e], sr[2 * e + 1]), sl2x2, nmsx2), y0, y1);
+        const uint32_t p0 = __float_as_uint(ex2(__uint_as_float(y0)));
+        const uint32_t p1 = __float_as_uint(ex2(__uint_as_float(y1)));
+        const uint64_t pp = f2_pack(p0, p1);
+        ls2[e & 3] = e < 4 ? pp : f2_add(ls2[e & 3], pp);
+        const uint32_t h0 = p0 & 0xFFFF0000u;
+        const uint32_t h1 = p1 & 0xFFFF0000u;
+        uint32_t t0, t1;
+        f2_unpack(f2_sub(pp, f2_pack(h0, h1)), t0, t1);
         hw[e] = __byte_perm(h0, h1, 0x7632);
         tw[e] = __byte_perm(t0, t1, 0x7632);
       }
       tc_st32(tl + sb * kKT + 32 * hf, hw);
       tc_st32(tl + sb * kKT + 64 + 32 * hf, tw);
-      l += ((ls[0] + ls[1]) + (ls[2] + ls[3])) + ((ls[4] + ls[5]) + (ls[6] + ls[7]));
+      {
+        uint32_t a0, a1, b0, b1, c0, c1, d0, d1;
+        f2_unpack(ls2[0], a0, a1);
+        f2_unpack(ls2[1], b0, b1);
+        f2_unpack(ls2[2], c0, c1);
+        f2_unpack(ls2[3], d0, d1);
+        l += ((__uint_as_float(a0) + __uint_as_float(a1)) + (__uint_as_float(b0) + __uint_as_float(b1))) +
+             ((__uint_as_float(c0) + __uint_as_float(c1)) + (__uint_as_float(d0) + __uint_as_float(d1)));
+      }
       tc_fence_before();
       mbar_arrive(p_full + 8 * sb);
     }
