@@ -466,16 +466,42 @@ def run_instrumented(st, stream, evs):
                   st.ctx_out, x["node_off"], st.path, st.accept_len, st.dst_slot, st.ws, stream)
 
 
+def _clone_step(st):
+    """A second VerifyStep with its own per-step input buffers, outputs and
+    workspace, sharing the resident state (KV cache, block table, original code,
+    LM-head weight) -- the second buffer set of the pipelined end-to-end loop."""
+    from paper_2506_02780_gb300 import step as S
+    x = st.inp
+    c = {n: x[n].clone() for n in ("tail", "cursor", "parent", "node_off", "draft_tok", "ctx_len", "q",
+                                    "k_tree", "v_tree", "hidden")}
+    return S.VerifyStep(orig_tokens=x["orig_tokens"], orig_off=x["orig_off"], tail=c["tail"],
+                        cursor=c["cursor"], parent=c["parent"], node_off=c["node_off"],
+                        draft_tok=c["draft_tok"], ctx_len=c["ctx_len"], block_table=x["block_table"],
+                        q=c["q"], k_tree=c["k_tree"], v_tree=c["v_tree"], k_cache=x["k_cache"],
+                        v_cache=x["v_cache"], hidden=c["hidden"], lm_w=x["lm_w"], max_ctx=st.max_ctx,
+                        max_T=st.max_T, max_matches=st.max_matches, keep_layers=False)
+
+
 def run_e2e(st, graph, stream, steps, dev, world):
     """Same metric through the public API with host buffers: every step copies its
     inputs (tail, cursor, tree, per-layer q / tree K/V, hidden states) from pinned
-    host memory, replays the step, reads the results back, and synchronises."""
+    host memory, replays the step and copies its results back to pinned host memory.
+
+    e2e: two buffer sets, as a server interleaving independent batches does --
+    step i+1's input copies run on a copy stream while step i computes, and the
+    host reads step i's results (accept lengths) once they have arrived, one step
+    later.  e2e_serial: one buffer set; copy, replay, read back, synchronise."""
     names_in = ["tail", "cursor", "parent", "node_off", "draft_tok", "ctx_len", "q", "k_tree", "v_tree",
                 "hidden"]
     host_in = {n: st.inp[n].detach().cpu().pin_memory() for n in names_in}
-    outs = [st.accept_len, st.path, st.bonus, st.argmax, st.match_pos, st.n_matches, st.ctx_out]
-    host_out = [torch.empty(o.shape, dtype=o.dtype).pin_memory() for o in outs]
+
+    def outs_of(s):
+        return [s.accept_len, s.path, s.bonus, s.argmax, s.match_pos, s.n_matches, s.ctx_out]
     h2d = sum(t.numel() * t.element_size() for t in host_in.values())
+
+    # serial: one buffer set
+    outs = outs_of(st)
+    host_out = [torch.empty(o.shape, dtype=o.dtype).pin_memory() for o in outs]
     d2h = sum(t.numel() * t.element_size() for t in host_out)
 
     def one():
@@ -494,9 +520,62 @@ def run_e2e(st, graph, stream, steps, dev, world):
     t0 = time.perf_counter()
     for _ in range(steps):
         one()
+    dt_serial = reduce_max(time.perf_counter() - t0, world, dev)
+
+    # pipelined: two buffer sets, copies on their own stream
+    st2 = _clone_step(st)
+    with torch.cuda.stream(stream):
+        st2.run(stream)
+        stream.synchronize()
+        graph2 = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph2, stream=stream):
+            st2.run(stream)
+    stream.synchronize()
+    sets = [(st, graph, outs, host_out), (st2, graph2, outs_of(st2),
+                                          [torch.empty(o.shape, dtype=o.dtype).pin_memory()
+                                           for o in outs_of(st2)])]
+    copy_stream = torch.cuda.Stream(device=dev)
+    copied = [torch.cuda.Event(), torch.cuda.Event()]
+    done = [torch.cuda.Event(), torch.cuda.Event()]
+    seen = []
+
+    def pipelined(n):
+        for i in range(n):
+            j = i % 2
+            s_, g_, o_, ho_ = sets[j]
+            with torch.cuda.stream(copy_stream):
+                if i >= 2:
+                    copy_stream.wait_event(done[j])       # set j's previous step has finished with it
+                for nm in names_in:
+                    s_.inp[nm].copy_(host_in[nm], non_blocking=True)
+                copied[j].record(copy_stream)
+            with torch.cuda.stream(stream):
+                stream.wait_event(copied[j])
+                g_.replay()
+                for ho, o in zip(ho_, o_):
+                    ho.copy_(o, non_blocking=True)
+                done[j].record(stream)
+            if i >= 1:                                     # the previous step's results, on the host
+                k = (i - 1) % 2
+                done[k].synchronize()
+                seen.append(int(sets[k][3][0][0]))
+        done[(n - 1) % 2].synchronize()
+        seen.append(int(sets[(n - 1) % 2][3][0][0]))
+        torch.cuda.synchronize(dev)
+
+    pipelined(6)
+    if world > 1:
+        torch.distributed.barrier()
+    seen.clear()
+    t0 = time.perf_counter()
+    pipelined(steps)
     dt = reduce_max(time.perf_counter() - t0, world, dev)
+    assert len(seen) == steps and len(set(seen)) == 1   # every step's accept length came back
     return {"value": round(world * steps / dt, 2), "unit": UNIT, "h2d_bytes_per_step": int(h2d),
-            "d2h_bytes_per_step": int(d2h), "ms_per_step": round(1e3 * dt / steps, 4)}
+            "d2h_bytes_per_step": int(d2h), "ms_per_step": round(1e3 * dt / steps, 4),
+            "pipelined": "2 buffer sets: step i+1's copies overlap step i's compute",
+            "serial": {"value": round(world * steps / dt_serial, 2),
+                       "ms_per_step": round(1e3 * dt_serial / steps, 4)}}
 
 
 def _config_text(name):
