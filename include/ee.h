@@ -104,6 +104,30 @@ ee_status ee_workspace_init(void* ws, size_t ws_bytes, ee_stream_t stream);
 ee_status ee_read_errors(void* ws, ee_stream_t stream, int32_t* bits);
 
 /*
+ * ee_selftest_timeout -- diagnostic of the device-side failure detection (no
+ * step of the verification path calls it).  Launches one 64-thread CTA that
+ * makes the two kinds of bounded wait the pipelines use run out, without any
+ * fault or trap:
+ *   (a) warp 0 waits on a shared-memory mbarrier that nothing arrives at; it
+ *       gives up after the device wait limit and raises the CTA's abort flag;
+ *   (b) warp 1 starts the same kind of wait half a limit later; it must leave
+ *       through the abort flag raised by (a), before its own limit;
+ *   (c) thread 0 then waits, with acquire loads, for a global counter in the
+ *       workspace head that no launch ever writes (the cross-CTA arrival wait
+ *       of the attention merge), and gives up after the limit.
+ * Then it sets EE_DEVERR_TIMEOUT in the device error word, as every pipeline
+ * does after a wait gave up; ee_read_errors() reports and clears it.  The
+ * call runs for about two wait limits (2 x 2e9 SM cycles, ~2 s at 2.07 GHz).
+ *   out  device int64[7]: [0] the wait limit in SM cycles, [1] result of (a)
+ *        (1 = the wait completed, 0 = it gave up), [2] cycles (a) waited,
+ *        [3] result of (b), [4] cycles (b) waited, [5] result of (c),
+ *        [6] cycles (c) waited.
+ * Errors: EE_ERR_INVALID_ARG for a NULL or misaligned ws or out, or ws_bytes
+ * below the fixed workspace head.
+ */
+ee_status ee_selftest_timeout(void* ws, size_t ws_bytes, int64_t* out, ee_stream_t stream);
+
+/*
  * ee_match_reuse -- reuse-span lookup (Sec. III-A, prefix matching that switches
  * Generate back to Reuse).  For each sequence s, with c = orig_tokens[
  * orig_off[s] .. orig_off[s+1]) and t = tail[s*n .. s*n+n) (the last n generated

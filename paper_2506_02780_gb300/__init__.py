@@ -27,10 +27,12 @@ STATUS = {0: "ok", 1: "invalid argument", 2: "unsupported configuration", 3: "CU
           4: "device error word set", 5: "workspace too small"}
 DEVERR = {0x01: "MATCH_ARGS", 0x02: "TREE", 0x04: "PAGE", 0x08: "CTX", 0x10: "FP16_RANGE",
           0x20: "TIMEOUT", 0x40: "PATH"}
+DEVERR_TIMEOUT = 0x20
 
 EXPORTS = ("ee_version", "ee_status_string", "ee_workspace_size", "ee_workspace_init",
            "ee_read_errors", "ee_match_reuse", "ee_tree_prepare", "ee_tree_verify_attn", "ee_attn_plan",
-           "ee_lmhead_accept", "ee_lmhead_verify", "ee_lmhead_accept_static", "ee_kv_compact")
+           "ee_lmhead_accept", "ee_lmhead_verify", "ee_lmhead_accept_static", "ee_kv_compact",
+           "ee_selftest_timeout")
 
 VERIFY_MODES = {"greedy": 0, "direct": 1, "topk": 2, "entropy": 3}
 
@@ -72,6 +74,7 @@ _SIGS = {
                                  _P], _I),
     "ee_kv_compact": ([_P, _P, _I64, _P, _P, _I64, _I, _I, _P, _I, _P, _P, _P, _P, _P, _I, _I, _I, _I,
                        _P, _P, _SZ, _P], _I),
+    "ee_selftest_timeout": ([_P, _SZ, _P, _P], _I),
 }
 
 
@@ -135,6 +138,14 @@ def ee_read_errors(ws, stream=None) -> int:
     if st not in (0, 4):
         raise EEError("ee_read_errors", st)
     return int(bits.value)
+
+
+def ee_selftest_timeout(ws, out, stream=None):
+    """Run the bounded-wait self-test; `out` is a device int64[7] (see ee.h)."""
+    _check(out, torch.int64, "out")
+    if out.numel() < 7:
+        raise ValueError("out needs 7 int64")
+    _ok("ee_selftest_timeout", lib().ee_selftest_timeout(_p(ws), ws.numel(), _p(out), _stream(stream)))
 
 
 def new_workspace(B, total_nodes, n_q, max_ctx, device="cuda", stream=None):

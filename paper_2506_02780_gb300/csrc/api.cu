@@ -1,6 +1,7 @@
 // Library-level entry points of libee: version, status strings, workspace
 // sizing/initialisation and the device error word.
 #include "ee_common.cuh"
+#include "ee_ptx.cuh"
 
 extern "C" const char* ee_version(void) { return "libee 0.1 (sm_103a)"; }
 
@@ -43,5 +44,58 @@ extern "C" ee_status ee_read_errors(void* ws, ee_stream_t stream, int32_t* bits)
     EE_CUDA_OK(cudaStreamSynchronize((cudaStream_t)stream));
     return EE_ERR_DEVICE;
   }
+  return EE_OK;
+}
+
+namespace ee {
+namespace {
+
+// Makes the two kinds of bounded wait of the pipelines run out (an mbarrier
+// nothing arrives at, a global counter nothing raises) and records how each
+// ended; see ee_selftest_timeout in ee.h.
+__global__ void __launch_bounds__(64) selftest_timeout_kernel(int32_t* err, const uint32_t* never_set,
+                                                              int64_t* out) {
+  __shared__ __align__(8) uint64_t s_bar[2];
+  __shared__ volatile int s_abort;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    mbar_init(smem_u32(&s_bar[0]), 1);
+    mbar_init(smem_u32(&s_bar[1]), 1);
+    s_abort = 0;
+  }
+  __syncthreads();
+  if (lane == 0) {
+    if (warp == 1) {   // start half a limit after warp 0
+      const long long d0 = cycles();
+      while (cycles() - d0 < kWaitLimitCycles / 2) {
+      }
+    }
+    const long long t0 = cycles();
+    // phase 0 of a fresh barrier completes only when its one arrival comes
+    const bool ok = mbar_wait(smem_u32(&s_bar[warp]), 0u, &s_abort);
+    out[1 + 2 * warp] = ok ? 1 : 0;
+    out[2 + 2 * warp] = cycles() - t0;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    const long long t0 = cycles();
+    const bool ok = wait_count_geq(never_set, 1u);
+    out[5] = ok ? 1 : 0;
+    out[6] = cycles() - t0;
+    out[0] = kWaitLimitCycles;
+    if (s_abort || !ok) flag_error(err, EE_DEVERR_TIMEOUT);
+  }
+}
+
+}  // namespace
+}  // namespace ee
+
+extern "C" ee_status ee_selftest_timeout(void* ws, size_t ws_bytes, int64_t* out, ee_stream_t stream) {
+  if (!ws || !out || ws_bytes < ee::kWorkspaceBytes || !ee::aligned(ws, 256) || !ee::aligned(out, 8))
+    return EE_ERR_INVALID_ARG;
+  const uint32_t* never_set =
+      reinterpret_cast<const uint32_t*>(static_cast<const char*>(ws) + ee::kNeverSetOff);
+  ee::selftest_timeout_kernel<<<1, 64, 0, (cudaStream_t)stream>>>(ee::err_word(ws), never_set, out);
+  EE_CUDA_OK(cudaGetLastError());
   return EE_OK;
 }

@@ -662,13 +662,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
   if (p.coop) {
     if (threadIdx.x == 0) {
       red_add_release(cnt, 1u);     // this CTA's slot (ordered before by the fences and barrier)
-      const long long t0 = cycles();
-      bool ready = true;
-      while (ld_acquire(cnt) < (uint32_t)p.S)
-        if (cycles() - t0 > kWaitLimitCycles) {
-          ready = false;
-          break;
-        }
+      const bool ready = wait_count_geq(cnt, (uint32_t)p.S);
       if (!ready) flag_error(p.err, EE_DEVERR_TIMEOUT);
       s_ready = ready;
     }

@@ -19,6 +19,7 @@ namespace ee {
 //   [0, 4)              device error word (EE_DEVERR_* bits)
 //   [16, 20)            LM-head "CTAs finished" ticket counter
 //   [24, 28)            verification finalize "CTAs finished" ticket counter
+//   [32, 36)            never-written flag (zero): the self-test's wait target
 //   [256, 256+8*EE_MAX_LM_NODES)  LM-head packed running argmax per node
 //   [kLmVerifyOff, +kLmVerifyBytes) LM-head verification partials
 //   [kAttnPartOff, ...)           attention partial slots, kAttnPartBytes per
@@ -27,6 +28,7 @@ namespace ee {
 // ---------------------------------------------------------------------------
 constexpr size_t kErrOff = 0;
 constexpr size_t kTicketOff = 16;
+constexpr size_t kNeverSetOff = 32;
 constexpr size_t kArgmaxOff = 256;
 constexpr size_t kWorkspaceBytes = 256 + 8 * (size_t)EE_MAX_LM_NODES + 256;   // the fixed head
 constexpr int kNumSMsMax = 152;       // LM-head grid bound (one persistent CTA per SM)

@@ -189,6 +189,14 @@ __device__ __forceinline__ uint32_t ld_acquire(const uint32_t* a) {
   asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(a) : "memory");
   return v;
 }
+// Bounded wait for a global counter that other CTAs raise to reach `target`:
+// false when the time limit passed first.
+__device__ __forceinline__ bool wait_count_geq(const uint32_t* cnt, uint32_t target) {
+  const long long t0 = cycles();
+  while (ld_acquire(cnt) < target)
+    if (cycles() - t0 > kWaitLimitCycles) return false;
+  return true;
+}
 // Packed fp32 pairs (sm_100 family): two lanes of fp32 arithmetic per instruction.
 __device__ __forceinline__ uint64_t f2_pack(uint32_t lo, uint32_t hi) {
   uint64_t d;

@@ -147,3 +147,12 @@ def test_compact_rejects_aliasing_ctx(L):
     assert f(*alias) == 1
     hd = list(args); hd[18] = 96
     assert f(*hd) == 2
+
+
+def test_selftest_timeout_rejects_bad_args(L):
+    f = L.ee_selftest_timeout
+    assert f(None, 1 << 20, FAKE, None) == 1                     # no workspace
+    assert f(FAKE, 1 << 20, None, None) == 1                     # no output
+    assert f(FAKE, 64, FAKE, None) == 1                          # below the fixed head
+    assert f(ctypes.c_void_p(0x10008), 1 << 20, FAKE, None) == 1   # ws not 256-aligned
+    assert f(FAKE, 1 << 20, ctypes.c_void_p(0x10004), None) == 1   # out not 8-aligned
