@@ -87,8 +87,10 @@ const char* ee_status_string(ee_status s);
  * Workspace bytes needed by every entry point for problems up to these sizes:
  * B sequences, total_nodes tree nodes in all, n_q query heads, max_ctx cached
  * positions in the longest sequence.  The buffer must be 256-byte aligned.
- * 3,219,968 bytes when max_ctx is 0, else 3,219,968 + B * n_q * 16 * 66,816
- * (the attention's partial slots; about 30 MB for one sequence with 28 heads).
+ * 3,219,968 bytes when max_ctx is 0, else 3,219,968 + max(B * n_q * 16, 304)
+ * * 66,816 (the attention's partial slots: one per CTA of a split launch, two
+ * per resident CTA of a balanced one; about 30 MB for one sequence with 28
+ * heads).
  * Returns 0 for negative arguments.
  */
 size_t ee_workspace_size(int32_t B, int32_t total_nodes, int32_t n_q, int32_t head_dim,
@@ -180,10 +182,15 @@ ee_status ee_tree_prepare(const int32_t* parent, const int32_t* node_off, int32_
  * all bf16 arrays 16-byte aligned.  Q.K^T runs on bf16 tensor cores with fp32
  * accumulation in TMEM; P.V runs on bf16 tensor cores with P carried as two
  * bf16 parts (head + tail, about 2^-14 relative) and V as stored; softmax and
- * the output are fp32.  One launch per call: a thread-block cluster of up to
- * 8 CTAs per 128 query rows splits the context; each CTA writes its partial
- * result to its slot in `ws` (L2-resident) and, after one cluster barrier,
- * each CTA merges a share of the rows.  EE_ERR_WORKSPACE when ws_bytes is
+ * the output are fp32.  One launch per call, in one of three forms the host
+ * picks from the sizes (ee_attn_plan): the context of each 128 query rows is
+ * cut into equal chunks, one CTA each, met at a thread-block cluster barrier
+ * or (cooperative launch) a counter; or, balanced, one CTA per SM takes an
+ * equal share of all row blocks' 128-key tiles, read from the device's
+ * ctx_len and node_off (ragged batches, and row-block counts that do not
+ * divide the SM count).  Split work writes partial results to slots in `ws`
+ * (L2-resident); once a row block's pieces are all written, each of their
+ * CTAs merges a share of its rows.  EE_ERR_WORKSPACE when ws_bytes is
  * below ee_workspace_size(B, total_nodes, n_q, head_dim, max_ctx).
  * Device errors: EE_DEVERR_PAGE (the key is skipped), EE_DEVERR_CTX,
  * EE_DEVERR_TIMEOUT (outputs undefined).
@@ -247,7 +254,9 @@ ee_status ee_lmhead_verify(const ee_bf16* hidden, const ee_bf16* lm_w, int32_t h
  * chunks per 128 query rows (1..16), *chunk = keys per chunk, *mode = 0
  * (one chunk, no merge), 1 (chunks of a row block form a thread-block
  * cluster) or 2 (cooperative launch, merge counters in the workspace),
- * *ctas = CTAs launched.  Needs the device (occupancy queries): EE_ERR_CUDA
+ * *ctas = CTAs launched.  Mode 3 (balanced, cooperative, one CTA per SM):
+ * *splits = CTAs that share the work at most, *chunk = keys per CTA when
+ * every sequence holds max_ctx positions and max_T nodes.  Needs the device (occupancy queries): EE_ERR_CUDA
  * without one; EE_ERR_INVALID_ARG for sizes ee_tree_verify_attn rejects.
  */
 ee_status ee_attn_plan(int32_t B, int32_t max_T, int32_t n_q, int32_t n_kv, int32_t max_ctx,

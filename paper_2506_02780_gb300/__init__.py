@@ -198,7 +198,7 @@ def ee_attn_plan(B, max_T, n_q, n_kv, max_ctx) -> dict:
     st = lib().ee_attn_plan(B, max_T, n_q, n_kv, max_ctx, *[ctypes.byref(x) for x in v])
     _ok("ee_attn_plan", st)
     return {"splits": v[0].value, "chunk": v[1].value,
-            "mode": ("single", "cluster", "cooperative")[v[2].value], "ctas": v[3].value}
+            "mode": ("single", "cluster", "cooperative", "balanced")[v[2].value], "ctas": v[3].value}
 
 
 def ee_lmhead_accept(hidden, lm_w, draft_tok, parent, depth, anc, node_off, max_T, argmax, accept_len,

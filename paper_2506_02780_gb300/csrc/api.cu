@@ -22,8 +22,10 @@ extern "C" size_t ee_workspace_size(int32_t B, int32_t total_nodes, int32_t n_q,
   if (B < 0 || total_nodes < 0 || n_q < 0 || head_dim < 0 || max_ctx < 0) return 0;
   if (max_ctx == 0) return ee::kAttnPartOff;      // one chunk per row block: no attention slots
   // attention CTAs of a split launch: B x n_kv x ceil(max_T * g / 128) row
-  // blocks (<= B x n_q, as max_T <= 128) x at most 16 chunks
-  return ee::kAttnPartOff + (size_t)B * n_q * ee::kAttnMaxSplits * ee::kAttnPartBytes;
+  // blocks (<= B x n_q, as max_T <= 128) x at most 16 chunks; a balanced
+  // launch: two slots per resident CTA (one per SM)
+  const size_t slots = std::max((size_t)B * n_q * ee::kAttnMaxSplits, 2 * (size_t)ee::kNumSMsMax);
+  return ee::kAttnPartOff + slots * ee::kAttnPartBytes;
 }
 
 extern "C" ee_status ee_workspace_init(void* ws, size_t ws_bytes, ee_stream_t stream) {

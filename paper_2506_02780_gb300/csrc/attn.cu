@@ -81,16 +81,17 @@ constexpr uint32_t kOffV = kOffK + kKST * kKVBytes;
 constexpr uint32_t kOffQ = kOffV + kVST * kKVBytes;  // Q block, 128 rows x 128 bf16, SW128 K-major
 constexpr uint32_t kOffPages = kOffQ + kKVBytes;
 constexpr uint32_t kOffBar = kOffPages + 4 * kMaxCtaPages;
-constexpr uint32_t kNumBars = 2 * kKST + 2 * kVST + 2 * kSB + 2 + 2;
+constexpr uint32_t kNumBars = 2 * kKST + 2 * kVST + 2 * kSB + 2 + 3;
 constexpr uint32_t kSmemBytes = 1024 + kOffBar + 8 * kNumBars + 64;
 constexpr uint32_t kTmemCols = 512;              // S0 [0,128) S1 [128,256) S2 [256,384) O [384,512)
 constexpr uint32_t kColO = 384;
 constexpr float kRescaleLog2 = 8.0f;
 constexpr int kMaxCluster = 8;                   // portable thread-block cluster size
 constexpr int kMaxSplits = ee::kAttnMaxSplits;   // chunks per row block (cooperative launch)
+constexpr int kMaxBalSeqs = 512;                 // sequences of a balanced launch
 // warp roles (warp 3 is idle after set-up); softmax warps 4..11, two per TMEM
 // lane quarter
-constexpr int kWarpK = 0, kWarpMma = 1, kWarpV = 2, kWarpSoft0 = 4;
+constexpr int kWarpK = 0, kWarpMma = 1, kWarpV = 2, kWarpSched = 3, kWarpSoft0 = 4;
 constexpr int kSoftThreads = 8 * 32;
 
 static_assert(kRows == ee::kAttnRows, "row block size");
@@ -109,6 +110,7 @@ struct AttnParams {
   int32_t* err;
   int num_pages, max_pages, max_ctx, n_q, n_kv, g, total_nodes, max_T, nrb, chunk, S;
   int coop;                    // 1: cooperative launch, counters; 0: cluster barrier
+  int B;                       // sequences (the balanced mode's work list)
   float scale_log2;
 };
 
@@ -140,8 +142,12 @@ __device__ __forceinline__ unsigned tile_mask(const int32_t* s_pages, int t, int
 // without keys have (m, l) = (-inf, 0) and weight 0; their O words, never
 // written, are not used.
 template <int S>
-__device__ __forceinline__ void merge_rows(const AttnParams& p, const uint8_t* slot0, int row0, int r0,
-                                           int nown, int o, int hk) {
+__device__ __forceinline__ void merge_rows(const AttnParams& p, size_t slot_a, size_t slot_b, int stride,
+                                           int row0, int r0, int nown, int o, int hk) {
+  // partial s lives in slot slot_a (s = 0) or slot_b + (s - 1) * stride
+  auto slot = [&](int s) -> const uint8_t* {
+    return p.part + (s == 0 ? slot_a : slot_b + (size_t)(s - 1) * stride) * kAttnPartBytes;
+  };
   constexpr int kRpc = (kRows + S - 1) / S;
   constexpr int kTprMin = kThreads / kRpc;
   constexpr int kCh = (kD / 4 + kTprMin - 1) / kTprMin;   // chunks per thread, at most
@@ -151,14 +157,14 @@ __device__ __forceinline__ void merge_rows(const AttnParams& p, const uint8_t* s
   float2 ml[S];
 #pragma unroll
   for (int s = 0; s < S; ++s)
-    ml[s] = __ldcg(reinterpret_cast<const float2*>(slot0 + (size_t)s * kAttnPartBytes + kAttnMlOff) + r0 + j);
+    ml[s] = __ldcg(reinterpret_cast<const float2*>(slot(s) + kAttnMlOff) + r0 + j);
   float4 v[kCh][S];
 #pragma unroll
   for (int k = 0; k < kCh; ++k) {
     const int c = cg + k * tpr;
 #pragma unroll
     for (int s = 0; s < S; ++s)
-      v[k][s] = c < kD / 4 ? __ldcg(reinterpret_cast<const float4*>(slot0 + (size_t)s * kAttnPartBytes) +
+      v[k][s] = c < kD / 4 ? __ldcg(reinterpret_cast<const float4*>(slot(s)) +
                                     (size_t)c * kRows + r0 + j)
                            : make_float4(0.f, 0.f, 0.f, 0.f);
   }
@@ -192,6 +198,15 @@ __device__ __forceinline__ void merge_rows(const AttnParams& p, const uint8_t* s
   }
 }
 
+// A row block's partial that this CTA merges with the other pieces of the same
+// row block (balanced mode): the unit, the number of pieces K, this CTA's
+// piece index k, and where the pieces' slots are (piece 0 at slot0, piece
+// s >= 1 at slot1 + 2 (s - 1)).
+struct BalPiece {
+  int hk, rb, o, R, K, k, slot0, slot1;
+};
+
+template <bool kBal>
 __global__ void __launch_bounds__(kThreads, 1)
 attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__ CUtensorMap tmVc,
                const __grid_constant__ CUtensorMap tmKt, const __grid_constant__ CUtensorMap tmVt,
@@ -204,6 +219,13 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
   __shared__ int s_kissued[kKST], s_vissued[kVST];
   __shared__ float s_xmax[2][2][kRows];             // [tile parity][half][row]: softmax pair exchange
   __shared__ float s_xl[2][kRows];                  // [half][row]: final row sums
+  // balanced mode: per sequence (node offset, T, context length, tiles) and the
+  // exclusive prefix of the sequences' work in tiles
+  __shared__ int4 s_seq[kBal ? kMaxBalSeqs : 1];
+  __shared__ int s_wpre[kBal ? kMaxBalSeqs + 1 : 1];
+  __shared__ int s_sched[6];                        // balanced: next tile, end tile, W, N, tiles, segments
+  __shared__ BalPiece s_pc[2];                      // balanced: this CTA's pieces of split units
+  __shared__ int s_npc;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t sbase = smem_u32(smem);
@@ -212,7 +234,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
   const uint32_t k_full = bar0, k_empty = k_full + 8 * kKST;
   const uint32_t v_full = k_empty + 8 * kKST, v_empty = v_full + 8 * kVST;
   const uint32_t s_full = v_empty + 8 * kVST, p_full = s_full + 8 * kSB, o_done = p_full + 8 * kSB;
-  const uint32_t drain = o_done + 16, q_ready = drain + 8;
+  const uint32_t drain = o_done + 16, q_ready = drain + 8, o_final = q_ready + 8;
 
   // on-chip set-up first: it touches no global memory, so it overlaps the end
   // of the previous kernel in the stream
@@ -222,6 +244,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmKt)) : "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmVt)) : "memory");
     s_abort = 0;
+    s_npc = 0;
     for (int i = 0; i < kKST; ++i) {
       mbar_init(k_full + 8 * i, 1);
       mbar_init(k_empty + 8 * i, 1);
@@ -239,6 +262,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
     for (int i = 0; i < 2; ++i) mbar_init(o_done + 8 * i, 1);
     mbar_init(drain, 1);
     mbar_init(q_ready, 2 * kRows);
+    mbar_init(o_final, 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     fence_async_smem();
   }
@@ -251,380 +275,548 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
   }
 
   pdl_wait();   // no global access before the previous kernel's writes are visible
-  const int b = blockIdx.z;
-  const int hk = blockIdx.y;
-  const int rb = blockIdx.x / p.S;                 // the S chunks of a row block are consecutive
-  const int split = blockIdx.x % p.S;              // == cluster rank in the cluster mode
-  // this chunk's page ids, issued now beside the sequence's node range and
-  // context length so that the round trips overlap (validated below)
-  constexpr int kPgPerThread = (kMaxCtaPages + kThreads - 1) / kThreads;
-  const int pg_first = split * (p.chunk / EE_PAGE);
-  const int npg_cap = max(0, min(p.chunk / EE_PAGE, p.max_pages - pg_first));
-  int32_t pgr[kPgPerThread];
+  const int g = p.g;
+
+  // ---- balanced mode: the shared work list ---------------------------------------
+  // Work is counted in 128-key tiles: sequence b brings n_kv x nrb_b units (a
+  // KV head's row block) of ceil(ctx_b / 128) context tiles + 1 tree tile.
+  // Units are ordered sequence, KV head, row block; CTA c takes the tiles
+  // [c W / N, (c + 1) W / N) of that order, so a CTA may finish one unit and
+  // start the next (at most two of its segments are pieces of split units).
+  // N is capped so that every CTA gets at least m = max(2, ceil(t_max / 14))
+  // tiles, which bounds the pieces of any unit by 15.
+  // Warp 3 (otherwise idle) builds it: lane l takes sequences [16 l, 16 l + 16).
+  if constexpr (kBal) {
+    if (warp == kWarpSched) {
+      constexpr int kPer = kMaxBalSeqs / 32;
+      int wl[kPer];
+      int wsum = 0, tmax = 0;
 #pragma unroll
-  for (int k = 0; k < kPgPerThread; ++k) {
-    const int i = threadIdx.x + k * kThreads;
-    pgr[k] = i < npg_cap ? ld_nc_pinned(p.block_table + (size_t)b * p.max_pages + pg_first + i) : -1;
+      for (int k = 0; k < kPer; ++k) {   // loads first (clamped indices), all in flight
+        const int bb = min(lane * kPer + k, p.B - 1);
+        s_seq[lane * kPer + k] = make_int4(p.node_off[bb], p.node_off[bb + 1], p.ctx_len[bb], 0);
+      }
+      __syncwarp();
+#pragma unroll
+      for (int k = 0; k < kPer; ++k) {
+        const int bb = lane * kPer + k;
+        wl[k] = 0;
+        if (bb < p.B) {
+          const int4 sq = s_seq[bb];
+          const int Tb = sq.y - sq.x;
+          const bool bad = Tb < 1 || Tb > EE_MAX_TREE || Tb > p.max_T || sq.x < 0 || sq.x + Tb > p.total_nodes;
+          if (bad && blockIdx.x == 0) flag_error(p.err, EE_DEVERR_TREE);
+          int c = sq.z;
+          if (c < 0 || c > p.max_ctx) {
+            if (blockIdx.x == 0) flag_error(p.err, EE_DEVERR_CTX);
+            c = c < 0 ? 0 : p.max_ctx;
+          }
+          const int tiles = (c + kKT - 1) / kKT + 1;
+          if (!bad) {
+            wl[k] = p.n_kv * ((Tb * g + kRows - 1) / kRows) * tiles;
+            tmax = max(tmax, tiles);
+          }
+          s_seq[bb] = make_int4(sq.x, bad ? 0 : Tb, c, tiles);
+        }
+        wsum += wl[k];
+      }
+      // warp-wide exclusive scan of the lanes' sums (lane order is sequence order)
+      int incl = wsum;
+#pragma unroll
+      for (int d = 1; d < 32; d <<= 1) {
+        const int v = __shfl_up_sync(0xffffffffu, incl, d);
+        if (lane >= d) incl += v;
+      }
+      const int W = __shfl_sync(0xffffffffu, incl, 31);
+      const int tmax_all = __reduce_max_sync(0xffffffffu, tmax);
+      int run = incl - wsum;
+#pragma unroll
+      for (int k = 0; k < kPer; ++k) {
+        const int bb = lane * kPer + k;
+        if (bb < p.B) s_wpre[bb] = run;
+        run += wl[k];
+      }
+      if (lane == 0) {
+        const int m = max(2, (tmax_all + 13) / 14);
+        const int N = W > 0 ? min((int)gridDim.x, max(1, W / m)) : 0;
+        const bool mine = (int)blockIdx.x < N;
+        s_sched[0] = mine ? (int)blockIdx.x * W / N : 0;
+        s_sched[1] = mine ? ((int)blockIdx.x + 1) * W / N : 0;
+        s_sched[2] = W;
+        s_sched[3] = N;
+        s_sched[4] = 0;
+        s_sched[5] = 0;
+        s_wpre[p.B] = W;
+      }
+    }
+    __syncthreads();
   }
-  const int o = p.node_off[b];
-  const int T = p.node_off[b + 1] - o;
-  int ctx = p.ctx_len[b];
-  const int R = T * p.g;
-  const bool bad_tree = T < 1 || T > EE_MAX_TREE || T > p.max_T || o < 0 || o + T > p.total_nodes;
-  if (bad_tree && threadIdx.x == 0 && blockIdx.x == 0 && hk == 0) flag_error(p.err, EE_DEVERR_TREE);
-  if (bad_tree || rb * kRows >= R) {                // uniform over the CTA (and the row block)
+
+  const int qhalf = lane >> 4, qc = lane & 15;
+  int32_t* s_pages = reinterpret_cast<int32_t*>(smem + kOffPages);
+  uint32_t tmem = 0;
+  bool skip = false;          // uniform mode: the row block has no work
+  // uniform mode: the (row block, chunk) of this CTA, and the row block's node
+  // offset and rows for the merge
+  const int split = kBal ? 0 : (int)(blockIdx.x % p.S);   // == cluster rank in the cluster mode
+  int u_o = 0, u_R = 0;
+
+  for (;;) {
+    // ---------------- the next segment of this CTA's work ----------------
+    constexpr int kPgPerThread = (kMaxCtaPages + kThreads - 1) / kThreads;
+    int b, hk, rb, o, T, ctx, k_begin, k_end;
+    bool with_tree, alone;
+    size_t slot;
+    int32_t pgr[kPgPerThread];
+    int x_next = 0;
+    // tiles this CTA processed before this segment (ring slots and phases count
+    // over all segments), and the segments done; kept in shared memory so that
+    // no register carries them across the softmax loop
+    const int tb = kBal ? s_sched[4] : 0;
+    const int nseg = kBal ? s_sched[5] : 0;
+    if constexpr (kBal) {
+      const int x = s_sched[0], x_end = s_sched[1], W = s_sched[2], N = s_sched[3];
+      if (x >= x_end) break;
+      int lo = 0, hi = p.B;   // s_wpre[lo] <= x < s_wpre[hi]
+      while (hi - lo > 1) {
+        const int mid = (lo + hi) >> 1;
+        if (s_wpre[mid] <= x) lo = mid; else hi = mid;
+      }
+      b = lo;
+      const int4 sq = s_seq[b];
+      o = sq.x;
+      T = sq.y;
+      ctx = sq.z;
+      const int tiles = sq.w;
+      const int nrb_b = (T * g + kRows - 1) / kRows;
+      const int local = x - s_wpre[b];
+      const int u = local / tiles, t0 = local - u * tiles;
+      hk = u / nrb_b;
+      rb = u - hk * nrb_b;
+      const int len = min(tiles - t0, x_end - x);
+      const int n_ctx_b = tiles - 1;
+      k_begin = min(t0, n_ctx_b) * kKT;
+      k_end = t0 < n_ctx_b ? min(ctx, min(t0 + len, n_ctx_b) * kKT) : k_begin;
+      with_tree = t0 + len == tiles;
+      // the CTAs holding the unit's first and last tiles
+      const int U0 = x - t0;
+      const int c0 = ((U0 + 1) * N - 1) / W;
+      const int c1 = ((U0 + tiles) * N - 1) / W;
+      alone = c0 == c1;
+      // a piece is this CTA's first segment (slot 2c) or its last (slot 2c + 1)
+      slot = 2 * (size_t)blockIdx.x + (nseg > 0 ? 1 : 0);
+      if (!alone && threadIdx.x == 0 && s_npc < 2) {
+        const int start0 = c0 * W / N;
+        s_pc[s_npc] = BalPiece{hk, rb, o, T * g, c1 - c0 + 1, (int)blockIdx.x - c0,
+                               2 * c0 + (U0 > start0 ? 1 : 0), 2 * (c0 + 1)};
+        s_npc = s_npc + 1;
+      }
+      x_next = x + len;
+      const int pg_first = k_begin / EE_PAGE;
+      const int npg = (k_end - k_begin + EE_PAGE - 1) / EE_PAGE;   // <= kMaxCtaPages: see the plan
+#pragma unroll
+      for (int k = 0; k < kPgPerThread; ++k) {
+        const int i = threadIdx.x + k * kThreads;
+        pgr[k] = i < npg ? ld_nc_pinned(p.block_table + (size_t)b * p.max_pages + pg_first + i) : -1;
+      }
+    } else {
+      b = blockIdx.z;
+      hk = blockIdx.y;
+      rb = blockIdx.x / p.S;                     // the S chunks of a row block are consecutive
+      // this chunk's page ids, issued now beside the sequence's node range and
+      // context length so that the round trips overlap (validated below)
+      const int pg_first = split * (p.chunk / EE_PAGE);
+      const int npg_cap = max(0, min(p.chunk / EE_PAGE, p.max_pages - pg_first));
+#pragma unroll
+      for (int k = 0; k < kPgPerThread; ++k) {
+        const int i = threadIdx.x + k * kThreads;
+        pgr[k] = i < npg_cap ? ld_nc_pinned(p.block_table + (size_t)b * p.max_pages + pg_first + i) : -1;
+      }
+      o = p.node_off[b];
+      T = p.node_off[b + 1] - o;
+      ctx = p.ctx_len[b];
+      const bool bad_tree = T < 1 || T > EE_MAX_TREE || T > p.max_T || o < 0 || o + T > p.total_nodes;
+      if (bad_tree && threadIdx.x == 0 && blockIdx.x == 0 && hk == 0) flag_error(p.err, EE_DEVERR_TREE);
+      if (bad_tree || rb * kRows >= T * g) {     // uniform over the CTA (and the row block)
+        skip = true;
+        break;
+      }
+      if (ctx < 0 || ctx > p.max_ctx) {
+        if (threadIdx.x == 0 && blockIdx.x == 0 && hk == 0) flag_error(p.err, EE_DEVERR_CTX);
+        ctx = ctx < 0 ? 0 : p.max_ctx;
+      }
+      // everything above is uniform over the row block's CTAs; from here on every
+      // CTA reaches the merge synchronisation
+      const int S = attn_splits_for(ctx, p.chunk);   // chunks this sequence uses, <= p.S
+      const bool active = split < S;
+      k_begin = split * p.chunk;
+      k_end = active ? min(ctx, k_begin + p.chunk) : k_begin;
+      with_tree = active && split == S - 1;
+      alone = p.S == 1;
+      slot = ((size_t)blockIdx.z * gridDim.y + blockIdx.y) * gridDim.x + blockIdx.x;
+      u_o = o;
+      u_R = T * g;
+    }
+    const int R = T * g;
+    const int n_ctx_tiles = k_end > k_begin ? (k_end - k_begin + kKT - 1) / kKT : 0;
+    const int n_tiles = n_ctx_tiles + (with_tree ? 1 : 0);
+
+    // softmax threads issue the coalesced loads of the block's Q rows now (a
+    // half-warp reads one 256-byte row; rows past R read row R - 1 and are
+    // zeroed later) so that they leave before the K/V stream starts; the values
+    // are consumed after the barrier below
+    uint4 qv[kRows / 16];
+    if (warp >= kWarpSoft0) {
+#pragma unroll
+      for (int k = 0; k < kRows / 16; ++k) {
+        const int rq = 2 * ((warp - kWarpSoft0) + 8 * k) + qhalf;   // 0..127
+        const int rrq = min(rb * kRows + rq, R - 1);
+        const int nq = rrq / g;
+        qv[k] = __ldg(reinterpret_cast<const uint4*>(
+                          p.q + ((size_t)(o + nq) * p.n_q + hk * g + (rrq - nq * g)) * kD) +
+                      qc);
+      }
+    }
+    {
+      // pages that hold keys of this segment (k_end <= ctx <= max_pages * 16);
+      // the previous segment's readers are past the barrier that ended it
+      const int npg = (k_end - k_begin + EE_PAGE - 1) / EE_PAGE;
+#pragma unroll
+      for (int k = 0; k < kPgPerThread; ++k) {
+        const int i = threadIdx.x + k * kThreads;
+        if (i < npg) {
+          const int pg = pgr[k];
+          const bool ok = pg >= 0 && pg < p.num_pages;
+          if (!ok) flag_error(p.err, EE_DEVERR_PAGE);
+          s_pages[i] = ok ? pg : -1;
+        }
+      }
+    }
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
-    if (warp == kWarpMma)
-      asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(s_tmem),
-                   "r"(kTmemCols)
-                   : "memory");
-    return;
-  }
-  if (ctx < 0 || ctx > p.max_ctx) {
-    if (threadIdx.x == 0 && blockIdx.x == 0 && hk == 0) flag_error(p.err, EE_DEVERR_CTX);
-    ctx = ctx < 0 ? 0 : p.max_ctx;
-  }
-  // everything above is uniform over the row block's CTAs; from here on every
-  // CTA reaches the merge synchronisation
-  const int S = attn_splits_for(ctx, p.chunk);     // chunks this sequence uses, <= p.S
-  const bool active = split < S;
-  const int k_begin = split * p.chunk;
-  const int k_end = active ? min(ctx, k_begin + p.chunk) : k_begin;
-  const int n_ctx_tiles = k_end > k_begin ? (k_end - k_begin + kKT - 1) / kKT : 0;
-  const int n_tiles = active ? n_ctx_tiles + ((split == S - 1) ? 1 : 0) : 0;   // + the tree tile
+    tmem = s_tmem;
+    // every thread has read the schedule position: advance it for the next segment
+    if (kBal && threadIdx.x == 0) {
+      s_sched[0] = x_next;
+      s_sched[4] = tb + n_tiles;
+      s_sched[5] = nseg + 1;
+    }
 
-  // softmax threads issue the coalesced loads of the block's Q rows now (a
-  // half-warp reads one 256-byte row; rows past R read row R - 1 and are
-  // zeroed later) so that they leave before the K/V stream starts; the values
-  // are consumed after the barrier below
-  const int qhalf = lane >> 4, qc = lane & 15;
-  uint4 qv[kRows / 16];
-  if (warp >= kWarpSoft0) {
-#pragma unroll
-    for (int k = 0; k < kRows / 16; ++k) {
-      const int rq = 2 * ((warp - kWarpSoft0) + 8 * k) + qhalf;   // 0..127
-      const int rrq = min(rb * kRows + rq, R - 1);
-      const int nq = rrq / p.g;
-      qv[k] = __ldg(reinterpret_cast<const uint4*>(
-                        p.q + ((size_t)(o + nq) * p.n_q + hk * p.g + (rrq - nq * p.g)) * kD) +
-                    qc);
-    }
-  }
-  int32_t* s_pages = reinterpret_cast<int32_t*>(smem + kOffPages);
-  {
-    // pages that hold keys of this chunk: <= npg_cap (k_end <= ctx <= max_pages * 16)
-    const int npg = (k_end - k_begin + EE_PAGE - 1) / EE_PAGE;
-#pragma unroll
-    for (int k = 0; k < kPgPerThread; ++k) {
-      const int i = threadIdx.x + k * kThreads;
-      if (i < npg) {
-        const int pg = pgr[k];
-        const bool ok = pg >= 0 && pg < p.num_pages;
-        if (!ok) flag_error(p.err, EE_DEVERR_PAGE);
-        s_pages[i] = ok ? pg : -1;
-      }
-    }
-  }
-  tc_fence_before();
-  __syncthreads();
-  tc_fence_after();
-  const uint32_t tmem = s_tmem;
-
-  bool have = false;          // softmax threads: this row's partial is complete
-  float row_m = -INFINITY, row_l = 0.f;
-  if (warp == kWarpK || warp == kWarpV) {
-    // ---------------- TMA producers: warp 0 streams K, warp 2 streams V ----------------
-    // lane 0 waits for the slot and posts the byte count; lane i < 8 then issues
-    // the two boxes of the tile's 16-row block i
-    const bool isK = warp == kWarpK;
-    const int nst = isK ? kKST : kVST;
-    const uint32_t full0 = isK ? k_full : v_full, empty0 = isK ? k_empty : v_empty;
-    const uint32_t ring = isK ? sK : sV;
-    const CUtensorMap* mc = isK ? &tmKc : &tmVc;
-    const CUtensorMap* mt = isK ? &tmKt : &tmVt;
-    int* issued = isK ? s_kissued : s_vissued;
-    for (int t = 0; t < n_tiles; ++t) {
-      const int st = t % nst, use = t / nst;
-      bool go = true;
-      if (lane == 0) go = mbar_wait(empty0 + 8 * st, (uint32_t)(use & 1) ^ 1u, &s_abort);
-      // the last V stage holds the staged Q rows until they are in TMEM
-      if (!__shfl_sync(0xffffffffu, go, 0)) break;
-      const uint32_t full = full0 + 8 * st;
-      const uint32_t dst = ring + st * kKVBytes;
-      if (lane == 0) mbar_expect_tx(full, 2 * kKVHalf);
-      __syncwarp();
-      if (t < n_ctx_tiles) {
-        // every 16-row block is written: blocks without a loaded page are read at
-        // row -16, wholly out of range, which the TMA unit fills with zeros (a
-        // stale V row would turn 0 * P into NaN)
-        if (lane < kKT / 16) {
-          const int pos = k_begin + t * kKT + 16 * lane;
-          const int pg = pos < k_end ? s_pages[t * (kKT / 16) + lane] : -1;
-          const int row0 = pg >= 0 ? (pg * p.n_kv + hk) * EE_PAGE : -EE_PAGE;
-          tma_load_2d(dst + lane * 2048, mc, full, 0, row0);
-          tma_load_2d(dst + kKVHalf + lane * 2048, mc, full, 64, row0);
-        }
-      } else if (lane == 0) {
-        tma_load_3d(dst, mt, full, 0, hk, o);
-        tma_load_3d(dst + kKVHalf, mt, full, 64, hk, o);
-      }
-      __syncwarp();
-      if (lane == 0) issued[st] = use;
-    }
-  } else if (warp == kWarpMma) {
-    // ---------- MMA issuer: Q.K^T(0..kSB-1), then P.V(t), Q.K^T(t+kSB) ----------
-    if (lane == 0) {
-      tc_fence_after();
-      const uint32_t id_qk = idesc_f16(kRows, kKT, 1, 1, 0);
-      const uint32_t sQ = sbase + kOffQ;
-      const uint32_t id_pv = idesc_f16(kRows, kD, 1, 1, 1);
-      auto issue_qk = [&](int t) -> bool {
-        if (!mbar_wait(k_full + 8 * (t % kKST), (uint32_t)((t / kKST) & 1), &s_abort)) return false;
-        tc_fence_after();
-        const uint32_t kb = sK + (t % kKST) * kKVBytes;
-#pragma unroll
-        for (int kk = 0; kk < kD / 16; ++kk) {
-          const uint32_t off = (kk & 3) * 32;
-          tc_mma(tmem + (t % kSB) * kKT, smem_desc_sw128(sQ + (kk >> 2) * kKVHalf + off),
-                 smem_desc_sw128(kb + (kk >> 2) * kKVHalf + off), id_qk, kk > 0 ? 1u : 0u);
-        }
-        tc_commit(k_empty + 8 * (t % kKST));
-        tc_commit(s_full + 8 * (t % kSB));
-        return true;
-      };
-      bool ok = mbar_wait(q_ready, 0, &s_abort);
-      for (int t = 0; t < kSB && t < n_tiles && ok; ++t) ok = issue_qk(t);
-      for (int t = 0; t < n_tiles && ok; ++t) {
-        if (!mbar_wait(p_full + 8 * (t % kSB), (uint32_t)((t / kSB) & 1), &s_abort) ||
-            !mbar_wait(v_full + 8 * (t % kVST), (uint32_t)((t / kVST) & 1), &s_abort))
-          break;
-        tc_fence_after();
-        const uint32_t pa = tmem + (t % kSB) * kKT;        // bf16 P head: cols 0..63, tail: 64..127
-        const uint32_t vb = sV + (t % kVST) * kKVBytes;
-#pragma unroll
-        for (int part = 0; part < 2; ++part)
-#pragma unroll
-          for (int j = 0; j < kKT / 16; ++j)
-            tc_mma_ts(tmem + kColO, pa + 64 * part + 8 * j,
-                      smem_desc_sw128_mn(vb + j * 2048, kKVHalf, 1024), id_pv,
-                      (t > 0 || part > 0 || j > 0) ? 1u : 0u);
-        tc_commit(v_empty + 8 * (t % kVST));
-        tc_commit(o_done + 8 * (t & 1));
-        if (t + kSB < n_tiles) ok = issue_qk(t + kSB);
-      }
-    }
-  } else if (warp >= kWarpSoft0) {
-    // ---------------- softmax: one query row and half of every tile per thread ----------------
-    // Warps w and w + 4 share TMEM lane quarter w & 3 (32 query rows); half hf
-    // of the pair takes keys [64 hf, 64 hf + 64) of every tile and O columns
-    // [64 hf, 64 hf + 64).  The pair agrees on each tile's row maximum through
-    // shared memory at a 64-thread named barrier, so both halves take the same
-    // rescale decisions; each keeps the sum over its own keys, and the two sums
-    // are added (half 0 first) at the end.  Two warps per sub-partition hide
-    // each other's latencies.  Every exit from the tile loop happens right
-    // after the pair barrier and on a decision both warps share.
-    const int qd = warp & 3;
-    const int hf = (warp - kWarpSoft0) >> 2;
-    const uint32_t pair_bar = 2 + qd;
-    const int r = qd * 32 + lane;                     // == TMEM lane of this quarter
-    const int rr = rb * kRows + r;
-    const bool vrow = rr < R;
-    const int node = vrow ? rr / p.g : 0;
-    const uint64_t ancw = vrow ? p.anc[2 * (size_t)(o + node) + hf] : 0ull;   // this half's tree keys
-    const uint32_t tl = tmem + ((uint32_t)(qd * 32) << 16);
-    // the block's Q rows into shared memory as the A operand of Q.K^T: 128 rows
-    // x 128 bf16 in two 64-column slabs, 128-byte swizzled K-major (the layout
-    // TMA gives the K tiles): 16-byte chunk j of row r at slab (j / 8),
-    // (r / 8) * 1024 + (r % 8) * 128 + ((j % 8) ^ (r % 8)) * 16; rows past R are
-    // zero.  The rows were loaded (coalesced) before the set-up barrier.
-    {
-      uint8_t* qs = smem + kOffQ;
-#pragma unroll
-      for (int k = 0; k < kRows / 16; ++k) {
-        const int rq = 2 * ((warp - kWarpSoft0) + 8 * k) + qhalf;
-        const int j = qc & 7;
-        *reinterpret_cast<uint4*>(qs + (qc >> 3) * kKVHalf + (rq >> 3) * 1024 + (rq & 7) * 128 +
-                                  ((j ^ (rq & 7)) << 4)) =
-            rb * kRows + rq < R ? qv[k] : make_uint4(0u, 0u, 0u, 0u);
-      }
-      fence_async_smem();   // generic-proxy writes, read by the tensor core
-      mbar_arrive(q_ready);
-    }
-    // m_used is kept in raw score units (scale > 0, so the max commutes with it)
-    float m_used = -INFINITY, l = 0.f;
-    const float sl2 = p.scale_log2;
-    const float kFail = __int_as_float(0x7fffffff);   // NaN: "this half's wait failed"
-    bool ok = true;
-    for (int t = 0; t < n_tiles; ++t) {
-      const int sb = t % kSB;     // S buffer of this tile
-      const int xb = t & 1;       // pair-exchange slot
-      // wait outcomes are warp-uniform: the TMEM accesses that follow are
-      // warp-collective (.sync.aligned)
-      const bool got =
-          __all_sync(0xffffffffu, mbar_wait(s_full + 8 * sb, (uint32_t)((t / kSB) & 1), &s_abort));
-      uint32_t sr[64];
-      float tmax = -INFINITY;
-      if (got) {
-        tc_fence_after();
-        tc_ld32(tl + sb * kKT + 64 * hf, *reinterpret_cast<uint32_t(*)[32]>(&sr[0]));
-        tc_ld32(tl + sb * kKT + 64 * hf + 32, *reinterpret_cast<uint32_t(*)[32]>(&sr[32]));
-        // visibility of this half's 64 keys as one 64-bit word
-        uint64_t kw;
+    if (warp == kWarpK || warp == kWarpV) {
+      // ---------------- TMA producers: warp 0 streams K, warp 2 streams V ----------------
+      // lane 0 waits for the slot and posts the byte count; lane i < 8 then issues
+      // the two boxes of the tile's 16-row block i.  Ring slots and phases count
+      // the CTA's tiles over all its segments.
+      const bool isK = warp == kWarpK;
+      const int nst = isK ? kKST : kVST;
+      const uint32_t full0 = isK ? k_full : v_full, empty0 = isK ? k_empty : v_empty;
+      const uint32_t ring = isK ? sK : sV;
+      const CUtensorMap* mc = isK ? &tmKc : &tmVc;
+      const CUtensorMap* mt = isK ? &tmKt : &tmVt;
+      int* issued = isK ? s_kissued : s_vissued;
+      for (int t = 0; t < n_tiles; ++t) {
+        const int tg = tb + t;
+        const int st = tg % nst, use = tg / nst;
+        bool go = true;
+        if (lane == 0) go = mbar_wait(empty0 + 8 * st, (uint32_t)(use & 1) ^ 1u, &s_abort);
+        if (!__shfl_sync(0xffffffffu, go, 0)) break;
+        const uint32_t full = full0 + 8 * st;
+        const uint32_t dst = ring + st * kKVBytes;
+        if (lane == 0) mbar_expect_tx(full, 2 * kKVHalf);
+        __syncwarp();
         if (t < n_ctx_tiles) {
-          const unsigned m = tile_mask(s_pages, t, k_begin, k_end);
-          const int nv = min(max(k_end - (k_begin + t * kKT) - 64 * hf, 0), 64);
-          uint64_t pgw = 0ull;
-#pragma unroll
-          for (int i = 0; i < 4; ++i) pgw |= ((m >> (4 * hf + i)) & 1u) ? (0xFFFFull << (16 * i)) : 0ull;
-          kw = pgw & (nv >= 64 ? ~0ull : ((1ull << nv) - 1ull));
-        } else {
-          const int th = min(max(T - 64 * hf, 0), 64);
-          kw = ancw & (th >= 64 ? ~0ull : ((1ull << th) - 1ull));
+          // every 16-row block is written: blocks without a loaded page are read at
+          // row -16, wholly out of range, which the TMA unit fills with zeros (a
+          // stale V row would turn 0 * P into NaN)
+          if (lane < kKT / 16) {
+            const int pos = k_begin + t * kKT + 16 * lane;
+            const int pg = pos < k_end ? s_pages[t * (kKT / 16) + lane] : -1;
+            const int row0 = pg >= 0 ? (pg * p.n_kv + hk) * EE_PAGE : -EE_PAGE;
+            tma_load_2d(dst + lane * 2048, mc, full, 0, row0);
+            tma_load_2d(dst + kKVHalf + lane * 2048, mc, full, 64, row0);
+          }
+        } else if (lane == 0) {
+          tma_load_3d(dst, mt, full, 0, hk, o);
+          tma_load_3d(dst + kKVHalf, mt, full, 64, hk, o);
         }
-        if (!vrow) kw = 0ull;
-        if (!__all_sync(0xffffffffu, kw == ~0ull)) {
-#pragma unroll
-          for (int c = 0; c < 64; ++c)
-            if (!((kw >> c) & 1ull)) sr[c] = __float_as_uint(-INFINITY);
-        }
-        float mx[8];
-#pragma unroll
-        for (int c = 0; c < 8; ++c) mx[c] = __uint_as_float(sr[c]);
-#pragma unroll
-        for (int c = 8; c < 64; ++c) mx[c & 7] = fmaxf(mx[c & 7], __uint_as_float(sr[c]));
-        tmax = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
-                     fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
+        __syncwarp();
+        if (lane == 0) issued[st] = use;
       }
-      // the pair swaps its halves' maxima; both S halves are in registers before
-      // either warp overwrites S with P
-      s_xmax[xb][hf][r] = got ? tmax : kFail;
-      tc_fence_before();
-      asm volatile("bar.sync %0, 64;" ::"r"(pair_bar) : "memory");
-      tc_fence_after();
-      const float other = s_xmax[xb][hf ^ 1][r];
-      if (!__all_sync(0xffffffffu, got && other == other)) {
-        ok = false;
-        break;
-      }
-      tmax = fmaxf(tmax, other);
-      const float m_new = fmaxf(m_used, tmax);
-      const bool need = (m_new - m_used) * sl2 > kRescaleLog2;   // true when m_used = -inf < m_new
-      if (t >= 1 && __any_sync(0xffffffffu, need)) {
-        // O must hold P.V(t-1) before this half's columns are rescaled; a failed
-        // wait sets the abort flag, and the pair stops at the next barrier
-        if (__all_sync(0xffffffffu,
-                       mbar_wait(o_done + 8 * ((t - 1) & 1), (uint32_t)(((t - 1) >> 1) & 1), &s_abort))) {
+    } else if (warp == kWarpMma) {
+      // ---------- MMA issuer: Q.K^T(0..kSB-1), then P.V(t), Q.K^T(t+kSB) ----------
+      if (lane == 0) {
+        tc_fence_after();
+        const uint32_t id_qk = idesc_f16(kRows, kKT, 1, 1, 0);
+        const uint32_t sQ = sbase + kOffQ;
+        const uint32_t id_pv = idesc_f16(kRows, kD, 1, 1, 1);
+        auto issue_qk = [&](int t) -> bool {
+          const int tg = tb + t;
+          if (!mbar_wait(k_full + 8 * (tg % kKST), (uint32_t)((tg / kKST) & 1), &s_abort)) return false;
           tc_fence_after();
-          const float f = need ? ex2((m_used - m_new) * sl2) : 1.f;
-#pragma unroll 1
-          for (int c4 = 0; c4 < 2; ++c4) {
-            uint32_t ov[32];
-            tc_ld32(tl + kColO + 64 * hf + 32 * c4, ov);
+          const uint32_t kb = sK + (tg % kKST) * kKVBytes;
 #pragma unroll
-            for (int e = 0; e < 32; ++e) ov[e] = __float_as_uint(__uint_as_float(ov[e]) * f);
-            tc_st32(tl + kColO + 64 * hf + 32 * c4, ov);
+          for (int kk = 0; kk < kD / 16; ++kk) {
+            const uint32_t off = (kk & 3) * 32;
+            tc_mma(tmem + (tg % kSB) * kKT, smem_desc_sw128(sQ + (kk >> 2) * kKVHalf + off),
+                   smem_desc_sw128(kb + (kk >> 2) * kKVHalf + off), id_qk, kk > 0 ? 1u : 0u);
           }
-        } else {
-          ok = false;
-        }
-      }
-      if (need) {
-        l *= ex2((m_used - m_new) * sl2);
-        m_used = m_new;
-      }
-      const float nms = m_used == -INFINITY ? 0.f : -m_used * sl2;
-      // p = 2^(s*scale_log2 - m); P = head + tail, both bf16 (top 16 bits): this
-      // half's head pairs go to columns 32 hf.. of the S buffer, its tail pairs
-      // to 64 + 32 hf..
-      // (pairs of columns run on packed fp32x2 arithmetic: the scale-and-shift,
-      // the running sums and the tail subtraction take one instruction per pair)
-      const uint64_t sl2x2 = f2_pack(__float_as_uint(sl2), __float_as_uint(sl2));
-      const uint64_t nmsx2 = f2_pack(__float_as_uint(nms), __float_as_uint(nms));
-      uint64_t ls2[4];
-      uint32_t hw[32], tw[32];
+          tc_commit(k_empty + 8 * (tg % kKST));
+          tc_commit(s_full + 8 * (tg % kSB));
+          return true;
+        };
+        bool ok = mbar_wait(q_ready, (uint32_t)(nseg & 1), &s_abort);
+        for (int t = 0; t < kSB && t < n_tiles && ok; ++t) ok = issue_qk(t);
+        for (int t = 0; t < n_tiles && ok; ++t) {
+          const int tg = tb + t;
+          if (!mbar_wait(p_full + 8 * (tg % kSB), (uint32_t)((tg / kSB) & 1), &s_abort) ||
+              !mbar_wait(v_full + 8 * (tg % kVST), (uint32_t)((tg / kVST) & 1), &s_abort))
+            break;
+          tc_fence_after();
+          const uint32_t pa = tmem + (tg % kSB) * kKT;       // bf16 P head: cols 0..63, tail: 64..127
+          const uint32_t vb = sV + (tg % kVST) * kKVBytes;
 #pragma unroll
-      for (int e = 0; e < 32; ++e) {
-        uint32_t y0, y1;
-        f2_unpack(f2_fma(f2_pack(sr[2 * e], sr[2 * e + 1]), sl2x2, nmsx2), y0, y1);
-        const uint32_t p0 = __float_as_uint(ex2(__uint_as_float(y0)));
-        const uint32_t p1 = __float_as_uint(ex2(__uint_as_float(y1)));
-        const uint64_t pp = f2_pack(p0, p1);
-        ls2[e & 3] = e < 4 ? pp : f2_add(ls2[e & 3], pp);
-        const uint32_t h0 = p0 & 0xFFFF0000u;
-        const uint32_t h1 = p1 & 0xFFFF0000u;
-        uint32_t t0, t1;
-        f2_unpack(f2_sub(pp, f2_pack(h0, h1)), t0, t1);
-        hw[e] = __byte_perm(h0, h1, 0x7632);
-        tw[e] = __byte_perm(t0, t1, 0x7632);
+          for (int part = 0; part < 2; ++part)
+#pragma unroll
+            for (int j = 0; j < kKT / 16; ++j)
+              tc_mma_ts(tmem + kColO, pa + 64 * part + 8 * j,
+                        smem_desc_sw128_mn(vb + j * 2048, kKVHalf, 1024), id_pv,
+                        (t > 0 || part > 0 || j > 0) ? 1u : 0u);
+          tc_commit(v_empty + 8 * (tg % kVST));
+          tc_commit(o_done + 8 * (tg & 1));
+          if (t + kSB < n_tiles) ok = issue_qk(t + kSB);
+        }
+        // one phase per segment: every product of the segment is complete
+        if (n_tiles > 0) tc_commit(o_final);
       }
-      tc_st32(tl + sb * kKT + 32 * hf, hw);
-      tc_st32(tl + sb * kKT + 64 + 32 * hf, tw);
+    } else if (warp >= kWarpSoft0) {
+      // ---------------- softmax: one query row and half of every tile per thread ----------------
+      // Warps w and w + 4 share TMEM lane quarter w & 3 (32 query rows); half hf
+      // of the pair takes keys [64 hf, 64 hf + 64) of every tile and O columns
+      // [64 hf, 64 hf + 64).  The pair agrees on each tile's row maximum through
+      // shared memory at a 64-thread named barrier, so both halves take the same
+      // rescale decisions; each keeps the sum over its own keys, and the two sums
+      // are added (half 0 first) at the end.  Two warps per sub-partition hide
+      // each other's latencies.  Every exit from the tile loop happens right
+      // after the pair barrier and on a decision both warps share.
+      const int qd = warp & 3;
+      const int hf = (warp - kWarpSoft0) >> 2;
+      const uint32_t pair_bar = 2 + qd;
+      const int r = qd * 32 + lane;                     // == TMEM lane of this quarter
+      const int rr = rb * kRows + r;
+      const bool vrow = rr < R;
+      const int node = vrow ? rr / g : 0;
+      const uint64_t ancw = vrow ? p.anc[2 * (size_t)(o + node) + hf] : 0ull;   // this half's tree keys
+      const uint32_t tl = tmem + ((uint32_t)(qd * 32) << 16);
+      // the block's Q rows into shared memory as the A operand of Q.K^T: 128 rows
+      // x 128 bf16 in two 64-column slabs, 128-byte swizzled K-major (the layout
+      // TMA gives the K tiles): 16-byte chunk j of row r at slab (j / 8),
+      // (r / 8) * 1024 + (r % 8) * 128 + ((j % 8) ^ (r % 8)) * 16; rows past R are
+      // zero.  The rows were loaded (coalesced) before the set-up barrier; the
+      // previous segment's Q.K^T products completed before its last P.V did.
       {
-        uint32_t a0, a1, b0, b1, c0, c1, d0, d1;
-        f2_unpack(ls2[0], a0, a1);
-        f2_unpack(ls2[1], b0, b1);
-        f2_unpack(ls2[2], c0, c1);
-        f2_unpack(ls2[3], d0, d1);
-        l += ((__uint_as_float(a0) + __uint_as_float(a1)) + (__uint_as_float(b0) + __uint_as_float(b1))) +
-             ((__uint_as_float(c0) + __uint_as_float(c1)) + (__uint_as_float(d0) + __uint_as_float(d1)));
-      }
-      tc_fence_before();
-      mbar_arrive(p_full + 8 * sb);
-    }
-    // wait for the last P.V; the pair adds its two sums, then each half writes
-    // its 64 columns out: O / l itself when the CTA is alone, else the partial
-    // (O, m, l) to this CTA's slot
-    const bool fin =
-        ok && n_tiles > 0 &&
-        mbar_wait(o_done + 8 * ((n_tiles - 1) & 1), (uint32_t)(((n_tiles - 1) >> 1) & 1), &s_abort);
-    have = __all_sync(0xffffffffu, fin);
-    s_xl[hf][r] = have ? l : kFail;
-    asm volatile("bar.sync %0, 64;" ::"r"(pair_bar) : "memory");
-    const float l_sum = s_xl[0][r] + s_xl[1][r];     // NaN when either half failed
-    const bool both = have && l_sum == l_sum;
-    row_m = (both && vrow && m_used != -INFINITY) ? m_used * sl2 : -INFINITY;
-    row_l = (both && vrow && m_used != -INFINITY) ? l_sum : 0.f;
-    const bool alone = p.S == 1;
-    const size_t cta = ((size_t)blockIdx.z * gridDim.y + blockIdx.y) * gridDim.x + blockIdx.x;
-    float4* dst;
-    size_t dstride;                                   // float4 between column chunks
-    float inv = 1.f;
-    if (alone) {
-      const size_t orow = (size_t)(o + node) * p.n_q + hk * p.g + (rr - node * p.g);
-      dst = reinterpret_cast<float4*>(p.out + orow * kD);
-      dstride = 1;
-      inv = row_l > 0.f ? 1.f / row_l : 0.f;
-    } else {
-      dst = reinterpret_cast<float4*>(p.part + cta * kAttnPartBytes) + r;
-      dstride = kRows;
-    }
-    const bool store = alone ? vrow : row_l > 0.f;
-    // the TMEM read is warp-collective: the whole warp reads when any lane stores
-    if (__any_sync(0xffffffffu, store)) {
-      tc_fence_after();
-#pragma unroll 1
-      for (int c4 = 0; c4 < 2; ++c4) {
-        uint32_t ov[32];
-        tc_ld32(tl + kColO + 64 * hf + 32 * c4, ov);
-        if (store) {
+        uint8_t* qs = smem + kOffQ;
 #pragma unroll
-          for (int e = 0; e < 8; ++e) {
-            const float4 v = make_float4(__uint_as_float(ov[4 * e]) * inv, __uint_as_float(ov[4 * e + 1]) * inv,
-                                         __uint_as_float(ov[4 * e + 2]) * inv,
-                                         __uint_as_float(ov[4 * e + 3]) * inv);
-            __stcg(dst + (size_t)(16 * hf + 8 * c4 + e) * dstride, v);
+        for (int k = 0; k < kRows / 16; ++k) {
+          const int rq = 2 * ((warp - kWarpSoft0) + 8 * k) + qhalf;
+          const int j = qc & 7;
+          *reinterpret_cast<uint4*>(qs + (qc >> 3) * kKVHalf + (rq >> 3) * 1024 + (rq & 7) * 128 +
+                                    ((j ^ (rq & 7)) << 4)) =
+              rb * kRows + rq < R ? qv[k] : make_uint4(0u, 0u, 0u, 0u);
+        }
+        fence_async_smem();   // generic-proxy writes, read by the tensor core
+        mbar_arrive(q_ready);
+      }
+      // m_used is kept in raw score units (scale > 0, so the max commutes with it)
+      float m_used = -INFINITY, l = 0.f;
+      const float sl2 = p.scale_log2;
+      const float kFail = __int_as_float(0x7fffffff);   // NaN: "this half's wait failed"
+      bool ok = true;
+      // the loop runs over the CTA's tile count tg (ring phases), with the
+      // segment's first tile at tg = tb; key positions and staged page ids are
+      // addressed from bases shifted back by tb tiles, so that no register
+      // holds tb across the loop
+      const int tg_end = tb + n_tiles, tg_ctx_end = tb + n_ctx_tiles;
+      const int kb0 = k_begin - tb * kKT;
+      const int32_t* pages0 = s_pages - (kKT / 16) * tb;
+      for (int tg = tb; tg < tg_end; ++tg) {
+        const int sb = tg % kSB;    // S buffer of this tile
+        const int xb = tg & 1;      // pair-exchange slot
+        // wait outcomes are warp-uniform: the TMEM accesses that follow are
+        // warp-collective (.sync.aligned)
+        const bool got =
+            __all_sync(0xffffffffu, mbar_wait(s_full + 8 * sb, (uint32_t)((tg / kSB) & 1), &s_abort));
+        uint32_t sr[64];
+        float tmax = -INFINITY;
+        if (got) {
+          tc_fence_after();
+          tc_ld32(tl + sb * kKT + 64 * hf, *reinterpret_cast<uint32_t(*)[32]>(&sr[0]));
+          tc_ld32(tl + sb * kKT + 64 * hf + 32, *reinterpret_cast<uint32_t(*)[32]>(&sr[32]));
+          // visibility of this half's 64 keys as one 64-bit word
+          uint64_t kw;
+          if (tg < tg_ctx_end) {
+            const unsigned m = tile_mask(pages0, tg, kb0, k_end);
+            const int nv = min(max(k_end - (kb0 + tg * kKT) - 64 * hf, 0), 64);
+            uint64_t pgw = 0ull;
+#pragma unroll
+            for (int i = 0; i < 4; ++i) pgw |= ((m >> (4 * hf + i)) & 1u) ? (0xFFFFull << (16 * i)) : 0ull;
+            kw = pgw & (nv >= 64 ? ~0ull : ((1ull << nv) - 1ull));
+          } else {
+            const int th = min(max(T - 64 * hf, 0), 64);
+            kw = ancw & (th >= 64 ? ~0ull : ((1ull << th) - 1ull));
+          }
+          if (!vrow) kw = 0ull;
+          if (!__all_sync(0xffffffffu, kw == ~0ull)) {
+#pragma unroll
+            for (int c = 0; c < 64; ++c)
+              if (!((kw >> c) & 1ull)) sr[c] = __float_as_uint(-INFINITY);
+          }
+          float mx[8];
+#pragma unroll
+          for (int c = 0; c < 8; ++c) mx[c] = __uint_as_float(sr[c]);
+#pragma unroll
+          for (int c = 8; c < 64; ++c) mx[c & 7] = fmaxf(mx[c & 7], __uint_as_float(sr[c]));
+          tmax = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
+                       fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
+        }
+        // the pair swaps its halves' maxima; both S halves are in registers before
+        // either warp overwrites S with P
+        s_xmax[xb][hf][r] = got ? tmax : kFail;
+        tc_fence_before();
+        asm volatile("bar.sync %0, 64;" ::"r"(pair_bar) : "memory");
+        tc_fence_after();
+        const float other = s_xmax[xb][hf ^ 1][r];
+        if (!__all_sync(0xffffffffu, got && other == other)) {
+          ok = false;
+          break;
+        }
+        tmax = fmaxf(tmax, other);
+        const float m_new = fmaxf(m_used, tmax);
+        const bool need = (m_new - m_used) * sl2 > kRescaleLog2;   // true when m_used = -inf < m_new
+        if (tg > 0 && __any_sync(0xffffffffu, need)) {
+          // O must hold P.V(tg-1) before this half's columns are rescaled; a failed
+          // wait sets the abort flag, and the pair stops at the next barrier.  At a
+          // segment's first tile that product belongs to the previous segment (its
+          // completion was already waited for) and the rescale is harmless: the
+          // segment's first P.V overwrites O.
+          if (__all_sync(0xffffffffu,
+                         mbar_wait(o_done + 8 * ((tg - 1) & 1), (uint32_t)(((tg - 1) >> 1) & 1), &s_abort))) {
+            tc_fence_after();
+            const float f = need ? ex2((m_used - m_new) * sl2) : 1.f;
+#pragma unroll 1
+            for (int c4 = 0; c4 < 2; ++c4) {
+              uint32_t ov[32];
+              tc_ld32(tl + kColO + 64 * hf + 32 * c4, ov);
+#pragma unroll
+              for (int e = 0; e < 32; ++e) ov[e] = __float_as_uint(__uint_as_float(ov[e]) * f);
+              tc_st32(tl + kColO + 64 * hf + 32 * c4, ov);
+            }
+          } else {
+            ok = false;
+          }
+        }
+        if (need) {
+          l *= ex2((m_used - m_new) * sl2);
+          m_used = m_new;
+        }
+        const float nms = m_used == -INFINITY ? 0.f : -m_used * sl2;
+        // p = 2^(s*scale_log2 - m); P = head + tail, both bf16 (top 16 bits): this
+        // half's head pairs go to columns 32 hf.. of the S buffer, its tail pairs
+        // to 64 + 32 hf..
+        // (pairs of columns run on packed fp32x2 arithmetic: the scale-and-shift,
+        // the running sums and the tail subtraction take one instruction per pair)
+        const uint64_t sl2x2 = f2_pack(__float_as_uint(sl2), __float_as_uint(sl2));
+        const uint64_t nmsx2 = f2_pack(__float_as_uint(nms), __float_as_uint(nms));
+        uint64_t ls2[4];
+        uint32_t hw[32], tw[32];
+#pragma unroll
+        for (int e = 0; e < 32; ++e) {
+          uint32_t y0, y1;
+          f2_unpack(f2_fma(f2_pack(sr[2 * e], sr[2 * e + 1]), sl2x2, nmsx2), y0, y1);
+          const uint32_t p0 = __float_as_uint(ex2(__uint_as_float(y0)));
+          const uint32_t p1 = __float_as_uint(ex2(__uint_as_float(y1)));
+          const uint64_t pp = f2_pack(p0, p1);
+          ls2[e & 3] = e < 4 ? pp : f2_add(ls2[e & 3], pp);
+          const uint32_t h0 = p0 & 0xFFFF0000u;
+          const uint32_t h1 = p1 & 0xFFFF0000u;
+          uint32_t t0, t1;
+          f2_unpack(f2_sub(pp, f2_pack(h0, h1)), t0, t1);
+          hw[e] = __byte_perm(h0, h1, 0x7632);
+          tw[e] = __byte_perm(t0, t1, 0x7632);
+        }
+        tc_st32(tl + sb * kKT + 32 * hf, hw);
+        tc_st32(tl + sb * kKT + 64 + 32 * hf, tw);
+        {
+          uint32_t a0, a1, b0, b1, c0, c1, d0, d1;
+          f2_unpack(ls2[0], a0, a1);
+          f2_unpack(ls2[1], b0, b1);
+          f2_unpack(ls2[2], c0, c1);
+          f2_unpack(ls2[3], d0, d1);
+          l += ((__uint_as_float(a0) + __uint_as_float(a1)) + (__uint_as_float(b0) + __uint_as_float(b1))) +
+               ((__uint_as_float(c0) + __uint_as_float(c1)) + (__uint_as_float(d0) + __uint_as_float(d1)));
+        }
+        tc_fence_before();
+        mbar_arrive(p_full + 8 * sb);
+      }
+      // wait for the last P.V; the pair adds its two sums, then each half writes
+      // its 64 columns out: O / l itself when the segment is a whole row block,
+      // else the partial (O, m, l) to the segment's slot.  The wait is on a
+      // barrier of its own: here the tensor pipe may still owe P.V(n-3) and
+      // P.V(n-1), two phases of the same o_done barrier, which a parity wait
+      // cannot tell apart (inside the loop at most one phase is pending, since
+      // S(t) completes after P.V(t-3))
+      const bool fin = ok && n_tiles > 0 && mbar_wait(o_final, (uint32_t)(nseg & 1), &s_abort);
+      const bool have = __all_sync(0xffffffffu, fin);
+      s_xl[hf][r] = have ? l : kFail;
+      asm volatile("bar.sync %0, 64;" ::"r"(pair_bar) : "memory");
+      const float l_sum = s_xl[0][r] + s_xl[1][r];     // NaN when either half failed
+      const bool both = have && l_sum == l_sum;
+      const float row_m = (both && vrow && m_used != -INFINITY) ? m_used * sl2 : -INFINITY;
+      const float row_l = (both && vrow && m_used != -INFINITY) ? l_sum : 0.f;
+      float4* dst;
+      size_t dstride;                                   // float4 between column chunks
+      float inv = 1.f;
+      if (alone) {
+        const size_t orow = (size_t)(o + node) * p.n_q + hk * g + (rr - node * g);
+        dst = reinterpret_cast<float4*>(p.out + orow * kD);
+        dstride = 1;
+        inv = row_l > 0.f ? 1.f / row_l : 0.f;
+      } else {
+        dst = reinterpret_cast<float4*>(p.part + slot * kAttnPartBytes) + r;
+        dstride = kRows;
+      }
+      const bool store = alone ? vrow : row_l > 0.f;
+      // the TMEM read is warp-collective: the whole warp reads when any lane stores
+      if (__any_sync(0xffffffffu, store)) {
+        tc_fence_after();
+#pragma unroll 1
+        for (int c4 = 0; c4 < 2; ++c4) {
+          uint32_t ov[32];
+          tc_ld32(tl + kColO + 64 * hf + 32 * c4, ov);
+          if (store) {
+#pragma unroll
+            for (int e = 0; e < 8; ++e) {
+              const float4 v = make_float4(__uint_as_float(ov[4 * e]) * inv, __uint_as_float(ov[4 * e + 1]) * inv,
+                                           __uint_as_float(ov[4 * e + 2]) * inv,
+                                           __uint_as_float(ov[4 * e + 3]) * inv);
+              __stcg(dst + (size_t)(16 * hf + 8 * c4 + e) * dstride, v);
+            }
           }
         }
       }
+      if (!alone) {
+        if (hf == 0)
+          __stcg(reinterpret_cast<float2*>(p.part + slot * kAttnPartBytes + kAttnMlOff) + r,
+                 make_float2(row_m, row_l));
+        __threadfence();
+      }
     }
-    if (!alone) {
-      if (hf == 0)
-        __stcg(reinterpret_cast<float2*>(p.part + cta * kAttnPartBytes + kAttnMlOff) + r,
-               make_float2(row_m, row_l));
-      __threadfence();
-    }
+    if constexpr (!kBal) break;
+    // end of the segment: every role is done with its pages, Q, S buffers and O
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (s_abort) break;
   }
 
   // ---- CTA teardown: drain on abort, free TMEM --------------------------------
@@ -647,56 +839,111 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
     }
     __syncwarp();
     tc_fence_after();
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols)
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(s_tmem), "r"(kTmemCols)
                  : "memory");
   }
-  if (p.S == 1) return;
 
-  // ---- merge ----------------------------------------------------------------------------
-  // once every slot of the row block is complete and visible, chunk `split`
-  // merges rows [r0, r0 + nown) of the row block
-  const size_t cta0 = ((size_t)blockIdx.z * gridDim.y + blockIdx.y) * gridDim.x + (size_t)rb * p.S;
-  const uint8_t* slot0 = p.part + cta0 * kAttnPartBytes;
-  uint32_t* cnt = reinterpret_cast<uint32_t*>(p.part + cta0 * kAttnPartBytes + kAttnCntOff);
-  __shared__ int s_ready;
-  if (p.coop) {
+  __shared__ int s_ready[2];
+  if constexpr (kBal) {
+    // ---- merge of split row blocks (balanced mode) ----------------------------------
+    // every CTA counts all its pieces before it waits for any (the launch is
+    // cooperative, so all CTAs are resident and every count arrives)
+    const int npieces = s_npc;     // written by thread 0 before the teardown barrier
+    if (npieces == 0) return;
+    uint32_t* cnt[2];
+#pragma unroll
+    for (int i = 0; i < 2; ++i)
+      cnt[i] = reinterpret_cast<uint32_t*>(p.part + (size_t)s_pc[i < npieces ? i : 0].slot0 * kAttnPartBytes +
+                                           kAttnCntOff);
     if (threadIdx.x == 0) {
-      red_add_release(cnt, 1u);     // this CTA's slot (ordered before by the fences and barrier)
-      const bool ready = wait_count_geq(cnt, (uint32_t)p.S);
-      if (!ready) flag_error(p.err, EE_DEVERR_TIMEOUT);
-      s_ready = ready;
+      for (int i = 0; i < npieces; ++i) red_add_release(cnt[i], 1u);
+      for (int i = 0; i < npieces; ++i) {
+        const bool ready = wait_count_geq(cnt[i], (uint32_t)s_pc[i].K);
+        if (!ready) flag_error(p.err, EE_DEVERR_TIMEOUT);
+        s_ready[i] = ready;
+      }
     }
     __syncthreads();
-  } else {
-    cluster_sync();
-    if (threadIdx.x == 0) s_ready = 1;
-    __syncthreads();
-  }
-  const int rpc = (kRows + p.S - 1) / p.S;
-  const int r0 = split * rpc;
-  const int nown = s_ready ? max(0, min(rpc, min(kRows, R - rb * kRows) - r0)) : 0;
-  if (nown > 0) {
-    const int row0 = rb * kRows + r0;
-    switch (p.S) {
-#define EE_MERGE_CASE(n) \
-  case n:                \
-    merge_rows<n>(p, slot0, row0, r0, nown, o, hk); \
+    for (int i = 0; i < npieces; ++i) {
+      const BalPiece q = s_pc[i];
+      const int rpc = (kRows + q.K - 1) / q.K;
+      const int r0 = q.k * rpc;
+      const int nown = s_ready[i] ? max(0, min(rpc, min(kRows, q.R - q.rb * kRows) - r0)) : 0;
+      if (nown > 0) {
+        const int row0 = q.rb * kRows + r0;
+        switch (q.K) {
+#define EE_MERGE_CASE(n)                                                                   \
+  case n:                                                                                  \
+    merge_rows<n>(p, (size_t)q.slot0, (size_t)q.slot1, 2, row0, r0, nown, q.o, q.hk); \
     break;
-      EE_MERGE_CASE(2) EE_MERGE_CASE(3) EE_MERGE_CASE(4) EE_MERGE_CASE(5) EE_MERGE_CASE(6)
-      EE_MERGE_CASE(7) EE_MERGE_CASE(8) EE_MERGE_CASE(9) EE_MERGE_CASE(10) EE_MERGE_CASE(11)
-      EE_MERGE_CASE(12) EE_MERGE_CASE(13) EE_MERGE_CASE(14) EE_MERGE_CASE(15) EE_MERGE_CASE(16)
+          EE_MERGE_CASE(2) EE_MERGE_CASE(3) EE_MERGE_CASE(4) EE_MERGE_CASE(5) EE_MERGE_CASE(6)
+          EE_MERGE_CASE(7) EE_MERGE_CASE(8) EE_MERGE_CASE(9) EE_MERGE_CASE(10) EE_MERGE_CASE(11)
+          EE_MERGE_CASE(12) EE_MERGE_CASE(13) EE_MERGE_CASE(14) EE_MERGE_CASE(15) EE_MERGE_CASE(16)
 #undef EE_MERGE_CASE
-      default:
-        break;
+          default:
+            break;
+        }
+      }
     }
-  }
-  if (p.coop) {
-    // every CTA of the row block has passed its wait once all have counted
-    // themselves here: the last returns both counters to zero
+    // every piece's CTA has passed its wait once all have counted themselves
+    // here: the last returns both counters to zero
     __syncthreads();
-    if (threadIdx.x == 0 && s_ready && atomicAdd(cnt + 1, 1u) == (uint32_t)p.S - 1) {
-      cnt[0] = 0u;
-      cnt[1] = 0u;
+    if (threadIdx.x == 0)
+      for (int i = 0; i < npieces; ++i)
+        if (s_ready[i] && atomicAdd(cnt[i] + 1, 1u) == (uint32_t)s_pc[i].K - 1) {
+          cnt[i][0] = 0u;
+          cnt[i][1] = 0u;
+        }
+    return;
+  } else {
+    if (skip || p.S == 1) return;
+
+    // ---- merge (uniform modes) -------------------------------------------------------
+    // once every slot of the row block is complete and visible, chunk `split`
+    // merges rows [r0, r0 + nown) of the row block
+    const int R = u_R, o = u_o;
+    const int rb = blockIdx.x / p.S;
+    const size_t cta0 = ((size_t)blockIdx.z * gridDim.y + blockIdx.y) * gridDim.x + (size_t)rb * p.S;
+    uint32_t* cnt = reinterpret_cast<uint32_t*>(p.part + cta0 * kAttnPartBytes + kAttnCntOff);
+    if (p.coop) {
+      if (threadIdx.x == 0) {
+        red_add_release(cnt, 1u);     // this CTA's slot (ordered before by the fences and barrier)
+        const bool ready = wait_count_geq(cnt, (uint32_t)p.S);
+        if (!ready) flag_error(p.err, EE_DEVERR_TIMEOUT);
+        s_ready[0] = ready;
+      }
+      __syncthreads();
+    } else {
+      cluster_sync();
+      if (threadIdx.x == 0) s_ready[0] = 1;
+      __syncthreads();
+    }
+    const int rpc = (kRows + p.S - 1) / p.S;
+    const int r0 = split * rpc;
+    const int nown = s_ready[0] ? max(0, min(rpc, min(kRows, R - rb * kRows) - r0)) : 0;
+    if (nown > 0) {
+      const int row0 = rb * kRows + r0;
+      switch (p.S) {
+#define EE_MERGE_CASE(n)                                                                  \
+  case n:                                                                                 \
+    merge_rows<n>(p, cta0, cta0 + 1, 1, row0, r0, nown, o, (int)blockIdx.y); \
+    break;
+        EE_MERGE_CASE(2) EE_MERGE_CASE(3) EE_MERGE_CASE(4) EE_MERGE_CASE(5) EE_MERGE_CASE(6)
+        EE_MERGE_CASE(7) EE_MERGE_CASE(8) EE_MERGE_CASE(9) EE_MERGE_CASE(10) EE_MERGE_CASE(11)
+        EE_MERGE_CASE(12) EE_MERGE_CASE(13) EE_MERGE_CASE(14) EE_MERGE_CASE(15) EE_MERGE_CASE(16)
+#undef EE_MERGE_CASE
+        default:
+          break;
+      }
+    }
+    if (p.coop) {
+      // every CTA of the row block has passed its wait once all have counted
+      // themselves here: the last returns both counters to zero
+      __syncthreads();
+      if (threadIdx.x == 0 && s_ready[0] && atomicAdd(cnt + 1, 1u) == (uint32_t)p.S - 1) {
+        cnt[0] = 0u;
+        cnt[1] = 0u;
+      }
     }
   }
 }
@@ -717,7 +964,7 @@ int active_clusters(int S) {
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     int n = 0;
-    if (cudaOccupancyMaxActiveClusters(&n, attn_tc_kernel, &cfg) != cudaSuccess || n < 1) {
+    if (cudaOccupancyMaxActiveClusters(&n, attn_tc_kernel<false>, &cfg) != cudaSuccess || n < 1) {
       cudaGetLastError();
       n = std::max(1, kNumSMs / S);
     }
@@ -726,14 +973,15 @@ int active_clusters(int S) {
   return cache[S];
 }
 
-// CTAs of this kernel the GPU holds at once (asked once; -1 if unknown).
+// CTAs of one instantiation the GPU holds at once (asked once; -1 if unknown).
+template <bool kBal>
 int resident_ctas() {
   static int cap = 0;
   if (!cap) {
     int dev = 0, sms = 0, per = 0;
     if (cudaGetDevice(&dev) != cudaSuccess ||
         cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
-        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per, attn_tc_kernel, kThreads, kSmemBytes) !=
+        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per, attn_tc_kernel<kBal>, kThreads, kSmemBytes) !=
             cudaSuccess ||
         per < 1) {
       cudaGetLastError();
@@ -743,6 +991,19 @@ int resident_ctas() {
     }
   }
   return cap;
+}
+
+// Both instantiations take the full dynamic shared memory (set once).
+cudaError_t set_attrs() {
+  static bool done = false;
+  if (done) return cudaSuccess;
+  cudaError_t e = cudaFuncSetAttribute(attn_tc_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)kSmemBytes);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(attn_tc_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)kSmemBytes);
+  done = e == cudaSuccess;
+  return e;
 }
 
 // Chunk length for s chunks (the last one also carries the tree tile), the
@@ -760,15 +1021,22 @@ void chunk_for(int max_ctx, int s, int* chunk, int* used, int* tiles) {
 struct Split {
   int S = 1, chunk = EE_PAGE;
   bool coop = false;
+  bool bal = false;            // balanced work list (cooperative, one CTA per SM)
+  int ctas = 0;                // balanced: grid size; CTAs sharing the work (at most); tiles per CTA
+  int bal_ctas = 0, bal_tiles = 0;
 };
 
-// Number of chunks per row block, their length and the synchronisation mode.
-// Cost = waves x (tiles of the busiest CTA + a fixed per-CTA cost of about 3):
+// Launch plan.  Cost, in half-tiles, = 2 x waves x (tiles of the busiest CTA
+// + a fixed per-CTA cost of about 3):
 //   cluster mode: S <= 8, waves from the clusters the GPU holds at once (one
 //   slot fewer per wave once a second wave is needed);
 //   cooperative mode: one wave by construction, S up to 16 with n_rb x S
-//   CTAs no more than the GPU holds.  Ties go to the cooperative mode.
-Split choose_split(int max_ctx, int n_rb) {
+//   CTAs no more than the GPU holds.  Ties go to the cooperative mode;
+//   balanced mode: every resident CTA takes an equal share of all units'
+//   tiles (w_max at most, t_max per unit at most) and may cross one unit
+//   boundary (about 1.5 tiles more); it needs 2 partial slots per CTA, a
+//   share of at most 256 context tiles (the staged page ids) and B <= 512.
+Split choose_split(int max_ctx, int n_rb, long w_max, int t_max, int B, size_t part_slots) {
   Split best;
   if (max_ctx <= 0) return best;
   const int min_splits = (max_ctx + kMaxCtaPages * EE_PAGE - 1) / (kMaxCtaPages * EE_PAGE);
@@ -782,26 +1050,41 @@ Split choose_split(int max_ctx, int n_rb) {
     const long act = active_clusters(used);
     long waves = (n_rb + act - 1) / act;
     if (waves >= 2 && act > 1) waves = (n_rb + act - 2) / (act - 1);
-    const long cost = waves * (tiles + 3);
+    const long cost = 2 * waves * (tiles + 3);
     if (best_cost < 0 || cost < best_cost) {
       best_cost = cost;
       best.S = used;
       best.chunk = chunk;
     }
   }
-  const int cap = resident_ctas();
+  const int cap = resident_ctas<false>();
   if (cap > 0) {
     for (int s = std::max(2, min_splits); s <= kMaxSplits && (long)s * n_rb <= cap; ++s) {
       int chunk, used, tiles;
       chunk_for(max_ctx, s, &chunk, &used, &tiles);
       if (used < 2) continue;
-      const long cost = tiles + 3;
+      const long cost = 2 * (tiles + 3);
       if (cost <= best_cost) {
         best_cost = cost;
         best.S = used;
         best.chunk = chunk;
         best.coop = true;
       }
+    }
+  }
+  const int capb = resident_ctas<true>();
+  if (capb > 0 && B <= kMaxBalSeqs && w_max <= (long)(kMaxCtaPages / (kKT / EE_PAGE)) * capb &&
+      part_slots >= 2 * (size_t)capb) {
+    const long m = std::max(2, (t_max + 13) / 14);
+    const long n_eff = std::min<long>(capb, std::max<long>(1, w_max / m));
+    const long share = (w_max + n_eff - 1) / n_eff;
+    const long cost = 2 * share + 9;
+    if (cost < best_cost) {
+      best.bal = true;
+      best.coop = true;
+      best.ctas = capb;
+      best.bal_ctas = (int)n_eff;
+      best.bal_tiles = (int)share;
     }
   }
   return best;
@@ -815,21 +1098,25 @@ extern "C" ee_status ee_attn_plan(int32_t B, int32_t max_T, int32_t n_q, int32_t
   if (B < 1 || max_T < 1 || max_T > EE_MAX_TREE || n_q < 1 || n_kv < 1 || n_q % n_kv != 0 ||
       max_ctx < 0 || !splits || !chunk || !mode || !ctas)
     return EE_ERR_INVALID_ARG;
-  static bool attr_set = false;
-  if (!attr_set) {
-    EE_CUDA_OK(cudaFuncSetAttribute(attn_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                    (int)kSmemBytes));
-    attr_set = true;
-  }
+  EE_CUDA_OK(set_attrs());
   const int nrb = (max_T * (n_q / n_kv) + kRows - 1) / kRows;
-  const Split sp = choose_split(max_ctx, nrb * n_kv * B);
-  *splits = sp.S;
-  *chunk = sp.chunk;
-  *mode = sp.S == 1 ? 0 : (sp.coop ? 2 : 1);
-  *ctas = nrb * sp.S * n_kv * B;
+  const int t_max = (max_ctx + kKT - 1) / kKT + 1;
+  // the partial slots of a workspace sized by ee_workspace_size
+  const size_t slots = std::max((size_t)B * n_q * kAttnMaxSplits, 2 * (size_t)kNumSMsMax);
+  const Split sp = choose_split(max_ctx, nrb * n_kv * B, (long)B * n_kv * nrb * t_max, t_max, B, slots);
+  if (sp.bal) {
+    *splits = sp.bal_ctas;
+    *chunk = sp.bal_tiles * kKT;
+    *mode = 3;
+    *ctas = sp.ctas;
+  } else {
+    *splits = sp.S;
+    *chunk = sp.chunk;
+    *mode = sp.S == 1 ? 0 : (sp.coop ? 2 : 1);
+    *ctas = nrb * sp.S * n_kv * B;
+  }
   return EE_OK;
 }
-
 extern "C" ee_status ee_tree_verify_attn(const ee_bf16* q, const ee_bf16* k_tree,
                                          const ee_bf16* v_tree, const ee_bf16* k_cache,
                                          const ee_bf16* v_cache, int32_t num_pages,
@@ -857,12 +1144,7 @@ extern "C" ee_status ee_tree_verify_attn(const ee_bf16* q, const ee_bf16* k_tree
   // a CTA stages at most kMaxCtaPages page ids, and a cluster holds at most 8 chunks
   if ((int64_t)max_ctx > (int64_t)kMaxCluster * kMaxCtaPages * EE_PAGE) return EE_ERR_UNSUPPORTED;
 
-  static bool attr_set = false;
-  if (!attr_set) {
-    EE_CUDA_OK(cudaFuncSetAttribute(attn_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                    (int)kSmemBytes));
-    attr_set = true;
-  }
+  EE_CUDA_OK(set_attrs());
   // tensor maps: cache [pages * n_kv * 16 rows][128], tree [total][n_kv][128]
   CUtensorMap tmKc, tmVc, tmKt, tmVt;
   {
@@ -881,10 +1163,12 @@ extern "C" ee_status ee_tree_verify_attn(const ee_bf16* q, const ee_bf16* k_tree
   }
   const int g = n_q / n_kv;
   const int nrb = (max_T * g + kRows - 1) / kRows;
-  const Split sp = choose_split(max_ctx, nrb * n_kv * B);
-  const int S = sp.S, chunk = sp.chunk;
+  const int t_max = (max_ctx + kKT - 1) / kKT + 1;
+  const size_t slots = ws_bytes > kAttnPartOff ? (ws_bytes - kAttnPartOff) / kAttnPartBytes : 0;
+  const Split sp = choose_split(max_ctx, nrb * n_kv * B, (long)B * n_kv * nrb * t_max, t_max, B, slots);
+  const int S = sp.bal ? 1 : sp.S, chunk = sp.chunk;
   // a split launch writes one partial slot per CTA after the zeroed part
-  if (S > 1 && ws_bytes < kAttnPartOff + (size_t)nrb * S * n_kv * B * kAttnPartBytes)
+  if (!sp.bal && S > 1 && ws_bytes < kAttnPartOff + (size_t)nrb * S * n_kv * B * kAttnPartBytes)
     return EE_ERR_WORKSPACE;
 
   AttnParams p;
@@ -907,11 +1191,12 @@ extern "C" ee_status ee_tree_verify_attn(const ee_bf16* q, const ee_bf16* k_tree
   p.nrb = nrb;
   p.chunk = chunk;
   p.S = S;
-  p.coop = (S > 1 && sp.coop) ? 1 : 0;
+  p.coop = (S > 1 && sp.coop) || sp.bal ? 1 : 0;
+  p.B = B;
   p.scale_log2 = scale * 1.4426950408889634f;
 
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(nrb * S, n_kv, B);
+  cfg.gridDim = sp.bal ? dim3(sp.ctas, 1, 1) : dim3(nrb * S, n_kv, B);
   cfg.blockDim = dim3(kThreads);
   cfg.dynamicSmemBytes = kSmemBytes;
   cfg.stream = (cudaStream_t)stream;
@@ -931,6 +1216,9 @@ extern "C" ee_status ee_tree_verify_attn(const ee_bf16* q, const ee_bf16* k_tree
     attr[1].val.clusterDim.z = 1;
     cfg.numAttrs = 2;
   }
-  EE_CUDA_OK(cudaLaunchKernelEx(&cfg, attn_tc_kernel, tmKc, tmVc, tmKt, tmVt, p));
+  if (sp.bal)
+    EE_CUDA_OK(cudaLaunchKernelEx(&cfg, attn_tc_kernel<true>, tmKc, tmVc, tmKt, tmVt, p));
+  else
+    EE_CUDA_OK(cudaLaunchKernelEx(&cfg, attn_tc_kernel<false>, tmKc, tmVc, tmKt, tmVt, p));
   return EE_OK;
 }

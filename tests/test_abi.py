@@ -58,16 +58,18 @@ def test_workspace_size(L):
     per node), and, when the
     context is split, one attention partial slot per CTA: 128 rows x 128 fp32
     + 128 x (m, l) + a 256-byte counter trailer, for at most B x n_q row blocks
-    x 16 chunks.  Independent of the node count."""
+    x 16 chunks, and at least two per SM (152) for the balanced launch.
+    Independent of the node count."""
     head = L.ee_workspace_size(1, 64, 28, 128, 0)
     assert head == L.ee_workspace_size(8, 2048, 56, 128, 0)
     assert head % 256 == 0
     assert head == 16896 + 152 * 256 * 80 + 8 * 2048 + 4 * 2048 * 8 + 4 * 2048
     slot = 128 * 128 * 4 + 128 * 8 + 256
     assert slot % 256 == 0
-    for B, n_q, ctx in ((1, 28, 4096), (8, 56, 262144), (3, 8, 16)):
-        assert L.ee_workspace_size(B, 64, n_q, 128, ctx) == head + B * n_q * 16 * slot
-        assert L.ee_workspace_size(B, 2048, n_q, 128, ctx) == head + B * n_q * 16 * slot
+    for B, n_q, ctx in ((1, 28, 4096), (8, 56, 262144), (3, 8, 16), (1, 8, 512)):
+        n_slots = max(B * n_q * 16, 2 * 152)
+        assert L.ee_workspace_size(B, 64, n_q, 128, ctx) == head + n_slots * slot
+        assert L.ee_workspace_size(B, 2048, n_q, 128, ctx) == head + n_slots * slot
     assert L.ee_workspace_size(-1, 64, 28, 128, 16) == 0
     assert L.ee_workspace_size(1, 64, 28, 128, -1) == 0
 

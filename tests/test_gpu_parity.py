@@ -114,6 +114,77 @@ def test_repeat_runs_bit_identical():
 
 
 # ----------------------------------------------------------------------------
+# balanced attention launch (one CTA per SM, an equal share of all row blocks'
+# tiles, row blocks split across CTAs and merged through counters)
+# ----------------------------------------------------------------------------
+
+_RAGGED = [W.TreeSpec(100, [(0, 14), (50, 14)], W.chain_path(60)),   # T = 128
+           W.TreeSpec(1, [], [0]),                                    # a decode step
+           W.TreeSpec(60, [(10, 17)], W.chain_path(30)),              # T = 77
+           W.TreeSpec(100, [(3, 28)], [0, 1, 2, 3, 100, 101, 102]),   # T = 128, path into a branch
+           W.TreeSpec(40, [], W.chain_path(20))]                      # T = 40
+
+
+@pytest.mark.parametrize("ctxs", [
+    [5000, 0, 3001, 4500, 17],      # ragged; an empty cache; a one-page context
+    [4999, 4096, 1, 127, 2049],
+])
+def test_balanced_ragged(ctxs):
+    """Five sequences of 1 to 128 nodes over ragged contexts with 6 query heads
+    per KV head: 60 row blocks leave a quarter of the SMs idle in an equal-chunk
+    launch, so the planner picks the balanced launch; CTAs' shares cross row
+    blocks, whole small row blocks sit inside one CTA, and large ones are split
+    over several CTAs.  Every node and head is checked against the oracle."""
+    E = _E()
+    w = W.build("tiny", seed=31, device="cuda", trees=_RAGGED, ctxs=ctxs, n_q=12, n_kv=2)
+    plan = E.ee_attn_plan(w.B, w.max_T, w.n_q, w.n_kv, int(w.ctx_len.max()))
+    assert plan["mode"] == "balanced", plan
+    full_check(w)
+
+
+def test_balanced_many_pieces():
+    """One sequence, 8 KV heads x 5 row blocks of 158 tiles: each row block is
+    split over 4 to 5 CTAs (sampled nodes, every head)."""
+    E = _E()
+    w = W.build("tiny", seed=32, device="cuda", trees=[_RAGGED[0]], ctx=20000, n_q=40, n_kv=8)
+    plan = E.ee_attn_plan(w.B, w.max_T, w.n_q, w.n_kv, int(w.ctx_len.max()))
+    assert plan["mode"] == "balanced", plan
+    full_check(w, attn_nodes=_sample_nodes(w, 12, 3))
+
+
+def test_balanced_repeat_bit_identical():
+    """The merge order of a split row block is fixed (piece order), so repeated
+    balanced launches give identical outputs, and the counters return to zero."""
+    E = _E()
+    from paper_2506_02780_gb300 import step as S
+    w = W.build("tiny", seed=33, device="cuda", trees=_RAGGED, ctxs=[5000, 0, 3001, 4500, 17],
+                n_q=12, n_kv=2)
+    st = S.from_workload(w)
+    assert E.ee_attn_plan(w.B, w.max_T, w.n_q, w.n_kv, st.max_ctx)["mode"] == "balanced"
+    outs = []
+    for _ in range(8):
+        st.run()
+        torch.cuda.synchronize()
+        outs.append(st.attn_out.clone())
+    assert E.ee_read_errors(st.ws) == 0
+    for o in outs[1:]:
+        assert torch.equal(outs[0], o)
+
+
+def test_launch_plans_of_the_configurations():
+    """The plans the configurations are timed with: 7b fills 144 SMs with 9
+    equal chunks of 16 row blocks; 33b (56 row blocks of 257 tiles) and the
+    ragged batch take the balanced launch."""
+    E = _E()
+    p7 = E.ee_attn_plan(1, 64, 28, 4, 4096)
+    assert p7["mode"] == "cooperative" and p7["splits"] == 9 and p7["ctas"] == 144, p7
+    p33 = E.ee_attn_plan(1, 128, 56, 8, 32768)
+    assert p33["mode"] == "balanced", p33
+    pb = E.ee_attn_plan(8, 96, 28, 4, 16384)
+    assert pb["mode"] == "balanced", pb
+
+
+# ----------------------------------------------------------------------------
 # device-detected bad input: error word set, access skipped, context usable
 # ----------------------------------------------------------------------------
 

@@ -271,6 +271,12 @@ def _plan(name, rng, overrides):
     if "trees" in o:
         specs = o.pop("trees")
         seqs = [dict(seqs[i % len(seqs)], spec=sp) for i, sp in enumerate(specs)]
+    if "ctxs" in o:
+        # one context length per sequence (after ``trees`` fixed the count)
+        cs = [int(c) for c in o.pop("ctxs")]
+        if len(cs) != len(seqs):
+            raise ValueError("ctxs needs one entry per sequence")
+        seqs = [dict(sp, ctx=c) for sp, c in zip(seqs, cs)]
     if o:
         raise ValueError(f"unused overrides {sorted(o)}")
     return shape, seqs
@@ -337,7 +343,8 @@ def build(name: str, seed: int | None = None, device="cpu", *, q_std: float = 1.
 
     ``name`` is one of CONFIG_NAMES; ``seed`` defaults to 1234 + the config's
     index.  Overrides (``ctx``, ``layers``, ``vocab``, ``hidden``, ``n_q``,
-    ``n_kv``, ``n``, ``trees``, and for the sweep ``B``) shrink or reshape a
+    ``n_kv``, ``n``, ``trees``, ``ctxs`` (one context length per sequence), and
+    for the sweep ``B``) shrink or reshape a
     configuration for tests.  ``q_std`` scales the queries (a large value makes
     the softmax peaky).  ``dup_rows`` > 0 copies that many planted target rows of
     the LM-head weight to a higher token id, creating exact logit ties.
