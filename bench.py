@@ -60,8 +60,9 @@ def parse_args():
 # DRAM bytes (read + write) per launch from one ncu capture of the kernel as it
 # now stands (profiles/ names the capture); a kernel changed since has no entry.
 TRAFFIC = {
-    ("tree_verify_attn", "7b"): 9061632,          # profiles/attn_tc_7b.md
-    ("tree_verify_attn", "33b"): 139859968,       # profiles/attn_tc_33b.md
+    ("tree_verify_attn", "7b"): 9061120,          # profiles/attn_tc_7b.md
+    ("tree_verify_attn", "33b"): 158299648,       # profiles/attn_tc_33b.md
+    ("tree_verify_attn", "batched"): 245043456,   # profiles/attn_tc_batched.md
     ("lmhead_accept", "7b"): 1095463424,          # profiles/lmhead_accept_7b.md
 }
 

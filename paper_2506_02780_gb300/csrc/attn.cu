@@ -223,7 +223,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
   // exclusive prefix of the sequences' work in tiles
   __shared__ int4 s_seq[kBal ? kMaxBalSeqs : 1];
   __shared__ int s_wpre[kBal ? kMaxBalSeqs + 1 : 1];
-  __shared__ int s_sched[6];                        // balanced: next tile, end tile, W, N, tiles, segments
+  __shared__ int s_sched[7];   // balanced: range start, range end, W, N, tiles done, segments done, next end
   __shared__ BalPiece s_pc[2];                      // balanced: this CTA's pieces of split units
   __shared__ int s_npc;
 
@@ -346,6 +346,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
         s_sched[3] = N;
         s_sched[4] = 0;
         s_sched[5] = 0;
+        s_sched[6] = s_sched[1];
         s_wpre[p.B] = W;
       }
     }
@@ -369,18 +370,25 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
     size_t slot;
     int32_t pgr[kPgPerThread];
     int x_next = 0;
+    int rot = 0;                // tiles run in the order rot, rot + 1, ..., n_tiles - 1, 0, ..., rot - 1
     // tiles this CTA processed before this segment (ring slots and phases count
     // over all segments), and the segments done; kept in shared memory so that
     // no register carries them across the softmax loop
     const int tb = kBal ? s_sched[4] : 0;
     const int nseg = kBal ? s_sched[5] : 0;
     if constexpr (kBal) {
-      const int x = s_sched[0], x_end = s_sched[1], W = s_sched[2], N = s_sched[3];
-      if (x >= x_end) break;
-      int lo = 0, hi = p.B;   // s_wpre[lo] <= x < s_wpre[hi]
+      // The CTA walks its range from the end: its last segment (the head of a
+      // row block) first.  Within a segment the tiles run rotated so that the
+      // CTA reads tile x of a row block at about its local time x mod P (P =
+      // the share): the CTAs holding other row blocks of the same KV head then
+      // read the same K/V tiles at about the same time, and L2 serves the
+      // repeats (each KV head's tiles are read by all its row blocks).
+      const int x_begin = s_sched[0], y = s_sched[6], W = s_sched[2], N = s_sched[3];
+      if (y <= x_begin) break;
+      int lo = 0, hi = p.B;   // s_wpre[lo] <= y - 1 < s_wpre[hi]
       while (hi - lo > 1) {
         const int mid = (lo + hi) >> 1;
-        if (s_wpre[mid] <= x) lo = mid; else hi = mid;
+        if (s_wpre[mid] <= y - 1) lo = mid; else hi = mid;
       }
       b = lo;
       const int4 sq = s_seq[b];
@@ -389,29 +397,34 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
       ctx = sq.z;
       const int tiles = sq.w;
       const int nrb_b = (T * g + kRows - 1) / kRows;
-      const int local = x - s_wpre[b];
-      const int u = local / tiles, t0 = local - u * tiles;
+      const int u = (y - 1 - s_wpre[b]) / tiles;
       hk = u / nrb_b;
       rb = u - hk * nrb_b;
-      const int len = min(tiles - t0, x_end - x);
+      const int U0 = s_wpre[b] + u * tiles;          // the unit's first tile in the work list
+      const int seg0 = max(U0, x_begin);
+      const int t0 = seg0 - U0;
+      const int len = y - seg0;
       const int n_ctx_b = tiles - 1;
       k_begin = min(t0, n_ctx_b) * kKT;
       k_end = t0 < n_ctx_b ? min(ctx, min(t0 + len, n_ctx_b) * kKT) : k_begin;
       with_tree = t0 + len == tiles;
+      const int P = (W + N - 1) / N;
+      int ph = (tb - t0) % P;
+      ph += ph < 0 ? P : 0;
+      rot = ph < len ? ph : 0;
       // the CTAs holding the unit's first and last tiles
-      const int U0 = x - t0;
       const int c0 = ((U0 + 1) * N - 1) / W;
       const int c1 = ((U0 + tiles) * N - 1) / W;
       alone = c0 == c1;
-      // a piece is this CTA's first segment (slot 2c) or its last (slot 2c + 1)
-      slot = 2 * (size_t)blockIdx.x + (nseg > 0 ? 1 : 0);
+      // a piece starts the CTA's range (slot 2c) or ends it (slot 2c + 1)
+      slot = 2 * (size_t)blockIdx.x + (seg0 > x_begin ? 1 : 0);
       if (!alone && threadIdx.x == 0 && s_npc < 2) {
         const int start0 = c0 * W / N;
         s_pc[s_npc] = BalPiece{hk, rb, o, T * g, c1 - c0 + 1, (int)blockIdx.x - c0,
                                2 * c0 + (U0 > start0 ? 1 : 0), 2 * (c0 + 1)};
         s_npc = s_npc + 1;
       }
-      x_next = x + len;
+      x_next = seg0;
       const int pg_first = k_begin / EE_PAGE;
       const int npg = (k_end - k_begin + EE_PAGE - 1) / EE_PAGE;   // <= kMaxCtaPages: see the plan
 #pragma unroll
@@ -498,7 +511,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
     tmem = s_tmem;
     // every thread has read the schedule position: advance it for the next segment
     if (kBal && threadIdx.x == 0) {
-      s_sched[0] = x_next;
+      s_sched[6] = x_next;
       s_sched[4] = tb + n_tiles;
       s_sched[5] = nseg + 1;
     }
@@ -525,13 +538,14 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
         const uint32_t dst = ring + st * kKVBytes;
         if (lane == 0) mbar_expect_tx(full, 2 * kKVHalf);
         __syncwarp();
-        if (t < n_ctx_tiles) {
+        const int i = t + rot < n_tiles ? t + rot : t + rot - n_tiles;   // the segment's tile
+        if (i < n_ctx_tiles) {
           // every 16-row block is written: blocks without a loaded page are read at
           // row -16, wholly out of range, which the TMA unit fills with zeros (a
           // stale V row would turn 0 * P into NaN)
           if (lane < kKT / 16) {
-            const int pos = k_begin + t * kKT + 16 * lane;
-            const int pg = pos < k_end ? s_pages[t * (kKT / 16) + lane] : -1;
+            const int pos = k_begin + i * kKT + 16 * lane;
+            const int pg = pos < k_end ? s_pages[i * (kKT / 16) + lane] : -1;
             const int row0 = pg >= 0 ? (pg * p.n_kv + hk) * EE_PAGE : -EE_PAGE;
             tma_load_2d(dst + lane * 2048, mc, full, 0, row0);
             tma_load_2d(dst + kKVHalf + lane * 2048, mc, full, 64, row0);
@@ -633,12 +647,10 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
       const float kFail = __int_as_float(0x7fffffff);   // NaN: "this half's wait failed"
       bool ok = true;
       // the loop runs over the CTA's tile count tg (ring phases), with the
-      // segment's first tile at tg = tb; key positions and staged page ids are
-      // addressed from bases shifted back by tb tiles, so that no register
-      // holds tb across the loop
-      const int tg_end = tb + n_tiles, tg_ctx_end = tb + n_ctx_tiles;
-      const int kb0 = k_begin - tb * kKT;
-      const int32_t* pages0 = s_pages - (kKT / 16) * tb;
+      // segment's first tile at tg = tb; step tg processes the segment's tile
+      // tg + d (mod n_tiles)
+      const int tg_end = tb + n_tiles;
+      const int d = rot - tb;
       for (int tg = tb; tg < tg_end; ++tg) {
         const int sb = tg % kSB;    // S buffer of this tile
         const int xb = tg & 1;      // pair-exchange slot
@@ -654,9 +666,10 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
           tc_ld32(tl + sb * kKT + 64 * hf + 32, *reinterpret_cast<uint32_t(*)[32]>(&sr[32]));
           // visibility of this half's 64 keys as one 64-bit word
           uint64_t kw;
-          if (tg < tg_ctx_end) {
-            const unsigned m = tile_mask(pages0, tg, kb0, k_end);
-            const int nv = min(max(k_end - (kb0 + tg * kKT) - 64 * hf, 0), 64);
+          const int i = tg + d < n_tiles ? tg + d : tg + d - n_tiles;
+          if (i < n_ctx_tiles) {
+            const unsigned m = tile_mask(s_pages, i, k_begin, k_end);
+            const int nv = min(max(k_end - (k_begin + i * kKT) - 64 * hf, 0), 64);
             uint64_t pgw = 0ull;
 #pragma unroll
             for (int i = 0; i < 4; ++i) pgw |= ((m >> (4 * hf + i)) & 1u) ? (0xFFFFull << (16 * i)) : 0ull;
@@ -704,13 +717,14 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
             tc_fence_after();
             const float f = need ? ex2((m_used - m_new) * sl2) : 1.f;
 #pragma unroll 1
-            for (int c4 = 0; c4 < 2; ++c4) {
-              uint32_t ov[32];
-              tc_ld32(tl + kColO + 64 * hf + 32 * c4, ov);
+            for (int c4 = 0; c4 < 4; ++c4) {
+              uint32_t ov[16];
+              tc_ld16(tl + kColO + 64 * hf + 16 * c4, ov);
 #pragma unroll
-              for (int e = 0; e < 32; ++e) ov[e] = __float_as_uint(__uint_as_float(ov[e]) * f);
-              tc_st32(tl + kColO + 64 * hf + 32 * c4, ov);
+              for (int e = 0; e < 16; ++e) ov[e] = __float_as_uint(__uint_as_float(ov[e]) * f);
+              tc_st16_nowait(tl + kColO + 64 * hf + 16 * c4, ov);
             }
+            tc_wait_st();
           } else {
             ok = false;
           }
@@ -728,24 +742,31 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
         const uint64_t sl2x2 = f2_pack(__float_as_uint(sl2), __float_as_uint(sl2));
         const uint64_t nmsx2 = f2_pack(__float_as_uint(nms), __float_as_uint(nms));
         uint64_t ls2[4];
-        uint32_t hw[32], tw[32];
+        // two halves of 16 column pairs: each half's head and tail words go
+        // out before the next half is computed (fewer live registers)
 #pragma unroll
-        for (int e = 0; e < 32; ++e) {
-          uint32_t y0, y1;
-          f2_unpack(f2_fma(f2_pack(sr[2 * e], sr[2 * e + 1]), sl2x2, nmsx2), y0, y1);
-          const uint32_t p0 = __float_as_uint(ex2(__uint_as_float(y0)));
-          const uint32_t p1 = __float_as_uint(ex2(__uint_as_float(y1)));
-          const uint64_t pp = f2_pack(p0, p1);
-          ls2[e & 3] = e < 4 ? pp : f2_add(ls2[e & 3], pp);
-          const uint32_t h0 = p0 & 0xFFFF0000u;
-          const uint32_t h1 = p1 & 0xFFFF0000u;
-          uint32_t t0, t1;
-          f2_unpack(f2_sub(pp, f2_pack(h0, h1)), t0, t1);
-          hw[e] = __byte_perm(h0, h1, 0x7632);
-          tw[e] = __byte_perm(t0, t1, 0x7632);
+        for (int hh = 0; hh < 2; ++hh) {
+          uint32_t hw[16], tw[16];
+#pragma unroll
+          for (int e2 = 0; e2 < 16; ++e2) {
+            const int e = 16 * hh + e2;
+            uint32_t y0, y1;
+            f2_unpack(f2_fma(f2_pack(sr[2 * e], sr[2 * e + 1]), sl2x2, nmsx2), y0, y1);
+            const uint32_t p0 = __float_as_uint(ex2(__uint_as_float(y0)));
+            const uint32_t p1 = __float_as_uint(ex2(__uint_as_float(y1)));
+            const uint64_t pp = f2_pack(p0, p1);
+            ls2[e & 3] = e < 4 ? pp : f2_add(ls2[e & 3], pp);
+            const uint32_t h0 = p0 & 0xFFFF0000u;
+            const uint32_t h1 = p1 & 0xFFFF0000u;
+            uint32_t t0, t1;
+            f2_unpack(f2_sub(pp, f2_pack(h0, h1)), t0, t1);
+            hw[e2] = __byte_perm(h0, h1, 0x7632);
+            tw[e2] = __byte_perm(t0, t1, 0x7632);
+          }
+          tc_st16_nowait(tl + sb * kKT + 32 * hf + 16 * hh, hw);
+          tc_st16_nowait(tl + sb * kKT + 64 + 32 * hf + 16 * hh, tw);
         }
-        tc_st32(tl + sb * kKT + 32 * hf, hw);
-        tc_st32(tl + sb * kKT + 64 + 32 * hf, tw);
+        tc_wait_st();
         {
           uint32_t a0, a1, b0, b1, c0, c1, d0, d1;
           f2_unpack(ls2[0], a0, a1);
