@@ -23,6 +23,12 @@ tests/test_oracle_pins.py):
   accept_path      pinned: token-by-token replay of Eq. (piecewise), brute force
                    over all root-to-node paths, hand-worked golden cases
   kv_compact       pinned: sequential append into a slot dictionary, canaries
+  tree_kv_to_cache / tree_kv_from_cache
+                   pinned: round trip, slot-dictionary placement
+  kv_compact_inplace
+                   pinned: equals kv_compact on the committed positions after
+                   tree_kv_to_cache (random trees and paths), chains move
+                   nothing, a hand-worked overlapping move
   entropy_top_tau  pinned: closed forms of Eq. (entropy) / top_tau (H=0, uniform)
   verify_accept    pinned: reduces to accept_path (greedy; top-1; all-reuse trees),
                    top-V = direct, brute force over root-to-node paths, H = 0 and
@@ -38,6 +44,9 @@ from .ee_oracle import (  # noqa: F401
     lm_head_argmax,
     accept_path,
     kv_compact,
+    tree_kv_to_cache,
+    tree_kv_from_cache,
+    kv_compact_inplace,
     entropy_top_tau,
     VERIFY_MODES,
     node_ranking,

@@ -333,6 +333,87 @@ def kv_compact(k_tree, v_tree, k_cache, v_cache, block_table, ctx_len, node_off,
 
 
 # ----------------------------------------------------------------------------
+# In-place speculative K/V: the tree's K/V live in the cache slots after the
+# context (the accepted prefix extension of Sec. III-A without a separate
+# tree buffer)
+# ----------------------------------------------------------------------------
+
+def _slot(block_table, s, pos, num_pages):
+    page = int(block_table[s, pos // PAGE])
+    if page < 0 or page >= num_pages:
+        raise ValueError("no page allocated for position %d" % pos)
+    return page, pos % PAGE
+
+
+def tree_kv_to_cache(k_tree, v_tree, k_cache, v_cache, block_table, ctx_len, node_off):
+    """Place every tree node's K/V at cache position ctx + i (i = its local id),
+    every layer: where a K/V projection writes them when the tree is verified in
+    place.  Shapes as in kv_compact; copies are returned."""
+    kc = np.array(k_cache, copy=True)
+    vc = np.array(v_cache, copy=True)
+    kt, vt = np.asarray(k_tree), np.asarray(v_tree)
+    node_off = np.asarray(node_off)
+    for s in range(len(node_off) - 1):
+        o, T, ctx = int(node_off[s]), int(node_off[s + 1] - node_off[s]), int(ctx_len[s])
+        for i in range(T):
+            page, off = _slot(block_table, s, ctx + i, kc.shape[1])
+            kc[:, page, :, off, :] = kt[:, o + i, :, :]
+            vc[:, page, :, off, :] = vt[:, o + i, :, :]
+    return kc, vc
+
+
+def tree_kv_from_cache(k_cache, v_cache, block_table, ctx_len, node_off, n_layers=None):
+    """The tree's K/V as a [L, sumT, n_kv, d] array, read from positions ctx + i:
+    what attention over an in-place tree sees as the tree keys."""
+    kc, vc = np.asarray(k_cache), np.asarray(v_cache)
+    node_off = np.asarray(node_off)
+    L = kc.shape[0] if n_layers is None else n_layers
+    total = int(node_off[-1])
+    kt = np.zeros((L, total) + kc.shape[2:3] + kc.shape[4:], dtype=kc.dtype)
+    vt = np.zeros_like(kt)
+    for s in range(len(node_off) - 1):
+        o, T, ctx = int(node_off[s]), int(node_off[s + 1] - node_off[s]), int(ctx_len[s])
+        for i in range(T):
+            page, off = _slot(block_table, s, ctx + i, kc.shape[1])
+            kt[:, o + i] = kc[:L, page, :, off, :]
+            vt[:, o + i] = vc[:L, page, :, off, :]
+    return kt, vt
+
+
+def kv_compact_inplace(k_cache, v_cache, block_table, ctx_len, node_off, path, accept_len):
+    """Compaction when the tree's K/V already sit at positions ctx + i.
+
+    The accepted path (root first) must end up at positions ctx .. ctx + acc,
+    as kv_compact appends it.  Path entry k is node path[k] >= k (a parent's id
+    is below its child's), already at ctx + path[k]: entries with path[k] == k
+    stay, the others move down to ctx + k.  Moving in increasing k reads every
+    source before a later move overwrites it (a source ctx + path[k] is above
+    every earlier destination and at most the destination of a later entry
+    k' > k with path[k] == k').  Returns (k_cache', v_cache', dst_slot int32
+    [B, max_T] padded with -1, ctx_len' int32 [B] = ctx + accept_len + 1).
+    """
+    kc = np.array(k_cache, copy=True)
+    vc = np.array(v_cache, copy=True)
+    node_off = np.asarray(node_off)
+    B = len(node_off) - 1
+    max_T = path.shape[1]
+    dst = np.full((B, max_T), -1, dtype=np.int32)
+    ctx_out = np.asarray(ctx_len, dtype=np.int32).copy()
+    for s in range(B):
+        ctx = int(ctx_len[s])
+        for k in range(int(accept_len[s]) + 1):
+            node = int(path[s, k])
+            dpage, doff = _slot(block_table, s, ctx + k, kc.shape[1])
+            dst[s, k] = dpage * PAGE + doff
+            if node != k:
+                spage, soff = _slot(block_table, s, ctx + node, kc.shape[1])
+                kc[:, dpage, :, doff, :] = kc[:, spage, :, soff, :]
+                vc[:, dpage, :, doff, :] = vc[:, spage, :, soff, :]
+        ctx_out[s] = ctx + int(accept_len[s]) + 1
+    return kc, vc, dst, ctx_out
+
+
+# ----------------------------------------------------------------------------
 # Entropy-aware dynamic verification -- Eq. (entropy) and the top_tau rule
 # ----------------------------------------------------------------------------
 

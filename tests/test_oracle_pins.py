@@ -583,3 +583,116 @@ def test_verify_step_tiny_planted():
     assert r["ctx_out"][0] == 512 + 8
     assert r["bonus"][0] == w.planted_argmax[7]
     assert not np.isnan(r["attn"][0]).any()
+
+
+# ----------------------------------------------------------------------------
+# in-place speculative K/V: tree K/V at positions ctx + i, compaction by moves
+# ----------------------------------------------------------------------------
+
+def _inplace_case(seed, B=4, L=2, n_kv=2, d=4):
+    """Random trees (parent[i] drawn below i), a root-to-node path per tree,
+    ragged contexts (not page-aligned) and a shuffled block table."""
+    rng = np.random.default_rng(seed)
+    Ts = [int(rng.integers(1, 40)) for _ in range(B)]
+    ctx = np.asarray([int(rng.integers(0, 70)) for _ in range(B)], np.int32)
+    node_off = np.concatenate([[0], np.cumsum(Ts)]).astype(np.int32)
+    max_T = max(Ts)
+    max_pages = (int(ctx.max()) + max_T + 15) // 16 + 1
+    num_pages = B * max_pages
+    bt = rng.permutation(num_pages).astype(np.int32).reshape(B, max_pages)
+    path = np.full((B, max_T), -1, np.int32)
+    acc = np.zeros(B, np.int32)
+    for s, T in enumerate(Ts):
+        parent = [-1] + [int(rng.integers(0, i)) for i in range(1, T)]
+        u = int(rng.integers(0, T))
+        p = [u]
+        while parent[p[-1]] >= 0:
+            p.append(parent[p[-1]])
+        p = p[::-1]
+        path[s, :len(p)] = p
+        acc[s] = len(p) - 1
+    total = int(node_off[-1])
+    kt = rng.standard_normal((L, total, n_kv, d))
+    vt = rng.standard_normal((L, total, n_kv, d))
+    kc = rng.standard_normal((L, num_pages, n_kv, 16, d))
+    vc = rng.standard_normal((L, num_pages, n_kv, 16, d))
+    return dict(kt=kt, vt=vt, kc=kc, vc=vc, bt=bt, ctx=ctx, node_off=node_off, path=path, acc=acc,
+                Ts=Ts)
+
+
+@pytest.mark.parametrize("seed", [0, 1, 2])
+def test_tree_kv_placement_round_trip(seed):
+    c = _inplace_case(seed)
+    kc2, vc2 = O.tree_kv_to_cache(c["kt"], c["vt"], c["kc"], c["vc"], c["bt"], c["ctx"], c["node_off"])
+    # independent placement: a dict of slots, node by node
+    slots = {}
+    for s, T in enumerate(c["Ts"]):
+        for i in range(T):
+            pos = int(c["ctx"][s]) + i
+            slots[(int(c["bt"][s, pos // 16]), pos % 16)] = int(c["node_off"][s]) + i
+    for (page, off), src in slots.items():
+        np.testing.assert_array_equal(kc2[:, page, :, off], c["kt"][:, src])
+        np.testing.assert_array_equal(vc2[:, page, :, off], c["vt"][:, src])
+    keep = np.ones(c["kc"].shape[1:2] + (16,), bool)
+    for (page, off) in slots:
+        keep[page, off] = False
+    tk = c["kc"].transpose(0, 1, 3, 2, 4)
+    assert np.array_equal(kc2.transpose(0, 1, 3, 2, 4)[:, keep], tk[:, keep])
+    kt2, vt2 = O.tree_kv_from_cache(kc2, vc2, c["bt"], c["ctx"], c["node_off"])
+    np.testing.assert_array_equal(kt2, c["kt"])
+    np.testing.assert_array_equal(vt2, c["vt"])
+
+
+@pytest.mark.parametrize("seed", [3, 4, 5, 6, 7])
+def test_compact_inplace_equals_append(seed):
+    """With the tree's K/V placed at ctx + i, moving the path down gives the
+    cache kv_compact's append gives, on every position up to ctx + acc, and
+    leaves the context untouched."""
+    c = _inplace_case(seed)
+    placed_k, placed_v = O.tree_kv_to_cache(c["kt"], c["vt"], c["kc"], c["vc"], c["bt"], c["ctx"],
+                                            c["node_off"])
+    ik, iv, idst, ictx = O.kv_compact_inplace(placed_k, placed_v, c["bt"], c["ctx"], c["node_off"],
+                                              c["path"], c["acc"])
+    ak, av, adst, actx = O.kv_compact(c["kt"], c["vt"], c["kc"], c["vc"], c["bt"], c["ctx"],
+                                      c["node_off"], c["path"], c["acc"])
+    np.testing.assert_array_equal(idst, adst)
+    np.testing.assert_array_equal(ictx, actx)
+    for s in range(len(c["Ts"])):
+        for pos in range(int(c["ctx"][s]) + int(c["acc"][s]) + 1):
+            page, off = int(c["bt"][s, pos // 16]), pos % 16
+            np.testing.assert_array_equal(ik[:, page, :, off], ak[:, page, :, off])
+            np.testing.assert_array_equal(iv[:, page, :, off], av[:, page, :, off])
+            if pos < int(c["ctx"][s]):
+                np.testing.assert_array_equal(ik[:, page, :, off], c["kc"][:, page, :, off])
+
+
+def test_compact_inplace_chain_moves_nothing():
+    c = _inplace_case(8)
+    for s, T in enumerate(c["Ts"]):
+        a = min(T - 1, 5)
+        c["path"][s] = -1
+        c["path"][s, :a + 1] = np.arange(a + 1)
+        c["acc"][s] = a
+    pk, pv = O.tree_kv_to_cache(c["kt"], c["vt"], c["kc"], c["vc"], c["bt"], c["ctx"], c["node_off"])
+    ik, iv, _, _ = O.kv_compact_inplace(pk, pv, c["bt"], c["ctx"], c["node_off"], c["path"], c["acc"])
+    assert np.array_equal(ik, pk) and np.array_equal(iv, pv)
+
+
+def test_compact_inplace_overlapping_moves_golden():
+    """Path 0 -> 2 -> 3 (node 1 rejected): position ctx+1 takes node 2 from
+    ctx+2 before ctx+2 takes node 3 from ctx+3; ctx+3 keeps node 3."""
+    L, n_kv, d, T, ctx = 1, 1, 2, 4, 14                     # positions 14..17 straddle two pages
+    kt = np.arange(T, dtype=np.float64)[None, :, None, None] * np.ones((L, T, n_kv, d))
+    kc = np.full((L, 2, n_kv, 16, d), -1.0)
+    bt = np.asarray([[1, 0]], np.int32)
+    node_off = np.asarray([0, T], np.int32)
+    pk, pv = O.tree_kv_to_cache(kt, -kt, kc, kc.copy(), bt, [ctx], node_off)
+    path = np.asarray([[0, 2, 3, -1]], np.int32)
+    ik, iv, dst, ctx_out = O.kv_compact_inplace(pk, pv, bt, np.asarray([ctx]), node_off, path,
+                                                np.asarray([2]))
+    def at(a, pos):
+        return a[0, bt[0, pos // 16], 0, pos % 16, 0]
+    assert [at(ik, ctx + k) for k in range(4)] == [0.0, 2.0, 3.0, 3.0]
+    assert [at(iv, ctx + k) for k in range(3)] == [0.0, -2.0, -3.0]
+    assert list(dst[0, :3]) == [1 * 16 + 14, 1 * 16 + 15, 0 * 16 + 0]
+    assert ctx_out[0] == ctx + 3
