@@ -12,6 +12,9 @@
  *   ee_tree_verify_attn  tree-masked attention over the paged cache (Sec. III-A)
  *   ee_lmhead_accept     LM head + argmax + longest accepted path   (Eq. piecewise)
  *   ee_kv_compact        accepted path's K/V appended to the cache  (Sec. III-A)
+ *   ee_tree_verify_attn_inplace / ee_kv_compact_inplace
+ *                        the same two steps with the tree's K/V already in
+ *                        the cache after the context (in-place speculative K/V)
  *
  * Conventions shared by every entry point
  * ---------------------------------------
@@ -204,6 +207,27 @@ ee_status ee_tree_verify_attn(const ee_bf16* q, const ee_bf16* k_tree, const ee_
                               void* ws, size_t ws_bytes, ee_stream_t stream);
 
 /*
+ * ee_tree_verify_attn_inplace -- the same attention when the tree's K/V are
+ * already in the cache (in-place speculative K/V): node i of sequence s
+ * (local id i) has its keys and values at position ctx_len[s] + i of its
+ * pages, where the target's K/V projection wrote them, instead of in
+ * k_tree / v_tree.  A node attends to positions 0 .. ctx - 1 and to positions
+ * ctx + j for every ancestor j in anc (itself included): out is the same as
+ * ee_tree_verify_attn's with k_tree / v_tree read from those positions (Sec.
+ * III-A; the paper has no separate tree buffer either).  block_table must hold
+ * a page for every position below ctx_len + T: max_ctx + max_T <=
+ * max_pages * EE_PAGE (else EE_ERR_INVALID_ARG), and a missing page sets
+ * EE_DEVERR_PAGE with its keys skipped.  Other arguments, layouts, precision
+ * and errors as ee_tree_verify_attn.  Pair it with ee_kv_compact_inplace.
+ */
+ee_status ee_tree_verify_attn_inplace(const ee_bf16* q, const ee_bf16* k_cache, const ee_bf16* v_cache,
+                                      int32_t num_pages, const int32_t* block_table, int32_t max_pages,
+                                      const int32_t* ctx_len, int32_t max_ctx, const int32_t* node_off,
+                                      const uint64_t* anc, int32_t B, int32_t total_nodes, int32_t max_T,
+                                      int32_t n_q, int32_t n_kv, int32_t head_dim, float scale, float* out,
+                                      void* ws, size_t ws_bytes, ee_stream_t stream);
+
+/*
  * ee_lmhead_verify -- the LM head with the verification rules the paper
  * compares (Sec. V-C, RQ3), including its entropy-aware dynamic verification
  * (Sec. III-B, Eq. (entropy) and the top_tau rule).  Same inputs, argmax,
@@ -249,7 +273,8 @@ ee_status ee_lmhead_verify(const ee_bf16* hidden, const ee_bf16* lm_w, int32_t h
                            ee_stream_t stream);
 
 /*
- * ee_attn_plan -- the launch plan ee_tree_verify_attn uses for these sizes
+ * ee_attn_plan -- the launch plan ee_tree_verify_attn (inplace = 0) or
+ * ee_tree_verify_attn_inplace (inplace = 1) uses for these sizes
  * (introspection only; the paper has no counterpart).  *splits = context
  * chunks per 128 query rows (1..16), *chunk = keys per chunk, *mode = 0
  * (one chunk, no merge), 1 (chunks of a row block form a thread-block
@@ -260,7 +285,7 @@ ee_status ee_lmhead_verify(const ee_bf16* hidden, const ee_bf16* lm_w, int32_t h
  * without one; EE_ERR_INVALID_ARG for sizes ee_tree_verify_attn rejects.
  */
 ee_status ee_attn_plan(int32_t B, int32_t max_T, int32_t n_q, int32_t n_kv, int32_t max_ctx,
-                       int32_t* splits, int32_t* chunk, int32_t* mode, int32_t* ctas);
+                       int32_t inplace, int32_t* splits, int32_t* chunk, int32_t* mode, int32_t* ctas);
 
 /*
  * ee_lmhead_accept -- LM head fused with greedy decode and acceptance
@@ -346,6 +371,31 @@ ee_status ee_kv_compact(const ee_bf16* k_tree, const ee_bf16* v_tree, int64_t tr
                         const int32_t* path, const int32_t* accept_len, int32_t B, int32_t max_T,
                         int32_t n_kv, int32_t head_dim, int32_t* dst_slot,
                         void* ws, size_t ws_bytes, ee_stream_t stream);
+
+/*
+ * ee_kv_compact_inplace -- ee_kv_compact's result when the tree's K/V already
+ * sit at positions ctx_len_in[s] + i (in-place speculative K/V, see
+ * ee_tree_verify_attn_inplace).  Path entry k is node path[k] >= k (a parent's
+ * id is below its child's): entries with path[k] == k are already in place --
+ * every entry of a reuse chain -- and the others move from position
+ * ctx + path[k] down to ctx + k, every layer.  Positions after ctx + accept_len
+ * keep the rejected nodes' K/V (they lie beyond the new ctx_len).
+ *   k_cache/v_cache bf16, layer l at + l*cache_layer_stride elements, each layer
+ *                   [num_pages][n_kv][EE_PAGE][head_dim]
+ *   node_off int32 [B+1] with node_off[B] <= total_nodes; path, accept_len,
+ *   dst_slot, ctx_len_in / ctx_len_out as ee_kv_compact.
+ * HBM traffic: 2 (K, V) x 2 (read, write) x n_kv x 256 bytes per moved entry
+ * and layer; a chain moves nothing.
+ * Device errors: EE_DEVERR_PATH (path[k] < k or >= T, or a bad accept_len:
+ * the sequence is skipped), EE_DEVERR_PAGE (a missing page for a moved entry:
+ * the sequence is skipped).
+ */
+ee_status ee_kv_compact_inplace(ee_bf16* k_cache, ee_bf16* v_cache, int64_t cache_layer_stride, int32_t L,
+                                int32_t num_pages, const int32_t* block_table, int32_t max_pages,
+                                const int32_t* ctx_len_in, int32_t* ctx_len_out, const int32_t* node_off,
+                                const int32_t* path, const int32_t* accept_len, int32_t B,
+                                int32_t total_nodes, int32_t max_T, int32_t n_kv, int32_t head_dim,
+                                int32_t* dst_slot, void* ws, size_t ws_bytes, ee_stream_t stream);
 
 #ifdef __cplusplus
 }

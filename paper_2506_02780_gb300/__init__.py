@@ -32,7 +32,7 @@ DEVERR_TIMEOUT = 0x20
 EXPORTS = ("ee_version", "ee_status_string", "ee_workspace_size", "ee_workspace_init",
            "ee_read_errors", "ee_match_reuse", "ee_tree_prepare", "ee_tree_verify_attn", "ee_attn_plan",
            "ee_lmhead_accept", "ee_lmhead_verify", "ee_lmhead_accept_static", "ee_kv_compact",
-           "ee_selftest_timeout")
+           "ee_selftest_timeout", "ee_tree_verify_attn_inplace", "ee_kv_compact_inplace")
 
 VERIFY_MODES = {"greedy": 0, "direct": 1, "topk": 2, "entropy": 3}
 
@@ -64,8 +64,12 @@ _SIGS = {
     "ee_tree_prepare": ([_P, _P, _I, _I, _P, _P, _P, _SZ, _P], _I),
     "ee_tree_verify_attn": ([_P, _P, _P, _P, _P, _I, _P, _I, _P, _I, _P, _P, _I, _I, _I, _I, _I, _I,
                              _F, _P, _P, _SZ, _P], _I),
-    "ee_attn_plan": ([_I, _I, _I, _I, _I, ctypes.POINTER(_I), ctypes.POINTER(_I), ctypes.POINTER(_I),
+    "ee_attn_plan": ([_I, _I, _I, _I, _I, _I, ctypes.POINTER(_I), ctypes.POINTER(_I), ctypes.POINTER(_I),
                       ctypes.POINTER(_I)], _I),
+    "ee_tree_verify_attn_inplace": ([_P, _P, _P, _I, _P, _I, _P, _I, _P, _P, _I, _I, _I, _I, _I, _I, _F, _P,
+                                     _P, _SZ, _P], _I),
+    "ee_kv_compact_inplace": ([_P, _P, _I64, _I, _I, _P, _I, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _P, _P,
+                               _SZ, _P], _I),
     "ee_lmhead_accept": ([_P, _P, _I, _I, _P, _P, _P, _P, _P, _I, _I, _I, _P, _P, _P, _P, _P, _P, _SZ,
                           _P], _I),
     "ee_lmhead_verify": ([_P, _P, _I, _I, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _P, _P, _P, _P, _P,
@@ -192,10 +196,27 @@ def ee_tree_verify_attn(q, k_tree, v_tree, k_cache, v_cache, block_table, ctx_le
     _ok("ee_tree_verify_attn", st)
 
 
-def ee_attn_plan(B, max_T, n_q, n_kv, max_ctx) -> dict:
-    """The launch plan ee_tree_verify_attn uses for these sizes."""
+def ee_tree_verify_attn_inplace(q, k_cache, v_cache, block_table, ctx_len, max_ctx, node_off, anc, max_T,
+                                scale, out, ws, stream=None):
+    """Tree attention with the tree's K/V at cache positions ctx + i (one layer)."""
+    for t, nm in ((q, "q"), (k_cache, "k_cache"), (v_cache, "v_cache")):
+        _check(t, torch.bfloat16, nm)
+    _check(out, torch.float32, "out")
+    total, n_q, d = q.shape
+    num_pages, n_kv = k_cache.shape[0], k_cache.shape[1]
+    B, max_pages = block_table.shape
+    st = lib().ee_tree_verify_attn_inplace(_p(q), _p(k_cache), _p(v_cache), num_pages, _p(block_table),
+                                           max_pages, _p(ctx_len), max_ctx, _p(node_off), _p(anc), B, total,
+                                           max_T, n_q, n_kv, d, float(scale), _p(out), _p(ws), ws.numel(),
+                                           _stream(stream))
+    _ok("ee_tree_verify_attn_inplace", st)
+
+
+def ee_attn_plan(B, max_T, n_q, n_kv, max_ctx, inplace=False) -> dict:
+    """The launch plan ee_tree_verify_attn (or, inplace, ee_tree_verify_attn_inplace)
+    uses for these sizes."""
     v = [_I(0) for _ in range(4)]
-    st = lib().ee_attn_plan(B, max_T, n_q, n_kv, max_ctx, *[ctypes.byref(x) for x in v])
+    st = lib().ee_attn_plan(B, max_T, n_q, n_kv, max_ctx, int(bool(inplace)), *[ctypes.byref(x) for x in v])
     _ok("ee_attn_plan", st)
     return {"splits": v[0].value, "chunk": v[1].value,
             "mode": ("single", "cluster", "cooperative", "balanced")[v[2].value], "ctas": v[3].value}
@@ -264,3 +285,16 @@ def ee_kv_compact(k_tree, v_tree, k_cache, v_cache, block_table, ctx_len_in, ctx
                              _p(ctx_len_in), _p(ctx_len_out), _p(node_off), _p(path), _p(accept_len),
                              B, max_T, n_kv, d, _p(dst_slot), _p(ws), ws.numel(), _stream(stream))
     _ok("ee_kv_compact", st)
+
+
+def ee_kv_compact_inplace(k_cache, v_cache, block_table, ctx_len_in, ctx_len_out, node_off, path,
+                          accept_len, total_nodes, dst_slot, ws, stream=None):
+    """k_cache/v_cache [L, num_pages, n_kv, PAGE, d] holding the tree's K/V at ctx + i."""
+    L, num_pages, n_kv, _, d = k_cache.shape
+    B, max_pages = block_table.shape
+    max_T = path.shape[1]
+    st = lib().ee_kv_compact_inplace(_p(k_cache), _p(v_cache), num_pages * n_kv * EE_PAGE * d, L, num_pages,
+                                     _p(block_table), max_pages, _p(ctx_len_in), _p(ctx_len_out),
+                                     _p(node_off), _p(path), _p(accept_len), B, int(total_nodes), max_T, n_kv,
+                                     d, _p(dst_slot), _p(ws), ws.numel(), _stream(stream))
+    _ok("ee_kv_compact_inplace", st)

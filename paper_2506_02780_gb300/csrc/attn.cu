@@ -206,7 +206,13 @@ struct BalPiece {
   int hk, rb, o, R, K, k, slot0, slot1;
 };
 
-template <bool kBal>
+// kBal: balanced work list (else one (row block, chunk) per CTA).  kIP: the
+// tree's K/V sit in the cache at positions ctx .. ctx + T - 1 (in-place
+// speculative K/V), so a sequence's keys are positions [0, ctx + T) of its
+// pages, and a key at p >= ctx is visible to a row when bit p - ctx of the
+// row's ancestor mask is set; else they come from k_tree / v_tree as one extra
+// 128-key tile after the context.
+template <bool kBal, bool kIP>
 __global__ void __launch_bounds__(kThreads, 1)
 attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__ CUtensorMap tmVc,
                const __grid_constant__ CUtensorMap tmKt, const __grid_constant__ CUtensorMap tmVt,
@@ -311,7 +317,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
             if (blockIdx.x == 0) flag_error(p.err, EE_DEVERR_CTX);
             c = c < 0 ? 0 : p.max_ctx;
           }
-          const int tiles = (c + kKT - 1) / kKT + 1;
+          const int tiles = kIP ? (c + (bad ? 1 : Tb) + kKT - 1) / kKT : (c + kKT - 1) / kKT + 1;
           if (!bad) {
             wl[k] = p.n_kv * ((Tb * g + kRows - 1) / kRows) * tiles;
             tmax = max(tmax, tiles);
@@ -404,10 +410,10 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
       const int seg0 = max(U0, x_begin);
       const int t0 = seg0 - U0;
       const int len = y - seg0;
-      const int n_ctx_b = tiles - 1;
+      const int n_ctx_b = kIP ? tiles : tiles - 1;   // paged tiles of the unit
       k_begin = min(t0, n_ctx_b) * kKT;
-      k_end = t0 < n_ctx_b ? min(ctx, min(t0 + len, n_ctx_b) * kKT) : k_begin;
-      with_tree = t0 + len == tiles;
+      k_end = t0 < n_ctx_b ? min(kIP ? ctx + T : ctx, min(t0 + len, n_ctx_b) * kKT) : k_begin;
+      with_tree = !kIP && t0 + len == tiles;
       const int P = (W + N - 1) / N;
       int ph = (tb - t0) % P;
       ph += ph < 0 ? P : 0;
@@ -460,11 +466,12 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
       }
       // everything above is uniform over the row block's CTAs; from here on every
       // CTA reaches the merge synchronisation
-      const int S = attn_splits_for(ctx, p.chunk);   // chunks this sequence uses, <= p.S
+      const int span = kIP ? ctx + T : ctx;          // paged keys of the sequence
+      const int S = attn_splits_for(span, p.chunk);  // chunks this sequence uses, <= p.S
       const bool active = split < S;
       k_begin = split * p.chunk;
-      k_end = active ? min(ctx, k_begin + p.chunk) : k_begin;
-      with_tree = active && split == S - 1;
+      k_end = active ? min(span, k_begin + p.chunk) : k_begin;
+      with_tree = !kIP && active && split == S - 1;
       alone = p.S == 1;
       slot = ((size_t)blockIdx.z * gridDim.y + blockIdx.y) * gridDim.x + blockIdx.x;
       u_o = o;
@@ -620,7 +627,10 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
       const int rr = rb * kRows + r;
       const bool vrow = rr < R;
       const int node = vrow ? rr / g : 0;
-      const uint64_t ancw = vrow ? p.anc[2 * (size_t)(o + node) + hf] : 0ull;   // this half's tree keys
+      // this half's tree keys (separate tree tile), or the row's whole ancestor
+      // mask (in place: tree keys at any offset from a half's first key)
+      const uint64_t ancw = vrow ? p.anc[2 * (size_t)(o + node) + (kIP ? 0 : hf)] : 0ull;
+      const uint64_t anc_hi = (kIP && vrow) ? p.anc[2 * (size_t)(o + node) + 1] : 0ull;
       const uint32_t tl = tmem + ((uint32_t)(qd * 32) << 16);
       // the block's Q rows into shared memory as the A operand of Q.K^T: 128 rows
       // x 128 bf16 in two 64-column slabs, 128-byte swizzled K-major (the layout
@@ -672,8 +682,23 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
             const int nv = min(max(k_end - (k_begin + i * kKT) - 64 * hf, 0), 64);
             uint64_t pgw = 0ull;
 #pragma unroll
-            for (int i = 0; i < 4; ++i) pgw |= ((m >> (4 * hf + i)) & 1u) ? (0xFFFFull << (16 * i)) : 0ull;
+            for (int pb = 0; pb < 4; ++pb) pgw |= ((m >> (4 * hf + pb)) & 1u) ? (0xFFFFull << (16 * pb)) : 0ull;
             kw = pgw & (nv >= 64 ? ~0ull : ((1ull << nv) - 1ull));
+            if constexpr (kIP) {
+              // keys below ctx are context; key p >= ctx is tree node p - ctx
+              const int p0 = k_begin + i * kKT + 64 * hf;
+              const int nc = min(max(ctx - p0, 0), 64);
+              const int sh = p0 - ctx;    // ancestor bit of this half's first key
+              uint64_t tm;
+              if (sh >= 0)
+                tm = sh >= 128 ? 0ull
+                     : sh >= 64 ? (anc_hi >> (sh - 64))
+                     : sh == 0  ? ancw
+                                : ((ancw >> sh) | (anc_hi << (64 - sh)));
+              else
+                tm = sh <= -64 ? 0ull : (ancw << (-sh));
+              kw &= (nc >= 64 ? ~0ull : ((1ull << nc) - 1ull)) | tm;
+            }
           } else {
             const int th = min(max(T - 64 * hf, 0), 64);
             kw = ancw & (th >= 64 ? ~0ull : ((1ull << th) - 1ull));
@@ -985,7 +1010,7 @@ int active_clusters(int S) {
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     int n = 0;
-    if (cudaOccupancyMaxActiveClusters(&n, attn_tc_kernel<false>, &cfg) != cudaSuccess || n < 1) {
+    if (cudaOccupancyMaxActiveClusters(&n, attn_tc_kernel<false, false>, &cfg) != cudaSuccess || n < 1) {
       cudaGetLastError();
       n = std::max(1, kNumSMs / S);
     }
@@ -1002,7 +1027,7 @@ int resident_ctas() {
     int dev = 0, sms = 0, per = 0;
     if (cudaGetDevice(&dev) != cudaSuccess ||
         cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
-        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per, attn_tc_kernel<kBal>, kThreads, kSmemBytes) !=
+        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per, attn_tc_kernel<kBal, false>, kThreads, kSmemBytes) !=
             cudaSuccess ||
         per < 1) {
       cudaGetLastError();
@@ -1014,29 +1039,30 @@ int resident_ctas() {
   return cap;
 }
 
-// Both instantiations take the full dynamic shared memory (set once).
+// Every instantiation takes the full dynamic shared memory (set once).
 cudaError_t set_attrs() {
   static bool done = false;
   if (done) return cudaSuccess;
-  cudaError_t e = cudaFuncSetAttribute(attn_tc_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       (int)kSmemBytes);
-  if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(attn_tc_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)kSmemBytes);
+  cudaError_t e = cudaSuccess;
+  const void* fns[4] = {(const void*)attn_tc_kernel<false, false>, (const void*)attn_tc_kernel<true, false>,
+                        (const void*)attn_tc_kernel<false, true>, (const void*)attn_tc_kernel<true, true>};
+  for (const void* f : fns)
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
   done = e == cudaSuccess;
   return e;
 }
 
-// Chunk length for s chunks (the last one also carries the tree tile), the
-// chunks actually used and the 128-key tiles of the busiest CTA.
-void chunk_for(int max_ctx, int s, int* chunk, int* used, int* tiles) {
-  int c = (max_ctx + kKT + s - 1) / s;
+// Chunk length for s chunks of `span` paged keys (with tree_tile, the last one
+// also carries the 128-key tree tile), the chunks actually used and the
+// 128-key tiles of the busiest CTA.
+void chunk_for(int span, bool tree_tile, int s, int* chunk, int* used, int* tiles) {
+  int c = (span + (tree_tile ? kKT : 0) + s - 1) / s;
   c = (c + EE_PAGE - 1) / EE_PAGE * EE_PAGE;
   c = std::min(c, kMaxCtaPages * EE_PAGE);          // a CTA stages at most kMaxCtaPages page ids
   *chunk = c;
-  *used = attn_splits_for(max_ctx, c);
-  const int last = max_ctx - (*used - 1) * c;
-  *tiles = std::max((c + kKT - 1) / kKT, (last + kKT - 1) / kKT + 1);
+  *used = attn_splits_for(span, c);
+  const int last = span - (*used - 1) * c;
+  *tiles = std::max((c + kKT - 1) / kKT, (last + kKT - 1) / kKT + (tree_tile ? 1 : 0));
 }
 
 struct Split {
@@ -1057,14 +1083,14 @@ struct Split {
 //   tiles (w_max at most, t_max per unit at most) and may cross one unit
 //   boundary (about 1.5 tiles more); it needs 2 partial slots per CTA, a
 //   share of at most 256 context tiles (the staged page ids) and B <= 512.
-Split choose_split(int max_ctx, int n_rb, long w_max, int t_max, int B, size_t part_slots) {
+Split choose_split(int span, bool tree_tile, int n_rb, long w_max, int t_max, int B, size_t part_slots) {
   Split best;
-  if (max_ctx <= 0) return best;
-  const int min_splits = (max_ctx + kMaxCtaPages * EE_PAGE - 1) / (kMaxCtaPages * EE_PAGE);
+  if (span <= 0) return best;                      // the tree tile alone: one chunk
+  const int min_splits = (span + kMaxCtaPages * EE_PAGE - 1) / (kMaxCtaPages * EE_PAGE);
   long best_cost = -1;
   for (int s = std::max(1, min_splits); s <= kMaxCluster; ++s) {
     int chunk, used, tiles;
-    chunk_for(max_ctx, s, &chunk, &used, &tiles);
+    chunk_for(span, tree_tile, s, &chunk, &used, &tiles);
     // from the second wave on, clusters start as earlier ones finish, and free
     // SMs scattered over the GPCs can leave a slot unusable: plan such launches
     // with one cluster slot fewer
@@ -1082,7 +1108,7 @@ Split choose_split(int max_ctx, int n_rb, long w_max, int t_max, int B, size_t p
   if (cap > 0) {
     for (int s = std::max(2, min_splits); s <= kMaxSplits && (long)s * n_rb <= cap; ++s) {
       int chunk, used, tiles;
-      chunk_for(max_ctx, s, &chunk, &used, &tiles);
+      chunk_for(span, tree_tile, s, &chunk, &used, &tiles);
       if (used < 2) continue;
       const long cost = 2 * (tiles + 3);
       if (cost <= best_cost) {
@@ -1111,62 +1137,47 @@ Split choose_split(int max_ctx, int n_rb, long w_max, int t_max, int B, size_t p
   return best;
 }
 
-}  // namespace
-
-extern "C" ee_status ee_attn_plan(int32_t B, int32_t max_T, int32_t n_q, int32_t n_kv,
-                                  int32_t max_ctx, int32_t* splits, int32_t* chunk, int32_t* mode,
-                                  int32_t* ctas) {
-  if (B < 1 || max_T < 1 || max_T > EE_MAX_TREE || n_q < 1 || n_kv < 1 || n_q % n_kv != 0 ||
-      max_ctx < 0 || !splits || !chunk || !mode || !ctas)
-    return EE_ERR_INVALID_ARG;
-  EE_CUDA_OK(set_attrs());
+// The plan for these sizes: span = paged keys of the longest sequence
+// (max_ctx, or max_ctx + max_T in place), row blocks, work-list bound.
+Split plan_for(int B, int max_T, int n_q, int n_kv, int max_ctx, bool inplace, size_t slots) {
   const int nrb = (max_T * (n_q / n_kv) + kRows - 1) / kRows;
-  const int t_max = (max_ctx + kKT - 1) / kKT + 1;
-  // the partial slots of a workspace sized by ee_workspace_size
-  const size_t slots = std::max((size_t)B * n_q * kAttnMaxSplits, 2 * (size_t)kNumSMsMax);
-  const Split sp = choose_split(max_ctx, nrb * n_kv * B, (long)B * n_kv * nrb * t_max, t_max, B, slots);
-  if (sp.bal) {
-    *splits = sp.bal_ctas;
-    *chunk = sp.bal_tiles * kKT;
-    *mode = 3;
-    *ctas = sp.ctas;
-  } else {
-    *splits = sp.S;
-    *chunk = sp.chunk;
-    *mode = sp.S == 1 ? 0 : (sp.coop ? 2 : 1);
-    *ctas = nrb * sp.S * n_kv * B;
-  }
-  return EE_OK;
+  const int span = inplace ? max_ctx + max_T : max_ctx;
+  const int t_max = inplace ? (span + kKT - 1) / kKT : (max_ctx + kKT - 1) / kKT + 1;
+  return choose_split(span, !inplace, nrb * n_kv * B, (long)B * n_kv * nrb * t_max, t_max, B, slots);
 }
-extern "C" ee_status ee_tree_verify_attn(const ee_bf16* q, const ee_bf16* k_tree,
-                                         const ee_bf16* v_tree, const ee_bf16* k_cache,
-                                         const ee_bf16* v_cache, int32_t num_pages,
-                                         const int32_t* block_table, int32_t max_pages,
-                                         const int32_t* ctx_len, int32_t max_ctx,
-                                         const int32_t* node_off, const uint64_t* anc, int32_t B,
-                                         int32_t total_nodes, int32_t max_T, int32_t n_q,
-                                         int32_t n_kv, int32_t head_dim, float scale, float* out,
-                                         void* ws, size_t ws_bytes, ee_stream_t stream) {
+
+// Shared by ee_tree_verify_attn (tree K/V from k_tree / v_tree) and
+// ee_tree_verify_attn_inplace (tree K/V at cache positions ctx .. ctx + T - 1).
+ee_status verify_attn(const ee_bf16* q, const ee_bf16* k_tree, const ee_bf16* v_tree, const ee_bf16* k_cache,
+                      const ee_bf16* v_cache, int32_t num_pages, const int32_t* block_table, int32_t max_pages,
+                      const int32_t* ctx_len, int32_t max_ctx, const int32_t* node_off, const uint64_t* anc,
+                      int32_t B, int32_t total_nodes, int32_t max_T, int32_t n_q, int32_t n_kv, int32_t head_dim,
+                      float scale, float* out, void* ws, size_t ws_bytes, ee_stream_t stream, bool inplace) {
   if (B < 0 || total_nodes < 0 || n_q < 1 || n_kv < 1 || num_pages < 1 || max_pages < 1 ||
       max_ctx < 0 || max_T < 1)
     return EE_ERR_INVALID_ARG;
   if (head_dim != EE_HEAD_DIM || n_q % n_kv != 0 || max_T > EE_MAX_TREE) return EE_ERR_UNSUPPORTED;
-  if ((int64_t)max_ctx > (int64_t)max_pages * EE_PAGE) return EE_ERR_INVALID_ARG;
+  // every key position must have a block-table entry: the context, and in
+  // place the tree's positions after it
+  const int64_t span = (int64_t)max_ctx + (inplace ? max_T : 0);
+  if (span > (int64_t)max_pages * EE_PAGE) return EE_ERR_INVALID_ARG;
   if (!(scale > 0.f) || !std::isfinite(scale)) return EE_ERR_INVALID_ARG;
   if (B == 0 || total_nodes == 0) return EE_OK;
-  if (!q || !k_tree || !v_tree || !k_cache || !v_cache || !block_table || !ctx_len || !node_off ||
-      !anc || !out || !ws)
+  if (!q || (!inplace && (!k_tree || !v_tree)) || !k_cache || !v_cache || !block_table || !ctx_len ||
+      !node_off || !anc || !out || !ws)
     return EE_ERR_INVALID_ARG;
-  if (!aligned(q, 16) || !aligned(k_tree, 16) || !aligned(v_tree, 16) || !aligned(k_cache, 16) ||
-      !aligned(v_cache, 16) || !aligned(out, 16) || !aligned(anc, 8) || !aligned(ws, 256))
+  if (!aligned(q, 16) || (!inplace && (!aligned(k_tree, 16) || !aligned(v_tree, 16))) ||
+      !aligned(k_cache, 16) || !aligned(v_cache, 16) || !aligned(out, 16) || !aligned(anc, 8) ||
+      !aligned(ws, 256))
     return EE_ERR_INVALID_ARG;
   if (ws_bytes < kWorkspaceBytes) return EE_ERR_WORKSPACE;
   if ((int64_t)num_pages * n_kv * EE_PAGE >= ((int64_t)1 << 31)) return EE_ERR_UNSUPPORTED;
   // a CTA stages at most kMaxCtaPages page ids, and a cluster holds at most 8 chunks
-  if ((int64_t)max_ctx > (int64_t)kMaxCluster * kMaxCtaPages * EE_PAGE) return EE_ERR_UNSUPPORTED;
+  if (span > (int64_t)kMaxCluster * kMaxCtaPages * EE_PAGE) return EE_ERR_UNSUPPORTED;
 
   EE_CUDA_OK(set_attrs());
   // tensor maps: cache [pages * n_kv * 16 rows][128], tree [total][n_kv][128]
+  // (in place the tree maps are not read: the cache maps stand in)
   CUtensorMap tmKc, tmVc, tmKt, tmVt;
   {
     const uint64_t dims[2] = {(uint64_t)head_dim, (uint64_t)num_pages * n_kv * EE_PAGE};
@@ -1175,7 +1186,10 @@ extern "C" ee_status ee_tree_verify_attn(const ee_bf16* q, const ee_bf16* k_tree
     if (!encode_bf16_tmap(&tmKc, k_cache, 2, dims, strides, box)) return EE_ERR_CUDA;
     if (!encode_bf16_tmap(&tmVc, v_cache, 2, dims, strides, box)) return EE_ERR_CUDA;
   }
-  {
+  if (inplace) {
+    tmKt = tmKc;
+    tmVt = tmVc;
+  } else {
     const uint64_t dims[3] = {(uint64_t)head_dim, (uint64_t)n_kv, (uint64_t)total_nodes};
     const uint64_t strides[2] = {(uint64_t)head_dim * 2, (uint64_t)n_kv * head_dim * 2};
     const uint32_t box[3] = {64, 1, (uint32_t)kKT};
@@ -1184,9 +1198,8 @@ extern "C" ee_status ee_tree_verify_attn(const ee_bf16* q, const ee_bf16* k_tree
   }
   const int g = n_q / n_kv;
   const int nrb = (max_T * g + kRows - 1) / kRows;
-  const int t_max = (max_ctx + kKT - 1) / kKT + 1;
   const size_t slots = ws_bytes > kAttnPartOff ? (ws_bytes - kAttnPartOff) / kAttnPartBytes : 0;
-  const Split sp = choose_split(max_ctx, nrb * n_kv * B, (long)B * n_kv * nrb * t_max, t_max, B, slots);
+  const Split sp = plan_for(B, max_T, n_q, n_kv, max_ctx, inplace, slots);
   const int S = sp.bal ? 1 : sp.S, chunk = sp.chunk;
   // a split launch writes one partial slot per CTA after the zeroed part
   if (!sp.bal && S > 1 && ws_bytes < kAttnPartOff + (size_t)nrb * S * n_kv * B * kAttnPartBytes)
@@ -1237,9 +1250,67 @@ extern "C" ee_status ee_tree_verify_attn(const ee_bf16* q, const ee_bf16* k_tree
     attr[1].val.clusterDim.z = 1;
     cfg.numAttrs = 2;
   }
-  if (sp.bal)
-    EE_CUDA_OK(cudaLaunchKernelEx(&cfg, attn_tc_kernel<true>, tmKc, tmVc, tmKt, tmVt, p));
+  if (sp.bal && inplace)
+    EE_CUDA_OK(cudaLaunchKernelEx(&cfg, attn_tc_kernel<true, true>, tmKc, tmVc, tmKt, tmVt, p));
+  else if (sp.bal)
+    EE_CUDA_OK(cudaLaunchKernelEx(&cfg, attn_tc_kernel<true, false>, tmKc, tmVc, tmKt, tmVt, p));
+  else if (inplace)
+    EE_CUDA_OK(cudaLaunchKernelEx(&cfg, attn_tc_kernel<false, true>, tmKc, tmVc, tmKt, tmVt, p));
   else
-    EE_CUDA_OK(cudaLaunchKernelEx(&cfg, attn_tc_kernel<false>, tmKc, tmVc, tmKt, tmVt, p));
+    EE_CUDA_OK(cudaLaunchKernelEx(&cfg, attn_tc_kernel<false, false>, tmKc, tmVc, tmKt, tmVt, p));
   return EE_OK;
+}
+
+}  // namespace
+
+extern "C" ee_status ee_attn_plan(int32_t B, int32_t max_T, int32_t n_q, int32_t n_kv,
+                                  int32_t max_ctx, int32_t inplace, int32_t* splits, int32_t* chunk,
+                                  int32_t* mode, int32_t* ctas) {
+  if (B < 1 || max_T < 1 || max_T > EE_MAX_TREE || n_q < 1 || n_kv < 1 || n_q % n_kv != 0 ||
+      max_ctx < 0 || (inplace != 0 && inplace != 1) || !splits || !chunk || !mode || !ctas)
+    return EE_ERR_INVALID_ARG;
+  EE_CUDA_OK(set_attrs());
+  const int nrb = (max_T * (n_q / n_kv) + kRows - 1) / kRows;
+  // the partial slots of a workspace sized by ee_workspace_size
+  const size_t slots = std::max((size_t)B * n_q * kAttnMaxSplits, 2 * (size_t)kNumSMsMax);
+  const Split sp = plan_for(B, max_T, n_q, n_kv, max_ctx, inplace != 0, slots);
+  if (sp.bal) {
+    *splits = sp.bal_ctas;
+    *chunk = sp.bal_tiles * kKT;
+    *mode = 3;
+    *ctas = sp.ctas;
+  } else {
+    *splits = sp.S;
+    *chunk = sp.chunk;
+    *mode = sp.S == 1 ? 0 : (sp.coop ? 2 : 1);
+    *ctas = nrb * sp.S * n_kv * B;
+  }
+  return EE_OK;
+}
+
+extern "C" ee_status ee_tree_verify_attn(const ee_bf16* q, const ee_bf16* k_tree,
+                                         const ee_bf16* v_tree, const ee_bf16* k_cache,
+                                         const ee_bf16* v_cache, int32_t num_pages,
+                                         const int32_t* block_table, int32_t max_pages,
+                                         const int32_t* ctx_len, int32_t max_ctx,
+                                         const int32_t* node_off, const uint64_t* anc, int32_t B,
+                                         int32_t total_nodes, int32_t max_T, int32_t n_q,
+                                         int32_t n_kv, int32_t head_dim, float scale, float* out,
+                                         void* ws, size_t ws_bytes, ee_stream_t stream) {
+  return verify_attn(q, k_tree, v_tree, k_cache, v_cache, num_pages, block_table, max_pages, ctx_len, max_ctx,
+                     node_off, anc, B, total_nodes, max_T, n_q, n_kv, head_dim, scale, out, ws, ws_bytes, stream,
+                     false);
+}
+
+extern "C" ee_status ee_tree_verify_attn_inplace(const ee_bf16* q, const ee_bf16* k_cache,
+                                                 const ee_bf16* v_cache, int32_t num_pages,
+                                                 const int32_t* block_table, int32_t max_pages,
+                                                 const int32_t* ctx_len, int32_t max_ctx,
+                                                 const int32_t* node_off, const uint64_t* anc, int32_t B,
+                                                 int32_t total_nodes, int32_t max_T, int32_t n_q,
+                                                 int32_t n_kv, int32_t head_dim, float scale, float* out,
+                                                 void* ws, size_t ws_bytes, ee_stream_t stream) {
+  return verify_attn(q, nullptr, nullptr, k_cache, v_cache, num_pages, block_table, max_pages, ctx_len, max_ctx,
+                     node_off, anc, B, total_nodes, max_T, n_q, n_kv, head_dim, scale, out, ws, ws_bytes, stream,
+                     true);
 }

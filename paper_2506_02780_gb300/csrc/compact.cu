@@ -6,11 +6,19 @@
 // Pure data movement: one warp per (layer, sequence, path entry) copies the
 // n_kv K rows and n_kv V rows (head_dim bf16 = 256 bytes each) with 16-byte
 // vector loads/stores.  HBM-bound: 2 * 2 * n_kv * 256 bytes per entry and layer.
+//
+// ee_kv_compact_inplace: the same result when the tree's K/V already sit at
+// positions ctx + i.  Path entry k is node path[k] >= k: entries with
+// path[k] == k are in place (all of a reuse chain's), the others move down
+// from ctx + path[k] to ctx + k.  A destination can be a later entry's source,
+// so one CTA per (layer, sequence, KV head) first reads every moving row into
+// shared memory and, after a barrier, writes them all.
 #include "ee_common.cuh"
 
 namespace {
 
 constexpr int kWarpsPerBlock = 8;
+constexpr int kVecPerRow = EE_HEAD_DIM * 2 / 16;   // uint4 per head row
 
 __global__ void __launch_bounds__(32 * kWarpsPerBlock)
 kv_compact_kernel(const uint4* __restrict__ k_tree, const uint4* __restrict__ v_tree,
@@ -58,7 +66,6 @@ kv_compact_kernel(const uint4* __restrict__ k_tree, const uint4* __restrict__ v_
   const int row = pos % EE_PAGE;
   if (lead) dst_slot[(size_t)b * max_T + k] = page * EE_PAGE + row;
   // 16 uint4 per head row; K rows then V rows
-  constexpr int kVecPerRow = EE_HEAD_DIM * 2 / 16;
   const int64_t tl = tree_layer_stride / 8 * l;   // strides are in bf16 elements
   const int64_t cl = cache_layer_stride / 8 * l;
   const int nvec = 2 * n_kv * kVecPerRow;
@@ -70,6 +77,83 @@ kv_compact_kernel(const uint4* __restrict__ k_tree, const uint4* __restrict__ v_
     const int64_t dst = cl + (((int64_t)page * n_kv + h) * EE_PAGE + row) * kVecPerRow + c;
     if (which == 0) k_cache[dst] = k_tree[src];
     else v_cache[dst] = v_tree[src];
+  }
+}
+
+constexpr int kInplaceThreads = 256;
+constexpr size_t kInplaceSmem = (size_t)EE_MAX_TREE * 2 * kVecPerRow * 16;   // K and V rows, 64 KB
+
+__global__ void __launch_bounds__(kInplaceThreads)
+kv_compact_inplace_kernel(uint4* __restrict__ k_cache, uint4* __restrict__ v_cache, int64_t cache_layer_stride,
+                          int num_pages, const int32_t* __restrict__ block_table, int max_pages,
+                          const int32_t* __restrict__ ctx_in, int32_t* __restrict__ ctx_out,
+                          const int32_t* __restrict__ node_off, const int32_t* __restrict__ path,
+                          const int32_t* __restrict__ accept_len, int max_T, int n_kv, int total_nodes,
+                          int32_t* __restrict__ dst_slot, int32_t* err) {
+  extern __shared__ uint4 stage[];   // [entry][K 16 | V 16] uint4
+  ee::pdl_allow_next();
+  ee::pdl_wait();   // no global access before the previous kernel's writes are visible
+  const int h = blockIdx.x, b = blockIdx.y, l = blockIdx.z;
+  const bool lead = h == 0 && l == 0;
+  const int o = node_off[b];
+  const int T = node_off[b + 1] - o;
+  const int acc = accept_len[b];
+  const int ctx = ctx_in[b];
+  const bool seq_ok = acc >= 0 && acc < T && acc < max_T && ctx >= 0 && o >= 0 && o + T <= total_nodes;
+  // entry k (thread k): its node, source and destination slots; a bad node or
+  // page anywhere stops the whole sequence (every CTA of it decides alike)
+  const int k = threadIdx.x;
+  bool bad = false;
+  int src_slot = -1, dslot = -1, node = -1;
+  if (seq_ok && k <= acc) {
+    node = path[(size_t)b * max_T + k];
+    const int dpos = ctx + k, spos = ctx + node;
+    const int dpg = dpos / EE_PAGE < max_pages ? block_table[(size_t)b * max_pages + dpos / EE_PAGE] : -1;
+    const int spg = (node >= 0 && spos / EE_PAGE < max_pages) ? block_table[(size_t)b * max_pages + spos / EE_PAGE]
+                                                                : -1;
+    if (node < k || node >= T) {
+      bad = true;
+      if (lead) ee::flag_error(err, EE_DEVERR_PATH);
+    } else if (dpg < 0 || dpg >= num_pages || spg < 0 || spg >= num_pages) {
+      bad = true;
+      if (lead) ee::flag_error(err, EE_DEVERR_PAGE);
+    } else {
+      dslot = dpg * EE_PAGE + dpos % EE_PAGE;
+      src_slot = spg * EE_PAGE + spos % EE_PAGE;
+    }
+  }
+  const bool stop = __syncthreads_or(bad) || !seq_ok;
+  if (lead && k < max_T) dst_slot[(size_t)b * max_T + k] = (!stop && k <= acc) ? dslot : -1;
+  if (lead && k == 0) {
+    if (!seq_ok) ee::flag_error(err, EE_DEVERR_PATH);
+    else ctx_out[b] = ctx + acc + 1;
+  }
+  if (stop) return;
+  __shared__ int s_src[EE_MAX_TREE], s_dst[EE_MAX_TREE];
+  if (k <= acc) {
+    s_src[k] = node != k ? src_slot : -1;      // -1: already in place
+    s_dst[k] = dslot;
+  }
+  __syncthreads();
+  // row (slot, head h) of layer l starts at uint4 ((slot / PAGE * n_kv + h) * PAGE + slot % PAGE) * 16
+  const int64_t cl = cache_layer_stride / 8 * l;
+  auto row = [&](int slot) -> int64_t {
+    return cl + (((int64_t)(slot / EE_PAGE) * n_kv + h) * EE_PAGE + slot % EE_PAGE) * kVecPerRow;
+  };
+  const int n = (acc + 1) * 2 * kVecPerRow;
+  for (int v = threadIdx.x; v < n; v += kInplaceThreads) {   // gather every moving row
+    const int e = v / (2 * kVecPerRow), r = v % (2 * kVecPerRow);
+    if (s_src[e] < 0) continue;
+    const int64_t a = row(s_src[e]) + (r % kVecPerRow);
+    stage[v] = r < kVecPerRow ? k_cache[a] : v_cache[a];
+  }
+  __syncthreads();
+  for (int v = threadIdx.x; v < n; v += kInplaceThreads) {   // then scatter them
+    const int e = v / (2 * kVecPerRow), r = v % (2 * kVecPerRow);
+    if (s_src[e] < 0) continue;
+    const int64_t a = row(s_dst[e]) + (r % kVecPerRow);
+    if (r < kVecPerRow) k_cache[a] = stage[v];
+    else v_cache[a] = stage[v];
   }
 }
 
@@ -107,5 +191,41 @@ extern "C" ee_status ee_kv_compact(const ee_bf16* k_tree, const ee_bf16* v_tree,
       tree_layer_stride, reinterpret_cast<uint4*>(k_cache), reinterpret_cast<uint4*>(v_cache),
       cache_layer_stride, num_pages, block_table, max_pages, ctx_len_in, ctx_len_out, node_off, path,
       accept_len, max_T, n_kv, total_nodes, dst_slot, ee::err_word(ws)));
+  return EE_OK;
+}
+
+extern "C" ee_status ee_kv_compact_inplace(ee_bf16* k_cache, ee_bf16* v_cache, int64_t cache_layer_stride,
+                                           int32_t L, int32_t num_pages, const int32_t* block_table,
+                                           int32_t max_pages, const int32_t* ctx_len_in, int32_t* ctx_len_out,
+                                           const int32_t* node_off, const int32_t* path,
+                                           const int32_t* accept_len, int32_t B, int32_t total_nodes,
+                                           int32_t max_T, int32_t n_kv, int32_t head_dim, int32_t* dst_slot,
+                                           void* ws, size_t ws_bytes, ee_stream_t stream) {
+  if (B < 0 || L < 0 || max_T < 1 || max_T > EE_MAX_TREE || n_kv < 1 || num_pages < 1 || max_pages < 1 ||
+      total_nodes < 0)
+    return EE_ERR_INVALID_ARG;
+  if (head_dim != EE_HEAD_DIM) return EE_ERR_UNSUPPORTED;
+  if (B == 0) return EE_OK;
+  if (!k_cache || !v_cache || !block_table || !ctx_len_in || !ctx_len_out || !node_off || !path ||
+      !accept_len || !dst_slot || !ws)
+    return EE_ERR_INVALID_ARG;
+  if (ctx_len_in == ctx_len_out) return EE_ERR_INVALID_ARG;
+  if (!ee::aligned(k_cache, 16) || !ee::aligned(v_cache, 16) || cache_layer_stride % 8)
+    return EE_ERR_INVALID_ARG;
+  if (ws_bytes < ee::kWorkspaceBytes) return EE_ERR_WORKSPACE;
+  if (L == 0) return EE_OK;
+  static bool attr_set = false;
+  if (!attr_set) {
+    EE_CUDA_OK(cudaFuncSetAttribute(kv_compact_inplace_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    (int)kInplaceSmem));
+    attr_set = true;
+  }
+  static_assert(kInplaceThreads >= EE_MAX_TREE, "one thread per path entry");
+  dim3 grid(n_kv, B, L);
+  EE_CUDA_OK(ee::launch_pdl(kv_compact_inplace_kernel, grid, dim3(kInplaceThreads), kInplaceSmem,
+                            (cudaStream_t)stream, 1, reinterpret_cast<uint4*>(k_cache),
+                            reinterpret_cast<uint4*>(v_cache), cache_layer_stride, num_pages, block_table,
+                            max_pages, ctx_len_in, ctx_len_out, node_off, path, accept_len, max_T, n_kv,
+                            total_nodes, dst_slot, ee::err_word(ws)));
   return EE_OK;
 }

@@ -91,11 +91,36 @@ def test_attn_plan_rejects_bad_args(L):
     out = [ctypes.c_int32(0) for _ in range(4)]
     ptrs = [ctypes.byref(x) for x in out]
     f = L.ee_attn_plan
-    assert f(0, 64, 28, 4, 4096, *ptrs) == 1          # no sequence
-    assert f(1, 129, 28, 4, 4096, *ptrs) == 1         # tree larger than 128 nodes
-    assert f(1, 64, 28, 5, 4096, *ptrs) == 1          # n_q not a multiple of n_kv
-    assert f(1, 64, 28, 4, -1, *ptrs) == 1            # negative context
-    assert f(1, 64, 28, 4, 4096, None, *ptrs[1:]) == 1
+    for inplace in (0, 1):
+        assert f(0, 64, 28, 4, 4096, inplace, *ptrs) == 1          # no sequence
+        assert f(1, 129, 28, 4, 4096, inplace, *ptrs) == 1         # tree larger than 128 nodes
+        assert f(1, 64, 28, 5, 4096, inplace, *ptrs) == 1          # n_q not a multiple of n_kv
+        assert f(1, 64, 28, 4, -1, inplace, *ptrs) == 1            # negative context
+        assert f(1, 64, 28, 4, 4096, inplace, None, *ptrs[1:]) == 1
+    assert f(1, 64, 28, 4, 4096, 2, *ptrs) == 1                    # inplace is 0 or 1
+
+
+def test_inplace_entry_points_reject_bad_args(L):
+    ws = ctypes.c_void_p(0x20000)
+    a = L.ee_tree_verify_attn_inplace
+    base = [FAKE, FAKE, FAKE, 10, FAKE, 4, FAKE, 40, FAKE, FAKE, 1, 16, 16, 8, 2, 128,
+            ctypes.c_float(0.088), FAKE, ws, 1 << 26, None]
+    assert a(*base[:7], 49, *base[8:]) == 1          # max_ctx + max_T = 65 > max_pages * 16
+    bad = list(base); bad[15] = 64
+    assert a(*bad) == 2                               # head_dim other than 128
+    bad = list(base); bad[0] = None
+    assert a(*bad) == 1
+    c = L.ee_kv_compact_inplace
+    cb = [FAKE, FAKE, 10 * 2 * 16 * 128, 2, 10, FAKE, 4, FAKE, ctypes.c_void_p(0x30000), FAKE, FAKE, FAKE,
+          1, 16, 16, 2, 128, FAKE, ws, 1 << 26, None]
+    bad = list(cb); bad[8] = FAKE
+    assert c(*bad) == 1                               # ctx_len_out aliases ctx_len_in
+    bad = list(cb); bad[14] = 129
+    assert c(*bad) == 1                               # max_T above 128
+    bad = list(cb); bad[16] = 64
+    assert c(*bad) == 2
+    bad = list(cb); bad[19] = 64
+    assert c(*bad) == 5                               # workspace below the head
 
 
 def test_match_rejects_bad_args(L):
