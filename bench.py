@@ -49,7 +49,7 @@ def parse_args():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-clocks", action="store_true")
     ap.add_argument("--no-variants", action="store_true",
-                    help="skip the verification-rule variants (entropy k=3, k=5)")
+                    help="skip the step variants (entropy k=3, k=5; in-place speculative K/V)")
     ap.add_argument("--profile", action="store_true",
                     help="run --steps eager steps and exit (for ncu captures: few launches, no timing)")
     ap.add_argument("--layers", type=int, default=None,
@@ -372,6 +372,31 @@ def run_ours(args, rank, world, local_rank):
                 "accept_len": [int(a) for a in sv.accept_len.cpu().tolist()[:8]],
                 "greedy_accept_len": [int(a) for a in st.accept_len.cpu().tolist()[:8]]}
             del pool, sv
+    # the same step with in-place speculative K/V: the tree's K/V already in the
+    # cache after each context, compaction moving only the path entries that are
+    # out of place (none for a reuse chain)
+    if not args.no_variants:
+        sv = S.from_workload(w, device=dev, keep_layers=False, inplace_kv=True)
+        pool = []
+        with torch.cuda.stream(stream):
+            sv.run(stream)
+            stream.synchronize()
+            for _ in range(2):
+                g = torch.cuda.CUDAGraph()
+                with torch.cuda.graph(g, stream=stream):
+                    sv.run(stream)
+                pool.append(g)
+        for i in range(max(3, args.warmup // 4)):
+            pool[i % 2].replay()
+        stream.synchronize()
+        ms_v = timed(pool, max(8, args.steps // 4))
+        assert E.ee_read_errors(sv.ws, stream) == 0
+        variants["inplace_kv"] = {
+            "value": round(world * 1e3 / ms_v, 2), "ms_per_step": round(ms_v, 5),
+            "attention_launch": E.ee_attn_plan(w.B, w.max_T, w.n_q, w.n_kv, int(w.ctx_len.max()),
+                                               inplace=True),
+            "accept_len": [int(a) for a in sv.accept_len.cpu().tolist()[:8]]}
+        del pool, sv
     assert E.ee_read_errors(st.ws, stream) == 0
 
     # ---- end to end: host inputs -> device -> step -> host results ---------

@@ -15,19 +15,23 @@
 // shared memory and, after a barrier, writes them all.
 #include "ee_common.cuh"
 
+// Both kernels start before the LM head that produces path / accept_len has
+// finished (programmatic dependent launch).  Everything another kernel may
+// have written is read after griddepcontrol.wait with plain coherent loads
+// (__ldcg), never through const __restrict__ parameters: the compiler may
+// treat such loads as invariant and issue them before the wait.
+
 namespace {
 
 constexpr int kWarpsPerBlock = 8;
 constexpr int kVecPerRow = EE_HEAD_DIM * 2 / 16;   // uint4 per head row
 
 __global__ void __launch_bounds__(32 * kWarpsPerBlock)
-kv_compact_kernel(const uint4* __restrict__ k_tree, const uint4* __restrict__ v_tree,
-                  int64_t tree_layer_stride, uint4* __restrict__ k_cache, uint4* __restrict__ v_cache,
-                  int64_t cache_layer_stride, int num_pages, const int32_t* __restrict__ block_table,
-                  int max_pages, const int32_t* __restrict__ ctx_in, int32_t* __restrict__ ctx_out,
-                  const int32_t* __restrict__ node_off, const int32_t* __restrict__ path,
-                  const int32_t* __restrict__ accept_len, int max_T, int n_kv, int total_nodes,
-                  int32_t* __restrict__ dst_slot, int32_t* err) {
+kv_compact_kernel(const uint4* k_tree, const uint4* v_tree, int64_t tree_layer_stride, uint4* k_cache,
+                  uint4* v_cache, int64_t cache_layer_stride, int num_pages, const int32_t* block_table,
+                  int max_pages, const int32_t* ctx_in, int32_t* ctx_out, const int32_t* node_off,
+                  const int32_t* path, const int32_t* accept_len, int max_T, int n_kv, int total_nodes,
+                  int32_t* dst_slot, int32_t* err) {
   ee::pdl_allow_next();
   ee::pdl_wait();   // no global access before the previous kernel's writes are visible
   const int lane = threadIdx.x & 31;
@@ -35,10 +39,10 @@ kv_compact_kernel(const uint4* __restrict__ k_tree, const uint4* __restrict__ v_
   const int b = blockIdx.y;
   const int l = blockIdx.z;
   if (k >= max_T) return;
-  const int o = node_off[b];
-  const int T = node_off[b + 1] - o;
-  const int acc = accept_len[b];
-  const int ctx = ctx_in[b];
+  const int o = __ldcg(node_off + b);
+  const int T = __ldcg(node_off + b + 1) - o;
+  const int acc = __ldcg(accept_len + b);
+  const int ctx = __ldcg(ctx_in + b);
   const bool lead = (l == 0 && lane == 0);
   if (acc < 0 || acc >= T || acc >= max_T || ctx < 0 || o < 0 || o + T > total_nodes) {
     if (lead) {
@@ -52,10 +56,10 @@ kv_compact_kernel(const uint4* __restrict__ k_tree, const uint4* __restrict__ v_
     return;
   }
   if (lead && k == 0) ctx_out[b] = ctx + acc + 1;
-  const int node = path[(size_t)b * max_T + k];
+  const int node = __ldcg(path + (size_t)b * max_T + k);
   const int pos = ctx + k;
   const int pg = pos / EE_PAGE;
-  const int page = pg < max_pages ? block_table[(size_t)b * max_pages + pg] : -1;
+  const int page = pg < max_pages ? __ldcg(block_table + (size_t)b * max_pages + pg) : -1;
   if (node < 0 || node >= T || page < 0 || page >= num_pages) {
     if (lead) {
       ee::flag_error(err, (node < 0 || node >= T) ? EE_DEVERR_PATH : EE_DEVERR_PAGE);
@@ -75,8 +79,8 @@ kv_compact_kernel(const uint4* __restrict__ k_tree, const uint4* __restrict__ v_
     const int h = rem / kVecPerRow, c = rem % kVecPerRow;
     const int64_t src = tl + ((int64_t)(o + node) * n_kv + h) * kVecPerRow + c;
     const int64_t dst = cl + (((int64_t)page * n_kv + h) * EE_PAGE + row) * kVecPerRow + c;
-    if (which == 0) k_cache[dst] = k_tree[src];
-    else v_cache[dst] = v_tree[src];
+    if (which == 0) k_cache[dst] = __ldcg(k_tree + src);
+    else v_cache[dst] = __ldcg(v_tree + src);
   }
 }
 
@@ -84,21 +88,19 @@ constexpr int kInplaceThreads = 256;
 constexpr size_t kInplaceSmem = (size_t)EE_MAX_TREE * 2 * kVecPerRow * 16;   // K and V rows, 64 KB
 
 __global__ void __launch_bounds__(kInplaceThreads)
-kv_compact_inplace_kernel(uint4* __restrict__ k_cache, uint4* __restrict__ v_cache, int64_t cache_layer_stride,
-                          int num_pages, const int32_t* __restrict__ block_table, int max_pages,
-                          const int32_t* __restrict__ ctx_in, int32_t* __restrict__ ctx_out,
-                          const int32_t* __restrict__ node_off, const int32_t* __restrict__ path,
-                          const int32_t* __restrict__ accept_len, int max_T, int n_kv, int total_nodes,
-                          int32_t* __restrict__ dst_slot, int32_t* err) {
+kv_compact_inplace_kernel(uint4* k_cache, uint4* v_cache, int64_t cache_layer_stride, int num_pages,
+                          const int32_t* block_table, int max_pages, const int32_t* ctx_in, int32_t* ctx_out,
+                          const int32_t* node_off, const int32_t* path, const int32_t* accept_len, int max_T,
+                          int n_kv, int total_nodes, int32_t* dst_slot, int32_t* err) {
   extern __shared__ uint4 stage[];   // [entry][K 16 | V 16] uint4
   ee::pdl_allow_next();
   ee::pdl_wait();   // no global access before the previous kernel's writes are visible
   const int h = blockIdx.x, b = blockIdx.y, l = blockIdx.z;
   const bool lead = h == 0 && l == 0;
-  const int o = node_off[b];
-  const int T = node_off[b + 1] - o;
-  const int acc = accept_len[b];
-  const int ctx = ctx_in[b];
+  const int o = __ldcg(node_off + b);
+  const int T = __ldcg(node_off + b + 1) - o;
+  const int acc = __ldcg(accept_len + b);
+  const int ctx = __ldcg(ctx_in + b);
   const bool seq_ok = acc >= 0 && acc < T && acc < max_T && ctx >= 0 && o >= 0 && o + T <= total_nodes;
   // entry k (thread k): its node, source and destination slots; a bad node or
   // page anywhere stops the whole sequence (every CTA of it decides alike)
@@ -106,11 +108,11 @@ kv_compact_inplace_kernel(uint4* __restrict__ k_cache, uint4* __restrict__ v_cac
   bool bad = false;
   int src_slot = -1, dslot = -1, node = -1;
   if (seq_ok && k <= acc) {
-    node = path[(size_t)b * max_T + k];
+    node = __ldcg(path + (size_t)b * max_T + k);
     const int dpos = ctx + k, spos = ctx + node;
-    const int dpg = dpos / EE_PAGE < max_pages ? block_table[(size_t)b * max_pages + dpos / EE_PAGE] : -1;
-    const int spg = (node >= 0 && spos / EE_PAGE < max_pages) ? block_table[(size_t)b * max_pages + spos / EE_PAGE]
-                                                                : -1;
+    const int dpg = dpos / EE_PAGE < max_pages ? __ldcg(block_table + (size_t)b * max_pages + dpos / EE_PAGE) : -1;
+    const int spg =
+        (node >= 0 && spos / EE_PAGE < max_pages) ? __ldcg(block_table + (size_t)b * max_pages + spos / EE_PAGE) : -1;
     if (node < k || node >= T) {
       bad = true;
       if (lead) ee::flag_error(err, EE_DEVERR_PATH);
@@ -145,7 +147,7 @@ kv_compact_inplace_kernel(uint4* __restrict__ k_cache, uint4* __restrict__ v_cac
     const int e = v / (2 * kVecPerRow), r = v % (2 * kVecPerRow);
     if (s_src[e] < 0) continue;
     const int64_t a = row(s_src[e]) + (r % kVecPerRow);
-    stage[v] = r < kVecPerRow ? k_cache[a] : v_cache[a];
+    stage[v] = r < kVecPerRow ? __ldcg(k_cache + a) : __ldcg(v_cache + a);
   }
   __syncthreads();
   for (int v = threadIdx.x; v < n; v += kInplaceThreads) {   // then scatter them

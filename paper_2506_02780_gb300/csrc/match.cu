@@ -18,10 +18,13 @@ constexpr int kTile = kThreads * kPer;
 constexpr int kWarps = kThreads / 32;
 
 __global__ void __launch_bounds__(kThreads)
-match_reuse_kernel(const int32_t* __restrict__ tok, const int64_t* __restrict__ off,
-                   const int32_t* __restrict__ tail, int n, const int32_t* __restrict__ cursor,
-                   int max_matches, int32_t* __restrict__ match_pos, int32_t* __restrict__ n_matches,
+match_reuse_kernel(const int32_t* __restrict__ tok, const int64_t* off, const int32_t* tail, int n,
+                   const int32_t* cursor, int max_matches, int32_t* match_pos, int32_t* n_matches,
                    int32_t* err) {
+  // tok (the original code) is read-only data for the whole run; the per-step
+  // inputs (off, tail, cursor) may come from an earlier kernel and are read
+  // with plain loads after the dependent-launch wait (a const __restrict__
+  // load may be treated as invariant and issued before the wait)
   __shared__ int32_t s_c[kTile + EE_MAX_NGRAM];
   __shared__ int32_t s_tail[EE_MAX_NGRAM];
   __shared__ int32_t s_wtot[kWarps];

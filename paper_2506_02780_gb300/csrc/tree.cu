@@ -11,9 +11,11 @@
 namespace {
 
 __global__ void __launch_bounds__(EE_MAX_TREE)
-tree_prepare_kernel(const int32_t* __restrict__ parent, const int32_t* __restrict__ node_off,
-                    int32_t* __restrict__ depth, uint64_t* __restrict__ anc, int total_nodes,
-                    int32_t* err) {
+tree_prepare_kernel(const int32_t* parent, const int32_t* node_off, int32_t* depth, uint64_t* anc,
+                    int total_nodes, int32_t* err) {
+  // parent / node_off may come from an earlier kernel: plain loads after the
+  // dependent-launch wait (no const __restrict__, whose loads may be issued
+  // before it)
   __shared__ int32_t s_par[EE_MAX_TREE];
   ee::pdl_allow_next();
   ee::pdl_wait();   // no global access before the previous kernel's writes are visible

@@ -8,6 +8,9 @@ buffers and the workspace and issues, on one stream:
     ee_match_reuse -> ee_tree_prepare -> L x ee_tree_verify_attn
         -> ee_lmhead_accept -> ee_kv_compact
 
+or, with ``inplace_kv``, ee_tree_verify_attn_inplace and ee_kv_compact_inplace
+over tree K/V that sit in the cache after each sequence's context.
+
 No arithmetic happens here; every step runs in libee's kernels.  The whole
 sequence can be captured into a CUDA graph (``capture``).
 """
@@ -17,8 +20,9 @@ import math
 
 import torch
 
-from . import (EE_HEAD_DIM, ee_kv_compact, ee_lmhead_accept, ee_lmhead_verify, ee_match_reuse,
-               ee_tree_prepare, ee_tree_verify_attn, new_workspace)
+from . import (EE_HEAD_DIM, ee_kv_compact, ee_kv_compact_inplace, ee_lmhead_accept, ee_lmhead_verify,
+               ee_match_reuse, ee_tree_prepare, ee_tree_verify_attn, ee_tree_verify_attn_inplace,
+               new_workspace)
 
 
 class VerifyStep:
@@ -30,12 +34,16 @@ class VerifyStep:
     lm_w [V, H] in bf16.  ``max_ctx`` bounds ctx_len (host-side value).
     ``verify`` = (mode, k) switches the LM head to ee_lmhead_verify with that
     rule for the edit content marked by ``gen_mask`` (uint8 [total]); None
-    keeps the greedy ee_lmhead_accept.
+    keeps the greedy ee_lmhead_accept.  ``inplace_kv`` verifies with the tree's
+    K/V in the cache at positions ctx + i (in-place speculative K/V): at set-up
+    they are copied there from k_tree / v_tree, where a K/V projection would
+    have written them, and the block table gets the columns max_ctx + max_T
+    positions need (-1 padded).
     """
 
     def __init__(self, *, orig_tokens, orig_off, tail, cursor, parent, node_off, draft_tok, ctx_len,
                  block_table, q, k_tree, v_tree, k_cache, v_cache, hidden, lm_w, max_ctx, max_T,
-                 max_matches=8, scale=None, keep_layers=True, verify=None, gen_mask=None):
+                 max_matches=8, scale=None, keep_layers=True, verify=None, gen_mask=None, inplace_kv=False):
         self.inp = dict(orig_tokens=orig_tokens, orig_off=orig_off, tail=tail, cursor=cursor,
                         parent=parent, node_off=node_off, draft_tok=draft_tok, ctx_len=ctx_len,
                         block_table=block_table, q=q, k_tree=k_tree, v_tree=v_tree, k_cache=k_cache,
@@ -70,7 +78,29 @@ class VerifyStep:
             self.topk_ids = torch.empty((self.total, k), **i32)
             self.top_tau = torch.empty(self.total, **i32)
             self.h_norm = torch.empty(self.total, dtype=torch.float32, device=dev)
+        self.inplace_kv = bool(inplace_kv)
+        if self.inplace_kv:
+            self._place_tree_kv()
         self.graph = None
+
+    def _place_tree_kv(self):
+        """Set-up for in-place verification (not part of a step): copy node i's
+        K/V to cache position ctx + i of its sequence, every layer, and give the
+        block table a column for every position below max_ctx + max_T."""
+        x = self.inp
+        bt, node_off, ctx = x["block_table"], x["node_off"], x["ctx_len"]
+        cols = -(-(self.max_ctx + self.max_T) // 16)
+        if bt.shape[1] < cols:
+            pad = torch.full((self.B, cols - bt.shape[1]), -1, dtype=bt.dtype, device=bt.device)
+            x["block_table"] = bt = torch.cat([bt, pad], dim=1).contiguous()
+        T = (node_off[1:] - node_off[:-1]).long()
+        seq = torch.repeat_interleave(torch.arange(self.B, device=bt.device), T)
+        pos = ctx.long()[seq] + (torch.arange(self.total, device=bt.device) - node_off.long()[seq])
+        page = bt.long()[seq, pos // 16]
+        row = pos % 16
+        for name in ("k", "v"):
+            cache, tree = x[name + "_cache"], x[name + "_tree"]
+            cache[:, page, :, row, :] = tree.permute(1, 0, 2, 3)
 
     def run(self, stream=None, logits=None, layers=None):
         """Enqueue one whole step (``layers`` restricts attention, for tests)."""
@@ -80,9 +110,14 @@ class VerifyStep:
         ee_tree_prepare(x["parent"], x["node_off"], self.depth, self.anc, self.ws, stream)
         for l in (range(self.L) if layers is None else layers):
             out = self.attn_out[l if self.attn_out.shape[0] == self.L else 0]
-            ee_tree_verify_attn(x["q"][l], x["k_tree"][l], x["v_tree"][l], x["k_cache"][l],
-                                x["v_cache"][l], x["block_table"], x["ctx_len"], self.max_ctx,
-                                x["node_off"], self.anc, self.max_T, self.scale, out, self.ws, stream)
+            if self.inplace_kv:
+                ee_tree_verify_attn_inplace(x["q"][l], x["k_cache"][l], x["v_cache"][l], x["block_table"],
+                                            x["ctx_len"], self.max_ctx, x["node_off"], self.anc, self.max_T,
+                                            self.scale, out, self.ws, stream)
+            else:
+                ee_tree_verify_attn(x["q"][l], x["k_tree"][l], x["v_tree"][l], x["k_cache"][l],
+                                    x["v_cache"][l], x["block_table"], x["ctx_len"], self.max_ctx,
+                                    x["node_off"], self.anc, self.max_T, self.scale, out, self.ws, stream)
         if self.verify is None:
             ee_lmhead_accept(x["hidden"], x["lm_w"], x["draft_tok"], x["parent"], self.depth, self.anc,
                              x["node_off"], self.max_T, self.argmax, self.accept_len, self.path,
@@ -93,9 +128,14 @@ class VerifyStep:
                              self.accept_len, self.path, self.bonus, self.ws, gen_mask=self.gen_mask,
                              topk_ids=self.topk_ids, top_tau=self.top_tau, h_norm=self.h_norm,
                              logits=logits, stream=stream)
-        ee_kv_compact(x["k_tree"], x["v_tree"], x["k_cache"], x["v_cache"], x["block_table"],
-                      x["ctx_len"], self.ctx_out, x["node_off"], self.path, self.accept_len,
-                      self.dst_slot, self.ws, stream)
+        if self.inplace_kv:
+            ee_kv_compact_inplace(x["k_cache"], x["v_cache"], x["block_table"], x["ctx_len"], self.ctx_out,
+                                  x["node_off"], self.path, self.accept_len, self.total, self.dst_slot,
+                                  self.ws, stream)
+        else:
+            ee_kv_compact(x["k_tree"], x["v_tree"], x["k_cache"], x["v_cache"], x["block_table"],
+                          x["ctx_len"], self.ctx_out, x["node_off"], self.path, self.accept_len,
+                          self.dst_slot, self.ws, stream)
 
     def capture(self, stream):
         """Capture one step into a CUDA graph on ``stream`` (a side stream)."""
@@ -114,9 +154,10 @@ class VerifyStep:
         return 2 + self.L + 2 + (0 if self.verify is None else 1)
 
 
-def from_workload(w, device="cuda", keep_layers=True, verify=None):
+def from_workload(w, device="cuda", keep_layers=True, verify=None, inplace_kv=False):
     """VerifyStep over a workloads.Workload (its float tensors already on ``device``);
-    ``verify`` = (mode, k) uses that rule on the workload's generated branches."""
+    ``verify`` = (mode, k) uses that rule on the workload's generated branches;
+    ``inplace_kv`` verifies with the tree's K/V placed in the cache."""
     def i32(a):
         return torch.as_tensor(a, dtype=torch.int32).to(device)
     return VerifyStep(
@@ -126,4 +167,5 @@ def from_workload(w, device="cuda", keep_layers=True, verify=None):
         q=w.q, k_tree=w.k_tree, v_tree=w.v_tree, k_cache=w.k_cache, v_cache=w.v_cache,
         hidden=w.hidden_states, lm_w=w.lm_w, max_ctx=int(w.ctx_len.max()), max_T=w.max_T,
         max_matches=w.max_matches, keep_layers=keep_layers, verify=verify,
-        gen_mask=torch.as_tensor(w.gen_mask).to(device) if verify is not None else None)
+        gen_mask=torch.as_tensor(w.gen_mask).to(device) if verify is not None else None,
+        inplace_kv=inplace_kv)

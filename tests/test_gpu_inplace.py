@@ -142,3 +142,53 @@ def test_inplace_7b_full_size():
     rng = np.random.default_rng(0)
     nodes = sorted(set(rng.choice(w.total_nodes, 10, replace=False).tolist()) | {0, w.total_nodes - 1})
     assert check_inplace(w, nodes=nodes, expect_mode="cooperative") == 0   # the planted path is the chain
+
+
+@pytest.mark.parametrize("name,kw", [("tiny", {}),
+                                     ("batched", dict(layers=2, vocab=8192, hidden=512))])
+def test_step_inplace_kv(name, kw):
+    """VerifyStep with inplace_kv: set-up places the tree's K/V in the cache;
+    the step's attention, acceptance and compaction match the oracle."""
+    E = _E()
+    from paper_2506_02780_gb300 import step as S
+    w = W.build(name, seed=45, device="cuda", **kw)
+    st = S.from_workload(w, inplace_kv=True)
+    kc0, vc0 = U.raw16(w.k_cache), U.raw16(w.v_cache)     # after placement, before the step
+    ref_k, ref_v = O.tree_kv_to_cache(U.raw16(w.k_tree), U.raw16(w.v_tree), kc0, vc0, w.block_table,
+                                      w.ctx_len, w.node_off)
+    assert np.array_equal(kc0, ref_k) and np.array_equal(vc0, ref_v)   # placement as the oracle places
+    st.run()
+    torch.cuda.synchronize()
+    assert E.ee_read_errors(st.ws) == 0
+    anc = U.check_tree(w, st)
+    U.check_attention(w, st, range(w.layers), anc)
+    acc, path = U.check_accept(w, st)
+    rk, rv, rdst, rctx = O.kv_compact_inplace(kc0, vc0, w.block_table, w.ctx_len, w.node_off, path, acc)
+    np.testing.assert_array_equal(st.dst_slot.cpu().numpy(), rdst)
+    np.testing.assert_array_equal(st.ctx_out.cpu().numpy(), rctx)
+    assert np.array_equal(U.raw16(w.k_cache), rk) and np.array_equal(U.raw16(w.v_cache), rv)
+
+
+@pytest.mark.parametrize("inplace", [False, True])
+def test_compaction_waits_for_the_lm_head(inplace):
+    """The compaction starts before the LM head has finished (programmatic
+    dependent launch) and must read path / accept_len only after its wait.  The
+    outputs are poisoned before every step, and later calls in one process
+    overlap the launches: a premature read shows as a device error or a wrong
+    new context length."""
+    E = _E()
+    from paper_2506_02780_gb300 import step as S
+    w = W.build("batched", seed=45, device="cuda", layers=2, vocab=8192, hidden=512)
+    st = S.from_workload(w, inplace_kv=inplace)
+    want = None
+    for _ in range(4):
+        st.accept_len.fill_(-7)
+        st.path.fill_(-7)
+        st.ctx_out.fill_(-5)
+        st.run()
+        torch.cuda.synchronize()
+        assert E.ee_read_errors(st.ws) == 0
+        got = st.ctx_out.cpu().numpy()
+        np.testing.assert_array_equal(got, w.ctx_len + st.accept_len.cpu().numpy() + 1)
+        want = got if want is None else want
+        np.testing.assert_array_equal(got, want)
