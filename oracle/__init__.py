@@ -25,6 +25,10 @@ tests/test_oracle_pins.py):
   kv_compact       pinned: sequential append into a slot dictionary, canaries
   tree_kv_to_cache / tree_kv_from_cache
                    pinned: round trip, slot-dictionary placement
+  chain_attention  pinned: equals tree_attention on chain trees (T <= 128) with the
+                   draft placed in the cache; torch SDPA (fp64, causal) over
+                   prefix + draft for longer drafts
+  accept_chain     pinned: equals accept_path on chain parents; token replay
   kv_compact_inplace
                    pinned: equals kv_compact on the committed positions after
                    tree_kv_to_cache (random trees and paths), chains move
@@ -47,6 +51,8 @@ from .ee_oracle import (  # noqa: F401
     tree_kv_to_cache,
     tree_kv_from_cache,
     kv_compact_inplace,
+    chain_attention,
+    accept_chain,
     entropy_top_tau,
     VERIFY_MODES,
     node_ranking,

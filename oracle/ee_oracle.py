@@ -414,6 +414,79 @@ def kv_compact_inplace(k_cache, v_cache, block_table, ctx_len, node_off, path, a
 
 
 # ----------------------------------------------------------------------------
+# Long reuse drafts: a linear draft of up to 2048 tokens verified in place
+# (Sec. III-A: the reused span of the original code needs no draft length)
+# ----------------------------------------------------------------------------
+
+def chain_attention(q, k_cache, v_cache, block_table, ctx_len, node_off, scale=None, nodes=None, heads=None):
+    """Attention of a linear draft verified in place, ONE layer.
+
+    The draft's K/V sit at positions ctx .. ctx + T - 1 after the prefix, and
+    draft token i (local id, position ctx + i) attends to positions 0 .. ctx + i:
+    ordinary causal attention over prefix + draft, as one target pass over the
+    appended span computes it.  Shapes as in tree_attention (no tree arrays);
+    ``nodes`` / ``heads`` restrict the computation, other entries are NaN.
+    """
+    q = _f64(q)
+    kc, vc = _f64(k_cache), _f64(v_cache)
+    total, n_q, d = q.shape
+    n_kv = kc.shape[1]
+    if n_q % n_kv:
+        raise ValueError("n_q must be a multiple of n_kv")
+    g = n_q // n_kv
+    if scale is None:
+        scale = 1.0 / math.sqrt(d)
+    node_off = np.asarray(node_off)
+    want_nodes = set(range(total)) if nodes is None else set(int(x) for x in nodes)
+    want_heads = list(range(n_q)) if heads is None else [int(h) for h in heads]
+    out = np.full((total, n_q, d), np.nan)
+    for s in range(len(node_off) - 1):
+        o, T = int(node_off[s]), int(node_off[s + 1] - node_off[s])
+        ctx = int(ctx_len[s])
+        for hk in range(n_kv):
+            hs = [h for h in want_heads if h // g == hk]
+            if not hs:
+                continue
+            keys = _context_kv(kc, block_table[s], ctx + T, hk)
+            vals = _context_kv(vc, block_table[s], ctx + T, hk)
+            for i in range(T):
+                if o + i not in want_nodes:
+                    continue
+                for h in hs:
+                    sc = scale * (keys[:ctx + i + 1] @ q[o + i, h])
+                    p = np.exp(sc - sc.max())
+                    p /= p.sum()
+                    out[o + i, h] = p @ vals[:ctx + i + 1]
+    return out
+
+
+def accept_chain(argmax, draft_tok, node_off, max_T=None):
+    """Eq. (piecewise) on a linear draft: d_1 .. d_j are accepted for the
+    largest j with decode(p_k) = d_k for every k <= j, where p_k comes from the
+    logits at d_{k-1} (the root for k = 1).  Returns (accept_len = j,
+    path = 0 .. j padded with -1 to max_T, bonus = argmax at d_j)."""
+    argmax = np.asarray(argmax)
+    draft_tok = np.asarray(draft_tok)
+    node_off = np.asarray(node_off)
+    B = len(node_off) - 1
+    Ts = np.diff(node_off)
+    if max_T is None:
+        max_T = int(Ts.max())
+    accept_len = np.zeros(B, dtype=np.int32)
+    path = np.full((B, max_T), -1, dtype=np.int32)
+    bonus = np.zeros(B, dtype=np.int32)
+    for s in range(B):
+        o, T = int(node_off[s]), int(Ts[s])
+        j = 0
+        while j + 1 < T and int(draft_tok[o + j + 1]) == int(argmax[o + j]):
+            j += 1
+        accept_len[s] = j
+        path[s, :j + 1] = np.arange(j + 1)
+        bonus[s] = int(argmax[o + j])
+    return accept_len, path, bonus
+
+
+# ----------------------------------------------------------------------------
 # Entropy-aware dynamic verification -- Eq. (entropy) and the top_tau rule
 # ----------------------------------------------------------------------------
 

@@ -696,3 +696,81 @@ def test_compact_inplace_overlapping_moves_golden():
     assert [at(iv, ctx + k) for k in range(3)] == [0.0, -2.0, -3.0]
     assert list(dst[0, :3]) == [1 * 16 + 14, 1 * 16 + 15, 0 * 16 + 0]
     assert ctx_out[0] == ctx + 3
+
+
+# ----------------------------------------------------------------------------
+# long reuse drafts: a linear draft verified in place
+# ----------------------------------------------------------------------------
+
+def _placed_cache(w):
+    kc, vc = O.tree_kv_to_cache(w.k_tree.view(torch.int16).numpy(), w.v_tree.view(torch.int16).numpy(),
+                                w.k_cache.view(torch.int16).numpy(), w.v_cache.view(torch.int16).numpy(),
+                                w.block_table, w.ctx_len, w.node_off)
+    return torch.from_numpy(kc).view(torch.bfloat16), torch.from_numpy(vc).view(torch.bfloat16)
+
+
+def test_chain_attention_equals_tree_attention_on_chains():
+    """Up to 128 nodes a linear draft is a chain tree: in-place chain attention
+    equals tree attention over the separate tree arrays."""
+    trees = [W.TreeSpec(9, [], [0, 1]), W.TreeSpec(128, [], [0]), W.TreeSpec(1, [], [0])]
+    w = W.build("tiny", trees=trees, ctxs=[45, 300, 0])
+    kc, vc = _placed_cache(w)
+    _, anc = O.tree_prepare(w.parent, w.node_off)
+    ref = O.tree_attention(w.q[0], w.k_tree[0], w.v_tree[0], w.k_cache[0], w.v_cache[0],
+                           w.block_table, w.ctx_len, w.node_off, anc)
+    out = O.chain_attention(w.q[0], kc[0], vc[0], w.block_table, w.ctx_len, w.node_off)
+    np.testing.assert_allclose(out, ref, rtol=0, atol=1e-12)
+
+
+def test_chain_attention_long_draft_is_causal_sdpa():
+    """A 300-token draft after a 45-token prefix: torch SDPA (fp64) with the
+    causal mask over the whole sequence, every head."""
+    T, ctx = 300, 45
+    w = W.build("tiny", trees=[W.TreeSpec(T, [], [0, 1])], ctx=ctx)
+    kc, vc = _placed_cache(w)
+    out = O.chain_attention(w.q[0], kc[0], vc[0], w.block_table, w.ctx_len, w.node_off)
+    g = w.n_q // w.n_kv
+    keys = torch.stack([_linear_kv(w, 0, 0, hk, range(T), "k") for hk in range(w.n_kv)])
+    vals = torch.stack([_linear_kv(w, 0, 0, hk, range(T), "v") for hk in range(w.n_kv)])
+    keys = keys.repeat_interleave(g, dim=0)
+    vals = vals.repeat_interleave(g, dim=0)
+    qq = w.q[0, :T].double().permute(1, 0, 2)
+    mask = torch.arange(ctx + T)[None, :] <= (ctx + torch.arange(T))[:, None]
+    ref = F.scaled_dot_product_attention(qq[None], keys[None], vals[None], attn_mask=mask)[0]
+    np.testing.assert_allclose(out[:T], ref.permute(1, 0, 2).numpy(), rtol=0, atol=1e-12)
+
+
+@pytest.mark.parametrize("seed", [0, 1, 2])
+def test_accept_chain_equals_tree_rule_on_chains(seed):
+    """accept_chain is accept_path on chain parents, for drafts up to 2048 tokens,
+    and a token-by-token replay fixes its length."""
+    rng = np.random.default_rng(seed)
+    Ts = [1, 2, 300, 2048, 700]
+    node_off = np.concatenate([[0], np.cumsum(Ts)]).astype(np.int32)
+    total = int(node_off[-1])
+    argmax = rng.integers(0, 5, total).astype(np.int32)
+    draft = np.empty(total, np.int32)
+    parent = np.empty(total, np.int32)
+    for s, T in enumerate(Ts):
+        o = int(node_off[s])
+        stop = int(rng.integers(1, T + 1))              # first rejected position (T: none)
+        for i in range(T):
+            parent[o + i] = i - 1
+            if i == 0:
+                draft[o] = 99
+            elif i < stop:
+                draft[o + i] = argmax[o + i - 1]
+            else:
+                draft[o + i] = (argmax[o + i - 1] + 1) % 5 if i == stop else int(rng.integers(0, 5))
+    acc, path, bonus = O.accept_chain(argmax, draft, node_off)
+    acc2, path2, bonus2 = O.accept_path(argmax, draft, parent, node_off)
+    np.testing.assert_array_equal(acc, acc2)
+    np.testing.assert_array_equal(path, path2)
+    np.testing.assert_array_equal(bonus, bonus2)
+    for s, T in enumerate(Ts):                            # replay
+        o, j = int(node_off[s]), 0
+        for k in range(1, T):
+            if draft[o + k] != argmax[o + k - 1]:
+                break
+            j = k
+        assert acc[s] == j and bonus[s] == argmax[o + j]
