@@ -43,7 +43,7 @@ def parse_args():
     ap.add_argument("--steps", type=int, default=2000)
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--config", default="7b", choices=["7b", "batched", "33b", "tiny"])
+    ap.add_argument("--config", default="7b", choices=["7b", "batched", "33b", "tiny", "long"])
     ap.add_argument("--graphs", type=int, default=8, help="graphs replayed round-robin")
     ap.add_argument("--e2e-steps", type=int, default=300)
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -190,22 +190,37 @@ def oracle_step_time(w, attn_nodes=None, lm_rows=None):
     n_att = w.total_nodes if attn_nodes is None else max(1, min(int(attn_nodes), w.total_nodes))
     rows_n = max(1, w.vocab // 16) if lm_rows is None else max(1, min(int(lm_rows), w.vocab))
     nodes = np.linspace(0, w.total_nodes - 1, n_att).round().astype(int).tolist()
+    raw = lambda x: x.detach().cpu().contiguous().view(torch.int16).numpy()  # noqa: E731
+    chain = w.max_T > 128     # linear drafts verified in place (long reuse drafts)
+    if chain:                 # set-up, not timed: the drafts' K/V where a K/V projection writes them
+        pk, pv = O.tree_kv_to_cache(raw(w.k_tree[:1]), raw(w.v_tree[:1]), raw(w.k_cache[:1]),
+                                    raw(w.v_cache[:1]), w.block_table, w.ctx_len, w.node_off)
+        pk_t, pv_t = torch.from_numpy(pk[0]).view(torch.bfloat16), torch.from_numpy(pv[0]).view(torch.bfloat16)
     t0 = time.perf_counter()
     O.match_reuse(w.orig_tokens, w.orig_off, w.tail, w.cursor, w.max_matches)
     t1 = time.perf_counter()
-    depth, anc = O.tree_prepare(w.parent, w.node_off)
+    if not chain:
+        depth, anc = O.tree_prepare(w.parent, w.node_off)
     t2 = time.perf_counter()
-    O.tree_attention(w.q[0], w.k_tree[0], w.v_tree[0], w.k_cache[0], w.v_cache[0], w.block_table,
-                     w.ctx_len, w.node_off, anc, nodes=nodes)
+    if chain:
+        O.chain_attention(w.q[0], pk_t, pv_t, w.block_table, w.ctx_len, w.node_off, nodes=nodes)
+    else:
+        O.tree_attention(w.q[0], w.k_tree[0], w.v_tree[0], w.k_cache[0], w.v_cache[0], w.block_table,
+                         w.ctx_len, w.node_off, anc, nodes=nodes)
     t3 = time.perf_counter()
     logits, _ = O.lm_head_logits(w.hidden_states, w.lm_w, rows=slice(0, rows_n))
     am = np.argmax(logits, axis=1).astype(np.int32)
     t4 = time.perf_counter()
-    acc, path, bonus = O.accept_path(am, w.draft_tok, w.parent, w.node_off, w.max_T)
+    if chain:
+        acc, path, bonus = O.accept_chain(am, w.draft_tok, w.node_off, w.max_T)
+    else:
+        acc, path, bonus = O.accept_path(am, w.draft_tok, w.parent, w.node_off, w.max_T)
     t5 = time.perf_counter()
-    raw = lambda x: x.detach().cpu().contiguous().view(torch.int16).numpy()  # noqa: E731
-    O.kv_compact(raw(w.k_tree[:1]), raw(w.v_tree[:1]), raw(w.k_cache[:1]), raw(w.v_cache[:1]),
-                 w.block_table, w.ctx_len, w.node_off, path, acc)
+    if chain:
+        O.kv_compact_inplace(pk, pv, w.block_table, w.ctx_len, w.node_off, path, acc)
+    else:
+        O.kv_compact(raw(w.k_tree[:1]), raw(w.v_tree[:1]), raw(w.k_cache[:1]), raw(w.v_cache[:1]),
+                     w.block_table, w.ctx_len, w.node_off, path, acc)
     t6 = time.perf_counter()
     a_scale = w.layers * w.total_nodes / n_att
     l_scale = w.vocab / rows_n
@@ -350,7 +365,7 @@ def run_ours(args, rank, world, local_rank):
     # the same step under the entropy-aware rule (Sec. III-B) for the generated
     # branches, with the paper's two settings of k (Sec. IV-E: 3 and 5)
     variants = {}
-    if not args.no_variants and w.lm_w is not None:
+    if not args.no_variants and w.lm_w is not None and not st.chain:   # the rules take trees
         for k in (3, 5):
             sv = S.from_workload(w, device=dev, keep_layers=False, verify=("entropy", k))
             pool = []
@@ -375,7 +390,7 @@ def run_ours(args, rank, world, local_rank):
     # the same step with in-place speculative K/V: the tree's K/V already in the
     # cache after each context, compaction moving only the path entries that are
     # out of place (none for a reuse chain)
-    if not args.no_variants:
+    if not args.no_variants and not st.chain:     # linear drafts are verified in place already
         sv = S.from_workload(w, device=dev, keep_layers=False, inplace_kv=True)
         pool = []
         with torch.cuda.stream(stream):
@@ -422,8 +437,8 @@ def run_ours(args, rank, world, local_rank):
         cand = {
             "lmhead_accept": dict(ms=float(per[1]), bytes=alg["lm_bytes"], flops=alg["lm_flops"],
                                   launches=1),
-            "tree_verify_attn": dict(ms=attn_ms, bytes=alg["attn_bytes"], flops=alg["attn_flops"],
-                                     launches=L),
+            ("chain_verify_attn" if st.chain else "tree_verify_attn"):
+                dict(ms=attn_ms, bytes=alg["attn_bytes"], flops=alg["attn_flops"], launches=L),
         }
         for name, c in cand.items():
             t_s = c["ms"] * 1e-3
@@ -452,8 +467,8 @@ def run_ours(args, rank, world, local_rank):
                        l2="inputs larger than L2 (%.2f GB touched per step)" %
                           ((alg["lm_bytes"] + w.layers * alg["attn_bytes"]) / 1e9),
                        parallelism=f"replicas x{world}",
-                       attention_launch=E.ee_attn_plan(w.B, w.max_T, w.n_q, w.n_kv,
-                                                       int(w.ctx_len.max()))),
+                       attention_launch=E.ee_attn_plan(w.B, w.max_T, w.n_q, w.n_kv, int(w.ctx_len.max()),
+                                                       inplace="chain" if st.chain else False)),
         "draft_tokens_per_s": round(steps_per_s * alg["draft_nodes"], 1),
         "roofline": roofline, "roofline_kernels": rl, "kernels": kernels,
         "e2e": e2e, "gpu_launches": st.launches_per_step() * args.steps, "clocks": clk,
@@ -471,25 +486,7 @@ def run_ours(args, rank, world, local_rank):
 def run_instrumented(st, stream, evs):
     """One step; with `evs` (three events) recorded before the first attention
     layer, after the last one and after the LM head (inside capture)."""
-    from paper_2506_02780_gb300 import (ee_kv_compact, ee_lmhead_accept, ee_match_reuse,
-                                        ee_tree_prepare, ee_tree_verify_attn)
-    x = st.inp
-    rec = (lambda k: evs[k].record(stream)) if evs else (lambda k: None)
-    ee_match_reuse(x["orig_tokens"], x["orig_off"], x["tail"], x["cursor"], st.max_matches,
-                   st.match_pos, st.n_matches, st.ws, stream)
-    ee_tree_prepare(x["parent"], x["node_off"], st.depth, st.anc, st.ws, stream)
-    rec(0)
-    for l in range(st.L):
-        ee_tree_verify_attn(x["q"][l], x["k_tree"][l], x["v_tree"][l], x["k_cache"][l], x["v_cache"][l],
-                            x["block_table"], x["ctx_len"], st.max_ctx, x["node_off"], st.anc, st.max_T,
-                            st.scale, st.attn_out[0], st.ws, stream)
-    rec(1)
-    ee_lmhead_accept(x["hidden"], x["lm_w"], x["draft_tok"], x["parent"], st.depth, st.anc,
-                     x["node_off"], st.max_T, st.argmax, st.accept_len, st.path, st.bonus, st.ws,
-                     stream=stream)
-    rec(2)
-    ee_kv_compact(x["k_tree"], x["v_tree"], x["k_cache"], x["v_cache"], x["block_table"], x["ctx_len"],
-                  st.ctx_out, x["node_off"], st.path, st.accept_len, st.dst_slot, st.ws, stream)
+    st.run(stream, marks=(lambda k: evs[k].record(stream)) if evs else None)
 
 
 def _clone_step(st):
@@ -505,7 +502,8 @@ def _clone_step(st):
                         draft_tok=c["draft_tok"], ctx_len=c["ctx_len"], block_table=x["block_table"],
                         q=c["q"], k_tree=c["k_tree"], v_tree=c["v_tree"], k_cache=x["k_cache"],
                         v_cache=x["v_cache"], hidden=c["hidden"], lm_w=x["lm_w"], max_ctx=st.max_ctx,
-                        max_T=st.max_T, max_matches=st.max_matches, keep_layers=False)
+                        max_T=st.max_T, max_matches=st.max_matches, keep_layers=False,
+                        inplace_kv=st.inplace_kv, chain=st.chain)
 
 
 def run_e2e(st, graph, stream, steps, dev, world):
@@ -612,6 +610,9 @@ def _config_text(name):
         "batched": "8 sequences, ctx U[1k,16k], trees of 32-96 nodes, 7B shapes, 28 layers",
         "33b": "DeepSeek-Coder-33B shapes (H 7168, 56/8 heads, V 32256, 62 layers), ctx 32768, 128-node tree",
         "tiny": "1 sequence, ctx 512, 16-node tree, 8/2 heads, H 512, V 4096, 1 layer",
+        "long": "long reuse draft: Qwen2.5-Coder-7B shapes (H 3584, 28/4 heads, V 152064, 28 layers), "
+                "1 sequence, ctx 4096, a 2048-token linear draft copied from an 8000-token original code, "
+                "verified in place (causal attention over ctx + 2048, greedy longest-prefix acceptance)",
     }[name]
 
 

@@ -61,6 +61,7 @@ extern "C" {
 #define EE_MAX_NGRAM 32
 #define EE_MAX_MATCHES 1024
 #define EE_MAX_LM_NODES 2048
+#define EE_MAX_CHAIN 2048   /* nodes of one linear draft (long reuse drafts) */
 
 typedef uint16_t ee_bf16;                 /* raw bfloat16 bits */
 typedef struct CUstream_st* ee_stream_t;  /* same type as cudaStream_t */
@@ -193,8 +194,11 @@ ee_status ee_tree_prepare(const int32_t* parent, const int32_t* node_off, int32_
  * ctx_len and node_off (ragged batches, and row-block counts that do not
  * divide the SM count).  Split work writes partial results to slots in `ws`
  * (L2-resident); once a row block's pieces are all written, each of their
- * CTAs merges a share of its rows.  EE_ERR_WORKSPACE when ws_bytes is
- * below ee_workspace_size(B, total_nodes, n_q, head_dim, max_ctx).
+ * CTAs merges a share of its rows.  The plan uses only the partial slots the
+ * workspace holds: ee_workspace_size(B, total_nodes, n_q, head_dim, max_ctx)
+ * bytes admit every plan for trees; a smaller workspace runs a plan with fewer
+ * context chunks (one CTA per row block needs none).  EE_ERR_WORKSPACE when
+ * ws_bytes is below the fixed head or no plan fits.
  * Device errors: EE_DEVERR_PAGE (the key is skipped), EE_DEVERR_CTX,
  * EE_DEVERR_TIMEOUT (outputs undefined).
  */
@@ -273,8 +277,9 @@ ee_status ee_lmhead_verify(const ee_bf16* hidden, const ee_bf16* lm_w, int32_t h
                            ee_stream_t stream);
 
 /*
- * ee_attn_plan -- the launch plan ee_tree_verify_attn (inplace = 0) or
- * ee_tree_verify_attn_inplace (inplace = 1) uses for these sizes
+ * ee_attn_plan -- the launch plan ee_tree_verify_attn (inplace = 0),
+ * ee_tree_verify_attn_inplace (inplace = 1) or ee_chain_verify_attn
+ * (inplace = 2, max_T up to EE_MAX_CHAIN) uses for these sizes
  * (introspection only; the paper has no counterpart).  *splits = context
  * chunks per 128 query rows (1..16), *chunk = keys per chunk, *mode = 0
  * (one chunk, no merge), 1 (chunks of a row block form a thread-block
@@ -308,6 +313,11 @@ ee_status ee_attn_plan(int32_t B, int32_t max_T, int32_t n_q, int32_t n_kv, int3
  * 16-byte aligned.  Runs as one persistent tcgen05/TMEM GEMM (vocab rows on
  * the MMA M side) whose epilogue keeps the running argmax; the last CTA to
  * finish runs the acceptance.
+ * Linear drafts (long reuse drafts, Sec. III-A): with anc == NULL every
+ * sequence is a chain (node i's parent is i - 1; parent and depth may be
+ * NULL) of up to EE_MAX_CHAIN nodes (max_T <= EE_MAX_CHAIN): accept_len[s] is
+ * the largest j with draft_tok[i] == argmax[i - 1] for all 1 <= i <= j, path
+ * is 0 .. j.
  * Device errors: EE_DEVERR_TIMEOUT (outputs undefined).
  */
 ee_status ee_lmhead_accept(const ee_bf16* hidden, const ee_bf16* lm_w, int32_t hidden_dim,
@@ -359,7 +369,8 @@ ee_status ee_lmhead_accept_static(const ee_bf16* hidden, const ee_bf16* lm_w, in
  *                  [total_nodes][n_kv][head_dim]
  *   k_cache/v_cache bf16, layer l at + l*cache_layer_stride elements, each layer
  *                  [num_pages][n_kv][EE_PAGE][head_dim]
- *   path int32 [B][max_T], accept_len int32 [B] (from ee_lmhead_accept)
+ *   path int32 [B][max_T], accept_len int32 [B] (from ee_lmhead_accept);
+ *                  max_T <= EE_MAX_CHAIN (linear drafts)
  *   dst_slot int32 [B][max_T] out: page*EE_PAGE + row of each appended entry, -1 pad
  *   ctx_len_out must not alias ctx_len_in.
  * Device errors: EE_DEVERR_PAGE (entry skipped), EE_DEVERR_PATH.
@@ -373,6 +384,27 @@ ee_status ee_kv_compact(const ee_bf16* k_tree, const ee_bf16* v_tree, int64_t tr
                         void* ws, size_t ws_bytes, ee_stream_t stream);
 
 /*
+ * ee_chain_verify_attn -- attention of linear drafts verified in place (long
+ * reuse drafts: the paper verifies a long span of the original code in one
+ * pass, Sec. III-A).  Sequence s's draft of T_s <= EE_MAX_CHAIN tokens has its
+ * K/V at cache positions ctx .. ctx + T_s - 1 and draft token i (node i)
+ * attends to positions 0 .. ctx + i: ordinary causal attention over prefix +
+ * draft, out[i][h] = sum_j softmax_j(scale * q[i][h] . k_j) v_j.  Query rows
+ * past a row block's last node never see later keys, so a row block's work
+ * ends at its own last position (causal tile skipping).  block_table must
+ * cover max_ctx + max_T positions (else EE_ERR_INVALID_ARG); max_T <=
+ * EE_MAX_CHAIN.  Arguments, layouts, precision and device errors as
+ * ee_tree_verify_attn_inplace without anc.  Pair it with ee_lmhead_accept
+ * (anc NULL) and ee_kv_compact_inplace (nothing moves).
+ */
+ee_status ee_chain_verify_attn(const ee_bf16* q, const ee_bf16* k_cache, const ee_bf16* v_cache,
+                               int32_t num_pages, const int32_t* block_table, int32_t max_pages,
+                               const int32_t* ctx_len, int32_t max_ctx, const int32_t* node_off, int32_t B,
+                               int32_t total_nodes, int32_t max_T, int32_t n_q, int32_t n_kv,
+                               int32_t head_dim, float scale, float* out, void* ws, size_t ws_bytes,
+                               ee_stream_t stream);
+
+/*
  * ee_kv_compact_inplace -- ee_kv_compact's result when the tree's K/V already
  * sit at positions ctx_len_in[s] + i (in-place speculative K/V, see
  * ee_tree_verify_attn_inplace).  Path entry k is node path[k] >= k (a parent's
@@ -383,7 +415,8 @@ ee_status ee_kv_compact(const ee_bf16* k_tree, const ee_bf16* v_tree, int64_t tr
  *   k_cache/v_cache bf16, layer l at + l*cache_layer_stride elements, each layer
  *                   [num_pages][n_kv][EE_PAGE][head_dim]
  *   node_off int32 [B+1] with node_off[B] <= total_nodes; path, accept_len,
- *   dst_slot, ctx_len_in / ctx_len_out as ee_kv_compact.
+ *   dst_slot, ctx_len_in / ctx_len_out as ee_kv_compact.  Entries from
+ *   EE_MAX_TREE on (linear drafts only) must be in place.
  * HBM traffic: 2 (K, V) x 2 (read, write) x n_kv x 256 bytes per moved entry
  * and layer; a chain moves nothing.
  * Device errors: EE_DEVERR_PATH (path[k] < k or >= T, or a bad accept_len:

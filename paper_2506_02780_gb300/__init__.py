@@ -32,7 +32,8 @@ DEVERR_TIMEOUT = 0x20
 EXPORTS = ("ee_version", "ee_status_string", "ee_workspace_size", "ee_workspace_init",
            "ee_read_errors", "ee_match_reuse", "ee_tree_prepare", "ee_tree_verify_attn", "ee_attn_plan",
            "ee_lmhead_accept", "ee_lmhead_verify", "ee_lmhead_accept_static", "ee_kv_compact",
-           "ee_selftest_timeout", "ee_tree_verify_attn_inplace", "ee_kv_compact_inplace")
+           "ee_selftest_timeout", "ee_tree_verify_attn_inplace", "ee_kv_compact_inplace",
+           "ee_chain_verify_attn")
 
 VERIFY_MODES = {"greedy": 0, "direct": 1, "topk": 2, "entropy": 3}
 
@@ -68,6 +69,8 @@ _SIGS = {
                       ctypes.POINTER(_I)], _I),
     "ee_tree_verify_attn_inplace": ([_P, _P, _P, _I, _P, _I, _P, _I, _P, _P, _I, _I, _I, _I, _I, _I, _F, _P,
                                      _P, _SZ, _P], _I),
+    "ee_chain_verify_attn": ([_P, _P, _P, _I, _P, _I, _P, _I, _P, _I, _I, _I, _I, _I, _I, _F, _P, _P, _SZ, _P],
+                             _I),
     "ee_kv_compact_inplace": ([_P, _P, _I64, _I, _I, _P, _I, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _P, _P,
                                _SZ, _P], _I),
     "ee_lmhead_accept": ([_P, _P, _I, _I, _P, _P, _P, _P, _P, _I, _I, _I, _P, _P, _P, _P, _P, _P, _SZ,
@@ -212,11 +215,29 @@ def ee_tree_verify_attn_inplace(q, k_cache, v_cache, block_table, ctx_len, max_c
     _ok("ee_tree_verify_attn_inplace", st)
 
 
+def ee_chain_verify_attn(q, k_cache, v_cache, block_table, ctx_len, max_ctx, node_off, max_T, scale, out, ws,
+                         stream=None):
+    """Causal attention of linear drafts (up to EE_MAX_CHAIN tokens) whose K/V sit
+    at cache positions ctx + i (one layer)."""
+    for t, nm in ((q, "q"), (k_cache, "k_cache"), (v_cache, "v_cache")):
+        _check(t, torch.bfloat16, nm)
+    _check(out, torch.float32, "out")
+    total, n_q, d = q.shape
+    num_pages, n_kv = k_cache.shape[0], k_cache.shape[1]
+    B, max_pages = block_table.shape
+    st = lib().ee_chain_verify_attn(_p(q), _p(k_cache), _p(v_cache), num_pages, _p(block_table), max_pages,
+                                    _p(ctx_len), max_ctx, _p(node_off), B, total, max_T, n_q, n_kv, d,
+                                    float(scale), _p(out), _p(ws), ws.numel(), _stream(stream))
+    _ok("ee_chain_verify_attn", st)
+
+
 def ee_attn_plan(B, max_T, n_q, n_kv, max_ctx, inplace=False) -> dict:
-    """The launch plan ee_tree_verify_attn (or, inplace, ee_tree_verify_attn_inplace)
+    """The launch plan ee_tree_verify_attn (inplace False / 0),
+    ee_tree_verify_attn_inplace (True / 1) or ee_chain_verify_attn ("chain" / 2)
     uses for these sizes."""
+    kv = 2 if inplace == "chain" else int(inplace)
     v = [_I(0) for _ in range(4)]
-    st = lib().ee_attn_plan(B, max_T, n_q, n_kv, max_ctx, int(bool(inplace)), *[ctypes.byref(x) for x in v])
+    st = lib().ee_attn_plan(B, max_T, n_q, n_kv, max_ctx, kv, *[ctypes.byref(x) for x in v])
     _ok("ee_attn_plan", st)
     return {"splits": v[0].value, "chunk": v[1].value,
             "mode": ("single", "cluster", "cooperative", "balanced")[v[2].value], "ctas": v[3].value}

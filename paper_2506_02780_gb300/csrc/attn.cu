@@ -206,17 +206,32 @@ struct BalPiece {
   int hk, rb, o, R, K, k, slot0, slot1;
 };
 
-// kBal: balanced work list (else one (row block, chunk) per CTA).  kIP: the
-// tree's K/V sit in the cache at positions ctx .. ctx + T - 1 (in-place
-// speculative K/V), so a sequence's keys are positions [0, ctx + T) of its
-// pages, and a key at p >= ctx is visible to a row when bit p - ctx of the
-// row's ancestor mask is set; else they come from k_tree / v_tree as one extra
-// 128-key tile after the context.
-template <bool kBal, bool kIP>
+// Where the draft's K/V are (template kKV):
+//   kKVTree  -- k_tree / v_tree, one extra 128-key tile after the context;
+//   kKVInPlace -- in the cache at positions ctx .. ctx + T - 1 (in-place
+//     speculative K/V): a sequence's keys are positions [0, ctx + T) of its
+//     pages, and a key at p >= ctx is visible to a row when bit p - ctx of the
+//     row's ancestor mask is set;
+//   kKVChain -- as kKVInPlace for a linear draft of up to EE_MAX_CHAIN tokens:
+//     node i sees positions 0 .. ctx + i (causal), and a row block's keys end
+//     at its last node's position.
+constexpr int kKVTree = 0, kKVInPlace = 1, kKVChain = 2;
+
+// Chain drafts: 128-key tiles of row block r (its last node's position + 1 keys).
+__host__ __device__ inline int chain_rb_tiles(int ctx, int T, int g, int r) {
+  const int n_hi = min(T - 1, ((r + 1) * kRows - 1) / g);
+  return (ctx + n_hi + 1 + kKT - 1) / kKT;
+}
+
+// kBal: balanced work list (else one (row block, chunk) per CTA).
+template <bool kBal, int kKV>
 __global__ void __launch_bounds__(kThreads, 1)
 attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__ CUtensorMap tmVc,
                const __grid_constant__ CUtensorMap tmKt, const __grid_constant__ CUtensorMap tmVt,
                const AttnParams p) {
+  constexpr bool kIP = kKV != kKVTree;       // draft K/V in the cache
+  constexpr bool kChain = kKV == kKVChain;
+  constexpr int kMaxT = kChain ? EE_MAX_CHAIN : EE_MAX_TREE;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
@@ -310,17 +325,25 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
         if (bb < p.B) {
           const int4 sq = s_seq[bb];
           const int Tb = sq.y - sq.x;
-          const bool bad = Tb < 1 || Tb > EE_MAX_TREE || Tb > p.max_T || sq.x < 0 || sq.x + Tb > p.total_nodes;
+          const bool bad = Tb < 1 || Tb > kMaxT || Tb > p.max_T || sq.x < 0 || sq.x + Tb > p.total_nodes;
           if (bad && blockIdx.x == 0) flag_error(p.err, EE_DEVERR_TREE);
           int c = sq.z;
           if (c < 0 || c > p.max_ctx) {
             if (blockIdx.x == 0) flag_error(p.err, EE_DEVERR_CTX);
             c = c < 0 ? 0 : p.max_ctx;
           }
-          const int tiles = kIP ? (c + (bad ? 1 : Tb) + kKT - 1) / kKT : (c + kKT - 1) / kKT + 1;
+          // tiles of a unit (chain: of one KV head's row blocks, whose lengths differ)
+          const int nrb_b = bad ? 1 : (Tb * g + kRows - 1) / kRows;
+          int tiles = kIP ? (c + (bad ? 1 : Tb) + kKT - 1) / kKT : (c + kKT - 1) / kKT + 1;
+          int unit_max = tiles;
+          if constexpr (kChain) {
+            tiles = 0;
+            for (int r = 0; r < nrb_b && !bad; ++r) tiles += chain_rb_tiles(c, Tb, g, r);
+            unit_max = bad ? 1 : chain_rb_tiles(c, Tb, g, nrb_b - 1);
+          }
           if (!bad) {
-            wl[k] = p.n_kv * ((Tb * g + kRows - 1) / kRows) * tiles;
-            tmax = max(tmax, tiles);
+            wl[k] = p.n_kv * (kChain ? 1 : nrb_b) * tiles;
+            tmax = max(tmax, unit_max);
           }
           s_seq[bb] = make_int4(sq.x, bad ? 0 : Tb, c, tiles);
         }
@@ -401,18 +424,36 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
       o = sq.x;
       T = sq.y;
       ctx = sq.z;
-      const int tiles = sq.w;
-      const int nrb_b = (T * g + kRows - 1) / kRows;
-      const int u = (y - 1 - s_wpre[b]) / tiles;
-      hk = u / nrb_b;
-      rb = u - hk * nrb_b;
-      const int U0 = s_wpre[b] + u * tiles;          // the unit's first tile in the work list
+      int tiles = sq.w;
+      int U0;                                        // the unit's first tile in the work list
+      if constexpr (kChain) {
+        // sq.w = tiles of one KV head's row blocks; row block r has chain_rb_tiles
+        const int local = y - 1 - s_wpre[b];
+        hk = local / tiles;
+        const int rem = local - hk * tiles;
+        int r = 0, cum = 0, tu = chain_rb_tiles(ctx, T, g, 0);
+        while (rem >= cum + tu) {
+          cum += tu;
+          ++r;
+          tu = chain_rb_tiles(ctx, T, g, r);
+        }
+        rb = r;
+        U0 = s_wpre[b] + hk * tiles + cum;
+        tiles = tu;
+      } else {
+        const int nrb_b = (T * g + kRows - 1) / kRows;
+        const int u = (y - 1 - s_wpre[b]) / tiles;
+        hk = u / nrb_b;
+        rb = u - hk * nrb_b;
+        U0 = s_wpre[b] + u * tiles;
+      }
       const int seg0 = max(U0, x_begin);
       const int t0 = seg0 - U0;
       const int len = y - seg0;
       const int n_ctx_b = kIP ? tiles : tiles - 1;   // paged tiles of the unit
       k_begin = min(t0, n_ctx_b) * kKT;
-      k_end = t0 < n_ctx_b ? min(kIP ? ctx + T : ctx, min(t0 + len, n_ctx_b) * kKT) : k_begin;
+      const int unit_span = kChain ? ctx + min(T, ((rb + 1) * kRows - 1) / g + 1) : (kIP ? ctx + T : ctx);
+      k_end = t0 < n_ctx_b ? min(unit_span, min(t0 + len, n_ctx_b) * kKT) : k_begin;
       with_tree = !kIP && t0 + len == tiles;
       const int P = (W + N - 1) / N;
       int ph = (tb - t0) % P;
@@ -454,7 +495,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
       o = p.node_off[b];
       T = p.node_off[b + 1] - o;
       ctx = p.ctx_len[b];
-      const bool bad_tree = T < 1 || T > EE_MAX_TREE || T > p.max_T || o < 0 || o + T > p.total_nodes;
+      const bool bad_tree = T < 1 || T > kMaxT || T > p.max_T || o < 0 || o + T > p.total_nodes;
       if (bad_tree && threadIdx.x == 0 && blockIdx.x == 0 && hk == 0) flag_error(p.err, EE_DEVERR_TREE);
       if (bad_tree || rb * kRows >= T * g) {     // uniform over the CTA (and the row block)
         skip = true;
@@ -466,7 +507,8 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
       }
       // everything above is uniform over the row block's CTAs; from here on every
       // CTA reaches the merge synchronisation
-      const int span = kIP ? ctx + T : ctx;          // paged keys of the sequence
+      // paged keys of the row block (chain: up to its last node's position)
+      const int span = kChain ? ctx + min(T, ((rb + 1) * kRows - 1) / g + 1) : (kIP ? ctx + T : ctx);
       const int S = attn_splits_for(span, p.chunk);  // chunks this sequence uses, <= p.S
       const bool active = split < S;
       k_begin = split * p.chunk;
@@ -629,8 +671,8 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
       const int node = vrow ? rr / g : 0;
       // this half's tree keys (separate tree tile), or the row's whole ancestor
       // mask (in place: tree keys at any offset from a half's first key)
-      const uint64_t ancw = vrow ? p.anc[2 * (size_t)(o + node) + (kIP ? 0 : hf)] : 0ull;
-      const uint64_t anc_hi = (kIP && vrow) ? p.anc[2 * (size_t)(o + node) + 1] : 0ull;
+      const uint64_t ancw = (!kChain && vrow) ? p.anc[2 * (size_t)(o + node) + (kIP ? 0 : hf)] : 0ull;
+      const uint64_t anc_hi = (kKV == kKVInPlace && vrow) ? p.anc[2 * (size_t)(o + node) + 1] : 0ull;
       const uint32_t tl = tmem + ((uint32_t)(qd * 32) << 16);
       // the block's Q rows into shared memory as the A operand of Q.K^T: 128 rows
       // x 128 bf16 in two 64-column slabs, 128-byte swizzled K-major (the layout
@@ -684,7 +726,12 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
 #pragma unroll
             for (int pb = 0; pb < 4; ++pb) pgw |= ((m >> (4 * hf + pb)) & 1u) ? (0xFFFFull << (16 * pb)) : 0ull;
             kw = pgw & (nv >= 64 ? ~0ull : ((1ull << nv) - 1ull));
-            if constexpr (kIP) {
+            if constexpr (kChain) {
+              // causal: node sees positions up to ctx + node
+              const int p0 = k_begin + i * kKT + 64 * hf;
+              const int nvis = min(max(ctx + node + 1 - p0, 0), 64);
+              kw &= nvis >= 64 ? ~0ull : ((1ull << nvis) - 1ull);
+            } else if constexpr (kIP) {
               // keys below ctx are context; key p >= ctx is tree node p - ctx
               const int p0 = k_begin + i * kKT + 64 * hf;
               const int nc = min(max(ctx - p0, 0), 64);
@@ -1010,7 +1057,7 @@ int active_clusters(int S) {
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     int n = 0;
-    if (cudaOccupancyMaxActiveClusters(&n, attn_tc_kernel<false, false>, &cfg) != cudaSuccess || n < 1) {
+    if (cudaOccupancyMaxActiveClusters(&n, attn_tc_kernel<false, kKVTree>, &cfg) != cudaSuccess || n < 1) {
       cudaGetLastError();
       n = std::max(1, kNumSMs / S);
     }
@@ -1027,7 +1074,7 @@ int resident_ctas() {
     int dev = 0, sms = 0, per = 0;
     if (cudaGetDevice(&dev) != cudaSuccess ||
         cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
-        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per, attn_tc_kernel<kBal, false>, kThreads, kSmemBytes) !=
+        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per, attn_tc_kernel<kBal, kKVTree>, kThreads, kSmemBytes) !=
             cudaSuccess ||
         per < 1) {
       cudaGetLastError();
@@ -1044,8 +1091,9 @@ cudaError_t set_attrs() {
   static bool done = false;
   if (done) return cudaSuccess;
   cudaError_t e = cudaSuccess;
-  const void* fns[4] = {(const void*)attn_tc_kernel<false, false>, (const void*)attn_tc_kernel<true, false>,
-                        (const void*)attn_tc_kernel<false, true>, (const void*)attn_tc_kernel<true, true>};
+  const void* fns[6] = {(const void*)attn_tc_kernel<false, kKVTree>, (const void*)attn_tc_kernel<true, kKVTree>,
+                        (const void*)attn_tc_kernel<false, kKVInPlace>, (const void*)attn_tc_kernel<true, kKVInPlace>,
+                        (const void*)attn_tc_kernel<false, kKVChain>, (const void*)attn_tc_kernel<true, kKVChain>};
   for (const void* f : fns)
     if (e == cudaSuccess) e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
   done = e == cudaSuccess;
@@ -1094,6 +1142,7 @@ Split choose_split(int span, bool tree_tile, int n_rb, long w_max, int t_max, in
     // from the second wave on, clusters start as earlier ones finish, and free
     // SMs scattered over the GPCs can leave a slot unusable: plan such launches
     // with one cluster slot fewer
+    if (used > 1 && (size_t)n_rb * used > part_slots) continue;   // one partial slot per CTA
     const long act = active_clusters(used);
     long waves = (n_rb + act - 1) / act;
     if (waves >= 2 && act > 1) waves = (n_rb + act - 2) / (act - 1);
@@ -1109,7 +1158,7 @@ Split choose_split(int span, bool tree_tile, int n_rb, long w_max, int t_max, in
     for (int s = std::max(2, min_splits); s <= kMaxSplits && (long)s * n_rb <= cap; ++s) {
       int chunk, used, tiles;
       chunk_for(span, tree_tile, s, &chunk, &used, &tiles);
-      if (used < 2) continue;
+      if (used < 2 || (size_t)n_rb * used > part_slots) continue;
       const long cost = 2 * (tiles + 3);
       if (cost <= best_cost) {
         best_cost = cost;
@@ -1126,7 +1175,8 @@ Split choose_split(int span, bool tree_tile, int n_rb, long w_max, int t_max, in
     const long n_eff = std::min<long>(capb, std::max<long>(1, w_max / m));
     const long share = (w_max + n_eff - 1) / n_eff;
     const long cost = 2 * share + 9;
-    if (cost < best_cost) {
+    if (best_cost < 0 || cost < best_cost) {
+      best_cost = cost;
       best.bal = true;
       best.coop = true;
       best.ctas = capb;
@@ -1134,16 +1184,24 @@ Split choose_split(int span, bool tree_tile, int n_rb, long w_max, int t_max, in
       best.bal_tiles = (int)share;
     }
   }
+  if (best_cost < 0) best.S = 0;   // no plan fits the workspace's partial slots
   return best;
 }
 
-// The plan for these sizes: span = paged keys of the longest sequence
+// The plan for these sizes: span = paged keys of the longest row block
 // (max_ctx, or max_ctx + max_T in place), row blocks, work-list bound.
-Split plan_for(int B, int max_T, int n_q, int n_kv, int max_ctx, bool inplace, size_t slots) {
-  const int nrb = (max_T * (n_q / n_kv) + kRows - 1) / kRows;
-  const int span = inplace ? max_ctx + max_T : max_ctx;
-  const int t_max = inplace ? (span + kKT - 1) / kKT : (max_ctx + kKT - 1) / kKT + 1;
-  return choose_split(span, !inplace, nrb * n_kv * B, (long)B * n_kv * nrb * t_max, t_max, B, slots);
+Split plan_for(int B, int max_T, int n_q, int n_kv, int max_ctx, int kv, size_t slots) {
+  const int g = n_q / n_kv;
+  const int nrb = (max_T * g + kRows - 1) / kRows;
+  const int span = kv != kKVTree ? max_ctx + max_T : max_ctx;
+  const int t_max = kv != kKVTree ? (span + kKT - 1) / kKT : (max_ctx + kKT - 1) / kKT + 1;
+  long per_seq = (long)n_kv * nrb * t_max;
+  if (kv == kKVChain) {
+    per_seq = 0;
+    for (int r = 0; r < nrb; ++r) per_seq += chain_rb_tiles(max_ctx, max_T, g, r);
+    per_seq *= n_kv;
+  }
+  return choose_split(span, kv == kKVTree, nrb * n_kv * B, (long)B * per_seq, t_max, B, slots);
 }
 
 // Shared by ee_tree_verify_attn (tree K/V from k_tree / v_tree) and
@@ -1152,11 +1210,13 @@ ee_status verify_attn(const ee_bf16* q, const ee_bf16* k_tree, const ee_bf16* v_
                       const ee_bf16* v_cache, int32_t num_pages, const int32_t* block_table, int32_t max_pages,
                       const int32_t* ctx_len, int32_t max_ctx, const int32_t* node_off, const uint64_t* anc,
                       int32_t B, int32_t total_nodes, int32_t max_T, int32_t n_q, int32_t n_kv, int32_t head_dim,
-                      float scale, float* out, void* ws, size_t ws_bytes, ee_stream_t stream, bool inplace) {
+                      float scale, float* out, void* ws, size_t ws_bytes, ee_stream_t stream, int kv) {
+  const bool inplace = kv != kKVTree;
   if (B < 0 || total_nodes < 0 || n_q < 1 || n_kv < 1 || num_pages < 1 || max_pages < 1 ||
       max_ctx < 0 || max_T < 1)
     return EE_ERR_INVALID_ARG;
-  if (head_dim != EE_HEAD_DIM || n_q % n_kv != 0 || max_T > EE_MAX_TREE) return EE_ERR_UNSUPPORTED;
+  if (head_dim != EE_HEAD_DIM || n_q % n_kv != 0 || max_T > (kv == kKVChain ? EE_MAX_CHAIN : EE_MAX_TREE))
+    return EE_ERR_UNSUPPORTED;
   // every key position must have a block-table entry: the context, and in
   // place the tree's positions after it
   const int64_t span = (int64_t)max_ctx + (inplace ? max_T : 0);
@@ -1164,7 +1224,7 @@ ee_status verify_attn(const ee_bf16* q, const ee_bf16* k_tree, const ee_bf16* v_
   if (!(scale > 0.f) || !std::isfinite(scale)) return EE_ERR_INVALID_ARG;
   if (B == 0 || total_nodes == 0) return EE_OK;
   if (!q || (!inplace && (!k_tree || !v_tree)) || !k_cache || !v_cache || !block_table || !ctx_len ||
-      !node_off || !anc || !out || !ws)
+      !node_off || (kv != kKVChain && !anc) || !out || !ws)
     return EE_ERR_INVALID_ARG;
   if (!aligned(q, 16) || (!inplace && (!aligned(k_tree, 16) || !aligned(v_tree, 16))) ||
       !aligned(k_cache, 16) || !aligned(v_cache, 16) || !aligned(out, 16) || !aligned(anc, 8) ||
@@ -1199,7 +1259,8 @@ ee_status verify_attn(const ee_bf16* q, const ee_bf16* k_tree, const ee_bf16* v_
   const int g = n_q / n_kv;
   const int nrb = (max_T * g + kRows - 1) / kRows;
   const size_t slots = ws_bytes > kAttnPartOff ? (ws_bytes - kAttnPartOff) / kAttnPartBytes : 0;
-  const Split sp = plan_for(B, max_T, n_q, n_kv, max_ctx, inplace, slots);
+  const Split sp = plan_for(B, max_T, n_q, n_kv, max_ctx, kv, slots);
+  if (sp.S == 0) return EE_ERR_WORKSPACE;
   const int S = sp.bal ? 1 : sp.S, chunk = sp.chunk;
   // a split launch writes one partial slot per CTA after the zeroed part
   if (!sp.bal && S > 1 && ws_bytes < kAttnPartOff + (size_t)nrb * S * n_kv * B * kAttnPartBytes)
@@ -1250,14 +1311,16 @@ ee_status verify_attn(const ee_bf16* q, const ee_bf16* k_tree, const ee_bf16* v_
     attr[1].val.clusterDim.z = 1;
     cfg.numAttrs = 2;
   }
-  if (sp.bal && inplace)
-    EE_CUDA_OK(cudaLaunchKernelEx(&cfg, attn_tc_kernel<true, true>, tmKc, tmVc, tmKt, tmVt, p));
-  else if (sp.bal)
-    EE_CUDA_OK(cudaLaunchKernelEx(&cfg, attn_tc_kernel<true, false>, tmKc, tmVc, tmKt, tmVt, p));
-  else if (inplace)
-    EE_CUDA_OK(cudaLaunchKernelEx(&cfg, attn_tc_kernel<false, true>, tmKc, tmVc, tmKt, tmVt, p));
-  else
-    EE_CUDA_OK(cudaLaunchKernelEx(&cfg, attn_tc_kernel<false, false>, tmKc, tmVc, tmKt, tmVt, p));
+  decltype(&attn_tc_kernel<false, kKVTree>) fn;
+  switch (kv * 2 + (sp.bal ? 1 : 0)) {
+    case 0: fn = attn_tc_kernel<false, kKVTree>; break;
+    case 1: fn = attn_tc_kernel<true, kKVTree>; break;
+    case 2: fn = attn_tc_kernel<false, kKVInPlace>; break;
+    case 3: fn = attn_tc_kernel<true, kKVInPlace>; break;
+    case 4: fn = attn_tc_kernel<false, kKVChain>; break;
+    default: fn = attn_tc_kernel<true, kKVChain>; break;
+  }
+  EE_CUDA_OK(cudaLaunchKernelEx(&cfg, fn, tmKc, tmVc, tmKt, tmVt, p));
   return EE_OK;
 }
 
@@ -1266,14 +1329,16 @@ ee_status verify_attn(const ee_bf16* q, const ee_bf16* k_tree, const ee_bf16* v_
 extern "C" ee_status ee_attn_plan(int32_t B, int32_t max_T, int32_t n_q, int32_t n_kv,
                                   int32_t max_ctx, int32_t inplace, int32_t* splits, int32_t* chunk,
                                   int32_t* mode, int32_t* ctas) {
-  if (B < 1 || max_T < 1 || max_T > EE_MAX_TREE || n_q < 1 || n_kv < 1 || n_q % n_kv != 0 ||
-      max_ctx < 0 || (inplace != 0 && inplace != 1) || !splits || !chunk || !mode || !ctas)
+  if (B < 1 || max_T < 1 || inplace < 0 || inplace > 2 ||
+      max_T > (inplace == kKVChain ? EE_MAX_CHAIN : EE_MAX_TREE) || n_q < 1 || n_kv < 1 || n_q % n_kv != 0 ||
+      max_ctx < 0 || !splits || !chunk || !mode || !ctas)
     return EE_ERR_INVALID_ARG;
   EE_CUDA_OK(set_attrs());
   const int nrb = (max_T * (n_q / n_kv) + kRows - 1) / kRows;
   // the partial slots of a workspace sized by ee_workspace_size
   const size_t slots = std::max((size_t)B * n_q * kAttnMaxSplits, 2 * (size_t)kNumSMsMax);
-  const Split sp = plan_for(B, max_T, n_q, n_kv, max_ctx, inplace != 0, slots);
+  const Split sp = plan_for(B, max_T, n_q, n_kv, max_ctx, inplace, slots);
+  if (sp.S == 0) return EE_ERR_UNSUPPORTED;
   if (sp.bal) {
     *splits = sp.bal_ctas;
     *chunk = sp.bal_tiles * kKT;
@@ -1299,7 +1364,7 @@ extern "C" ee_status ee_tree_verify_attn(const ee_bf16* q, const ee_bf16* k_tree
                                          void* ws, size_t ws_bytes, ee_stream_t stream) {
   return verify_attn(q, k_tree, v_tree, k_cache, v_cache, num_pages, block_table, max_pages, ctx_len, max_ctx,
                      node_off, anc, B, total_nodes, max_T, n_q, n_kv, head_dim, scale, out, ws, ws_bytes, stream,
-                     false);
+                     kKVTree);
 }
 
 extern "C" ee_status ee_tree_verify_attn_inplace(const ee_bf16* q, const ee_bf16* k_cache,
@@ -1312,5 +1377,16 @@ extern "C" ee_status ee_tree_verify_attn_inplace(const ee_bf16* q, const ee_bf16
                                                  void* ws, size_t ws_bytes, ee_stream_t stream) {
   return verify_attn(q, nullptr, nullptr, k_cache, v_cache, num_pages, block_table, max_pages, ctx_len, max_ctx,
                      node_off, anc, B, total_nodes, max_T, n_q, n_kv, head_dim, scale, out, ws, ws_bytes, stream,
-                     true);
+                     kKVInPlace);
+}
+
+extern "C" ee_status ee_chain_verify_attn(const ee_bf16* q, const ee_bf16* k_cache, const ee_bf16* v_cache,
+                                          int32_t num_pages, const int32_t* block_table, int32_t max_pages,
+                                          const int32_t* ctx_len, int32_t max_ctx, const int32_t* node_off,
+                                          int32_t B, int32_t total_nodes, int32_t max_T, int32_t n_q,
+                                          int32_t n_kv, int32_t head_dim, float scale, float* out, void* ws,
+                                          size_t ws_bytes, ee_stream_t stream) {
+  return verify_attn(q, nullptr, nullptr, k_cache, v_cache, num_pages, block_table, max_pages, ctx_len, max_ctx,
+                     node_off, nullptr, B, total_nodes, max_T, n_q, n_kv, head_dim, scale, out, ws, ws_bytes,
+                     stream, kKVChain);
 }

@@ -102,47 +102,45 @@ kv_compact_inplace_kernel(uint4* k_cache, uint4* v_cache, int64_t cache_layer_st
   const int acc = __ldcg(accept_len + b);
   const int ctx = __ldcg(ctx_in + b);
   const bool seq_ok = acc >= 0 && acc < T && acc < max_T && ctx >= 0 && o >= 0 && o + T <= total_nodes;
-  // entry k (thread k): its node, source and destination slots; a bad node or
-  // page anywhere stops the whole sequence (every CTA of it decides alike)
-  const int k = threadIdx.x;
+  // entry k: its node, source and destination slots.  Only a tree (at most
+  // EE_MAX_TREE nodes) moves entries; a longer path (a linear draft) must be
+  // in place.  A bad node or page anywhere stops the whole sequence (every CTA
+  // of it decides alike).
+  __shared__ int s_src[EE_MAX_TREE], s_dst[EE_MAX_CHAIN];
   bool bad = false;
-  int src_slot = -1, dslot = -1, node = -1;
-  if (seq_ok && k <= acc) {
-    node = __ldcg(path + (size_t)b * max_T + k);
+  for (int k = threadIdx.x; seq_ok && k <= acc; k += kInplaceThreads) {
+    const int node = __ldcg(path + (size_t)b * max_T + k);
     const int dpos = ctx + k, spos = ctx + node;
     const int dpg = dpos / EE_PAGE < max_pages ? __ldcg(block_table + (size_t)b * max_pages + dpos / EE_PAGE) : -1;
     const int spg =
         (node >= 0 && spos / EE_PAGE < max_pages) ? __ldcg(block_table + (size_t)b * max_pages + spos / EE_PAGE) : -1;
-    if (node < k || node >= T) {
+    if (node < k || node >= T || (k >= EE_MAX_TREE && node != k)) {
       bad = true;
       if (lead) ee::flag_error(err, EE_DEVERR_PATH);
     } else if (dpg < 0 || dpg >= num_pages || spg < 0 || spg >= num_pages) {
       bad = true;
       if (lead) ee::flag_error(err, EE_DEVERR_PAGE);
     } else {
-      dslot = dpg * EE_PAGE + dpos % EE_PAGE;
-      src_slot = spg * EE_PAGE + spos % EE_PAGE;
+      s_dst[k] = dpg * EE_PAGE + dpos % EE_PAGE;
+      if (k < EE_MAX_TREE) s_src[k] = node != k ? spg * EE_PAGE + spos % EE_PAGE : -1;   // -1: in place
     }
   }
   const bool stop = __syncthreads_or(bad) || !seq_ok;
-  if (lead && k < max_T) dst_slot[(size_t)b * max_T + k] = (!stop && k <= acc) ? dslot : -1;
-  if (lead && k == 0) {
+  if (lead)
+    for (int k = threadIdx.x; k < max_T; k += kInplaceThreads)
+      dst_slot[(size_t)b * max_T + k] = (!stop && k <= acc) ? s_dst[k] : -1;
+  if (lead && threadIdx.x == 0) {
     if (!seq_ok) ee::flag_error(err, EE_DEVERR_PATH);
     else ctx_out[b] = ctx + acc + 1;
   }
   if (stop) return;
-  __shared__ int s_src[EE_MAX_TREE], s_dst[EE_MAX_TREE];
-  if (k <= acc) {
-    s_src[k] = node != k ? src_slot : -1;      // -1: already in place
-    s_dst[k] = dslot;
-  }
-  __syncthreads();
+  const int nm = min(acc, EE_MAX_TREE - 1);   // entries that may move: 0 .. nm
   // row (slot, head h) of layer l starts at uint4 ((slot / PAGE * n_kv + h) * PAGE + slot % PAGE) * 16
   const int64_t cl = cache_layer_stride / 8 * l;
   auto row = [&](int slot) -> int64_t {
     return cl + (((int64_t)(slot / EE_PAGE) * n_kv + h) * EE_PAGE + slot % EE_PAGE) * kVecPerRow;
   };
-  const int n = (acc + 1) * 2 * kVecPerRow;
+  const int n = (nm + 1) * 2 * kVecPerRow;
   for (int v = threadIdx.x; v < n; v += kInplaceThreads) {   // gather every moving row
     const int e = v / (2 * kVecPerRow), r = v % (2 * kVecPerRow);
     if (s_src[e] < 0) continue;
@@ -170,7 +168,7 @@ extern "C" ee_status ee_kv_compact(const ee_bf16* k_tree, const ee_bf16* v_tree,
                                    const int32_t* accept_len, int32_t B, int32_t max_T, int32_t n_kv,
                                    int32_t head_dim, int32_t* dst_slot, void* ws, size_t ws_bytes,
                                    ee_stream_t stream) {
-  if (B < 0 || L < 0 || max_T < 1 || max_T > EE_MAX_TREE || n_kv < 1 || num_pages < 1 ||
+  if (B < 0 || L < 0 || max_T < 1 || max_T > EE_MAX_CHAIN || n_kv < 1 || num_pages < 1 ||
       max_pages < 1)
     return EE_ERR_INVALID_ARG;
   if (head_dim != EE_HEAD_DIM) return EE_ERR_UNSUPPORTED;
@@ -203,7 +201,7 @@ extern "C" ee_status ee_kv_compact_inplace(ee_bf16* k_cache, ee_bf16* v_cache, i
                                            const int32_t* accept_len, int32_t B, int32_t total_nodes,
                                            int32_t max_T, int32_t n_kv, int32_t head_dim, int32_t* dst_slot,
                                            void* ws, size_t ws_bytes, ee_stream_t stream) {
-  if (B < 0 || L < 0 || max_T < 1 || max_T > EE_MAX_TREE || n_kv < 1 || num_pages < 1 || max_pages < 1 ||
+  if (B < 0 || L < 0 || max_T < 1 || max_T > EE_MAX_CHAIN || n_kv < 1 || num_pages < 1 || max_pages < 1 ||
       total_nodes < 0)
     return EE_ERR_INVALID_ARG;
   if (head_dim != EE_HEAD_DIM) return EE_ERR_UNSUPPORTED;
@@ -222,7 +220,6 @@ extern "C" ee_status ee_kv_compact_inplace(ee_bf16* k_cache, ee_bf16* v_cache, i
                                     (int)kInplaceSmem));
     attr_set = true;
   }
-  static_assert(kInplaceThreads >= EE_MAX_TREE, "one thread per path entry");
   dim3 grid(n_kv, B, L);
   EE_CUDA_OK(ee::launch_pdl(kv_compact_inplace_kernel, grid, dim3(kInplaceThreads), kInplaceSmem,
                             (cudaStream_t)stream, 1, reinterpret_cast<uint4*>(k_cache),

@@ -155,11 +155,33 @@ __device__ void accept_sequences(const AcceptArgs& a, const int32_t* am, const i
     else
       return *q;
   };
+  const bool chain = a.anc == nullptr;   // linear drafts (greedy only): node i's parent is i - 1
   for (int s = warp; s < a.B; s += nwarps) {
     const int o = a.node_off[s];
     const int T = a.node_off[s + 1] - o;
-    if (T < 1 || T > EE_MAX_TREE || T > a.max_T || o < 0 || o + T > a.total) {
+    if (T < 1 || T > (chain ? EE_MAX_CHAIN : EE_MAX_TREE) || T > a.max_T || o < 0 || o + T > a.total) {
       if (lane == 0) ee::flag_error(a.err, EE_DEVERR_TREE);
+      continue;
+    }
+    if (chain) {
+      // Eq. (piecewise) on a linear draft: the first node whose token differs
+      // from the argmax at its predecessor ends the accepted prefix
+      int first = T;
+      for (int base = 1; base < T; base += 32) {
+        const int i = base + lane;
+        const bool bad = i < T && a.draft_tok[o + i] != ld_i(am + o + i - 1);
+        const unsigned m = __ballot_sync(0xffffffffu, bad);
+        if (m) {
+          first = base + __ffs(m) - 1;
+          break;
+        }
+      }
+      const int acc = first - 1;
+      for (int j = lane; j < a.max_T; j += 32) a.path[(size_t)s * a.max_T + j] = j <= acc ? j : -1;
+      if (lane == 0) {
+        a.accept_len[s] = acc;
+        a.bonus[s] = ld_i(am + o + acc);
+      }
       continue;
     }
     // notok bit i: node i's edge from its parent is rejected
@@ -863,22 +885,25 @@ bool encode_2d(CUtensorMap* map, const void* base, uint64_t inner, uint64_t oute
 
 // Host-side argument checks shared by the LM-head entry points.  Sets *empty
 // when there is nothing to launch.
+// With allow_chain, anc == NULL selects linear drafts (parent and depth may
+// then be NULL, max_T up to EE_MAX_CHAIN).
 ee_status check_lm_args(const ee_bf16* hidden, const ee_bf16* lm_w, int32_t hidden_dim,
                         int32_t vocab, const int32_t* draft_tok, const int32_t* parent,
                         const int32_t* depth, const uint64_t* anc, const int32_t* node_off, int32_t B,
                         int32_t total_nodes, int32_t max_T, const int32_t* argmax,
                         const int32_t* accept_len, const int32_t* path, const int32_t* bonus,
-                        bool* empty) {
+                        bool* empty, bool allow_chain) {
   *empty = false;
+  const bool chain = allow_chain && anc == nullptr;
   if (B < 0 || total_nodes < 0 || hidden_dim < 8 || vocab < 1 || max_T < 1)
     return EE_ERR_INVALID_ARG;
-  if (hidden_dim % 8 != 0 || max_T > EE_MAX_TREE || total_nodes > EE_MAX_LM_NODES)
+  if (hidden_dim % 8 != 0 || max_T > (chain ? EE_MAX_CHAIN : EE_MAX_TREE) || total_nodes > EE_MAX_LM_NODES)
     return EE_ERR_UNSUPPORTED;
   if (B == 0 || total_nodes == 0) {
     *empty = true;
     return EE_OK;
   }
-  if (!hidden || !lm_w || !draft_tok || !parent || !depth || !anc || !node_off || !argmax ||
+  if (!hidden || !lm_w || !draft_tok || (!chain && (!parent || !depth || !anc)) || !node_off || !argmax ||
       !accept_len || !path || !bonus)
     return EE_ERR_INVALID_ARG;
   if (!ee::aligned(hidden, 16) || !ee::aligned(lm_w, 16)) return EE_ERR_INVALID_ARG;
@@ -1035,7 +1060,7 @@ extern "C" ee_status ee_lmhead_accept(const ee_bf16* hidden, const ee_bf16* lm_w
   bool empty = false;
   const ee_status st = check_lm_args(hidden, lm_w, hidden_dim, vocab, draft_tok, parent, depth, anc,
                                      node_off, B, total_nodes, max_T, argmax, accept_len, path,
-                                     bonus, &empty);
+                                     bonus, &empty, true);
   if (st != EE_OK || empty) return st;
   if (!ws || !ee::aligned(ws, 256)) return EE_ERR_INVALID_ARG;
   if (ws_bytes < ee::kWorkspaceBytes) return EE_ERR_WORKSPACE;
@@ -1063,7 +1088,7 @@ extern "C" ee_status ee_lmhead_verify(const ee_bf16* hidden, const ee_bf16* lm_w
   bool empty = false;
   const ee_status st = check_lm_args(hidden, lm_w, hidden_dim, vocab, draft_tok, parent, depth, anc,
                                      node_off, B, total_nodes, max_T, argmax, accept_len, path,
-                                     bonus, &empty);
+                                     bonus, &empty, false);
   if (st != EE_OK || empty) return st;
   if (!ws || !ee::aligned(ws, 256)) return EE_ERR_INVALID_ARG;
   if (ws_bytes < ee::kLmVerifyOff + ee::kLmVerifyBytes) return EE_ERR_WORKSPACE;
@@ -1127,7 +1152,7 @@ extern "C" ee_status ee_lmhead_accept_static(const ee_bf16* hidden, const ee_bf1
   bool empty = false;
   const ee_status st = check_lm_args(hidden, lm_w, hidden_dim, vocab, draft_tok, parent, depth, anc,
                                      node_off, B, total_nodes, max_T, argmax, accept_len, path,
-                                     bonus, &empty);
+                                     bonus, &empty, true);
   if (st != EE_OK || empty) return st;   // total_nodes > EE_MAX_LM_NODES -> EE_ERR_UNSUPPORTED
   void* scratch = nullptr;
   const ee_status ss = static_scratch(&scratch);

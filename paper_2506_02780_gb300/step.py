@@ -9,7 +9,10 @@ buffers and the workspace and issues, on one stream:
         -> ee_lmhead_accept -> ee_kv_compact
 
 or, with ``inplace_kv``, ee_tree_verify_attn_inplace and ee_kv_compact_inplace
-over tree K/V that sit in the cache after each sequence's context.
+over tree K/V that sit in the cache after each sequence's context; with
+``chain`` (linear drafts of up to 2048 tokens, long reuse drafts), no tree
+preparation, ee_chain_verify_attn, ee_lmhead_accept without ancestor masks and
+ee_kv_compact_inplace.
 
 No arithmetic happens here; every step runs in libee's kernels.  The whole
 sequence can be captured into a CUDA graph (``capture``).
@@ -20,9 +23,9 @@ import math
 
 import torch
 
-from . import (EE_HEAD_DIM, ee_kv_compact, ee_kv_compact_inplace, ee_lmhead_accept, ee_lmhead_verify,
-               ee_match_reuse, ee_tree_prepare, ee_tree_verify_attn, ee_tree_verify_attn_inplace,
-               new_workspace)
+from . import (EE_HEAD_DIM, ee_chain_verify_attn, ee_kv_compact, ee_kv_compact_inplace, ee_lmhead_accept,
+               ee_lmhead_verify, ee_match_reuse, ee_tree_prepare, ee_tree_verify_attn,
+               ee_tree_verify_attn_inplace, new_workspace)
 
 
 class VerifyStep:
@@ -43,7 +46,8 @@ class VerifyStep:
 
     def __init__(self, *, orig_tokens, orig_off, tail, cursor, parent, node_off, draft_tok, ctx_len,
                  block_table, q, k_tree, v_tree, k_cache, v_cache, hidden, lm_w, max_ctx, max_T,
-                 max_matches=8, scale=None, keep_layers=True, verify=None, gen_mask=None, inplace_kv=False):
+                 max_matches=8, scale=None, keep_layers=True, verify=None, gen_mask=None, inplace_kv=False,
+                 chain=False):
         self.inp = dict(orig_tokens=orig_tokens, orig_off=orig_off, tail=tail, cursor=cursor,
                         parent=parent, node_off=node_off, draft_tok=draft_tok, ctx_len=ctx_len,
                         block_table=block_table, q=q, k_tree=k_tree, v_tree=v_tree, k_cache=k_cache,
@@ -78,7 +82,10 @@ class VerifyStep:
             self.topk_ids = torch.empty((self.total, k), **i32)
             self.top_tau = torch.empty(self.total, **i32)
             self.h_norm = torch.empty(self.total, dtype=torch.float32, device=dev)
-        self.inplace_kv = bool(inplace_kv)
+        self.chain = bool(chain)
+        if self.chain and self.verify is not None:
+            raise ValueError("the verification rules take trees; linear drafts are greedy")
+        self.inplace_kv = bool(inplace_kv) or self.chain
         if self.inplace_kv:
             self._place_tree_kv()
         self.graph = None
@@ -102,15 +109,23 @@ class VerifyStep:
             cache, tree = x[name + "_cache"], x[name + "_tree"]
             cache[:, page, :, row, :] = tree.permute(1, 0, 2, 3)
 
-    def run(self, stream=None, logits=None, layers=None):
-        """Enqueue one whole step (``layers`` restricts attention, for tests)."""
+    def run(self, stream=None, logits=None, layers=None, marks=None):
+        """Enqueue one whole step (``layers`` restricts attention, for tests);
+        ``marks(k)`` is called before the first attention layer (k = 0), after
+        the last (1) and after the LM head (2), e.g. to record timing events."""
         x = self.inp
+        mark = marks if marks is not None else (lambda k: None)
         ee_match_reuse(x["orig_tokens"], x["orig_off"], x["tail"], x["cursor"], self.max_matches,
                        self.match_pos, self.n_matches, self.ws, stream)
-        ee_tree_prepare(x["parent"], x["node_off"], self.depth, self.anc, self.ws, stream)
+        if not self.chain:
+            ee_tree_prepare(x["parent"], x["node_off"], self.depth, self.anc, self.ws, stream)
+        mark(0)
         for l in (range(self.L) if layers is None else layers):
             out = self.attn_out[l if self.attn_out.shape[0] == self.L else 0]
-            if self.inplace_kv:
+            if self.chain:
+                ee_chain_verify_attn(x["q"][l], x["k_cache"][l], x["v_cache"][l], x["block_table"], x["ctx_len"],
+                                     self.max_ctx, x["node_off"], self.max_T, self.scale, out, self.ws, stream)
+            elif self.inplace_kv:
                 ee_tree_verify_attn_inplace(x["q"][l], x["k_cache"][l], x["v_cache"][l], x["block_table"],
                                             x["ctx_len"], self.max_ctx, x["node_off"], self.anc, self.max_T,
                                             self.scale, out, self.ws, stream)
@@ -118,7 +133,12 @@ class VerifyStep:
                 ee_tree_verify_attn(x["q"][l], x["k_tree"][l], x["v_tree"][l], x["k_cache"][l],
                                     x["v_cache"][l], x["block_table"], x["ctx_len"], self.max_ctx,
                                     x["node_off"], self.anc, self.max_T, self.scale, out, self.ws, stream)
-        if self.verify is None:
+        mark(1)
+        if self.chain:
+            ee_lmhead_accept(x["hidden"], x["lm_w"], x["draft_tok"], None, None, None, x["node_off"], self.max_T,
+                             self.argmax, self.accept_len, self.path, self.bonus, self.ws, logits=logits,
+                             stream=stream)
+        elif self.verify is None:
             ee_lmhead_accept(x["hidden"], x["lm_w"], x["draft_tok"], x["parent"], self.depth, self.anc,
                              x["node_off"], self.max_T, self.argmax, self.accept_len, self.path,
                              self.bonus, self.ws, logits=logits, stream=stream)
@@ -128,6 +148,7 @@ class VerifyStep:
                              self.accept_len, self.path, self.bonus, self.ws, gen_mask=self.gen_mask,
                              topk_ids=self.topk_ids, top_tau=self.top_tau, h_norm=self.h_norm,
                              logits=logits, stream=stream)
+        mark(2)
         if self.inplace_kv:
             ee_kv_compact_inplace(x["k_cache"], x["v_cache"], x["block_table"], x["ctx_len"], self.ctx_out,
                                   x["node_off"], self.path, self.accept_len, self.total, self.dst_slot,
@@ -149,15 +170,19 @@ class VerifyStep:
         return g
 
     def launches_per_step(self) -> int:
-        """Kernels this step launches: match, prepare, 1 per attention layer, LM head (+ the
-        verification finalize), compaction."""
-        return 2 + self.L + 2 + (0 if self.verify is None else 1)
+        """Kernels this step launches: match, prepare (not for linear drafts), 1 per attention
+        layer, LM head (+ the verification finalize), compaction."""
+        return (1 if self.chain else 2) + self.L + 2 + (0 if self.verify is None else 1)
 
 
-def from_workload(w, device="cuda", keep_layers=True, verify=None, inplace_kv=False):
+def from_workload(w, device="cuda", keep_layers=True, verify=None, inplace_kv=False, chain=None):
     """VerifyStep over a workloads.Workload (its float tensors already on ``device``);
     ``verify`` = (mode, k) uses that rule on the workload's generated branches;
-    ``inplace_kv`` verifies with the tree's K/V placed in the cache."""
+    ``inplace_kv`` verifies with the tree's K/V placed in the cache; ``chain``
+    (default: the workload's drafts are all linear and one exceeds 128 tokens)
+    verifies linear drafts in place."""
+    if chain is None:
+        chain = w.max_T > 128
     def i32(a):
         return torch.as_tensor(a, dtype=torch.int32).to(device)
     return VerifyStep(
@@ -168,4 +193,4 @@ def from_workload(w, device="cuda", keep_layers=True, verify=None, inplace_kv=Fa
         hidden=w.hidden_states, lm_w=w.lm_w, max_ctx=int(w.ctx_len.max()), max_T=w.max_T,
         max_matches=w.max_matches, keep_layers=keep_layers, verify=verify,
         gen_mask=torch.as_tensor(w.gen_mask).to(device) if verify is not None else None,
-        inplace_kv=inplace_kv)
+        inplace_kv=inplace_kv, chain=chain)

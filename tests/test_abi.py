@@ -97,7 +97,9 @@ def test_attn_plan_rejects_bad_args(L):
         assert f(1, 64, 28, 5, 4096, inplace, *ptrs) == 1          # n_q not a multiple of n_kv
         assert f(1, 64, 28, 4, -1, inplace, *ptrs) == 1            # negative context
         assert f(1, 64, 28, 4, 4096, inplace, None, *ptrs[1:]) == 1
-    assert f(1, 64, 28, 4, 4096, 2, *ptrs) == 1                    # inplace is 0 or 1
+    assert f(1, 64, 28, 4, 4096, 3, *ptrs) == 1                    # inplace is 0, 1 or 2 (chain)
+    assert f(1, 2049, 28, 4, 4096, 2, *ptrs) == 1                  # a chain above EE_MAX_CHAIN
+    assert f(1, 129, 28, 4, 4096, 1, *ptrs) == 1                   # a tree above EE_MAX_TREE
 
 
 def test_inplace_entry_points_reject_bad_args(L):
@@ -115,8 +117,8 @@ def test_inplace_entry_points_reject_bad_args(L):
           1, 16, 16, 2, 128, FAKE, ws, 1 << 26, None]
     bad = list(cb); bad[8] = FAKE
     assert c(*bad) == 1                               # ctx_len_out aliases ctx_len_in
-    bad = list(cb); bad[14] = 129
-    assert c(*bad) == 1                               # max_T above 128
+    bad = list(cb); bad[14] = 2049
+    assert c(*bad) == 1                               # a path above EE_MAX_CHAIN
     bad = list(cb); bad[16] = 64
     assert c(*bad) == 2
     bad = list(cb); bad[19] = 64
@@ -183,3 +185,25 @@ def test_selftest_timeout_rejects_bad_args(L):
     assert f(FAKE, 64, FAKE, None) == 1                          # below the fixed head
     assert f(ctypes.c_void_p(0x10008), 1 << 20, FAKE, None) == 1   # ws not 256-aligned
     assert f(FAKE, 1 << 20, ctypes.c_void_p(0x10004), None) == 1   # out not 8-aligned
+
+
+def test_chain_entry_points_reject_bad_args(L):
+    ws = ctypes.c_void_p(0x20000)
+    a = L.ee_chain_verify_attn
+    base = [FAKE, FAKE, FAKE, 200, FAKE, 160, FAKE, 512, FAKE, 1, 2048, 2048, 8, 2, 128,
+            ctypes.c_float(0.088), FAKE, ws, 1 << 26, None]
+    bad = list(base); bad[11] = 2049
+    assert a(*bad) == 2                               # draft above EE_MAX_CHAIN
+    bad = list(base); bad[5] = 159
+    assert a(*bad) == 1                               # 512 + 2048 positions need 160 pages
+    bad = list(base); bad[14] = 64
+    assert a(*bad) == 2
+    # the LM head takes linear drafts with anc NULL (parent / depth may be NULL too)
+    f = L.ee_lmhead_accept
+    lm = [FAKE, FAKE, 512, 4096, FAKE, None, None, None, FAKE, 1, 2048, 2049] + [FAKE] * 4 + [None, ws, 1 << 26, None]
+    assert f(*lm) == 2                                # max_T above EE_MAX_CHAIN
+    tree = [FAKE, FAKE, 512, 4096, FAKE, None, FAKE, FAKE, FAKE, 1, 2048, 129] + [FAKE] * 4 + [None, ws, 1 << 26, None]
+    assert f(*tree) == 2                              # a tree above EE_MAX_TREE
+    v = L.ee_lmhead_verify
+    assert v(FAKE, FAKE, 512, 4096, FAKE, None, None, None, FAKE, None, 1, 64, 64, 0, 1,
+             FAKE, None, None, None, FAKE, FAKE, FAKE, None, ws, 1 << 26, None) == 1   # rules need a tree

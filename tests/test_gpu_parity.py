@@ -214,9 +214,11 @@ def test_device_error_word():
     U.check_accept(w, st)
 
 
-def test_attention_rejects_small_workspace():
-    """A split launch needs one partial slot per CTA: a workspace sized for an
-    empty context is refused before anything is launched."""
+def test_attention_plans_within_a_small_workspace():
+    """A workspace with no room for partial slots (sized for an empty context)
+    runs the plan that needs none -- one CTA per row block over its whole
+    context -- and still matches the oracle; below the fixed head the call is
+    refused before anything is launched."""
     E = _E()
     from paper_2506_02780_gb300 import step as S
     w = W.build("tiny", seed=4, device="cuda")
@@ -224,11 +226,23 @@ def test_attention_rejects_small_workspace():
     small = E.new_workspace(w.B, w.total_nodes, w.n_q, 0)
     assert small.numel() < st.ws.numel()
     x = st.inp
+    anc = O.tree_prepare(w.parent, w.node_off)[1]
+    anc_d = torch.from_numpy(anc.view(np.int64)).cuda()
     out = torch.full_like(st.attn_out[0], 7.0)
+    E.ee_tree_verify_attn(x["q"][0], x["k_tree"][0], x["v_tree"][0], x["k_cache"][0], x["v_cache"][0],
+                          x["block_table"], x["ctx_len"], st.max_ctx, x["node_off"], anc_d, st.max_T, st.scale,
+                          out, small)
+    torch.cuda.synchronize()
+    assert E.ee_read_errors(small) == 0
+    ref = O.tree_attention(w.q[0], w.k_tree[0], w.v_tree[0], w.k_cache[0], w.v_cache[0], w.block_table,
+                           w.ctx_len, w.node_off, anc)
+    U.assert_close(out.cpu().numpy(), ref, "attention, one-chunk plan")
+    tiny_ws = small[:1024]
+    out.fill_(7.0)
     with pytest.raises(E.EEError) as ei:
-        E.ee_tree_verify_attn(x["q"][0], x["k_tree"][0], x["v_tree"][0], x["k_cache"][0],
-                              x["v_cache"][0], x["block_table"], x["ctx_len"], st.max_ctx,
-                              x["node_off"], st.anc, st.max_T, st.scale, out, small)
+        E.ee_tree_verify_attn(x["q"][0], x["k_tree"][0], x["v_tree"][0], x["k_cache"][0], x["v_cache"][0],
+                              x["block_table"], x["ctx_len"], st.max_ctx, x["node_off"], anc_d, st.max_T,
+                              st.scale, out, tiny_ws)
     assert ei.value.status == 5
     torch.cuda.synchronize()
     assert bool((out == 7.0).all())

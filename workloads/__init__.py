@@ -28,7 +28,7 @@ import torch
 
 PAGE = 16            # tokens per KV page
 HEAD_DIM = 128
-CONFIG_NAMES = ("tiny", "7b", "batched", "33b", "sweep")
+CONFIG_NAMES = ("tiny", "7b", "batched", "33b", "sweep", "long")
 BASE_SEED = 1234
 
 # Model shapes of the target models the paper's configurations are named after.
@@ -251,6 +251,14 @@ def _plan(name, rng, overrides):
                 spec.planted = chain_path(int(rng.integers(1, chain)))
             len_c = int(round(0.8 * ctx))
             seqs.append(dict(len_c=len_c, ctx=ctx, plen=int(0.6 * len_c), edits=3, spec=spec))
+    elif name == "long":
+        # a long reuse draft verified in one pass (Sec. III-A: a reused span of
+        # the original code needs no draft length): 7B shapes, one sequence, a
+        # 2048-token chain of the original code after the match point, accepted
+        # up to an edit 1500 tokens in
+        shape = dict(SHAPES["7b"], n=4)
+        seqs = [dict(len_c=8000, ctx=4096, plen=3000, edits=3,
+                     spec=TreeSpec(2048, [], chain_path(1500)))]
     elif name == "sweep":
         shape = dict(SHAPES["7b"], n=o.pop("n", 4))
         seqs = []
