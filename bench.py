@@ -64,6 +64,8 @@ TRAFFIC = {
     ("tree_verify_attn", "33b"): 158299648,       # profiles/attn_tc_33b.md
     ("tree_verify_attn", "batched"): 245043456,   # profiles/attn_tc_batched.md
     ("lmhead_accept", "7b"): 1095463424,          # profiles/lmhead_accept_7b.md
+    ("lmhead_accept", "long"): 1108085248,        # profiles/lmhead_accept_long.md
+    ("chain_verify_attn", "long"): 28688640,      # profiles/attn_chain_long.md
 }
 
 
