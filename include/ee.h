@@ -15,6 +15,9 @@
  *   ee_tree_verify_attn_inplace / ee_kv_compact_inplace
  *                        the same two steps with the tree's K/V already in
  *                        the cache after the context (in-place speculative K/V)
+ *   ee_chain_verify_attn causal attention of linear drafts of up to 2048
+ *                        tokens verified in place (long reuse drafts; the LM
+ *                        head takes them with anc NULL)
  *
  * Conventions shared by every entry point
  * ---------------------------------------
