@@ -29,6 +29,11 @@ tests/test_oracle_pins.py):
                    draft placed in the cache; torch SDPA (fp64, causal) over
                    prefix + draft for longer drafts
   accept_chain     pinned: equals accept_path on chain parents; token replay
+  build_reuse_tree / advance
+                   pinned: hand-worked trees and commits; a whole edit session
+                   (match, tree, a synthetic greedy target, acceptance, commit)
+                   reproduces the target's own greedy text (lossless greedy
+                   speculative decoding) from several starting points
   kv_compact_inplace
                    pinned: equals kv_compact on the committed positions after
                    tree_kv_to_cache (random trees and paths), chains move
@@ -53,6 +58,8 @@ from .ee_oracle import (  # noqa: F401
     kv_compact_inplace,
     chain_attention,
     accept_chain,
+    build_reuse_tree,
+    advance,
     entropy_top_tau,
     VERIFY_MODES,
     node_ranking,

@@ -487,6 +487,101 @@ def accept_chain(argmax, draft_tok, node_off, max_T=None):
 
 
 # ----------------------------------------------------------------------------
+# Reuse <-> Generate controller (Sec. III-A): the next draft tree from the match
+# points, and the commit of a verification step's result
+# ----------------------------------------------------------------------------
+
+def build_reuse_tree(orig_tokens, orig_off, match_pos, n_matches, last_tok, n, chain_len, n_branches,
+                     gen_tok=None):
+    """Draft tree of the next step, every sequence.
+
+    Sec. III-A: match points of the generated suffix in the remaining code are
+    new draft starts, and the code after each of them is a draft.  Node 0 is
+    the root, the last committed token.  Branch b (b < n_branches) holds the
+    chain_len tokens of c after the b-th match point p_b,
+    c[p_b + n + j] for j < chain_len, as a chain below the root; a branch with
+    no match point, and positions past the end of c, carry token -1 (no argmax
+    equals it, so such nodes are never accepted).  Then the generated branch:
+    gen_tok[s] (a draft model's proposal for edited content, G tokens, G = 0
+    allowed), also a chain below the root and marked in gen_mask.
+    Every sequence has T = 1 + n_branches * chain_len + G nodes.
+
+    Returns (draft_tok int32 [B*T], parent int32 [B*T] local ids,
+    node_off int32 [B+1], cpos int32 [B*T] = the node's position in c
+    (the root: p_0 + n - 1, its match; -1 for generated or empty nodes),
+    gen_mask uint8 [B*T]).
+    """
+    orig_tokens = np.asarray(orig_tokens)
+    orig_off = np.asarray(orig_off)
+    match_pos = np.asarray(match_pos)
+    B = len(orig_off) - 1
+    G = 0 if gen_tok is None else np.asarray(gen_tok).shape[1]
+    T = 1 + n_branches * chain_len + G
+    draft = np.full(B * T, -1, np.int32)
+    parent = np.zeros(B * T, np.int32)
+    cpos = np.full(B * T, -1, np.int32)
+    gmask = np.zeros(B * T, np.uint8)
+    for s in range(B):
+        o = s * T
+        c = orig_tokens[orig_off[s]:orig_off[s + 1]]
+        draft[o] = last_tok[s]
+        parent[o] = -1
+        if n_matches[s] > 0:
+            cpos[o] = match_pos[s, 0] + n - 1
+        for b in range(n_branches):
+            has = b < min(int(n_matches[s]), match_pos.shape[1])
+            for j in range(chain_len):
+                i = 1 + b * chain_len + j
+                parent[o + i] = 0 if j == 0 else i - 1
+                if has:
+                    q = int(match_pos[s, b]) + n + j
+                    if q < len(c):
+                        draft[o + i] = c[q]
+                        cpos[o + i] = q
+        for j in range(G):
+            i = 1 + n_branches * chain_len + j
+            parent[o + i] = 0 if j == 0 else i - 1
+            draft[o + i] = gen_tok[s][j]
+            gmask[o + i] = 1
+    node_off = (np.arange(B + 1) * T).astype(np.int32)
+    return draft, parent, node_off, cpos, gmask
+
+
+def advance(out_tok, out_len, draft_tok, cpos, node_off, path, accept_len, bonus, cursor, n):
+    """Commit one verification step (Sec. III-A).
+
+    The accepted draft tokens -- path nodes 1 .. accept_len (the root was
+    committed before) -- and the bonus token extend the generated sequence.
+    The tail becomes its last n tokens and the root of the next tree is the
+    bonus.  The cursor marks the start of the code not yet verified: when the
+    last accepted node came from c (cpos q >= 0), the code up to q is consumed
+    and the rest, from q + 1, stays the candidate draft; otherwise it stays.
+
+    Returns (out_tok', out_len', tail int32 [B, n], cursor', last_tok)."""
+    out = np.array(out_tok, copy=True)
+    out_len = np.asarray(out_len).astype(np.int32).copy()
+    cursor = np.asarray(cursor).astype(np.int32).copy()
+    B = len(out_len)
+    tail = np.zeros((B, n), np.int32)
+    last = np.zeros(B, np.int32)
+    for s in range(B):
+        o = int(node_off[s])
+        a = int(accept_len[s])
+        toks = [int(draft_tok[o + int(path[s, k])]) for k in range(1, a + 1)] + [int(bonus[s])]
+        L = int(out_len[s])
+        if L + len(toks) > out.shape[1]:
+            raise ValueError("committed-token buffer full")
+        out[s, L:L + len(toks)] = toks
+        out_len[s] = L + len(toks)
+        tail[s] = out[s, out_len[s] - n:out_len[s]]
+        q = int(cpos[o + int(path[s, a])])
+        if q >= 0:
+            cursor[s] = q + 1
+        last[s] = int(bonus[s])
+    return out, out_len, tail, cursor, last
+
+
+# ----------------------------------------------------------------------------
 # Entropy-aware dynamic verification -- Eq. (entropy) and the top_tau rule
 # ----------------------------------------------------------------------------
 

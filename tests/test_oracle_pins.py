@@ -774,3 +774,90 @@ def test_accept_chain_equals_tree_rule_on_chains(seed):
                 break
             j = k
         assert acc[s] == j and bonus[s] == argmax[o + j]
+
+
+# ----------------------------------------------------------------------------
+# Reuse <-> Generate controller
+# ----------------------------------------------------------------------------
+
+def test_build_reuse_tree_golden():
+    c = np.asarray([5, 6, 7, 8, 5, 6, 9, 1], np.int32)        # "5 6" occurs at 0 and 4
+    orig_off = np.asarray([0, len(c)], np.int64)
+    mp, nm = O.match_reuse(c, orig_off, np.asarray([[5, 6]]), np.asarray([0]), 4)
+    assert list(mp[0, :2]) == [0, 4] and nm[0] == 2
+    d, par, off, cpos, gm = O.build_reuse_tree(c, orig_off, mp, nm, [6], 2, 3, 3, gen_tok=[[40, 41]])
+    # root, branch 0: c[2..4], branch 1: c[6..7] then past the end, branch 2: none, generated 40 41
+    assert list(d) == [6, 7, 8, 5, 9, 1, -1, -1, -1, -1, 40, 41]
+    assert list(par) == [-1, 0, 1, 2, 0, 4, 5, 0, 7, 8, 0, 10]
+    assert list(cpos) == [1, 2, 3, 4, 6, 7, -1, -1, -1, -1, -1, -1]
+    assert list(gm) == [0] * 10 + [1, 1]
+    assert list(off) == [0, 12]
+
+
+def test_advance_golden():
+    out = np.zeros((1, 16), np.int32)
+    out[0, :4] = [1, 2, 5, 6]
+    d = np.asarray([6, 7, 8, 5, 9, 1, -1, -1, -1, -1, 40, 41], np.int32)
+    cpos = np.asarray([1, 2, 3, 4, 6, 7, -1, -1, -1, -1, -1, -1], np.int32)
+    path = np.full((1, 12), -1, np.int32)
+    path[0, :3] = [0, 1, 2]                                    # accepted 7, 8 (c[2], c[3])
+    o2, l2, tail, cur, last = O.advance(out, [4], d, cpos, [0, 12], path, [2], [33], [0], 2)
+    assert list(o2[0, :7]) == [1, 2, 5, 6, 7, 8, 33] and l2[0] == 7
+    assert list(tail[0]) == [8, 33] and cur[0] == 4 and last[0] == 33    # c[4..] stays the candidate
+    path[0, :3] = [0, 10, 11]                                  # the generated branch won
+    o3, l3, tail, cur, last = O.advance(out, [4], d, cpos, [0, 12], path, [2], [7], [3], 2)
+    assert list(o3[0, :7]) == [1, 2, 5, 6, 40, 41, 7] and cur[0] == 3     # no code consumed
+
+
+def _depths(parent, node_off):
+    dep = np.zeros(len(parent), np.int64)
+    for s in range(len(node_off) - 1):
+        o = int(node_off[s])
+        for i in range(1, int(node_off[s + 1]) - o):
+            dep[o + i] = dep[o + int(parent[o + i])] + 1
+    return dep
+
+
+def _edited(rng, c, vocab):
+    """c with a replaced span, an inserted span and a deleted span."""
+    c = list(c)
+    a = int(rng.integers(40, 80))
+    c[a:a + 5] = rng.integers(0, vocab, 5).tolist()
+    b = int(rng.integers(120, 160))
+    c[b:b] = rng.integers(0, vocab, 7).tolist()
+    e = int(rng.integers(200, 240))
+    del c[e:e + 6]
+    return np.asarray(c, np.int32)
+
+
+@pytest.mark.parametrize("seed,p0,gen", [(0, 20, 0), (1, 35, 3), (2, 8, 4), (3, 60, 2)])
+def test_session_reproduces_the_target_text(seed, p0, gen):
+    """A whole edit session on the host: match, tree, a synthetic greedy target
+    whose next token after k committed tokens is c'[k] (c' = the edited code),
+    tree acceptance, commit.  Greedy speculative decoding is lossless, so the
+    committed text is c' whatever the drafts; reuse makes it take far fewer
+    steps than tokens."""
+    rng = np.random.default_rng(seed)
+    vocab, n = 1000, 4
+    c = rng.integers(0, vocab, 300).astype(np.int32)
+    cp = _edited(rng, c, vocab)
+    orig_off = np.asarray([0, len(c)], np.int64)
+    out = np.zeros((1, len(cp) + 200), np.int32)
+    out[0, :p0] = cp[:p0]
+    out_len, cursor = np.asarray([p0], np.int32), np.asarray([0], np.int32)
+    last = np.asarray([cp[p0 - 1]], np.int32)
+    steps = 0
+    while out_len[0] < len(cp):
+        tail = out[:, out_len[0] - n:out_len[0]]
+        mp, nm = O.match_reuse(c, orig_off, tail, cursor, 4)
+        proposal = rng.integers(0, vocab, (1, gen)).astype(np.int32) if gen else None
+        d, par, off, cpos, _ = O.build_reuse_tree(c, orig_off, mp, nm, last, n, 24, 2, gen_tok=proposal)
+        dep = _depths(par, off)
+        pos = out_len[0] + dep
+        am = np.where(pos < len(cp), cp[np.minimum(pos, len(cp) - 1)], 0).astype(np.int32)
+        acc, path, bonus = O.accept_path(am, d, par, off)
+        out, out_len, tail, cursor, last = O.advance(out, out_len, d, cpos, off, path, acc, bonus, cursor, n)
+        steps += 1
+        assert steps < len(cp)
+    assert np.array_equal(out[0, :len(cp)], cp)
+    assert steps < (len(cp) - p0) // 3
