@@ -15,6 +15,10 @@
  *   ee_tree_verify_attn_inplace / ee_kv_compact_inplace
  *                        the same two steps with the tree's K/V already in
  *                        the cache after the context (in-place speculative K/V)
+ *   ee_build_reuse_tree / ee_advance
+ *                        the Reuse <-> Generate controller on the device: the
+ *                        next draft tree from the match points, the commit of
+ *                        a step's result (Sec. III-A)
  *   ee_chain_verify_attn causal attention of linear drafts of up to 2048
  *                        tokens verified in place (long reuse drafts; the LM
  *                        head takes them with anc NULL)
@@ -86,6 +90,7 @@ typedef enum {
 #define EE_DEVERR_FP16_RANGE   0x10  /* reserved (no current kernel sets it) */
 #define EE_DEVERR_TIMEOUT      0x20  /* a bounded device wait gave up */
 #define EE_DEVERR_PATH         0x40  /* path / accept_len inconsistent with the tree */
+#define EE_DEVERR_OVERFLOW     0x80  /* ee_advance: the committed-token buffer is full */
 
 const char* ee_version(void);
 const char* ee_status_string(ee_status s);
@@ -406,6 +411,55 @@ ee_status ee_chain_verify_attn(const ee_bf16* q, const ee_bf16* k_cache, const e
                                int32_t total_nodes, int32_t max_T, int32_t n_q, int32_t n_kv,
                                int32_t head_dim, float scale, float* out, void* ws, size_t ws_bytes,
                                ee_stream_t stream);
+
+/*
+ * ee_build_reuse_tree -- the next step's draft tree on the device (Sec. III-A:
+ * match points of the generated suffix in the remaining code are new draft
+ * starts, the code after each is a draft).  Every sequence gets
+ * T = 1 + n_branches * chain_len + gen_len <= EE_MAX_TREE nodes:
+ *   node 0            root: last_tok[s], the last committed token;
+ *   nodes 1 + b*chain_len + j  (b < n_branches, j < chain_len)
+ *                     branch b, a chain below the root: c[match_pos[s][b] + n + j]
+ *                     for b < min(n_matches[s], max_matches); -1 for an absent
+ *                     match and past the end of c (never accepted);
+ *   last gen_len nodes a chain below the root: gen_tok[s][0 .. gen_len), a
+ *                     draft model's proposal for edited content (gen_mask 1).
+ *   orig_tokens/orig_off as ee_match_reuse; match_pos int32 [B][max_matches],
+ *   n_matches int32 [B] (from ee_match_reuse); last_tok int32 [B];
+ *   gen_tok int32 [B][gen_len] or NULL when gen_len == 0.
+ *   Outputs: draft_tok, parent (local ids), cpos (position in c of the token,
+ *   the root's = match_pos[s][0] + n - 1, -1 for generated or empty nodes)
+ *   int32 [B*T]; node_off int32 [B+1] = s*T; gen_mask uint8 [B*T].
+ * Device errors: EE_DEVERR_MATCH_ARGS (a negative match position: its branch
+ * stays empty).
+ */
+ee_status ee_build_reuse_tree(const int32_t* orig_tokens, const int64_t* orig_off, int32_t B,
+                              const int32_t* match_pos, const int32_t* n_matches, int32_t max_matches,
+                              const int32_t* last_tok, int32_t n, int32_t chain_len, int32_t n_branches,
+                              const int32_t* gen_tok_or_null, int32_t gen_len, int32_t* draft_tok,
+                              int32_t* parent, int32_t* node_off, int32_t* cpos, uint8_t* gen_mask,
+                              void* ws, size_t ws_bytes, ee_stream_t stream);
+
+/*
+ * ee_advance -- commit one verification step on the device (Sec. III-A).  The
+ * accepted draft tokens (path nodes 1 .. accept_len; the root was committed
+ * before) and the bonus token are appended to the generated sequence
+ * out_tok[s][0 .. out_len[s]); then tail[s] = its last n tokens, last_tok[s] =
+ * bonus[s], and, when the last accepted node came from the code (cpos q >= 0),
+ * cursor[s] = q + 1: the code up to q is consumed and the rest stays the
+ * candidate draft; otherwise cursor[s] is unchanged.
+ *   out_tok int32 [B][cap], out_len int32 [B] (in/out, out_len >= n after
+ *   the commit); draft_tok / cpos / node_off from ee_build_reuse_tree (or any
+ *   tree with T <= EE_MAX_TREE); path / accept_len / bonus from the LM head;
+ *   tail int32 [B][n], cursor, last_tok int32 [B] (out; cursor in/out).
+ * Device errors: EE_DEVERR_PATH (bad path or accept_len), EE_DEVERR_OVERFLOW
+ * (out_tok has no room); the sequence is then left unchanged.
+ */
+ee_status ee_advance(int32_t* out_tok, int32_t* out_len, int32_t cap, const int32_t* draft_tok,
+                     const int32_t* cpos, const int32_t* node_off, const int32_t* path,
+                     const int32_t* accept_len, const int32_t* bonus, int32_t B, int32_t total_nodes,
+                     int32_t max_T, int32_t n, int32_t* tail, int32_t* cursor, int32_t* last_tok,
+                     void* ws, size_t ws_bytes, ee_stream_t stream);
 
 /*
  * ee_kv_compact_inplace -- ee_kv_compact's result when the tree's K/V already

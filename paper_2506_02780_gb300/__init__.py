@@ -26,14 +26,14 @@ EE_MAX_LM_NODES = 2048
 STATUS = {0: "ok", 1: "invalid argument", 2: "unsupported configuration", 3: "CUDA error",
           4: "device error word set", 5: "workspace too small"}
 DEVERR = {0x01: "MATCH_ARGS", 0x02: "TREE", 0x04: "PAGE", 0x08: "CTX", 0x10: "FP16_RANGE",
-          0x20: "TIMEOUT", 0x40: "PATH"}
+          0x20: "TIMEOUT", 0x40: "PATH", 0x80: "OVERFLOW"}
 DEVERR_TIMEOUT = 0x20
 
 EXPORTS = ("ee_version", "ee_status_string", "ee_workspace_size", "ee_workspace_init",
            "ee_read_errors", "ee_match_reuse", "ee_tree_prepare", "ee_tree_verify_attn", "ee_attn_plan",
            "ee_lmhead_accept", "ee_lmhead_verify", "ee_lmhead_accept_static", "ee_kv_compact",
            "ee_selftest_timeout", "ee_tree_verify_attn_inplace", "ee_kv_compact_inplace",
-           "ee_chain_verify_attn")
+           "ee_chain_verify_attn", "ee_build_reuse_tree", "ee_advance")
 
 VERIFY_MODES = {"greedy": 0, "direct": 1, "topk": 2, "entropy": 3}
 
@@ -71,6 +71,9 @@ _SIGS = {
                                      _P, _SZ, _P], _I),
     "ee_chain_verify_attn": ([_P, _P, _P, _I, _P, _I, _P, _I, _P, _I, _I, _I, _I, _I, _I, _F, _P, _P, _SZ, _P],
                              _I),
+    "ee_build_reuse_tree": ([_P, _P, _I, _P, _P, _I, _P, _I, _I, _I, _P, _I, _P, _P, _P, _P, _P, _P, _SZ, _P],
+                            _I),
+    "ee_advance": ([_P, _P, _I, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _P, _P, _P, _P, _SZ, _P], _I),
     "ee_kv_compact_inplace": ([_P, _P, _I64, _I, _I, _P, _I, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _P, _P,
                                _SZ, _P], _I),
     "ee_lmhead_accept": ([_P, _P, _I, _I, _P, _P, _P, _P, _P, _I, _I, _I, _P, _P, _P, _P, _P, _P, _SZ,
@@ -319,3 +322,25 @@ def ee_kv_compact_inplace(k_cache, v_cache, block_table, ctx_len_in, ctx_len_out
                                      _p(node_off), _p(path), _p(accept_len), B, int(total_nodes), max_T, n_kv,
                                      d, _p(dst_slot), _p(ws), ws.numel(), _stream(stream))
     _ok("ee_kv_compact_inplace", st)
+
+
+def ee_build_reuse_tree(orig_tokens, orig_off, match_pos, n_matches, last_tok, n, chain_len, n_branches,
+                        draft_tok, parent, node_off, cpos, gen_mask, ws, gen_tok=None, stream=None):
+    """Next draft tree: root, one reuse chain per match point, a generated branch."""
+    B = orig_off.numel() - 1
+    gen_len = 0 if gen_tok is None else gen_tok.shape[1]
+    _ok("ee_build_reuse_tree",
+        lib().ee_build_reuse_tree(_p(orig_tokens), _p(orig_off), B, _p(match_pos), _p(n_matches),
+                                  match_pos.shape[1], _p(last_tok), n, chain_len, n_branches, _p(gen_tok), gen_len,
+                                  _p(draft_tok), _p(parent), _p(node_off), _p(cpos), _p(gen_mask), _p(ws),
+                                  ws.numel(), _stream(stream)))
+
+
+def ee_advance(out_tok, out_len, draft_tok, cpos, node_off, path, accept_len, bonus, tail, cursor, last_tok, ws,
+               stream=None):
+    """Commit a step: accepted tokens + bonus appended, tail / cursor / root updated."""
+    B, cap = out_tok.shape
+    _ok("ee_advance",
+        lib().ee_advance(_p(out_tok), _p(out_len), cap, _p(draft_tok), _p(cpos), _p(node_off), _p(path),
+                         _p(accept_len), _p(bonus), B, draft_tok.numel(), path.shape[1], tail.shape[1], _p(tail),
+                         _p(cursor), _p(last_tok), _p(ws), ws.numel(), _stream(stream)))

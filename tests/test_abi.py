@@ -207,3 +207,25 @@ def test_chain_entry_points_reject_bad_args(L):
     v = L.ee_lmhead_verify
     assert v(FAKE, FAKE, 512, 4096, FAKE, None, None, None, FAKE, None, 1, 64, 64, 0, 1,
              FAKE, None, None, None, FAKE, FAKE, FAKE, None, ws, 1 << 26, None) == 1   # rules need a tree
+
+
+def test_controller_rejects_bad_args(L):
+    ws = ctypes.c_void_p(0x20000)
+    b = L.ee_build_reuse_tree
+    base = [FAKE, FAKE, 2, FAKE, FAKE, 4, FAKE, 4, 24, 4, None, 0] + [FAKE] * 5 + [ws, 1 << 26, None]
+    bad = list(base); bad[8] = 32
+    assert b(*bad) == 2                                # 1 + 4 x 32 nodes > 128
+    bad = list(base); bad[11] = 3
+    assert b(*bad) == 1                                # a generated branch without tokens
+    bad = list(base); bad[7] = 33
+    assert b(*bad) == 1                                # n above EE_MAX_NGRAM
+    bad = list(base); bad[18] = 64
+    assert b(*bad) == 5
+    a = L.ee_advance
+    abase = [FAKE, FAKE, 4096, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, 2, 194, 97, 4, FAKE, FAKE, FAKE, ws, 1 << 26, None]
+    bad = list(abase); bad[11] = 129
+    assert a(*bad) == 1                                # a tree above EE_MAX_TREE
+    bad = list(abase); bad[2] = 0
+    assert a(*bad) == 1
+    bad = list(abase); bad[13] = None
+    assert a(*bad) == 1
