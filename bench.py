@@ -414,6 +414,8 @@ def run_ours(args, rank, world, local_rank):
                                                inplace=True),
             "accept_len": [int(a) for a in sv.accept_len.cpu().tolist()[:8]]}
         del pool, sv
+    if not args.no_variants and not st.chain and args.config == "7b":
+        variants["edit_session"] = session_variant(w, dev, stream)
     assert E.ee_read_errors(st.ws, stream) == 0
 
     # ---- end to end: host inputs -> device -> step -> host results ---------
@@ -483,6 +485,91 @@ def run_ours(args, rank, world, local_rank):
                                "kind": "oracle", "sample": sample,
                                "threads_note": "numpy fp64, default BLAS threading"}
     return out
+
+
+def session_variant(w, dev, stream, K=16, replays=6):
+    """A whole edit session at the workload's shapes on the device (EditSession):
+    the workload's original code, an edited version of it (a replaced span, an
+    insertion, a deletion) as the synthetic target's greedy text, a committed
+    prefix of 200 tokens over a 4096-token context, trees of one reuse chain of
+    24 per match point (2) plus a 4-token generated branch from a noisy draft
+    model.  The device loop replays K captured steps at a time; the host loop
+    replays one step and reads the committed length back every step."""
+    import paper_2506_02780_gb300 as E
+    from paper_2506_02780_gb300.session import EditSession
+    rng = np.random.default_rng(11)
+    c = np.asarray(w.orig_tokens[w.orig_off[0]:w.orig_off[1]], np.int32)
+    cp = list(c)
+    cp[700:705] = rng.integers(0, w.vocab, 5).tolist()
+    cp[1500:1500] = rng.integers(0, w.vocab, 9).tolist()
+    del cp[2300:2306]
+    cp = np.asarray(cp, np.int32)
+    P0, ctx0, G, n = 200, 4096, 4, w.n
+    chain_len, nbr = 24, 2
+    T = 1 + nbr * chain_len + G
+    npg = -(-(ctx0 + len(cp) + 64 * T) // 16)
+    L, n_kv = w.layers, w.n_kv
+    g = torch.Generator(device=dev).manual_seed(11)
+    kc = torch.empty((L, npg, n_kv, 16, 128), dtype=torch.bfloat16, device=dev).normal_(0, 0.088, generator=g)
+    vc = torch.empty_like(kc).normal_(0, 0.088, generator=g)
+    bt = torch.randperm(npg, generator=g, device=dev).int().reshape(1, npg)
+    w_unit = (w.lm_w.float() / w.lm_w.float().norm(dim=1, keepdim=True)).bfloat16()
+    cap = len(cp) + 64 * T * 4
+    cp_pad = torch.zeros((1, cap + T + G), dtype=torch.int64, device=dev)
+    cp_pad[0, :len(cp)] = torch.as_tensor(cp)
+
+    def target_forward(ss):
+        want = cp_pad[0, ss.out_len.long()[0] + ss.depth.long()]
+        ss.hidden.copy_(w_unit[want] * 12.0)
+
+    def draft_proposal(ss):
+        k = ss.out_len.long()[:, None] + torch.arange(G, device=dev)[None, :]
+        t = cp_pad.gather(1, k)
+        ss.gen_tok.copy_(torch.where((k % 5) == 0, (t + 1) % w.vocab, t).int())
+
+    def make():
+        ss = EditSession(orig_tokens=torch.as_tensor(c, device=dev),
+                         orig_off=torch.as_tensor([0, len(c)], dtype=torch.int64, device=dev),
+                         committed=[cp[:P0].tolist()], ctx_len=[ctx0], k_cache=kc, v_cache=vc, block_table=bt,
+                         lm_w=w.lm_w, n_q=w.n_q, n=n, chain_len=chain_len, n_branches=nbr, gen_len=G, cap=cap,
+                         target_forward=target_forward, draft_proposal=draft_proposal, max_ctx=npg * 16 - T)
+        ss.q.normal_(0, 1, generator=g)
+        ss.k_tree.normal_(0, 0.088, generator=g)
+        ss.v_tree.normal_(0, 0.088, generator=g)
+        with torch.cuda.stream(stream):
+            ss.step(stream)
+        stream.synchronize()
+        return ss
+
+    dl = make()
+    dl.capture(K, stream)
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    len0 = int(dl.out_len[0])
+    with torch.cuda.stream(stream):
+        t0.record(stream)
+        for _ in range(replays):
+            dl.replay()
+        t1.record(stream)
+    t1.synchronize()
+    ms_dev = t0.elapsed_time(t1) / (K * replays)
+    toks = int(dl.out_len[0]) - len0
+    assert E.ee_read_errors(dl.ws, stream) == 0
+    ok = bool(np.array_equal(dl.out_tok[0, :int(dl.out_len[0])].cpu().numpy(), cp[:int(dl.out_len[0])]))
+    del dl
+    hl = make()
+    hl.capture(1, stream)
+    steps = K * replays
+    t_host = time.perf_counter()
+    for _ in range(steps):
+        hl.replay()
+        int(hl.out_len[0])                 # the host reads the state back each step
+    ms_host = (time.perf_counter() - t_host) * 1e3 / steps
+    assert E.ee_read_errors(hl.ws, stream) == 0
+    return {"device_loop_steps_per_s": round(1e3 / ms_dev, 2), "device_loop_ms_per_step": round(ms_dev, 5),
+            "committed_tokens_per_s": round(toks / (ms_dev * K * replays) * 1e3, 1),
+            "tokens_per_step": round(toks / (K * replays), 2), "steps_per_graph": K,
+            "host_loop_steps_per_s": round(1e3 / ms_host, 2), "committed_text_ok": ok,
+            "tree_nodes": T, "launches_per_step": hl.launches_per_step()}
 
 
 def run_instrumented(st, stream, evs):
