@@ -119,6 +119,12 @@ __device__ __forceinline__ float ex2(float x) {
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
   return y;
 }
+// three-input maximum (one instruction on sm_100-family GPUs)
+__device__ __forceinline__ float fmax3(float a, float b, float c) {
+  float r;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
+  return r;
+}
 
 // Loaded-page mask of context tile t: bit i set when the tile's 16-row block i
 // holds keys below k_end in a valid page.  s_pages holds the CTA's page ids
@@ -756,13 +762,18 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
             for (int c = 0; c < 64; ++c)
               if (!((kw >> c) & 1ull)) sr[c] = __float_as_uint(-INFINITY);
           }
+          // 8 independent chains of three-input maxima over the 64 values
           float mx[8];
 #pragma unroll
           for (int c = 0; c < 8; ++c) mx[c] = __uint_as_float(sr[c]);
 #pragma unroll
-          for (int c = 8; c < 64; ++c) mx[c & 7] = fmaxf(mx[c & 7], __uint_as_float(sr[c]));
-          tmax = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
-                       fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
+          for (int c = 8; c < 56; c += 16)         // values 8 .. 55, two per instruction
+#pragma unroll
+            for (int k = 0; k < 8; ++k)
+              mx[k] = fmax3(mx[k], __uint_as_float(sr[c + k]), __uint_as_float(sr[c + 8 + k]));
+#pragma unroll
+          for (int k = 0; k < 8; ++k) mx[k] = fmaxf(mx[k], __uint_as_float(sr[56 + k]));   // values 56 .. 63
+          tmax = fmax3(fmax3(mx[0], mx[1], mx[2]), fmax3(mx[3], mx[4], mx[5]), fmaxf(mx[6], mx[7]));
         }
         // the pair swaps its halves' maxima; both S halves are in registers before
         // either warp overwrites S with P
@@ -828,11 +839,13 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
             const uint32_t p1 = __float_as_uint(ex2(__uint_as_float(y1)));
             const uint64_t pp = f2_pack(p0, p1);
             ls2[e & 3] = e < 4 ? pp : f2_add(ls2[e & 3], pp);
+            // head = the top 16 bits (taken straight from p), tail = the top
+            // 16 bits of the exact remainder p - head
             const uint32_t h0 = p0 & 0xFFFF0000u;
             const uint32_t h1 = p1 & 0xFFFF0000u;
             uint32_t t0, t1;
             f2_unpack(f2_sub(pp, f2_pack(h0, h1)), t0, t1);
-            hw[e2] = __byte_perm(h0, h1, 0x7632);
+            hw[e2] = __byte_perm(p0, p1, 0x7632);
             tw[e2] = __byte_perm(t0, t1, 0x7632);
           }
           tc_st16_nowait(tl + sb * kKT + 32 * hf + 16 * hh, hw);
