@@ -2,17 +2,22 @@
 // paged KV cache plus the tree's own K/V, one layer per call (EfficientEdit
 // Sec. III-A: a single target forward pass over (prefix, draft) scores every
 // draft token; with a tree, each node sees the prefix and its own root path).
+// ee_tree_verify_attn_inplace and ee_chain_verify_attn are the same kernel
+// with the draft's K/V in the cache after the context (see kKV below).
 //
 // Work decomposition (split-KV):
 //   - For a (sequence, KV head) the query rows are the g = n_q / n_kv heads of
 //     the group times the T tree nodes, row r = node * g + head_in_group, so
 //     one K/V tile feeds g * T rows (GQA packing).  A CTA owns 128 rows: the
 //     M side of a tcgen05 MMA.
-//   - The context is cut into S <= 8 chunks of `chunk` keys (a multiple of the
-//     16-token page, at most 2048 pages); each (row block, chunk) is one CTA.  The CTA of
-//     the last chunk also processes the tree keys (one 128-key tile), masked by
-//     the ancestor bitmask.  A CTA first stages its chunk's page ids in shared
-//     memory.
+//   - A CTA processes segments: contiguous 128-key tile ranges of one row
+//     block.  Uniform launches cut each row block's context into S <= 16
+//     chunks of `chunk` keys (a multiple of the 16-token page, at most 2048
+//     pages), one CTA each; the last chunk also processes the tree keys (one
+//     128-key tile, masked by the ancestor bitmask).  Balanced launches give
+//     each of one CTA per SM an equal share of all row blocks' tiles (a CTA
+//     may finish one row block and start the next).  A CTA stages each
+//     segment's page ids in shared memory.
 //   - Q lives in shared memory (the softmax threads load the block's rows
 //     coalesced and store them in the 128-byte-swizzled K-major layout TMA
 //     gives the K tiles) and is the A operand of S = Q K^T; TMEM holds three S
@@ -32,10 +37,11 @@
 //     V is read straight from shared memory (MN-major).  P is carried to about
 //     2^-14 relative (fp16 would give 2^-11), V needs no conversion, and the
 //     split costs integer ops only, leaving the special-function pipe to exp2.
-//   - Warps 4-7 own one query row per thread (its TMEM lane): they read S,
-//     mask, keep the running max/sum, write P, and rescale O in TMEM only when
-//     a row's max grows by more than 2^8 (the stale max keeps every P <= 256,
-//     and the final O / l is unchanged).
+//   - Warps 4-11 own one query row per thread (its TMEM lane), two warps per
+//     lane quarter splitting each tile's keys: they read S, mask, keep the
+//     running max/sum, write P, and rescale O in TMEM only when a row's max
+//     grows by more than 2^8 (the stale max keeps every P <= 256, and the final
+//     O / l is unchanged).
 //   - Every chunk-CTA writes its unnormalised O rows and (max, sum) from TMEM
 //     to its own slot of the workspace (fp32, column-chunk major so that a
 //     warp's stores are contiguous; the slots stay in L2).  Once all S slots of
@@ -43,15 +49,17 @@
 //     [k * ceil(128 / S), ...) of all S slots with log-sum-exp weights and
 //     writes the fp32 output: one launch, no second pass, and L2 moves the
 //     partials several times faster than distributed shared memory does.
-//     With S = 1 the CTA writes O / l directly.  The S CTAs of a row block
-//     learn that all slots are written in one of two ways, chosen by the host:
+//     A segment that is a whole row block writes O / l directly.  The CTAs of
+//     a row block learn that all slots are written in one of two ways, chosen
+//     by the host:
 //       cluster: they form a thread-block cluster and meet at one cluster
 //         barrier (release / acquire at cluster scope);
 //       cooperative: the launch is cooperative (every CTA resident at once),
 //         each CTA adds 1 to the row block's counter (release) and waits for
 //         it to reach S (acquire); the last CTA to finish merging returns the
 //         counters to zero.  No GPC packing constraint: S can be any value up
-//         to 16, so the grid can cover every SM.
+//         to 16, so the grid can cover every SM.  Balanced launches count the
+//         pieces of each split row block the same way.
 //     Every CTA, also one whose chunk is empty for a short sequence, arrives:
 //     every wait before the arrival is bounded.
 //   - The next kernel in the stream may launch (programmatic dependent launch)
