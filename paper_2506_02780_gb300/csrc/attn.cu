@@ -31,12 +31,13 @@
 //     columns P lived in (the in-order tensor pipe finishes reading P first).
 //     With three S buffers the hand-off chain P(t) -> P.V(t) -> Q.K^T(t+3) ->
 //     softmax(t+3) spans three tiles, so it no longer sets the tile period.
-//   - P.V runs on bf16 operands: P is split exactly into a bf16 head (the top
-//     16 bits of the fp32 value) and a bf16 tail (the top 16 bits of the
-//     remainder), both written over S in TMEM and used as the MMA A operand;
-//     V is read straight from shared memory (MN-major).  P is carried to about
-//     2^-14 relative (fp16 would give 2^-11), V needs no conversion, and the
-//     split costs integer ops only, leaving the special-function pipe to exp2.
+//   - P.V runs on bf16 operands: P is split into a bf16 head (the fp32 value
+//     rounded to nearest bf16) and a bf16 tail (the exact remainder, rounded
+//     to nearest bf16), both written over S in TMEM and used as the MMA A
+//     operand; V is read straight from shared memory (MN-major).  P is carried
+//     to about 2^-17 relative (fp16 would give 2^-11) and V needs no
+//     conversion; per column pair the split is two packing conversions, a
+//     shift, a mask and one packed subtraction.
 //   - Warps 4-11 own one query row per thread (its TMEM lane), two warps per
 //     lane quarter splitting each tile's keys: they read S, mask, keep the
 //     running max/sum, write P, and rescale O in TMEM only when a row's max
@@ -126,6 +127,12 @@ __device__ __forceinline__ float ex2(float x) {
   float y;
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
   return y;
+}
+// {hi, lo} rounded to nearest bf16 and packed: lo in bits 0-15, hi in 16-31
+__device__ __forceinline__ uint32_t bf16x2_rn(float hi, float lo) {
+  uint32_t d;
+  asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(d) : "f"(hi), "f"(lo));
+  return d;
 }
 // three-input maximum (one instruction on sm_100-family GPUs)
 __device__ __forceinline__ float fmax3(float a, float b, float c) {
@@ -825,7 +832,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
           m_used = m_new;
         }
         const float nms = m_used == -INFINITY ? 0.f : -m_used * sl2;
-        // p = 2^(s*scale_log2 - m); P = head + tail, both bf16 (top 16 bits): this
+        // p = 2^(s*scale_log2 - m); P = head + tail, both bf16: this
         // half's head pairs go to columns 32 hf.. of the S buffer, its tail pairs
         // to 64 + 32 hf..
         // (pairs of columns run on packed fp32x2 arithmetic: the scale-and-shift,
@@ -847,14 +854,13 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
             const uint32_t p1 = __float_as_uint(ex2(__uint_as_float(y1)));
             const uint64_t pp = f2_pack(p0, p1);
             ls2[e & 3] = e < 4 ? pp : f2_add(ls2[e & 3], pp);
-            // head = the top 16 bits (taken straight from p), tail = the top
-            // 16 bits of the exact remainder p - head
-            const uint32_t h0 = p0 & 0xFFFF0000u;
-            const uint32_t h1 = p1 & 0xFFFF0000u;
+            // head = p rounded to bf16; tail = the remainder p - head (exact
+            // in fp32) rounded to bf16
+            const uint32_t hb = bf16x2_rn(__uint_as_float(p1), __uint_as_float(p0));
             uint32_t t0, t1;
-            f2_unpack(f2_sub(pp, f2_pack(h0, h1)), t0, t1);
-            hw[e2] = __byte_perm(p0, p1, 0x7632);
-            tw[e2] = __byte_perm(t0, t1, 0x7632);
+            f2_unpack(f2_sub(pp, f2_pack(hb << 16, hb & 0xFFFF0000u)), t0, t1);
+            hw[e2] = hb;
+            tw[e2] = bf16x2_rn(__uint_as_float(t1), __uint_as_float(t0));
           }
           tc_st16_nowait(tl + sb * kKT + 32 * hf + 16 * hh, hw);
           tc_st16_nowait(tl + sb * kKT + 64 + 32 * hf + 16 * hh, tw);
