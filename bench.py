@@ -460,6 +460,20 @@ def run_ours(args, rank, world, local_rank):
                              "traffic": TRAFFIC.get((name, args.config))})
         dom = max(cand, key=lambda n: cand[n]["ms"] * cand[n]["launches"])
         roofline = dict(rl[dom], kernel=dom)
+    step_rl = None
+    if rank == 0:
+        hbm = peaks["hbm_gbs"]
+        tf = peaks.get("bf16_tflops_sustained", peaks["bf16_tflops"])
+        # the step against the HBM roofline on the K/V and LM-head weight bytes it must read, and
+        # against the sum of its two big kernels' own floors (each the larger of bytes / HBM peak
+        # and flops / tensor peak)
+        kvw = w.layers * 2 * int(w.ctx_len.sum()) * w.n_kv * w.head_dim * 2 + w.vocab * w.hidden * 2
+        floor_s = (w.layers * max(alg["attn_bytes"] / (hbm * 1e9), alg["attn_flops"] / (tf * 1e12))
+                   + max(alg["lm_bytes"] / (hbm * 1e9), alg["lm_flops"] / (tf * 1e12)))
+        step_rl = {"kv_weight_bytes": kvw, "achieved_gbs": round(kvw / (ms_step * 1e-3) / 1e9, 1),
+                   "hbm_frac": round(kvw / (ms_step * 1e-3) / (hbm * 1e9), 4),
+                   "floor_us": round(floor_s * 1e6, 1), "frac_of_floor": round(floor_s / (ms_step * 1e-3), 4),
+                   "peaks": f"{peak_src}: HBM copy {hbm} GB/s, bf16 sustained {tf} TFLOP/s"}
 
     steps_per_s = world * 1e3 / ms_step
     out = {
@@ -474,7 +488,7 @@ def run_ours(args, rank, world, local_rank):
                        attention_launch=E.ee_attn_plan(w.B, w.max_T, w.n_q, w.n_kv, int(w.ctx_len.max()),
                                                        inplace="chain" if st.chain else False)),
         "draft_tokens_per_s": round(steps_per_s * alg["draft_nodes"], 1),
-        "roofline": roofline, "roofline_kernels": rl, "kernels": kernels,
+        "roofline": roofline, "roofline_kernels": rl, "step_roofline": step_rl, "kernels": kernels,
         "e2e": e2e, "gpu_launches": st.launches_per_step() * args.steps, "clocks": clk,
         "verify_variants": variants,
         "planted_accept": [int(a) for a in w.planted_accept[:8]],
