@@ -43,11 +43,15 @@ def parse_args():
     ap.add_argument("--steps", type=int, default=2000)
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--config", default="7b", choices=["7b", "batched", "33b", "tiny", "long"])
+    ap.add_argument("--config", default="7b", choices=["7b", "batched", "33b", "tiny", "long", "sweep"],
+                    help="workload of the timed step (sweep: --profile only, the match, tree and "
+                         "compaction kernels at the sweep's sizes)")
     ap.add_argument("--graphs", type=int, default=8, help="graphs replayed round-robin")
     ap.add_argument("--e2e-steps", type=int, default=300)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-clocks", action="store_true")
+    ap.add_argument("--no-rows", action="store_true",
+                    help="skip the sweep-size measurement of the match, tree and compaction kernels")
     ap.add_argument("--no-variants", action="store_true",
                     help="skip the step variants (entropy k=3, k=5; in-place speculative K/V)")
     ap.add_argument("--profile", action="store_true",
@@ -235,6 +239,111 @@ def oracle_step_time(w, attn_nodes=None, lm_rows=None):
     return full, t6 - t0, sample
 
 
+SWEEP_TEXT = ("sweep: 32 sequences of 65,536-token code (30% in repeated 8-token segments), n in {2, 4, 8}; "
+              "accept lengths U[1, 128] compacted over 28 layers of 7B-shaped K/V")
+
+
+def sweep_inputs(dev, n, layers):
+    """The reuse-matching and compaction sweep at full size (one seed per n)."""
+    return W.build("sweep", device=dev, n=n, layers=layers,
+                   seed=W.BASE_SEED + W.CONFIG_NAMES.index("sweep") + n)
+
+
+def sweep_rows(dev, stream, copies=16, reps=32):
+    """The hot path's small kernels at the sweep's sizes.  Device time per call
+    from a CUDA graph of `reps` calls between two events (the best of 5
+    replays).  The match cycles through `copies` copies of the code (134 MB,
+    more than L2 holds, so every call reads from DRAM); one compaction moves more
+    than L2 holds.  Algorithmic bytes: the code from each cursor on (4 B a token)
+    for the match; K and V of every committed entry read and written, all
+    layers, for the compaction; parents in, depth and ancestor masks out for the
+    tree."""
+    import paper_2506_02780_gb300 as E
+    peaks, src = load_peaks()
+    hbm = peaks["hbm_gbs"]
+    i32 = lambda a: torch.as_tensor(np.asarray(a), dtype=torch.int32, device=dev)  # noqa: E731
+
+    def timed(fn):
+        with torch.cuda.stream(stream):
+            fn(0)
+            stream.synchronize()
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=stream):
+                for k in range(reps):
+                    fn(k)
+            g.replay()
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            best = float("inf")
+            for _ in range(5):
+                a.record(stream)
+                g.replay()
+                b.record(stream)
+                b.synchronize()
+                best = min(best, a.elapsed_time(b) / reps)
+        return best * 1e-3          # seconds per call
+
+    def row(sec, nbytes, **extra):
+        gbs = nbytes / sec / 1e9
+        return dict(us=round(sec * 1e6, 2), bytes=int(nbytes), achieved_gbs=round(gbs, 1),
+                    frac=round(gbs / hbm, 4), **extra)
+
+    out = {"workload": SWEEP_TEXT, "peak": f"HBM copy {hbm} GB/s ({src})", "match_reuse": {}}
+    for n in (2, 4, 8):
+        w = sweep_inputs(dev, n, 28 if n == 4 else 1)
+        orig = [i32(w.orig_tokens) for _ in range(copies)]
+        off = torch.as_tensor(w.orig_off, device=dev)
+        tail, cur = i32(w.tail), i32(w.cursor)
+        mp = torch.empty((w.B, 16), dtype=torch.int32, device=dev)
+        nm = torch.empty(w.B, dtype=torch.int32, device=dev)
+        ws = E.new_workspace(w.B, w.total_nodes, 1, 0, device=dev)
+        sec = timed(lambda k: E.ee_match_reuse(orig[k % copies], off, tail, cur, 16, mp, nm, ws, stream))
+        region = sum(int(w.orig_off[s + 1] - w.orig_off[s]) - int(w.cursor[s]) for s in range(w.B))
+        out["match_reuse"][f"n{n}"] = row(sec, 4 * region)
+        if E.ee_read_errors(ws):
+            raise RuntimeError("device error in the match sweep")
+        if n == 4:
+            parent, node_off = i32(w.parent), i32(w.node_off)
+            depth = torch.empty(w.total_nodes, dtype=torch.int32, device=dev)
+            anc = torch.empty((w.total_nodes, 2), dtype=torch.int64, device=dev)
+            sec = timed(lambda k: E.ee_tree_prepare(parent, node_off, depth, anc, ws, stream))
+            out["tree_prepare"] = row(sec, w.total_nodes * (4 + 4 + 16) + 4 * (w.B + 1), nodes=w.total_nodes)
+            path = np.full((w.B, w.max_T), -1, np.int32)
+            for s in range(w.B):
+                path[s, :len(w.planted_path[s])] = w.planted_path[s]
+            path_d, acc_d, bt, ctx = i32(path), i32(w.planted_accept), i32(w.block_table), i32(w.ctx_len)
+            ctx_out = torch.empty(w.B, dtype=torch.int32, device=dev)
+            dst = torch.empty((w.B, w.max_T), dtype=torch.int32, device=dev)
+            sec = timed(lambda k: E.ee_kv_compact(w.k_tree, w.v_tree, w.k_cache, w.v_cache, bt, ctx, ctx_out,
+                                                  node_off, path_d, acc_d, dst, ws, stream))
+            entries = int((np.asarray(w.planted_accept) + 1).sum())
+            out["kv_compact"] = row(sec, entries * w.layers * w.n_kv * w.head_dim * 2 * 2 * 2, entries=entries,
+                                    layers=w.layers)
+            if E.ee_read_errors(ws):
+                raise RuntimeError("device error in the compaction sweep")
+        del w, orig
+    torch.cuda.empty_cache()
+    return out
+
+
+def oracle_rows_time():
+    """The oracle on the sweep's rows: the match (n = 4) whole, the compaction
+    of 2 of the 28 layers scaled by 14."""
+    import oracle as O
+    w = sweep_inputs("cpu", 4, 2)
+    raw = lambda x: x.detach().cpu().contiguous().view(torch.int16).numpy()  # noqa: E731
+    path = np.full((w.B, w.max_T), -1, np.int32)
+    for s in range(w.B):
+        path[s, :len(w.planted_path[s])] = w.planted_path[s]
+    t0 = time.perf_counter()
+    O.match_reuse(w.orig_tokens, w.orig_off, w.tail, w.cursor, 16)
+    t1 = time.perf_counter()
+    O.kv_compact(raw(w.k_tree), raw(w.v_tree), raw(w.k_cache), raw(w.v_cache), w.block_table, w.ctx_len,
+                 w.node_off, path, w.planted_accept)
+    t2 = time.perf_counter()
+    return {"match_reuse_n4_s": round(t1 - t0, 4), "kv_compact_s": round((t2 - t1) * 14, 4),
+            "sample": "sweep, n = 4: the match whole; the compaction of 2 of the 28 layers (x14)"}
+
+
 def cpu_cores():
     try:
         return len(os.sched_getaffinity(0))
@@ -255,6 +364,34 @@ def run_profile(args, local_rank):
     B.build_lib()
     dev = torch.device("cuda", local_rank)
     torch.cuda.set_device(dev)
+    if args.config == "sweep":
+        # the match (n = 4), tree and compaction kernels, each --steps times
+        w = sweep_inputs(dev, 4, 28 if args.layers is None else args.layers)
+        i32 = lambda a: torch.as_tensor(np.asarray(a), dtype=torch.int32, device=dev)  # noqa: E731
+        ws = E.new_workspace(w.B, w.total_nodes, 1, 0, device=dev)
+        mp = torch.empty((w.B, 16), dtype=torch.int32, device=dev)
+        nm = torch.empty(w.B, dtype=torch.int32, device=dev)
+        depth = torch.empty(w.total_nodes, dtype=torch.int32, device=dev)
+        anc = torch.empty((w.total_nodes, 2), dtype=torch.int64, device=dev)
+        path = np.full((w.B, w.max_T), -1, np.int32)
+        for s in range(w.B):
+            path[s, :len(w.planted_path[s])] = w.planted_path[s]
+        ctx_out = torch.empty(w.B, dtype=torch.int32, device=dev)
+        dst = torch.empty((w.B, w.max_T), dtype=torch.int32, device=dev)
+        orig, off, tail, cur = (i32(w.orig_tokens), torch.as_tensor(w.orig_off, device=dev), i32(w.tail),
+                                i32(w.cursor))
+        parent, node_off, path_d, acc_d = i32(w.parent), i32(w.node_off), i32(path), i32(w.planted_accept)
+        bt, ctx = i32(w.block_table), i32(w.ctx_len)
+        torch.cuda.synchronize(dev)
+        for _ in range(args.steps):
+            E.ee_match_reuse(orig, off, tail, cur, 16, mp, nm, ws)
+            E.ee_tree_prepare(parent, node_off, depth, anc, ws)
+            E.ee_kv_compact(w.k_tree, w.v_tree, w.k_cache, w.v_cache, bt, ctx, ctx_out, node_off, path_d, acc_d,
+                            dst, ws)
+        torch.cuda.synchronize(dev)
+        bits = E.ee_read_errors(ws)
+        print(json.dumps({"profile": "sweep", "steps": args.steps, "device_errors": bits}), flush=True)
+        return 0 if bits == 0 else 1
     over = {} if args.layers is None else {"layers": args.layers}
     w = W.build(args.config, device=dev, **over)
     st = S.from_workload(w, device=dev, keep_layers=False)
@@ -421,6 +558,9 @@ def run_ours(args, rank, world, local_rank):
     # ---- end to end: host inputs -> device -> step -> host results ---------
     e2e = run_e2e(st, plain[0], stream, args.e2e_steps, dev, world)
 
+    # the match, tree and compaction kernels at the sweep's sizes (after the timed regions)
+    rows = None if (args.no_rows or rank != 0) else sweep_rows(dev, stream)
+
     peaks, peak_src = load_peaks()
     per = (acc_ms / max(n_acc, 1)) if phase_events and n_acc else None
     kernels = {}
@@ -491,6 +631,7 @@ def run_ours(args, rank, world, local_rank):
         "roofline": roofline, "roofline_kernels": rl, "step_roofline": step_rl, "kernels": kernels,
         "e2e": e2e, "gpu_launches": st.launches_per_step() * args.steps, "clocks": clk,
         "verify_variants": variants,
+        "row_kernels": rows,
         "planted_accept": [int(a) for a in w.planted_accept[:8]],
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -498,6 +639,8 @@ def run_ours(args, rank, world, local_rank):
         out["cpu_baseline"] = {"value": round(1.0 / full, 6), "unit": UNIT, "cores": cpu_cores(),
                                "kind": "oracle", "sample": sample,
                                "threads_note": "numpy fp64, default BLAS threading"}
+        if rows is not None:
+            out["cpu_baseline"]["rows"] = oracle_rows_time()
     return out
 
 
@@ -768,6 +911,9 @@ def main():
         return
     if args.profile:
         sys.exit(run_profile(args, local_rank))
+    if args.config == "sweep":
+        sys.exit("the sweep has no verification step to time: its kernels are measured in every run's "
+                 "row_kernels, and --profile --config sweep launches them for ncu")
     if world > 1:
         torch.cuda.set_device(local_rank)
         torch.distributed.init_process_group("nccl", device_id=torch.device("cuda", local_rank))

@@ -3,9 +3,11 @@
 // prefix, so the K/V computed for them in the verification pass become cache
 // entries).  Path entry k of sequence s lands at position ctx + k.
 //
-// Pure data movement: one warp per (layer, sequence, path entry) copies the
-// n_kv K rows and n_kv V rows (head_dim bf16 = 256 bytes each) with 16-byte
-// vector loads/stores.  HBM-bound: 2 * 2 * n_kv * 256 bytes per entry and layer.
+// Pure data movement: one warp per (sequence, path entry, group of
+// kLayersPerWarp layers) copies the n_kv K rows and n_kv V rows (head_dim bf16
+// = 256 bytes each) of each of its layers with 16-byte vector loads/stores,
+// all of a batch's loads in flight before its stores.  HBM-bound:
+// 2 * 2 * n_kv * 256 bytes per entry and layer.
 //
 // ee_kv_compact_inplace: the same result when the tree's K/V already sit at
 // positions ctx + i.  Path entry k is node path[k] >= k: entries with
@@ -25,19 +27,21 @@ namespace {
 
 constexpr int kWarpsPerBlock = 8;
 constexpr int kVecPerRow = EE_HEAD_DIM * 2 / 16;   // uint4 per head row
+constexpr int kBatch = 16;                         // uint4 a lane holds between its loads and stores
+constexpr int kLayersPerWarp = 4;
 
 __global__ void __launch_bounds__(32 * kWarpsPerBlock)
 kv_compact_kernel(const uint4* k_tree, const uint4* v_tree, int64_t tree_layer_stride, uint4* k_cache,
                   uint4* v_cache, int64_t cache_layer_stride, int num_pages, const int32_t* block_table,
                   int max_pages, const int32_t* ctx_in, int32_t* ctx_out, const int32_t* node_off,
-                  const int32_t* path, const int32_t* accept_len, int max_T, int n_kv, int total_nodes,
+                  const int32_t* path, const int32_t* accept_len, int max_T, int n_kv, int total_nodes, int L,
                   int32_t* dst_slot, int32_t* err) {
   ee::pdl_allow_next();
   ee::pdl_wait();   // no global access before the previous kernel's writes are visible
   const int lane = threadIdx.x & 31;
   const int k = blockIdx.x * kWarpsPerBlock + (threadIdx.x >> 5);
   const int b = blockIdx.y;
-  const int l = blockIdx.z;
+  const int l = blockIdx.z;      // layer group
   if (k >= max_T) return;
   const int o = __ldcg(node_off + b);
   const int T = __ldcg(node_off + b + 1) - o;
@@ -70,17 +74,38 @@ kv_compact_kernel(const uint4* k_tree, const uint4* v_tree, int64_t tree_layer_s
   const int row = pos % EE_PAGE;
   if (lead) dst_slot[(size_t)b * max_T + k] = page * EE_PAGE + row;
   // 16 uint4 per head row; K rows then V rows
-  const int64_t tl = tree_layer_stride / 8 * l;   // strides are in bf16 elements
-  const int64_t cl = cache_layer_stride / 8 * l;
-  const int nvec = 2 * n_kv * kVecPerRow;
-  for (int v = lane; v < nvec; v += 32) {
-    const int which = v / (n_kv * kVecPerRow);  // 0 = K, 1 = V
-    const int rem = v % (n_kv * kVecPerRow);
-    const int h = rem / kVecPerRow, c = rem % kVecPerRow;
-    const int64_t src = tl + ((int64_t)(o + node) * n_kv + h) * kVecPerRow + c;
-    const int64_t dst = cl + (((int64_t)page * n_kv + h) * EE_PAGE + row) * kVecPerRow + c;
-    if (which == 0) k_cache[dst] = __ldcg(k_tree + src);
-    else v_cache[dst] = __ldcg(v_tree + src);
+  const int64_t tl = tree_layer_stride / 8;   // layer strides in uint4 (given in bf16 elements)
+  const int64_t cl = cache_layer_stride / 8;
+  // the warp's layers [l0, l1): up to kBatch vectors per lane are loaded
+  // before any is stored, so a warp has all its reads of a batch in flight
+  const int l0 = l * kLayersPerWarp, l1 = min(L, l0 + kLayersPerWarp);
+  const int nh = n_kv * kVecPerRow;               // uint4 of one K (or V) entry
+  const int nvec = 2 * nh;                        // per layer
+  const int tot = (l1 - l0) * nvec;
+  for (int v0 = 0; v0 < tot; v0 += 32 * kBatch) {
+    uint4 buf[kBatch];
+#pragma unroll
+    for (int u = 0; u < kBatch; ++u) {
+      const int v = v0 + 32 * u + lane;
+      if (v < tot) {
+        const int li = v / nvec, w = v - li * nvec;
+        const int which = w / nh;               // 0 = K, 1 = V
+        const int64_t src = tl * (l0 + li) + (int64_t)(o + node) * nh + (w - which * nh);
+        buf[u] = __ldcg((which ? v_tree : k_tree) + src);
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < kBatch; ++u) {
+      const int v = v0 + 32 * u + lane;
+      if (v < tot) {
+        const int li = v / nvec, w = v - li * nvec;
+        const int which = w / nh;
+        const int rem = w - which * nh;
+        const int h = rem / kVecPerRow, c = rem % kVecPerRow;
+        const int64_t dst = cl * (l0 + li) + (((int64_t)page * n_kv + h) * EE_PAGE + row) * kVecPerRow + c;
+        (which ? v_cache : k_cache)[dst] = buf[u];
+      }
+    }
   }
 }
 
@@ -184,13 +209,13 @@ extern "C" ee_status ee_kv_compact(const ee_bf16* k_tree, const ee_bf16* v_tree,
   if (L == 0) return EE_OK;
   if (tree_layer_stride % ((int64_t)n_kv * head_dim)) return EE_ERR_INVALID_ARG;
   const int total_nodes = (int)(tree_layer_stride / ((int64_t)n_kv * head_dim));
-  dim3 grid((max_T + kWarpsPerBlock - 1) / kWarpsPerBlock, B, L);
+  dim3 grid((max_T + kWarpsPerBlock - 1) / kWarpsPerBlock, B, (L + kLayersPerWarp - 1) / kLayersPerWarp);
   EE_CUDA_OK(ee::launch_pdl(
       kv_compact_kernel, grid, dim3(32 * kWarpsPerBlock), 0, (cudaStream_t)stream, 1,
       reinterpret_cast<const uint4*>(k_tree), reinterpret_cast<const uint4*>(v_tree),
       tree_layer_stride, reinterpret_cast<uint4*>(k_cache), reinterpret_cast<uint4*>(v_cache),
       cache_layer_stride, num_pages, block_table, max_pages, ctx_len_in, ctx_len_out, node_off, path,
-      accept_len, max_T, n_kv, total_nodes, dst_slot, ee::err_word(ws)));
+      accept_len, max_T, n_kv, total_nodes, (int)L, dst_slot, ee::err_word(ws)));
   return EE_OK;
 }
 

@@ -22,6 +22,7 @@ namespace ee {
 //   [32, 36)            never-written flag (zero): the self-test's wait target
 //   [256, 256+8*EE_MAX_LM_NODES)  LM-head packed running argmax per node
 //   [kLmVerifyOff, +kLmVerifyBytes) LM-head verification partials
+//   [kMatchOff, +kMatchBytes)     split reuse-span match: tickets and records
 //   [kAttnPartOff, ...)           attention partial slots, kAttnPartBytes per
 //                                 CTA of a split launch; the trailer of a row
 //                                 block's first slot holds its arrival counters
@@ -48,7 +49,12 @@ constexpr size_t kLmTkOff = kLmGthrOff + 8 * (size_t)EE_MAX_LM_NODES;
 constexpr size_t kLmTauOff = kLmTkOff + 4 * (size_t)EE_MAX_LM_NODES * kLmMaxK;
 constexpr size_t kLmVerifyBytes = kLmTauOff + 4 * (size_t)EE_MAX_LM_NODES;
 constexpr size_t kFinTicketOff = 24;   // in the head: finalize CTAs finished
-constexpr size_t kAttnPartOff = kLmVerifyOff + kLmVerifyBytes;   // attention partial slots
+// reuse-span match split over several CTAs per sequence: per sequence a 16-byte
+// ticket (zero between calls), then one record per CTA (its hit count and its
+// first max_matches hits)
+constexpr size_t kMatchOff = kLmVerifyOff + kLmVerifyBytes;
+constexpr size_t kMatchBytes = (size_t)1 << 20;
+constexpr size_t kAttnPartOff = kMatchOff + kMatchBytes;   // attention partial slots
 constexpr int kAttnRows = 128;        // query rows (node x head-in-group) per attention CTA
 constexpr int kAttnMaxSplits = 16;    // context chunks per row block
 // one CTA's partial: 128 rows x 128 fp32 of O (column-chunk major), then

@@ -55,7 +55,8 @@ def test_workspace_size(L):
     CTAs x 256 nodes x 80-byte records (8 top-k values, 8 ids, max and sum,
     padded to 16 bytes), then one 8-byte
     pruning threshold per node, the finalize step's 8 ranked ids and top_tau
-    per node), and, when the
+    per node), 1 MiB for the split reuse-span match (tickets and per-CTA
+    records), and, when the
     context is split, one attention partial slot per CTA: 128 rows x 128 fp32
     + 128 x (m, l) + a 256-byte counter trailer, for at most B x n_q row blocks
     x 16 chunks, and at least two per SM (152) for the balanced launch.
@@ -63,7 +64,7 @@ def test_workspace_size(L):
     head = L.ee_workspace_size(1, 64, 28, 128, 0)
     assert head == L.ee_workspace_size(8, 2048, 56, 128, 0)
     assert head % 256 == 0
-    assert head == 16896 + 152 * 256 * 80 + 8 * 2048 + 4 * 2048 * 8 + 4 * 2048
+    assert head == 16896 + 152 * 256 * 80 + 8 * 2048 + 4 * 2048 * 8 + 4 * 2048 + (1 << 20)
     slot = 128 * 128 * 4 + 128 * 8 + 256
     assert slot % 256 == 0
     for B, n_q, ctx in ((1, 28, 4096), (8, 56, 262144), (3, 8, 16), (1, 8, 512)):

@@ -301,6 +301,51 @@ def test_sweep_match_full_size(n):
     assert (cnt > 1).any()                    # repeated segments make some tails ambiguous
 
 
+@pytest.mark.parametrize("max_matches", [1, 16, 1024])
+def test_match_split_ranges(max_matches):
+    """Codes long enough for several CTAs per sequence (the scan is split into
+    ranges whose hits are concatenated by the last CTA to finish): hits planted
+    every 2,999 positions, none at all, dense (every 7th position, more than
+    1,024 hits), only before the cursor, and in a code shorter than one range;
+    positions and counts equal the oracle's.  The same inputs with a workspace
+    of only the fixed head (one CTA per sequence) give the same result."""
+    E = _E()
+    rng = np.random.default_rng(5)
+    n = 3
+    pat = np.array([1001, 1002, 1003], np.int32)            # tokens of c are drawn below 1000
+    lens = [65536, 20000, 40000, 30000, 100]
+    codes = []
+    for s, ln in enumerate(lens):
+        c = rng.integers(0, 1000, ln).astype(np.int32)
+        step = {0: 2999, 2: 7, 3: 1000, 4: 50}.get(s)
+        if step:
+            for p0 in range(5, ln - n - 1, step):
+                if s == 3 and p0 > 10000:
+                    break
+                c[p0:p0 + n] = pat
+        codes.append(c)
+    orig = np.concatenate(codes)
+    off = np.concatenate([[0], np.cumsum(lens)]).astype(np.int64)
+    tail = np.tile(pat, (len(lens), 1))
+    cursor = np.array([17, 0, 3, 12000, 0], np.int32)
+    pos, cnt = O.match_reuse(orig, off, tail, cursor, max_matches)
+    assert cnt[2] > 1024 and cnt[1] == 0 and cnt[3] == 0 and cnt[0] > 16
+    dev = "cuda"
+    args = (torch.as_tensor(orig, device=dev), torch.as_tensor(off, device=dev),
+            torch.as_tensor(tail, device=dev), torch.as_tensor(cursor, device=dev))
+    head = E.lib().ee_workspace_size(len(lens), 1, 1, 128, 0)
+    for ws in (E.new_workspace(len(lens), 64, 1, 0), torch.zeros(16896, dtype=torch.uint8, device=dev)):
+        for _ in range(2):                                   # the tickets are back at zero
+            mp = torch.full((len(lens), max_matches), 7, dtype=torch.int32, device=dev)
+            nm = torch.full((len(lens),), 7, dtype=torch.int32, device=dev)
+            E.ee_match_reuse(*args, max_matches, mp, nm, ws)
+            torch.cuda.synchronize()
+            assert E.ee_read_errors(ws) == 0
+            np.testing.assert_array_equal(mp.cpu().numpy(), pos)
+            np.testing.assert_array_equal(nm.cpu().numpy(), cnt)
+    assert head > 16896
+
+
 def test_sweep_compaction_full_size():
     E = _E()
     w = W.build("sweep", device="cuda")
