@@ -27,15 +27,19 @@ namespace {
 
 constexpr int kWarpsPerBlock = 8;
 constexpr int kVecPerRow = EE_HEAD_DIM * 2 / 16;   // uint4 per head row
-constexpr int kBatch = 16;                         // uint4 a lane holds between its loads and stores
+constexpr int kBatch = 8;                          // uint4 a lane holds between its loads and stores
 constexpr int kLayersPerWarp = 4;
 
+// kNkv > 0: the KV head count as a constant (the index arithmetic becomes
+// shifts); 0: taken from n_kv_arg
+template <int kNkv>
 __global__ void __launch_bounds__(32 * kWarpsPerBlock)
 kv_compact_kernel(const uint4* k_tree, const uint4* v_tree, int64_t tree_layer_stride, uint4* k_cache,
                   uint4* v_cache, int64_t cache_layer_stride, int num_pages, const int32_t* block_table,
                   int max_pages, const int32_t* ctx_in, int32_t* ctx_out, const int32_t* node_off,
-                  const int32_t* path, const int32_t* accept_len, int max_T, int n_kv, int total_nodes, int L,
-                  int32_t* dst_slot, int32_t* err) {
+                  const int32_t* path, const int32_t* accept_len, int max_T, int n_kv_arg, int total_nodes,
+                  int L, int32_t* dst_slot, int32_t* err) {
+  const int n_kv = kNkv > 0 ? kNkv : n_kv_arg;
   ee::pdl_allow_next();
   ee::pdl_wait();   // no global access before the previous kernel's writes are visible
   const int lane = threadIdx.x & 31;
@@ -210,8 +214,13 @@ extern "C" ee_status ee_kv_compact(const ee_bf16* k_tree, const ee_bf16* v_tree,
   if (tree_layer_stride % ((int64_t)n_kv * head_dim)) return EE_ERR_INVALID_ARG;
   const int total_nodes = (int)(tree_layer_stride / ((int64_t)n_kv * head_dim));
   dim3 grid((max_T + kWarpsPerBlock - 1) / kWarpsPerBlock, B, (L + kLayersPerWarp - 1) / kLayersPerWarp);
+  auto kern = n_kv == 1   ? kv_compact_kernel<1>
+              : n_kv == 2 ? kv_compact_kernel<2>
+              : n_kv == 4 ? kv_compact_kernel<4>
+              : n_kv == 8 ? kv_compact_kernel<8>
+                          : kv_compact_kernel<0>;
   EE_CUDA_OK(ee::launch_pdl(
-      kv_compact_kernel, grid, dim3(32 * kWarpsPerBlock), 0, (cudaStream_t)stream, 1,
+      kern, grid, dim3(32 * kWarpsPerBlock), 0, (cudaStream_t)stream, 1,
       reinterpret_cast<const uint4*>(k_tree), reinterpret_cast<const uint4*>(v_tree),
       tree_layer_stride, reinterpret_cast<uint4*>(k_cache), reinterpret_cast<uint4*>(v_cache),
       cache_layer_stride, num_pages, block_table, max_pages, ctx_len_in, ctx_len_out, node_off, path,
