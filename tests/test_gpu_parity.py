@@ -367,3 +367,66 @@ def test_sweep_compaction_full_size():
     np.testing.assert_array_equal(dst.cpu().numpy(), dref)
     np.testing.assert_array_equal(ctx_out.cpu().numpy(), cref)
     assert np.array_equal(U.raw16(w.k_cache), kc) and np.array_equal(U.raw16(w.v_cache), vc)
+
+
+@pytest.mark.parametrize("n_kv,n_q,layers", [(1, 8, 1), (3, 21, 5), (8, 56, 6), (2, 8, 4)])
+def test_compaction_head_counts_and_layer_groups(n_kv, n_q, layers):
+    """The compaction kernel's instances: KV head counts with a compiled-in
+    count (1, 2, 8) and the generic one (3); layer counts that fill the groups of
+    four exactly (4), leave a remainder (5, 6) or one layer.  Cache bytes, slots
+    and new context lengths bit-exact against the oracle's sequential append."""
+    E = _E()
+    w = W.build("sweep", B=6, layers=layers, n_kv=n_kv, n_q=n_q, seed=40 + n_kv)
+    dev = "cuda"
+    i32 = lambda a: torch.as_tensor(a, dtype=torch.int32, device=dev)  # noqa: E731
+    path = np.full((w.B, w.max_T), -1, np.int32)
+    for s in range(w.B):
+        path[s, :len(w.planted_path[s])] = w.planted_path[s]
+    k0, v0 = U.raw16(w.k_cache), U.raw16(w.v_cache)
+    kc_d = w.k_cache.to(dev)
+    vc_d = w.v_cache.to(dev)
+    ctx_out = torch.empty(w.B, dtype=torch.int32, device=dev)
+    dst = torch.empty((w.B, w.max_T), dtype=torch.int32, device=dev)
+    ws = E.new_workspace(w.B, w.total_nodes, 1, 0)
+    E.ee_kv_compact(w.k_tree.to(dev), w.v_tree.to(dev), kc_d, vc_d, i32(w.block_table), i32(w.ctx_len),
+                    ctx_out, i32(w.node_off), i32(path), i32(w.planted_accept), dst, ws)
+    torch.cuda.synchronize()
+    assert E.ee_read_errors(ws) == 0
+    kc, vc, dref, cref = O.kv_compact(U.raw16(w.k_tree), U.raw16(w.v_tree), k0, v0, w.block_table,
+                                      w.ctx_len, w.node_off, path, w.planted_accept)
+    np.testing.assert_array_equal(dst.cpu().numpy(), dref)
+    np.testing.assert_array_equal(ctx_out.cpu().numpy(), cref)
+    assert np.array_equal(U.raw16(kc_d), kc) and np.array_equal(U.raw16(vc_d), vc)
+
+
+@pytest.mark.parametrize("n", [9, 32])
+def test_match_long_ngrams_split(n):
+    """n-grams longer than the vectorised compare covers (the general loop),
+    over codes split across several CTAs per sequence: hits planted every 1,777
+    positions, including across range and tile boundaries."""
+    E = _E()
+    rng = np.random.default_rng(n)
+    pat = (2000 + np.arange(n)).astype(np.int32)
+    lens = [65536, 50000, 9000, 70000]
+    codes = []
+    for ln in lens:
+        c = rng.integers(0, 2000, ln).astype(np.int32)
+        for p0 in range(3, ln - n - 1, 1777):
+            c[p0:p0 + n] = pat
+        codes.append(c)
+    orig = np.concatenate(codes)
+    off = np.concatenate([[0], np.cumsum(lens)]).astype(np.int64)
+    tail = np.tile(pat, (len(lens), 1))
+    cursor = np.array([0, 4000, 8999 - n, 1], np.int32)
+    pos, cnt = O.match_reuse(orig, off, tail, cursor, 64)
+    dev = "cuda"
+    mp = torch.empty((len(lens), 64), dtype=torch.int32, device=dev)
+    nm = torch.empty(len(lens), dtype=torch.int32, device=dev)
+    ws = E.new_workspace(len(lens), 64, 1, 0)
+    E.ee_match_reuse(torch.as_tensor(orig, device=dev), torch.as_tensor(off, device=dev),
+                     torch.as_tensor(tail, device=dev), torch.as_tensor(cursor, device=dev), 64, mp, nm, ws)
+    torch.cuda.synchronize()
+    assert E.ee_read_errors(ws) == 0
+    np.testing.assert_array_equal(mp.cpu().numpy(), pos)
+    np.testing.assert_array_equal(nm.cpu().numpy(), cnt)
+    assert cnt[0] > 30
