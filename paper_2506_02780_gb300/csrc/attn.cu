@@ -452,10 +452,33 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
         const int local = y - 1 - s_wpre[b];
         hk = local / tiles;
         const int rem = local - hk * tiles;
-        int r = 0, cum = 0, tu = chain_rb_tiles(ctx, T, g, 0);
-        while (rem >= cum + tu) {
-          cum += tu;
-          ++r;
+        // the row block holding tile rem: every warp scans the row blocks' tile
+        // counts 32 at a time (a warp prefix sum; all warps reach the same answer)
+        const int nrb_b = (T * g + kRows - 1) / kRows;
+        int r = nrb_b - 1, cum = 0, tu = 0;
+        for (int r0 = 0, base = 0; r0 < nrb_b; r0 += 32) {
+          const int rr = r0 + lane;
+          const int t = rr < nrb_b ? chain_rb_tiles(ctx, T, g, rr) : 0;
+          int incl = t;
+#pragma unroll
+          for (int dd = 1; dd < 32; dd <<= 1) {
+            const int v = __shfl_up_sync(0xffffffffu, incl, dd);
+            if (lane >= dd) incl += v;
+          }
+          const int excl = base + incl - t;
+          const unsigned hit = __ballot_sync(0xffffffffu, rr < nrb_b && rem >= excl && rem < excl + t);
+          if (hit) {
+            const int src = __ffs(hit) - 1;
+            r = r0 + src;
+            cum = __shfl_sync(0xffffffffu, excl, src);
+            tu = __shfl_sync(0xffffffffu, t, src);
+            break;
+          }
+          base += __shfl_sync(0xffffffffu, incl, 31);
+        }
+        if (tu == 0) {   // not reached for a consistent work list
+          cum = 0;
+          for (int q = 0; q < r; ++q) cum += chain_rb_tiles(ctx, T, g, q);
           tu = chain_rb_tiles(ctx, T, g, r);
         }
         rb = r;
