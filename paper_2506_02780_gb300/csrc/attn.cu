@@ -339,6 +339,25 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
         s_seq[lane * kPer + k] = make_int4(p.node_off[bb], p.node_off[bb + 1], p.ctx_len[bb], 0);
       }
       __syncwarp();
+      // chain drafts: one KV head's tiles are a sum over its row blocks; for a
+      // few sequences the warp sums each one's row blocks 32 at a time (stored
+      // in .w), otherwise each lane walks its own sequences' row blocks
+      const bool coop = kChain && p.B <= 64;
+      if (coop) {
+        for (int bb = 0; bb < p.B; ++bb) {
+          const int4 sq = s_seq[bb];
+          const int Tb = sq.y - sq.x;
+          const bool bad = Tb < 1 || Tb > kMaxT || Tb > p.max_T || sq.x < 0 || sq.x + Tb > p.total_nodes;
+          const int c = min(max(sq.z, 0), p.max_ctx);
+          int acc = 0;
+          if (!bad)
+            for (int r = lane; r < (Tb * g + kRows - 1) / kRows; r += 32) acc += chain_rb_tiles(c, Tb, g, r);
+          acc = __reduce_add_sync(0xffffffffu, acc);
+          __syncwarp();
+          if (lane == 0) s_seq[bb].w = acc;
+        }
+        __syncwarp();
+      }
 #pragma unroll
       for (int k = 0; k < kPer; ++k) {
         const int bb = lane * kPer + k;
@@ -358,8 +377,11 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
           int tiles = kIP ? (c + (bad ? 1 : Tb) + kKT - 1) / kKT : (c + kKT - 1) / kKT + 1;
           int unit_max = tiles;
           if constexpr (kChain) {
-            tiles = 0;
-            for (int r = 0; r < nrb_b && !bad; ++r) tiles += chain_rb_tiles(c, Tb, g, r);
+            tiles = sq.w;
+            if (!coop) {
+              tiles = 0;
+              for (int r = 0; r < nrb_b && !bad; ++r) tiles += chain_rb_tiles(c, Tb, g, r);
+            }
             unit_max = bad ? 1 : chain_rb_tiles(c, Tb, g, nrb_b - 1);
           }
           if (!bad) {
