@@ -155,6 +155,11 @@ ee_status ee_selftest_timeout(void* ws, size_t ws_bytes, int64_t* out, ee_stream
  *   match_pos    int32 [B][max_matches] out: matches in ascending order, -1 pad
  *   n_matches    int32 [B]             out: total number of matches (may exceed
  *                                      max_matches; 1 <= max_matches <= 1024)
+ * A long code is scanned by several CTAs whose hits are concatenated through
+ * a region of the workspace (tickets that return to zero, per-CTA records);
+ * a workspace of ee_workspace_size() bytes holds it, and one of only the fixed
+ * head (EE_ERR_WORKSPACE below that) scans each sequence with one CTA.  The
+ * results do not depend on the split.
  * Device errors: EE_DEVERR_MATCH_ARGS (that sequence reports 0 matches).
  */
 ee_status ee_match_reuse(const int32_t* orig_tokens, const int64_t* orig_off, int32_t B,
