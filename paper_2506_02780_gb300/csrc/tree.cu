@@ -3,9 +3,11 @@
 // match points and generated branches share a prefix, so the step scores them
 // together as a tree whose nodes each see only their own root-to-node path.
 //
-// One CTA of 128 threads per sequence; thread i walks node i up to the root
-// through the parent array staged in shared memory (at most 127 steps, each a
-// shared-memory read), after a block-wide validation that parent[i] < i.
+// One CTA of 128 threads per sequence, thread i for node i.  After a
+// block-wide validation that parent[i] < i, the root paths are built by
+// pointer jumping in shared memory: node i keeps the nodes from itself up to
+// (not including) its current jump target and a jump target that doubles its
+// reach every round, so 7 rounds cover any path of a 128-node tree.
 #include "ee_common.cuh"
 
 namespace {
@@ -16,7 +18,8 @@ tree_prepare_kernel(const int32_t* parent, const int32_t* node_off, int32_t* dep
   // parent / node_off may come from an earlier kernel: plain loads after the
   // dependent-launch wait (no const __restrict__, whose loads may be issued
   // before it)
-  __shared__ int32_t s_par[EE_MAX_TREE];
+  __shared__ int32_t s_jmp[2][EE_MAX_TREE];
+  __shared__ uint64_t s_a0[2][EE_MAX_TREE], s_a1[2][EE_MAX_TREE];
   ee::pdl_allow_next();
   ee::pdl_wait();   // no global access before the previous kernel's writes are visible
   const int b = blockIdx.x;
@@ -27,32 +30,44 @@ tree_prepare_kernel(const int32_t* parent, const int32_t* node_off, int32_t* dep
     if (i == 0) ee::flag_error(err, EE_DEVERR_TREE);
     return;
   }
-  int p = 0;
+  int p = -1;
   bool ok = true;
   if (i < T) {
     p = parent[o + i];
     ok = (i == 0) ? (p == -1) : (p >= 0 && p < i);
-    s_par[i] = p;
   }
   const bool all_ok = __syncthreads_and(ok);
-  if (i >= T) return;
   if (!all_ok) {
     if (i == 0) ee::flag_error(err, EE_DEVERR_TREE);
-    depth[o + i] = 0;
-    anc[2 * (size_t)(o + i)] = 0;
-    anc[2 * (size_t)(o + i) + 1] = 0;
+    if (i < T) {
+      depth[o + i] = 0;
+      anc[2 * (size_t)(o + i)] = 0;
+      anc[2 * (size_t)(o + i) + 1] = 0;
+    }
     return;
   }
-  uint64_t a0 = 0, a1 = 0;
-  int d = 0;
-  int u = i;
-  while (u > 0) {            // terminates: parent[u] < u was checked for every node
-    if (u < 64) a0 |= 1ull << u; else a1 |= 1ull << (u - 64);
-    u = s_par[u];
-    ++d;
+  // every thread takes part in the rounds (nodes past T are isolated roots)
+  int j = i < T ? p : -1;
+  uint64_t a0 = i < 64 ? 1ull << i : 0ull, a1 = i < 64 ? 0ull : 1ull << (i - 64);
+  s_jmp[0][i] = j;
+  s_a0[0][i] = a0;
+  s_a1[0][i] = a1;
+  __syncthreads();
+#pragma unroll
+  for (int r = 0; r < 7; ++r) {   // 2^7 = 128 > the longest path
+    const int cur = r & 1;
+    if (j >= 0) {
+      a0 |= s_a0[cur][j];
+      a1 |= s_a1[cur][j];
+      j = s_jmp[cur][j];
+    }
+    s_jmp[cur ^ 1][i] = j;
+    s_a0[cur ^ 1][i] = a0;
+    s_a1[cur ^ 1][i] = a1;
+    __syncthreads();
   }
-  a0 |= 1ull;                // the root is on every path
-  depth[o + i] = d;
+  if (i >= T) return;
+  depth[o + i] = __popcll(a0) + __popcll(a1) - 1;   // the path holds the root and the node
   anc[2 * (size_t)(o + i)] = a0;
   anc[2 * (size_t)(o + i) + 1] = a1;
 }
