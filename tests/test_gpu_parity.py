@@ -430,3 +430,45 @@ def test_match_long_ngrams_split(n):
     np.testing.assert_array_equal(mp.cpu().numpy(), pos)
     np.testing.assert_array_equal(nm.cpu().numpy(), cnt)
     assert cnt[0] > 30
+
+
+def test_match_bad_sequences_in_a_split_batch():
+    """A batch whose long codes are split over several CTAs, with one sequence
+    whose offsets decrease and one with a negative cursor: the device error
+    word reports EE_DEVERR_MATCH_ARGS, those sequences report no match, and the
+    others equal the oracle's -- on two calls in a row (the tickets of the
+    split sequences return to zero; the bad ones take none)."""
+    E = _E()
+    rng = np.random.default_rng(8)
+    n = 4
+    pat = np.array([900, 901, 902, 903], np.int32)
+    lens = [60000, 30000, 50000, 20000]
+    codes = []
+    for ln in lens:
+        c = rng.integers(0, 800, ln).astype(np.int32)
+        for p0 in range(11, ln - n - 1, 997):
+            c[p0:p0 + n] = pat
+        codes.append(c)
+    orig = np.concatenate(codes)
+    off = np.concatenate([[0], np.cumsum(lens)]).astype(np.int64)
+    bad_off = off.copy()
+    bad_off[2] = bad_off[1] - 5               # sequence 1: end before start
+    cursor = np.array([0, 0, 0, -3], np.int32)  # sequence 3: negative cursor
+    tail = np.tile(pat, (len(lens), 1))
+    good = [0, 2]                               # sequence 2 spans [bad_off[2], off[3])
+    exp = {s: O.match_reuse(orig, bad_off[s:s + 2] - 0, tail[s:s + 1], cursor[s:s + 1], 16) for s in good}
+    dev = "cuda"
+    ws = E.new_workspace(len(lens), 64, 1, 0)
+    for _ in range(2):
+        mp = torch.full((len(lens), 16), 7, dtype=torch.int32, device=dev)
+        nm = torch.full((len(lens),), 7, dtype=torch.int32, device=dev)
+        E.ee_match_reuse(torch.as_tensor(orig, device=dev), torch.as_tensor(bad_off, device=dev),
+                         torch.as_tensor(tail, device=dev), torch.as_tensor(cursor, device=dev), 16, mp, nm, ws)
+        torch.cuda.synchronize()
+        assert E.ee_read_errors(ws) == 0x01
+        got_p, got_n = mp.cpu().numpy(), nm.cpu().numpy()
+        for s in good:
+            np.testing.assert_array_equal(got_p[s], exp[s][0][0])
+            assert got_n[s] == exp[s][1][0] > 16
+        for s in (1, 3):
+            assert got_n[s] == 0 and (got_p[s] == -1).all()
