@@ -19,7 +19,9 @@ tests/test_oracle_pins.py):
   tree_attention   pinned: torch SDPA in fp64 over each node's linear path,
                    single-key and equal-key closed forms, page-order invariance
   lm_head_argmax   pinned: planted argmax targets, duplicated-row ties,
-                   pure-Python dot products on a tiny case
+                   pure-Python dot products on a tiny case; the fp32
+                   accumulation bound against four fp32 summation orders and
+                   hand-built near ties (the candidate sets)
   accept_path      pinned: token-by-token replay of Eq. (piecewise), brute force
                    over all root-to-node paths, hand-worked golden cases
   kv_compact       pinned: sequential append into a slot dictionary, canaries

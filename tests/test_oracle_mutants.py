@@ -79,7 +79,10 @@ ATTN_PINS = ["test_attention_each_node_is_causal_attention_over_its_path",
              "test_attention_equal_keys_average_values", "test_attention_page_order_invariance",
              "test_attention_gqa_head_map"]
 LM_PINS = ["test_lm_head_pure_python_dot", "test_lm_head_planted_argmax",
-           "test_lm_head_duplicate_rows_lowest_id", "test_lm_head_identity_closed_form"]
+           "test_lm_head_duplicate_rows_lowest_id", "test_lm_head_identity_closed_form",
+           "test_lm_head_fp32_accumulation_stays_within_the_bound",
+           "test_lm_head_candidates_hold_every_argmax_within_the_bound",
+           "test_lm_head_candidates_at_a_gap_between_one_and_two_bounds"]
 ACCEPT_PINS = ["test_accept_golden", "test_accept_chain_replay_random", "test_accept_tree_bruteforce_random",
                "test_accept_planted"]
 COMPACT_PINS = ["test_compact_golden", "test_compact_sequential_append_and_canary"]
@@ -122,6 +125,9 @@ MUTANTS = [
      "am = logits.shape[1] - 1 - np.argmax(logits[:, ::-1], axis=1)", LM_PINS),
     ("lm_head_vocab_reversed", "lm_head_logits", "logits = x @ w.T", "logits = (w @ x.T).T[:, ::-1]",
      LM_PINS),
+    ("lm_head_bound_too_tight", "lm_head_logits", "err = 2.0 * x.shape[1] * _U32", "err = 1e-3 * _U32",
+     LM_PINS),
+    ("candidates_ignore_own_error", "lm_head_argmax", "logits[i] + err[i] >= lo", "logits[i] >= lo", LM_PINS),
     # acceptance, Eq. (piecewise)
     ("accept_judged_at_child", "accept_path", "int(argmax[o + p])", "int(argmax[o + i])", ACCEPT_PINS),
     ("accept_bonus_from_draft", "accept_path", "bonus[s] = int(argmax[o + best])",

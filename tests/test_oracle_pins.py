@@ -304,6 +304,81 @@ def test_lm_head_duplicate_rows_lowest_id():
         assert len(top) == 2 and am[i] == top.min()
 
 
+def test_lm_head_fp32_accumulation_stays_within_the_bound():
+    """Reading A7's bound holds for fp32 accumulation in any order: products of
+    two bf16 values are exact in fp32, and the sum of H rounded additions is off
+    by at most 2 H 2^-24 sum_k |x_k w_k| whatever the order (sequential, reversed,
+    16-wide blocks with fp32 partial sums as a tensor core forms them, BLAS)."""
+    H, V, n = 1024, 96, 3
+    g = torch.Generator().manual_seed(7)
+    x = torch.randn(n, H, generator=g).to(torch.bfloat16)
+    wm = (0.02 * torch.randn(V, H, generator=g)).to(torch.bfloat16)
+    logits, err = O.lm_head_logits(x, wm)
+    xf = x.float().numpy()
+    wf = wm.float().numpy()
+    prods = xf[:, None, :] * wf[None, :, :]                   # exact in fp32
+    orders = {}
+    acc = np.zeros((n, V), np.float32)
+    for k in range(H):
+        acc = (acc + prods[:, :, k]).astype(np.float32)
+    orders["sequential"] = acc
+    acc = np.zeros((n, V), np.float32)
+    for k in reversed(range(H)):
+        acc = (acc + prods[:, :, k]).astype(np.float32)
+    orders["reversed"] = acc
+    acc = np.zeros((n, V), np.float32)
+    for k0 in range(0, H, 16):
+        part = np.zeros((n, V), np.float32)
+        for k in range(k0, k0 + 16):
+            part = (part + prods[:, :, k]).astype(np.float32)
+        acc = (acc + part).astype(np.float32)
+    orders["blocked16"] = acc
+    orders["blas"] = (xf @ wf.T).astype(np.float32)
+    for name, y in orders.items():
+        dev = np.abs(y.astype(np.float64) - logits)
+        assert np.all(dev <= err), f"{name}: fp32 logits leave the bound by {(dev - err).max():.3e}"
+    assert err.max() < 1e-3 * np.abs(logits).max() + 1e-3    # and the bound is far from vacuous
+
+
+def test_lm_head_candidates_hold_every_argmax_within_the_bound():
+    """Any logits within err of the fp64 ones have their argmax among the
+    candidates -- including adversarial ones that raise a runner-up by err and
+    lower the maximum by err."""
+    rng = np.random.default_rng(3)
+    w = W.build("tiny", vocab=300, hidden=64, trees=[W.TreeSpec(6, [], [0])])
+    am, cands, logits = O.lm_head_argmax(w.hidden_states, w.lm_w)
+    _, err = O.lm_head_logits(w.hidden_states, w.lm_w)
+    for i in range(logits.shape[0]):
+        top = int(np.argmax(logits[i]))
+        for _ in range(50):
+            y = logits[i] + err[i] * rng.uniform(-1, 1, size=logits.shape[1])
+            assert int(np.argmax(y)) in set(cands[i].tolist())
+        for v in range(logits.shape[1]):
+            y = logits[i].copy()
+            y[top] -= err[i, top]
+            y[v] += err[i, v]
+            if int(np.argmax(y)) == v:
+                assert v in set(cands[i].tolist())
+
+
+def test_lm_head_candidates_at_a_gap_between_one_and_two_bounds():
+    """Hand-built near ties (H = 64, x = all ones, rows of ones differing in
+    element 0): the bound is err = 2 H 2^-24 sum_k |w_k| ~ 4.8e-4 per logit.
+    Row b trails row a by 2^-10 - 2^-12 = 7.3e-4: more than one bound, less
+    than two, so fp32 results may swap them and b is a candidate.  Row c
+    trails by 2^-10 + 2^-9 = 2.9e-3, more than both bounds: never the argmax."""
+    H = 64
+    x = torch.ones(1, H, dtype=torch.bfloat16)
+    w = torch.ones(4, H, dtype=torch.float32)
+    w[0, 0], w[1, 0], w[2, 0], w[3, 0] = -1.0, 2.0 ** -10, 2.0 ** -12, -(2.0 ** -9)   # rows: z, a, b, c
+    w = w.to(torch.bfloat16)
+    am, cands, logits = O.lm_head_argmax(x, w)
+    _, err = O.lm_head_logits(x, w)
+    gap_b, gap_c = logits[0, 1] - logits[0, 2], logits[0, 1] - logits[0, 3]
+    assert err[0, 1] < gap_b < err[0, 1] + err[0, 2] and gap_c > err[0, 1] + err[0, 3]
+    assert am[0] == 1 and list(cands[0]) == [1, 2]
+
+
 def test_lm_head_identity_closed_form():
     """W rows = unit vectors e_v (v < H): logits are the hidden coordinates."""
     H = 64
