@@ -7,7 +7,9 @@ workload's known tree (a 48-token reuse chain from the root, an 8-node branch
 off the root and one off chain node 24; ctx 4096; 28 query / 4 KV heads of
 128; vocab 152064, hidden 3584).
 """
+import os
 import subprocess
+import sys
 import tempfile
 
 import pytest
@@ -82,3 +84,14 @@ def test_clock_sampler_parses_nvidia_smi_rows():
 def test_clock_sampler_without_nvidia_smi_reports_nothing():
     s = bench.ClockSampler(0)
     assert s.stop() is None
+
+
+def test_reference_arm_runs_on_rank_0_only():
+    """Under torchrun the reference arm (the oracle on the host cores) runs on
+    rank 0 alone; every other rank exits 0 at once, without work or output."""
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    env = dict(os.environ, RANK="1", WORLD_SIZE="2", LOCAL_RANK="1")
+    r = subprocess.run([sys.executable, os.path.join(root, "bench.py"), "--impl", "reference", "--steps", "1",
+                        "--warmup", "3"], env=env, capture_output=True, text=True, timeout=300)
+    assert r.returncode == 0, r.stderr[-2000:]
+    assert r.stdout.strip() == ""
