@@ -160,6 +160,20 @@ MUTANTS = [
     ("controller_chain_starts_at_match", "build_reuse_tree", "q = int(match_pos[s, b]) + n + j",
      "q = int(match_pos[s, b]) + n - 1 + j", SESSION_PINS),
     ("controller_cursor_not_past_q", "advance", "cursor[s] = q + 1", "cursor[s] = q", SESSION_PINS),
+    ("controller_branch_without_match", "build_reuse_tree", "has = b < min(int(n_matches[s]), match_pos.shape[1])",
+     "has = b < match_pos.shape[1]", SESSION_PINS),
+    ("controller_branch_from_absent_match", "build_reuse_tree",
+     "has = b < min(int(n_matches[s]), match_pos.shape[1])",
+     "has = b < min(int(n_matches[s]), match_pos.shape[1]) or b == 0", SESSION_PINS),
+    ("controller_root_position_without_match", "build_reuse_tree", "if n_matches[s] > 0:", "if True:",
+     SESSION_PINS),
+    ("controller_root_position_past_match", "build_reuse_tree", "cpos[o] = match_pos[s, 0] + n - 1",
+     "cpos[o] = match_pos[s, 0] + n", SESSION_PINS),
+    ("advance_recommits_root", "advance", "for k in range(1, a + 1)", "for k in range(0, a + 1)", SESSION_PINS),
+    ("advance_tail_before_bonus", "advance", "tail[s] = out[s, out_len[s] - n:out_len[s]]",
+     "tail[s] = out[s, out_len[s] - n - 1:out_len[s] - 1]", SESSION_PINS),
+    ("inplace_reads_values_as_keys", "tree_kv_from_cache", "kt[:, o + i] = kc[:L, page, :, off, :]",
+     "kt[:, o + i] = vc[:L, page, :, off, :]", INPLACE_PINS),
 ]
 
 

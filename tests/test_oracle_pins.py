@@ -867,6 +867,14 @@ def test_build_reuse_tree_golden():
     assert list(cpos) == [1, 2, 3, 4, 6, 7, -1, -1, -1, -1, -1, -1]
     assert list(gm) == [0] * 10 + [1, 1]
     assert list(off) == [0, 12]
+    # no match point at all: the root alone holds a token, its position in c is unknown
+    c2 = np.asarray([3, 3, 4], np.int32)
+    off2 = np.asarray([0, 3], np.int64)
+    mp2, nm2 = O.match_reuse(c2, off2, np.asarray([[9, 9]]), np.asarray([0]), 2)
+    assert list(mp2[0]) == [-1, -1] and nm2[0] == 0
+    d, par, off, cpos, gm = O.build_reuse_tree(c2, off2, mp2, nm2, [9], 2, 2, 2)
+    assert list(d) == [9, -1, -1, -1, -1] and list(par) == [-1, 0, 1, 0, 3]
+    assert list(cpos) == [-1] * 5 and list(gm) == [0] * 5 and list(off) == [0, 5]
 
 
 def test_advance_golden():
