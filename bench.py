@@ -261,6 +261,46 @@ def oracle_step_time(w, attn_nodes=None, lm_rows=None):
     return full, t6 - t0, sample
 
 
+def oracle_repeat(w, budget_s):
+    """The default sample (every node of layer 0, 1/16 of the vocabulary)
+    repeated until about ``budget_s`` seconds of CPU work, each repetition
+    scaled to one full step.  Returns (mean full-step seconds, description)."""
+    fulls, spent_all, sample = [], 0.0, ""
+    while not fulls or (spent_all < budget_s and len(fulls) < 200):
+        full, spent, sample = oracle_step_time(w)
+        fulls.append(full)
+        spent_all += spent
+    return float(np.mean(fulls)), f"{sample}; repeated {len(fulls)} times ({spent_all:.1f} s of CPU work), mean"
+
+
+def oracle_single_thread(config, layers, budget_s=10.0, timeout_s=120):
+    """The same oracle sample timed in a child process held to one thread
+    (BLAS, OpenMP and torch; no GPU visible).  The child draws the
+    configuration's inputs on the CPU with one layer (the sample reads layer 0
+    only) and scales by the full layer count.  Never raises: a failure is
+    reported in the returned record."""
+    env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1",
+               NUMEXPR_NUM_THREADS="1", CUDA_VISIBLE_DEVICES="")
+    code = ("import json, sys, torch\n"
+            "torch.set_num_threads(1)\n"
+            f"sys.path.insert(0, {ROOT!r})\n"
+            "import bench, workloads as W\n"
+            f"w = W.build({config!r}, device='cpu', layers=1)\n"
+            f"w.layers = {int(layers)}\n"
+            f"full, sample = bench.oracle_repeat(w, {float(budget_s)!r})\n"
+            "print(json.dumps({'full_s': full, 'sample': sample}))\n")
+    try:
+        r = subprocess.run([sys.executable, "-c", code], env=env, capture_output=True, text=True,
+                           timeout=timeout_s)
+        if r.returncode != 0:
+            return {"error": (r.stderr or "")[-300:]}
+        d = json.loads(r.stdout.strip().splitlines()[-1])
+        return {"value": round(1.0 / d["full_s"], 6), "unit": UNIT, "cores": 1, "kind": "oracle",
+                "sample": d["sample"] + " (one thread, inputs drawn on the CPU)"}
+    except Exception as e:  # timing the baseline must never fail the benchmark
+        return {"error": f"{type(e).__name__}: {e}"[:300]}
+
+
 def oracle_sample_size(w, budget_s):
     """(attention nodes, LM-head vocabulary rows) of an oracle sample that takes
     about ``budget_s`` seconds: unit costs are calibrated on a minimal sample
@@ -683,18 +723,11 @@ def run_ours(args, rank, world, local_rank):
         "planted_accept": [int(a) for a in w.planted_accept[:8]],
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        # about 10 s of CPU work: the sample (every node of layer 0, 1/16 of the
-        # vocabulary) repeated, each repetition scaled to one full step
-        fulls, spent_all = [], 0.0
-        while not fulls or (spent_all < 10.0 and len(fulls) < 200):
-            full, spent, sample = oracle_step_time(w)
-            fulls.append(full)
-            spent_all += spent
-        full = float(np.mean(fulls))
-        sample = f"{sample}; repeated {len(fulls)} times ({spent_all:.1f} s of CPU work), mean"
+        full, sample = oracle_repeat(w, 10.0)
         out["cpu_baseline"] = {"value": round(1.0 / full, 6), "unit": UNIT, "cores": cpu_cores(),
                                "kind": "oracle", "sample": sample,
-                               "threads_note": "numpy fp64, default BLAS threading"}
+                               "threads_note": "numpy fp64, default BLAS threading",
+                               "single_thread": oracle_single_thread(args.config, w.layers)}
         if rows is not None:
             out["cpu_baseline"]["rows"] = oracle_rows_time()
     return out

@@ -95,3 +95,9 @@ def test_reference_arm_runs_on_rank_0_only():
                         "--warmup", "3"], env=env, capture_output=True, text=True, timeout=300)
     assert r.returncode == 0, r.stderr[-2000:]
     assert r.stdout.strip() == ""
+
+
+def test_single_thread_oracle_baseline_runs_in_a_child():
+    rec = bench.oracle_single_thread("tiny", 1, budget_s=0.5)
+    assert "error" not in rec, rec
+    assert rec["cores"] == 1 and rec["value"] > 0 and "one thread" in rec["sample"]
