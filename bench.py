@@ -273,20 +273,21 @@ def oracle_repeat(w, budget_s):
     return float(np.mean(fulls)), f"{sample}; repeated {len(fulls)} times ({spent_all:.1f} s of CPU work), mean"
 
 
-def oracle_single_thread(config, layers, budget_s=10.0, timeout_s=120):
+def oracle_single_thread(config, layers, vocab, budget_s=10.0, timeout_s=120):
     """The same oracle sample timed in a child process held to one thread
     (BLAS, OpenMP and torch; no GPU visible).  The child draws the
-    configuration's inputs on the CPU with one layer (the sample reads layer 0
-    only) and scales by the full layer count.  Never raises: a failure is
-    reported in the returned record."""
+    configuration's inputs on the CPU with only what the sample reads -- layer
+    0 and the first 1/16 of the vocabulary's weight rows -- and scales by the
+    full layer count and vocabulary.  Never raises: a failure is reported in
+    the returned record."""
     env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1",
                NUMEXPR_NUM_THREADS="1", CUDA_VISIBLE_DEVICES="")
     code = ("import json, sys, torch\n"
             "torch.set_num_threads(1)\n"
             f"sys.path.insert(0, {ROOT!r})\n"
             "import bench, workloads as W\n"
-            f"w = W.build({config!r}, device='cpu', layers=1)\n"
-            f"w.layers = {int(layers)}\n"
+            f"w = W.build({config!r}, device='cpu', layers=1, vocab={max(1, int(vocab) // 16)})\n"
+            f"w.layers, w.vocab = {int(layers)}, {int(vocab)}\n"
             f"full, sample = bench.oracle_repeat(w, {float(budget_s)!r})\n"
             "print(json.dumps({'full_s': full, 'sample': sample}))\n")
     try:
@@ -727,7 +728,7 @@ def run_ours(args, rank, world, local_rank):
         out["cpu_baseline"] = {"value": round(1.0 / full, 6), "unit": UNIT, "cores": cpu_cores(),
                                "kind": "oracle", "sample": sample,
                                "threads_note": "numpy fp64, default BLAS threading",
-                               "single_thread": oracle_single_thread(args.config, w.layers)}
+                               "single_thread": oracle_single_thread(args.config, w.layers, w.vocab)}
         if rows is not None:
             out["cpu_baseline"]["rows"] = oracle_rows_time()
     return out

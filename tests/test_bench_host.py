@@ -98,6 +98,7 @@ def test_reference_arm_runs_on_rank_0_only():
 
 
 def test_single_thread_oracle_baseline_runs_in_a_child():
-    rec = bench.oracle_single_thread("tiny", 1, budget_s=0.5)
+    rec = bench.oracle_single_thread("tiny", 1, 4096, budget_s=0.5)
     assert "error" not in rec, rec
     assert rec["cores"] == 1 and rec["value"] > 0 and "one thread" in rec["sample"]
+    assert "vocab rows 0..255 of 4096 (x16.0)" in rec["sample"]
