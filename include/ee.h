@@ -356,7 +356,10 @@ ee_status ee_lmhead_accept(const ee_bf16* hidden, const ee_bf16* lm_w, int32_t h
  *    ee_lmhead_accept.
  *  - The first call on each device looks up the array's device address
  *    (cudaGetSymbolAddress) with that device current; make that first call
- *    before any stream capture.
+ *    before any stream capture.  The array used is the current device's, so
+ *    `stream` must belong to the current device (NULL: the current device's
+ *    legacy stream); a stream of another device is rejected with
+ *    EE_ERR_INVALID_ARG.
  *  - Every call clears the array on `stream` before its launch, because the
  *    array keeps the previous call's contents.  All calls share the one array:
  *    calls that overlap on the GPU (different streams without ordering, or

@@ -1113,10 +1113,14 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
   }
 }
 
-// Clusters of `S` CTAs that fit on the GPU at once (asked once per size).
-int active_clusters(int S) {
-  static int cache[kMaxCluster + 1] = {};
-  if (!cache[S]) {
+// Clusters of `S` CTAs that fit on device `dev` at once (asked once per device
+// and size; `dev` is the current device).
+int active_clusters(int dev, int S) {
+  static std::mutex mu;
+  static int cache[kMaxDevices][kMaxCluster + 1] = {};
+  std::lock_guard<std::mutex> lock(mu);
+  int* cached = &cache[dev][S];
+  if (!*cached) {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(S * 64, 1, 1);
     cfg.blockDim = dim3(kThreads, 1, 1);
@@ -1133,19 +1137,22 @@ int active_clusters(int S) {
       cudaGetLastError();
       n = std::max(1, kNumSMs / S);
     }
-    cache[S] = n;
+    *cached = n;
   }
-  return cache[S];
+  return *cached;
 }
 
-// CTAs of one instantiation the GPU holds at once (asked once; -1 if unknown).
+// CTAs of one instantiation device `dev` (the current device) holds at once
+// (asked once per device; -1 if unknown).
 template <bool kBal>
-int resident_ctas() {
-  static int cap = 0;
+int resident_ctas(int dev) {
+  static std::mutex mu;
+  static int caps[kMaxDevices] = {};
+  std::lock_guard<std::mutex> lock(mu);
+  int& cap = caps[dev];
   if (!cap) {
-    int dev = 0, sms = 0, per = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess ||
-        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
+    int sms = 0, per = 0;
+    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
         cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per, attn_tc_kernel<kBal, kKVTree>, kThreads, kSmemBytes) !=
             cudaSuccess ||
         per < 1) {
@@ -1158,9 +1165,13 @@ int resident_ctas() {
   return cap;
 }
 
-// Every instantiation takes the full dynamic shared memory (set once).
-cudaError_t set_attrs() {
-  static bool done = false;
+// Every instantiation takes the full dynamic shared memory (set once per device;
+// `dev` is the current device).
+cudaError_t set_attrs(int dev) {
+  static std::mutex mu;
+  static bool done_dev[kMaxDevices] = {};
+  std::lock_guard<std::mutex> lock(mu);
+  bool& done = done_dev[dev];
   if (done) return cudaSuccess;
   cudaError_t e = cudaSuccess;
   const void* fns[6] = {(const void*)attn_tc_kernel<false, kKVTree>, (const void*)attn_tc_kernel<true, kKVTree>,
@@ -1203,7 +1214,7 @@ struct Split {
 //   tiles (w_max at most, t_max per unit at most) and may cross one unit
 //   boundary (about 1.5 tiles more); it needs 2 partial slots per CTA, a
 //   share of at most 256 context tiles (the staged page ids) and B <= 512.
-Split choose_split(int span, bool tree_tile, int n_rb, long w_max, int t_max, int B, size_t part_slots) {
+Split choose_split(int dev, int span, bool tree_tile, int n_rb, long w_max, int t_max, int B, size_t part_slots) {
   Split best;
   if (span <= 0) return best;                      // the tree tile alone: one chunk
   const int min_splits = (span + kMaxCtaPages * EE_PAGE - 1) / (kMaxCtaPages * EE_PAGE);
@@ -1215,7 +1226,7 @@ Split choose_split(int span, bool tree_tile, int n_rb, long w_max, int t_max, in
     // SMs scattered over the GPCs can leave a slot unusable: plan such launches
     // with one cluster slot fewer
     if (used > 1 && (size_t)n_rb * used > part_slots) continue;   // one partial slot per CTA
-    const long act = active_clusters(used);
+    const long act = active_clusters(dev, used);
     long waves = (n_rb + act - 1) / act;
     if (waves >= 2 && act > 1) waves = (n_rb + act - 2) / (act - 1);
     const long cost = 2 * waves * (tiles + 3);
@@ -1225,7 +1236,7 @@ Split choose_split(int span, bool tree_tile, int n_rb, long w_max, int t_max, in
       best.chunk = chunk;
     }
   }
-  const int cap = resident_ctas<false>();
+  const int cap = resident_ctas<false>(dev);
   if (cap > 0) {
     for (int s = std::max(2, min_splits); s <= kMaxSplits && (long)s * n_rb <= cap; ++s) {
       int chunk, used, tiles;
@@ -1240,7 +1251,7 @@ Split choose_split(int span, bool tree_tile, int n_rb, long w_max, int t_max, in
       }
     }
   }
-  const int capb = resident_ctas<true>();
+  const int capb = resident_ctas<true>(dev);
   if (capb > 0 && B <= kMaxBalSeqs && w_max <= (long)(kMaxCtaPages / (kKT / EE_PAGE)) * capb &&
       part_slots >= 2 * (size_t)capb) {
     const long m = std::max(2, (t_max + 13) / 14);
@@ -1262,7 +1273,7 @@ Split choose_split(int span, bool tree_tile, int n_rb, long w_max, int t_max, in
 
 // The plan for these sizes: span = paged keys of the longest row block
 // (max_ctx, or max_ctx + max_T in place), row blocks, work-list bound.
-Split plan_for(int B, int max_T, int n_q, int n_kv, int max_ctx, int kv, size_t slots) {
+Split plan_for(int dev, int B, int max_T, int n_q, int n_kv, int max_ctx, int kv, size_t slots) {
   const int g = n_q / n_kv;
   const int nrb = (max_T * g + kRows - 1) / kRows;
   const int span = kv != kKVTree ? max_ctx + max_T : max_ctx;
@@ -1273,7 +1284,7 @@ Split plan_for(int B, int max_T, int n_q, int n_kv, int max_ctx, int kv, size_t 
     for (int r = 0; r < nrb; ++r) per_seq += chain_rb_tiles(max_ctx, max_T, g, r);
     per_seq *= n_kv;
   }
-  return choose_split(span, kv == kKVTree, nrb * n_kv * B, (long)B * per_seq, t_max, B, slots);
+  return choose_split(dev, span, kv == kKVTree, nrb * n_kv * B, (long)B * per_seq, t_max, B, slots);
 }
 
 // Shared by ee_tree_verify_attn (tree K/V from k_tree / v_tree) and
@@ -1307,7 +1318,12 @@ ee_status verify_attn(const ee_bf16* q, const ee_bf16* k_tree, const ee_bf16* v_
   // a CTA stages at most kMaxCtaPages page ids, and a cluster holds at most 8 chunks
   if (span > (int64_t)kMaxCluster * kMaxCtaPages * EE_PAGE) return EE_ERR_UNSUPPORTED;
 
-  EE_CUDA_OK(set_attrs());
+  int dev = 0;
+  {
+    const ee_status ds = current_device(&dev);
+    if (ds != EE_OK) return ds;
+  }
+  EE_CUDA_OK(set_attrs(dev));
   // tensor maps: cache [pages * n_kv * 16 rows][128], tree [total][n_kv][128]
   // (in place the tree maps are not read: the cache maps stand in)
   CUtensorMap tmKc, tmVc, tmKt, tmVt;
@@ -1331,7 +1347,7 @@ ee_status verify_attn(const ee_bf16* q, const ee_bf16* k_tree, const ee_bf16* v_
   const int g = n_q / n_kv;
   const int nrb = (max_T * g + kRows - 1) / kRows;
   const size_t slots = ws_bytes > kAttnPartOff ? (ws_bytes - kAttnPartOff) / kAttnPartBytes : 0;
-  const Split sp = plan_for(B, max_T, n_q, n_kv, max_ctx, kv, slots);
+  const Split sp = plan_for(dev, B, max_T, n_q, n_kv, max_ctx, kv, slots);
   if (sp.S == 0) return EE_ERR_WORKSPACE;
   const int S = sp.bal ? 1 : sp.S, chunk = sp.chunk;
   // a split launch writes one partial slot per CTA after the zeroed part
@@ -1405,11 +1421,16 @@ extern "C" ee_status ee_attn_plan(int32_t B, int32_t max_T, int32_t n_q, int32_t
       max_T > (inplace == kKVChain ? EE_MAX_CHAIN : EE_MAX_TREE) || n_q < 1 || n_kv < 1 || n_q % n_kv != 0 ||
       max_ctx < 0 || !splits || !chunk || !mode || !ctas)
     return EE_ERR_INVALID_ARG;
-  EE_CUDA_OK(set_attrs());
+  int dev = 0;
+  {
+    const ee_status ds = current_device(&dev);
+    if (ds != EE_OK) return ds;
+  }
+  EE_CUDA_OK(set_attrs(dev));
   const int nrb = (max_T * (n_q / n_kv) + kRows - 1) / kRows;
   // the partial slots of a workspace sized by ee_workspace_size
   const size_t slots = std::max((size_t)B * n_q * kAttnMaxSplits, 2 * (size_t)kNumSMsMax);
-  const Split sp = plan_for(B, max_T, n_q, n_kv, max_ctx, inplace, slots);
+  const Split sp = plan_for(dev, B, max_T, n_q, n_kv, max_ctx, inplace, slots);
   if (sp.S == 0) return EE_ERR_UNSUPPORTED;
   if (sp.bal) {
     *splits = sp.bal_ctas;

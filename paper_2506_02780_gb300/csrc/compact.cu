@@ -248,11 +248,19 @@ extern "C" ee_status ee_kv_compact_inplace(ee_bf16* k_cache, ee_bf16* v_cache, i
     return EE_ERR_INVALID_ARG;
   if (ws_bytes < ee::kWorkspaceBytes) return EE_ERR_WORKSPACE;
   if (L == 0) return EE_OK;
-  static bool attr_set = false;
-  if (!attr_set) {
-    EE_CUDA_OK(cudaFuncSetAttribute(kv_compact_inplace_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                    (int)kInplaceSmem));
-    attr_set = true;
+  {
+    // the dynamic shared memory attribute, set once per device
+    int dev = 0;
+    const ee_status ds = ee::current_device(&dev);
+    if (ds != EE_OK) return ds;
+    static std::mutex mu;
+    static bool attr_set[ee::kMaxDevices] = {};
+    std::lock_guard<std::mutex> lock(mu);
+    if (!attr_set[dev]) {
+      EE_CUDA_OK(cudaFuncSetAttribute(kv_compact_inplace_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                      (int)kInplaceSmem));
+      attr_set[dev] = true;
+    }
   }
   dim3 grid(n_kv, B, L);
   EE_CUDA_OK(ee::launch_pdl(kv_compact_inplace_kernel, grid, dim3(kInplaceThreads), kInplaceSmem,

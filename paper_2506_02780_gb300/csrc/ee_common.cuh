@@ -8,6 +8,7 @@
 
 #include <algorithm>
 #include <cmath>
+#include <mutex>
 #include <utility>
 
 #include "../../include/ee.h"
@@ -66,6 +67,16 @@ constexpr size_t kAttnPartBytes = kAttnCntOff + 256;
 constexpr int kNumSMs = 152;
 
 __host__ __device__ inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+// Host-side set-up that CUDA applies per device (kernel attributes, occupancy
+// queries, device addresses of symbols) is cached per device ordinal: the
+// current device's index, or EE_ERR_UNSUPPORTED beyond kMaxDevices.  Each cache
+// is guarded by its own mutex, so host threads may call libee concurrently.
+constexpr int kMaxDevices = 64;
+inline ee_status current_device(int* dev) {
+  if (cudaGetDevice(dev) != cudaSuccess) return EE_ERR_CUDA;
+  return (*dev >= 0 && *dev < kMaxDevices) ? EE_OK : EE_ERR_UNSUPPORTED;
+}
 
 __device__ __forceinline__ void flag_error(int32_t* err, int bits) { atomicOr(err, bits); }
 

@@ -986,15 +986,23 @@ ee_status launch_lmhead(const ee_bf16* hidden, const ee_bf16* lm_w, int32_t hidd
   const size_t last = 1024 + (size_t)(EE_MAX_LM_NODES + 4) * 4;   // the last CTA: argmax per node
   const size_t smem_acc = std::max(smem, last);
   if (smem_acc > 227 * 1024) return EE_ERR_UNSUPPORTED;
-  static size_t attr_bytes[2] = {0, 0};
-  if (attr_bytes[va ? 1 : 0] < smem_acc) {
-    if (va)
-      EE_CUDA_OK(cudaFuncSetAttribute(lmhead_accept_kernel<true>,
-                                      cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_acc));
-    else
-      EE_CUDA_OK(cudaFuncSetAttribute(lmhead_accept_kernel<false>,
-                                      cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_acc));
-    attr_bytes[va ? 1 : 0] = smem_acc;
+  {
+    // the dynamic shared memory attribute, raised once per device and kernel
+    int dev = 0;
+    const ee_status ds = ee::current_device(&dev);
+    if (ds != EE_OK) return ds;
+    static std::mutex mu;
+    static size_t attr_bytes[ee::kMaxDevices][2] = {};
+    std::lock_guard<std::mutex> lock(mu);
+    if (attr_bytes[dev][va ? 1 : 0] < smem_acc) {
+      if (va)
+        EE_CUDA_OK(cudaFuncSetAttribute(lmhead_accept_kernel<true>,
+                                        cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_acc));
+      else
+        EE_CUDA_OK(cudaFuncSetAttribute(lmhead_accept_kernel<false>,
+                                        cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_acc));
+      attr_bytes[dev][va ? 1 : 0] = smem_acc;
+    }
   }
   const int num_tiles = p.n_vt * p.n_nt;
   int grid = (ee::kNumSMs / p.n_nt) * p.n_nt;   // multiple of n_nt: each CTA keeps one node tile
@@ -1120,15 +1128,22 @@ static __device__ __align__(256) unsigned char g_lm_scratch[kStaticScratchBytes]
 // Device address of g_lm_scratch per device ordinal, looked up once per device.
 // The host-side symbol `g_lm_scratch` is only a stand-in for the device array:
 // it must never be passed to a kernel.
-constexpr int kMaxDevices = 64;
-void* g_lm_scratch_ptr[kMaxDevices] = {};
+void* g_lm_scratch_ptr[ee::kMaxDevices] = {};
 
 std::mutex g_lm_scratch_mu;
 
-ee_status static_scratch(void** out) {
+// The current device's copy of the array; the launch stream must belong to
+// that device (the address, like the kernel attributes, is the current
+// device's), else EE_ERR_INVALID_ARG.
+ee_status static_scratch(ee_stream_t stream, void** out) {
   int dev = -1;
-  EE_CUDA_OK(cudaGetDevice(&dev));
-  if (dev < 0 || dev >= kMaxDevices) return EE_ERR_UNSUPPORTED;
+  const ee_status ds = ee::current_device(&dev);
+  if (ds != EE_OK) return ds;
+  if (stream) {
+    int sdev = -1;
+    EE_CUDA_OK(cudaStreamGetDevice((cudaStream_t)stream, &sdev));
+    if (sdev != dev) return EE_ERR_INVALID_ARG;
+  }
   std::lock_guard<std::mutex> lock(g_lm_scratch_mu);
   if (!g_lm_scratch_ptr[dev]) {
     void* ptr = nullptr;
@@ -1155,7 +1170,7 @@ extern "C" ee_status ee_lmhead_accept_static(const ee_bf16* hidden, const ee_bf1
                                      bonus, &empty, true);
   if (st != EE_OK || empty) return st;   // total_nodes > EE_MAX_LM_NODES -> EE_ERR_UNSUPPORTED
   void* scratch = nullptr;
-  const ee_status ss = static_scratch(&scratch);
+  const ee_status ss = static_scratch(stream, &scratch);
   if (ss != EE_OK) return ss;
   // the array keeps the previous call's contents: start from zero every call
   EE_CUDA_OK(cudaMemsetAsync(scratch, 0, kStaticScratchBytes, (cudaStream_t)stream));
