@@ -131,13 +131,32 @@ class Workload:
 def _original_code(rng, length, vocab, repeat_frac=0.0, seg=8):
     """Uniform tokens; optionally ``repeat_frac`` of them lie in copies of earlier
     ``seg``-token segments (repeated code lines make matches ambiguous).
-    Returns (tokens, list of (src, dst) copy starts)."""
+
+    The code is cut into ``seg``-token slots; a ``repeat_frac`` share of the
+    slots (slot 0 never) are destinations, each overwritten by a copy of an
+    earlier ``seg``-token span that starts anywhere but lies wholly inside
+    slots that are not destinations.  Copies never land on each other or on a
+    source, so every destination is an exact repeat of an earlier span: about
+    ``repeat_frac`` of all positions lie in an n-gram (n <= seg) that also
+    occurs earlier.  Returns (tokens, list of (src, dst) copy starts, by dst).
+    """
     c = rng.integers(0, vocab, size=length, dtype=np.int64).astype(np.int32)
-    n_seg = int(repeat_frac * length) // seg
+    n_slots = length // seg
+    n_seg = min(math.ceil(repeat_frac * length / seg), max(n_slots - 1, 0))
     copies = []
-    for _ in range(n_seg):
-        dst = int(rng.integers(seg, length - seg + 1))
-        src = int(rng.integers(0, dst - seg + 1))
+    if n_seg == 0:
+        return c, copies
+    dst_slots = np.sort(rng.choice(np.arange(1, n_slots), size=n_seg, replace=False))
+    is_dst = np.zeros(n_slots + 1, dtype=bool)
+    is_dst[dst_slots] = True
+    for ds in dst_slots:
+        dst = int(ds) * seg
+        for _ in range(64):      # a span starting anywhere before dst, clear of destinations
+            src = int(rng.integers(0, dst - seg + 1))
+            if not (is_dst[src // seg] or is_dst[(src + seg - 1) // seg]):
+                break
+        else:
+            continue             # no clear span found (rare, early slots): no copy
         c[dst:dst + seg] = c[src:src + seg]
         copies.append((src, dst))
     return c, copies
