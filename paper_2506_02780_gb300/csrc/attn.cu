@@ -55,12 +55,16 @@
 //     by the host:
 //       cluster: they form a thread-block cluster and meet at one cluster
 //         barrier (release / acquire at cluster scope);
-//       cooperative: the launch is cooperative (every CTA resident at once),
-//         each CTA adds 1 to the row block's counter (release) and waits for
-//         it to reach S (acquire); the last CTA to finish merging returns the
-//         counters to zero.  No GPC packing constraint: S can be any value up
-//         to 16, so the grid can cover every SM.  Balanced launches count the
-//         pieces of each split row block the same way.
+//       cooperative: the launch is cooperative (every CTA resident at once);
+//         the row block's 64-bit count grows by 720720 = lcm(1..16) per
+//         launch: each of its S CTAs reads the count (a multiple of 720720)
+//         before arriving, stores its partial, and after a CTA barrier one
+//         thread adds 720720 / S with a release reduction and waits (acquire)
+//         for the next multiple.  One release per CTA orders all its threads'
+//         stores, and nothing resets the count at the end of the kernel.  No
+//         GPC packing constraint: S can be any value up to 16, so the grid can
+//         cover every SM.  Balanced launches count the pieces of each split
+//         row block the same way.
 //     Every CTA, also one whose chunk is empty for a short sequence, arrives:
 //     every wait before the arrival is bounded.
 //   - The next kernel in the stream may launch (programmatic dependent launch)
@@ -225,7 +229,15 @@ __device__ __forceinline__ void merge_rows(const AttnParams& p, size_t slot_a, s
 // s >= 1 at slot1 + 2 (s - 1)).
 struct BalPiece {
   int hk, rb, o, R, K, k, slot0, slot1;
+  unsigned long long target;   // the count the row block's pieces raise it to
 };
+// A split row block's pieces meet at a 64-bit count in the trailer of its first
+// partial slot: every launch raises it by kCountGen in all (kCountGen / K per
+// piece, a release reduction after the piece's partial is stored), so a piece
+// reads a multiple of kCountGen at any time before its own arrival and waits
+// (acquire) for the next multiple.  The count is never reset; ee_workspace_init
+// zeroes it.
+constexpr unsigned long long kCountGen = 720720;   // lcm(1..16): K <= 16 divides it
 
 // Where the draft's K/V are (template kKV):
 //   kKVTree  -- k_tree / v_tree, one extra 128-key tile after the context;
@@ -433,6 +445,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
   // offset and rows for the merge
   const int split = kBal ? 0 : (int)(blockIdx.x % p.S);   // == cluster rank in the cluster mode
   int u_o = 0, u_R = 0;
+  unsigned long long u_target = 0;   // uniform cooperative mode: the row block's count target
 
   for (;;) {
     // ---------------- the next segment of this CTA's work ----------------
@@ -533,8 +546,11 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
       slot = 2 * (size_t)blockIdx.x + (seg0 > x_begin ? 1 : 0);
       if (!alone && threadIdx.x == 0 && s_npc < 2) {
         const int start0 = c0 * W / N;
-        s_pc[s_npc] = BalPiece{hk, rb, o, T * g, c1 - c0 + 1, (int)blockIdx.x - c0,
-                               2 * c0 + (U0 > start0 ? 1 : 0), 2 * (c0 + 1)};
+        const int slot0 = 2 * c0 + (U0 > start0 ? 1 : 0);
+        const unsigned long long c = ld_acquire64(
+            reinterpret_cast<const unsigned long long*>(p.part + (size_t)slot0 * kAttnPartBytes + kAttnCntOff));
+        s_pc[s_npc] = BalPiece{hk, rb, o, T * g, c1 - c0 + 1, (int)blockIdx.x - c0, slot0, 2 * (c0 + 1),
+                               (c / kCountGen + 1) * kCountGen};
         s_npc = s_npc + 1;
       }
       x_next = seg0;
@@ -584,6 +600,13 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
       slot = ((size_t)blockIdx.z * gridDim.y + blockIdx.y) * gridDim.x + blockIdx.x;
       u_o = o;
       u_R = T * g;
+      if (p.coop && p.S > 1 && threadIdx.x == 0) {
+        // read now (before this CTA's own arrival): a multiple of kCountGen
+        const size_t cta0 = ((size_t)blockIdx.z * gridDim.y + blockIdx.y) * gridDim.x + (size_t)rb * p.S;
+        const unsigned long long c = ld_acquire64(
+            reinterpret_cast<const unsigned long long*>(p.part + cta0 * kAttnPartBytes + kAttnCntOff));
+        u_target = (c / kCountGen + 1) * kCountGen;
+      }
     }
     const int R = T * g;
     const int n_ctx_tiles = k_end > k_begin ? (k_end - k_begin + kKT - 1) / kKT : 0;
@@ -973,7 +996,6 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
         if (hf == 0)
           __stcg(reinterpret_cast<float2*>(p.part + slot * kAttnPartBytes + kAttnMlOff) + r,
                  make_float2(row_m, row_l));
-        __threadfence();
       }
     }
     if constexpr (!kBal) break;
@@ -1015,15 +1037,17 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
     // cooperative, so all CTAs are resident and every count arrives)
     const int npieces = s_npc;     // written by thread 0 before the teardown barrier
     if (npieces == 0) return;
-    uint32_t* cnt[2];
+    unsigned long long* cnt[2];
 #pragma unroll
     for (int i = 0; i < 2; ++i)
-      cnt[i] = reinterpret_cast<uint32_t*>(p.part + (size_t)s_pc[i < npieces ? i : 0].slot0 * kAttnPartBytes +
-                                           kAttnCntOff);
+      cnt[i] = reinterpret_cast<unsigned long long*>(
+          p.part + (size_t)s_pc[i < npieces ? i : 0].slot0 * kAttnPartBytes + kAttnCntOff);
     if (threadIdx.x == 0) {
-      for (int i = 0; i < npieces; ++i) red_add_release(cnt[i], 1u);
+      // the partials of this CTA's pieces (every thread's stores precede the
+      // teardown barrier) are released with the count
+      for (int i = 0; i < npieces; ++i) red_add_release64(cnt[i], kCountGen / (unsigned)s_pc[i].K);
       for (int i = 0; i < npieces; ++i) {
-        const bool ready = wait_count_geq(cnt[i], (uint32_t)s_pc[i].K);
+        const bool ready = wait_count64_geq(cnt[i], s_pc[i].target);
         if (!ready) flag_error(p.err, EE_DEVERR_TIMEOUT);
         s_ready[i] = ready;
       }
@@ -1050,15 +1074,6 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
         }
       }
     }
-    // every piece's CTA has passed its wait once all have counted themselves
-    // here: the last returns both counters to zero
-    __syncthreads();
-    if (threadIdx.x == 0)
-      for (int i = 0; i < npieces; ++i)
-        if (s_ready[i] && atomicAdd(cnt[i] + 1, 1u) == (uint32_t)s_pc[i].K - 1) {
-          cnt[i][0] = 0u;
-          cnt[i][1] = 0u;
-        }
     return;
   } else {
     if (skip || p.S == 1) return;
@@ -1069,11 +1084,12 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
     const int R = u_R, o = u_o;
     const int rb = blockIdx.x / p.S;
     const size_t cta0 = ((size_t)blockIdx.z * gridDim.y + blockIdx.y) * gridDim.x + (size_t)rb * p.S;
-    uint32_t* cnt = reinterpret_cast<uint32_t*>(p.part + cta0 * kAttnPartBytes + kAttnCntOff);
+    unsigned long long* cnt = reinterpret_cast<unsigned long long*>(p.part + cta0 * kAttnPartBytes + kAttnCntOff);
     if (p.coop) {
       if (threadIdx.x == 0) {
-        red_add_release(cnt, 1u);     // this CTA's slot (ordered before by the fences and barrier)
-        const bool ready = wait_count_geq(cnt, (uint32_t)p.S);
+        // this CTA's partial (every thread's stores precede the teardown barrier)
+        red_add_release64(cnt, kCountGen / (unsigned)p.S);
+        const bool ready = wait_count64_geq(cnt, u_target);
         if (!ready) flag_error(p.err, EE_DEVERR_TIMEOUT);
         s_ready[0] = ready;
       }
@@ -1099,15 +1115,6 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
 #undef EE_MERGE_CASE
         default:
           break;
-      }
-    }
-    if (p.coop) {
-      // every CTA of the row block has passed its wait once all have counted
-      // themselves here: the last returns both counters to zero
-      __syncthreads();
-      if (threadIdx.x == 0 && s_ready[0] && atomicAdd(cnt + 1, 1u) == (uint32_t)p.S - 1) {
-        cnt[0] = 0u;
-        cnt[1] = 0u;
       }
     }
   }

@@ -59,8 +59,9 @@ constexpr size_t kAttnPartOff = kMatchOff + kMatchBytes;   // attention partial 
 constexpr int kAttnRows = 128;        // query rows (node x head-in-group) per attention CTA
 constexpr int kAttnMaxSplits = 16;    // context chunks per row block
 // one CTA's partial: 128 rows x 128 fp32 of O (column-chunk major), then
-// 128 x (m, l), then a 256-byte trailer (two uint32 counters, zeroed by
-// ee_workspace_init and returned to zero by every launch that uses them)
+// 128 x (m, l), then a 256-byte trailer whose first 8 bytes are the row
+// block's 64-bit arrival count (zeroed by ee_workspace_init; every launch that
+// uses it raises it by the same constant, so it is never reset)
 constexpr size_t kAttnMlOff = (size_t)kAttnRows * 128 * 4;
 constexpr size_t kAttnCntOff = kAttnMlOff + (size_t)kAttnRows * 8;
 constexpr size_t kAttnPartBytes = kAttnCntOff + 256;
