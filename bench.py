@@ -52,6 +52,8 @@ def parse_args():
     ap.add_argument("--no-clocks", action="store_true")
     ap.add_argument("--no-rows", action="store_true",
                     help="skip the sweep-size measurement of the match, tree and compaction kernels")
+    ap.add_argument("--no-configs", action="store_true",
+                    help="skip the 33b and batched configurations timed after the headline")
     ap.add_argument("--no-variants", action="store_true",
                     help="skip the step variants (entropy k=3, k=5; in-place speculative K/V)")
     ap.add_argument("--profile", action="store_true",
@@ -64,12 +66,10 @@ def parse_args():
 # DRAM bytes (read + write) per launch from one ncu capture of the kernel as it
 # now stands (profiles/ names the capture); a kernel changed since has no entry.
 TRAFFIC = {
-    ("tree_verify_attn", "7b"): 9063680,          # profiles/attn_tc_7b.md
+    ("tree_verify_attn", "7b"): 9063168,          # profiles/attn_tc_7b.md
     ("tree_verify_attn", "33b"): 160066048,       # profiles/attn_tc_33b.md
     ("tree_verify_attn", "batched"): 246875648,   # profiles/attn_tc_batched.md
-    # 7b LM head: null -- the kernel gained the linear-draft acceptance branch in
-    # its epilogue after profiles/lmhead_accept_7b.md was captured (1,095,463,424 B)
-    ("lmhead_accept", "7b"): None,
+    ("lmhead_accept", "7b"): 1095581184,          # profiles/lmhead_accept_7b.md
     ("lmhead_accept", "long"): 1108085248,        # profiles/lmhead_accept_long.md
     ("chain_verify_attn", "long"): 30021120,      # profiles/attn_chain_long.md
 }
@@ -734,6 +734,103 @@ def run_ours(args, rank, world, local_rank):
     return out
 
 
+def time_config(name, args, rank, dev, stream, steps):
+    """The same step on another configuration (33b, batched), timed like the
+    headline in the same process: plain CUDA graphs for ms_per_step, graphs with
+    three external events for the attention and LM-head phases, its own clock
+    record, and its roofline figures (per kernel: the bound of the larger of
+    bytes / HBM peak and flops / tensor peak; per step: the literal HBM fraction
+    on K/V and weight bytes and the fraction of the attainable floor)."""
+    import paper_2506_02780_gb300 as E
+    from paper_2506_02780_gb300 import step as S
+    w = W.build(name, seed=rank_seed(name, rank), device=dev)
+    alg = algorithmic(w)
+    st = S.from_workload(w, device=dev, keep_layers=False)
+    L = w.layers
+    mk = lambda: torch.cuda.Event(enable_timing=True, external=True)  # noqa: E731
+    plain, instr, evsets = [], [], []
+    with torch.cuda.stream(stream):
+        st.run(stream)
+        stream.synchronize()
+        for _ in range(2):
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=stream):
+                run_instrumented(st, stream, None)
+            plain.append(g)
+            g = torch.cuda.CUDAGraph()
+            evs = [mk() for _ in range(3)]
+            with torch.cuda.graph(g, stream=stream):
+                run_instrumented(st, stream, evs)
+            instr.append(g)
+            evsets.append(evs)
+    stream.synchronize()
+    assert E.ee_read_errors(st.ws, stream) == 0
+
+    def timed(pool, n):
+        t0 = torch.cuda.Event(enable_timing=True)
+        t1 = torch.cuda.Event(enable_timing=True)
+        with torch.cuda.stream(stream):
+            t0.record(stream)
+            for i in range(n):
+                pool[i % len(pool)].replay()
+            t1.record(stream)
+        t1.synchronize()
+        return t0.elapsed_time(t1) / n
+
+    for i in range(max(3, args.warmup // 4)):
+        plain[i % 2].replay()
+        instr[i % 2].replay()
+    stream.synchronize()
+    clocks = ClockSampler(dev.index)
+    if not args.no_clocks:
+        clocks.start()
+    torch.cuda.synchronize(dev)
+    ms = timed(plain, steps)
+    torch.cuda.synchronize(dev)
+    clk = None if args.no_clocks else clocks.stop()
+    acc = np.zeros(2)
+    n = max(2, steps // 4)
+    for i in range(n):
+        instr[i % 2].replay()
+        evs = evsets[i % 2]
+        evs[-1].synchronize()
+        acc += [evs[0].elapsed_time(evs[1]), evs[1].elapsed_time(evs[2])]
+    acc /= n
+    assert E.ee_read_errors(st.ws, stream) == 0
+    peaks, peak_src = load_peaks()
+    hbm = peaks["hbm_gbs"]
+    tf = peaks.get("bf16_tflops_sustained", peaks["bf16_tflops"])
+    attn_s, lm_s = 1e-3 * acc[0] / L, 1e-3 * acc[1]
+    rl = {}
+    for kname, t_s, nb, nf in (("tree_verify_attn", attn_s, alg["attn_bytes"], alg["attn_flops"]),
+                               ("lmhead_accept", lm_s, alg["lm_bytes"], alg["lm_flops"])):
+        gbs, tfs = nb / t_s / 1e9, nf / t_s / 1e12
+        floor = max(nb / (hbm * 1e9), nf / (tf * 1e12))
+        bound = "hbm" if nb / (hbm * 1e9) >= nf / (tf * 1e12) else "tensor"
+        rl[kname] = {"bound": bound, "achieved": round(gbs if bound == "hbm" else tfs, 2),
+                     "peak": hbm if bound == "hbm" else tf, "unit": "GB/s" if bound == "hbm" else "TFLOP/s",
+                     "frac": round((gbs / hbm) if bound == "hbm" else (tfs / tf), 4),
+                     "hbm_frac": round(gbs / hbm, 4), "frac_of_floor": round(floor / t_s, 4),
+                     "us_per_launch": round(1e6 * t_s, 2), "traffic": TRAFFIC.get((kname, name))}
+    kvw = L * 2 * int(w.ctx_len.sum()) * w.n_kv * w.head_dim * 2 + w.vocab * w.hidden * 2
+    floor_s = (L * max(alg["attn_bytes"] / (hbm * 1e9), alg["attn_flops"] / (tf * 1e12))
+               + max(alg["lm_bytes"] / (hbm * 1e9), alg["lm_flops"] / (tf * 1e12)))
+    out = {"workload": name + ": " + _config_text(name), "ms_per_step": round(ms, 5),
+           "value": round(1e3 / ms, 3), "unit": UNIT, "steps": steps,
+           "draft_tokens_per_s": round(1e3 / ms * alg["draft_nodes"], 1),
+           "kernels": {"attention_per_layer_us": round(1e6 * attn_s, 2), "lmhead_accept_us": round(1e6 * lm_s, 2)},
+           "roofline": dict(rl["tree_verify_attn"], kernel="tree_verify_attn"), "roofline_kernels": rl,
+           "step_roofline": {"kv_weight_bytes": kvw, "hbm_frac": round(kvw / (ms * 1e-3) / (hbm * 1e9), 4),
+                             "floor_us": round(floor_s * 1e6, 1), "frac_of_floor": round(floor_s / (ms * 1e-3), 4),
+                             "peaks": f"{peak_src}: HBM copy {hbm} GB/s, bf16 sustained {tf} TFLOP/s"},
+           "attention_launch": E.ee_attn_plan(w.B, w.max_T, w.n_q, w.n_kv, int(w.ctx_len.max())),
+           "clocks": clk, "config": W.describe(w)}
+    why = clocks_rejected(clk)
+    if why:
+        out["clocks_rejected"] = why
+    return out
+
+
 def session_variant(w, dev, stream, K=16, replays=6):
     """A whole edit session at the workload's shapes on the device (EditSession):
     the workload's original code, an edited version of it (a replaced span, an
@@ -1038,6 +1135,22 @@ def main():
         torch.cuda.set_device(local_rank)
         torch.distributed.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
     out = run_ours(args, rank, world, local_rank)
+    if args.config == "7b" and not args.no_configs and world == 1:
+        # the larger configurations, each timed after the headline in this process
+        import gc
+        gc.collect()
+        torch.cuda.empty_cache()
+        dev = torch.device("cuda", local_rank)
+        stream = torch.cuda.Stream(device=dev)
+        cfgs = {}
+        for name, n in (("33b", 40), ("batched", 100)):
+            try:
+                cfgs[name] = time_config(name, args, rank, dev, stream, n)
+            except Exception as e:  # a failed side measurement never hides the headline
+                cfgs[name] = {"error": f"{type(e).__name__}: {e}"[:300]}
+            gc.collect()
+            torch.cuda.empty_cache()
+        out["configs"] = cfgs
     if rank == 0:
         print(json.dumps(out), flush=True)
     if world > 1:

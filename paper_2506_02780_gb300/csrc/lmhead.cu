@@ -13,11 +13,17 @@
 //     issues tcgen05.mma.kind::f16 (bf16 x bf16 -> fp32) and commits each
 //     stage back to the producer; two TMEM accumulators let the epilogue drain
 //     tile i while tile i+1 accumulates.
-//   - Warps 2..5 (the epilogue) read the accumulator with tcgen05.ld (one TMEM
-//     lane = one vocabulary row per thread) and reduce each node's column to
-//     (max, lowest index) with a shuffle reduce-scatter; the running best per
-//     node stays in shared memory across the CTA's tiles and is published once
-//     with a 64-bit atomicMax on an order-preserving key.
+//   - Warps 2..9 (the epilogue, two per TMEM lane quarter taking alternate
+//     16-column chunks) read the accumulator with tcgen05.ld (one TMEM lane =
+//     one vocabulary row per thread) and reduce each node's column to (max,
+//     lowest index) with a shuffle reduce-scatter; the running best per node
+//     stays in shared memory across the CTA's tiles and is published once with
+//     a 64-bit atomicMax on an order-preserving key.
+//   - The LM head waits for the previous kernel before its first weight load:
+//     on sm_103a a TMA load issued before griddepcontrol.wait lands only after
+//     the previous grid has finished (measured in the attention kernel: 1.3 to
+//     1.5 us after the wait, the same as a load issued after it), so streaming
+//     W earlier buys nothing.
 //   - The last CTA to finish (ticket counter, no waiting) decodes the keys into
 //     argmax[], runs the acceptance for every sequence with one warp each
 //     (ancestor masks AND a per-node "edge accepted" mask), and resets the
