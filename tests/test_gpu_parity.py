@@ -472,3 +472,41 @@ def test_match_bad_sequences_in_a_split_batch():
             assert got_n[s] == exp[s][1][0] > 16
         for s in (1, 3):
             assert got_n[s] == 0 and (got_p[s] == -1).all()
+
+
+def test_split_row_block_counts_shared_by_plans():
+    """A workspace shared by launches with different plans (cooperative chunks
+    with different chunk counts, a balanced launch) keeps every result exact:
+    the row blocks' arrival counts are never reset, every launch raises them by
+    the same constant, so a count left by a 9-piece plan is a valid start for a
+    5-piece one.  Each call is bit-identical to the same call on a fresh
+    workspace, and close to the oracle."""
+    E = _E()
+    from paper_2506_02780_gb300 import step as S
+    cases = [W.build("tiny", seed=51, device="cuda", ctx=6000),
+             W.build("tiny", seed=52, device="cuda", ctx=1500),
+             W.build("tiny", seed=53, device="cuda", trees=_RAGGED, ctxs=[5000, 0, 3001, 4500, 17],
+                     n_q=12, n_kv=2)]
+    steps = [S.from_workload(w) for w in cases]
+    plans = [E.ee_attn_plan(w.B, w.max_T, w.n_q, w.n_kv, st.max_ctx) for w, st in zip(cases, steps)]
+    assert len({(p["mode"], p["splits"]) for p in plans}) == 3, plans
+    shared = E.new_workspace(5, max(w.total_nodes for w in cases), 12, 6000)
+    ref = []
+    for w, st in zip(cases, steps):                # fresh workspaces: the reference outputs
+        st.run()
+        torch.cuda.synchronize()
+        assert E.ee_read_errors(st.ws) == 0
+        ref.append(st.attn_out.clone())
+    anc = [U.check_tree(w, st) for w, st in zip(cases, steps)]
+    for rnd in range(3):
+        for i, (w, st) in enumerate(zip(cases, steps)):
+            x = st.inp
+            out = torch.full_like(st.attn_out[0], float("nan"))
+            E.ee_tree_verify_attn(x["q"][0], x["k_tree"][0], x["v_tree"][0], x["k_cache"][0], x["v_cache"][0],
+                                  x["block_table"], x["ctx_len"], st.max_ctx, x["node_off"], st.anc, st.max_T,
+                                  st.scale, out, shared)
+            torch.cuda.synchronize()
+            assert E.ee_read_errors(shared) == 0, (rnd, i)
+            assert torch.equal(out, ref[i][0]), (rnd, i, plans[i])
+    for i, (w, st) in enumerate(zip(cases, steps)):
+        U.check_attention(w, st, [0], anc[i], nodes=_sample_nodes(w, 12, 3))
