@@ -510,3 +510,32 @@ def test_split_row_block_counts_shared_by_plans():
             assert torch.equal(out, ref[i][0]), (rnd, i, plans[i])
     for i, (w, st) in enumerate(zip(cases, steps)):
         U.check_attention(w, st, [0], anc[i], nodes=_sample_nodes(w, 12, 3))
+
+
+@pytest.mark.parametrize("v_scale_log2", [24, -40])
+def test_split_values_far_from_unit_scale(v_scale_log2):
+    """Split row blocks hand partial (O, max, sum) over through the workspace and
+    merge them: values far above fp16's largest (2^24 times N(0, 1) / 11) and far
+    below its smallest normal (2^-40 times that) come out with the oracle's
+    relative accuracy, i.e. nothing on the way narrows the fp32 range.  The
+    values are scaled by an exact power of two, so the oracle sees the same bf16
+    inputs."""
+    E = _E()
+    from paper_2506_02780_gb300 import step as S
+    f = 2.0 ** v_scale_log2
+    w = W.build("tiny", seed=61, device="cuda", trees=_RAGGED, ctxs=[5000, 0, 3001, 4500, 17], n_q=12, n_kv=2)
+    w.v_cache.mul_(f)
+    w.v_tree.mul_(f)
+    st = S.from_workload(w)
+    plan = E.ee_attn_plan(w.B, w.max_T, w.n_q, w.n_kv, st.max_ctx)
+    assert plan["splits"] > 1 or plan["mode"] == 3, plan   # partials are merged
+    st.run()
+    torch.cuda.synchronize()
+    assert E.ee_read_errors(st.ws) == 0
+    anc = U.check_tree(w, st)
+    nodes = _sample_nodes(w, 16, 5)
+    ref = O.tree_attention(w.q[0], w.k_tree[0], w.v_tree[0], w.k_cache[0], w.v_cache[0], w.block_table,
+                           w.ctx_len, w.node_off, anc, nodes=nodes)[nodes]
+    got = st.attn_out[0].cpu().double().numpy()[nodes]
+    assert np.isfinite(got).all()
+    U.assert_close(got / f, ref / f, f"attention, values scaled by 2^{v_scale_log2}")
