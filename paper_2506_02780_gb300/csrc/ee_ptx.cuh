@@ -251,6 +251,14 @@ __device__ __forceinline__ bool wait_count_geq(const uint32_t* cnt, uint32_t tar
 __device__ __forceinline__ void red_add_release64(unsigned long long* a, unsigned long long v) {
   asm volatile("red.release.gpu.global.add.u64 [%0], %1;" ::"l"(a), "l"(v) : "memory");
 }
+// Fetch-and-add with acquire-release semantics at GPU scope: after a CTA
+// barrier, one thread's add publishes every write the CTA made before the
+// barrier and observes every write published by earlier adds.
+__device__ __forceinline__ unsigned int atom_add_acq_rel(unsigned int* a, unsigned int v) {
+  unsigned int old;
+  asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], %2;" : "=r"(old) : "l"(a), "r"(v) : "memory");
+  return old;
+}
 __device__ __forceinline__ unsigned long long ld_acquire64(const unsigned long long* a) {
   unsigned long long v;
   asm volatile("ld.acquire.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(a) : "memory");

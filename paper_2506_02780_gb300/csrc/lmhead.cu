@@ -27,7 +27,12 @@
 //   - The last CTA to finish (ticket counter, no waiting) decodes the keys into
 //     argmax[], runs the acceptance for every sequence with one warp each
 //     (ancestor masks AND a per-node "edge accepted" mask), and resets the
-//     workspace state for the next call.
+//     workspace state for the next call.  The tail is a chain of global round
+//     trips, kept short: the ticket is one acquire-release add after the CTA
+//     barrier (no separate fences), the node offsets load beside the key
+//     exchange, and the acceptance loads each node's inputs in one round trip.
+//   - The producer thread issues the ring's first stages right after it
+//     initialises the barriers, before the set-up barrier.
 //   - The kernel is bound by streaming W from HBM when the node count is below
 //     the ridge point (~250), by the tensor pipe above it.
 // Every mbarrier wait is bounded (2e9 SM cycles, about 1 s); on expiry the CTA sets
@@ -190,20 +195,33 @@ __device__ void accept_sequences(const AcceptArgs& a, const int32_t* am, const i
       }
       continue;
     }
-    // notok bit i: node i's edge from its parent is rejected
+    // notok bit i: node i's edge from its parent is rejected.  Each lane's
+    // nodes' parent, token, ancestor mask and depth are loaded together (one
+    // round trip); the deepest accepted node's mask comes from its lane.
     uint32_t notok[4];
     uint64_t a0[4], a1[4];
+    int par_[4], tok_[4], dep_[4];
+#pragma unroll
+    for (int c = 0; c < 4; ++c) {
+      const int i = c * 32 + lane;
+      const bool in = i < T;
+      par_[c] = in && i > 0 ? a.parent[o + i] : -1;
+      tok_[c] = in && i > 0 ? a.draft_tok[o + i] : 0;
+      dep_[c] = in ? a.depth[o + i] : 0;
+      a0[c] = in ? a.anc[2 * (size_t)(o + i)] : 0ull;
+      a1[c] = in ? a.anc[2 * (size_t)(o + i) + 1] : 0ull;
+    }
     int key_best = -1;
 #pragma unroll
     for (int c = 0; c < 4; ++c) {
       const int i = c * 32 + lane;
       bool bad = false;
       if (i < T && i > 0) {
-        const int par = a.parent[o + i];
+        const int par = par_[c];
         if (par < 0 || par >= i) {
           bad = true;
         } else {
-          const int tok = a.draft_tok[o + i];
+          const int tok = tok_[c];
           if (!kVerify || (a.gen_mask && !a.gen_mask[o + i])) {
             bad = tok != ld_i(am + o + par);               // reused code: greedy
           } else if (a.mode == EE_VERIFY_DIRECT) {
@@ -218,8 +236,6 @@ __device__ void accept_sequences(const AcceptArgs& a, const int32_t* am, const i
         }
       }
       notok[c] = __ballot_sync(0xffffffffu, bad);
-      a0[c] = i < T ? a.anc[2 * (size_t)(o + i)] : 0ull;
-      a1[c] = i < T ? a.anc[2 * (size_t)(o + i) + 1] : 0ull;
     }
     const uint64_t nz0 = (uint64_t)notok[0] | ((uint64_t)notok[1] << 32);
     const uint64_t nz1 = (uint64_t)notok[2] | ((uint64_t)notok[3] << 32);
@@ -227,7 +243,7 @@ __device__ void accept_sequences(const AcceptArgs& a, const int32_t* am, const i
     for (int c = 0; c < 4; ++c) {
       const int i = c * 32 + lane;
       if (i < T && (a0[c] & nz0) == 0 && (a1[c] & nz1) == 0) {
-        const int k = (a.depth[o + i] << 8) | (255 - i);
+        const int k = (dep_[c] << 8) | (255 - i);
         key_best = max(key_best, k);
       }
     }
@@ -235,7 +251,16 @@ __device__ void accept_sequences(const AcceptArgs& a, const int32_t* am, const i
     for (int d = 16; d >= 1; d >>= 1) key_best = max(key_best, __shfl_xor_sync(0xffffffffu, key_best, d));
     const int u = 255 - (key_best & 255);
     const int du = key_best >> 8;
-    const uint64_t w0 = a.anc[2 * (size_t)(o + u)], w1 = a.anc[2 * (size_t)(o + u) + 1];
+    uint64_t w0 = 0ull, w1 = 0ull;   // node u's ancestor mask, held by lane u % 32
+#pragma unroll
+    for (int c = 0; c < 4; ++c) {
+      const uint64_t x0 = __shfl_sync(0xffffffffu, a0[c], u & 31);
+      const uint64_t x1 = __shfl_sync(0xffffffffu, a1[c], u & 31);
+      if (c == (u >> 5)) {
+        w0 = x0;
+        w1 = x1;
+      }
+    }
     for (int j = lane; j < a.max_T; j += 32) a.path[(size_t)s * a.max_T + j] = -1;
     __syncwarp();
 #pragma unroll
@@ -305,6 +330,22 @@ lmhead_accept_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_const
     mbar_init(drain, 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    // the producer thread fills the ring's first stages now, before the set-up
+    // barrier (the ring is free and its barriers are initialised): the weight
+    // stream starts while the other warps allocate TMEM and clear their state
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmW)) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmX)) : "memory");
+    if ((int)blockIdx.x < p.n_vt * p.n_nt) {
+      const int vt = (int)blockIdx.x / p.n_nt, nt = (int)blockIdx.x % p.n_nt;
+      const int pre = min(S, p.nkb);
+      for (int kb = 0; kb < pre; ++kb) {
+        const uint32_t fb = full0 + 8 * kb;
+        mbar_expect_tx(fb, kABytes + bBytes);
+        tma_load_2d(smem_u32(sA + (size_t)kb * kABytes), &tmW, fb, kb * BK, vt * BM);
+        tma_load_2d(smem_u32(sB + (size_t)kb * bBytes), &tmX, fb, kb * BK, nt * BN);
+      }
+      s_issued = pre;
+    }
   }
   if (warp == 1) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
@@ -334,14 +375,14 @@ lmhead_accept_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_const
 
   if (warp == 0) {
     if (lane == 0) {
-      asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmW)) : "memory");
-      asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmX)) : "memory");
-      int stage = 0;
-      uint32_t phase = 0;
+      // the first min(S, nkb) stages of the first tile went out before the set-up barrier
+      const int pre = s_issued;
+      int stage = pre % S;
+      uint32_t phase = pre == S ? 1u : 0u;
       bool ok = true;
       for (int t = blockIdx.x; t < num_tiles && ok; t += gridDim.x) {
         const int vt = t / p.n_nt, nt = t % p.n_nt;
-        for (int kb = 0; kb < p.nkb; ++kb) {
+        for (int kb = (t == (int)blockIdx.x ? pre : 0); kb < p.nkb; ++kb) {
           if (!mbar_wait(empty0 + 8 * stage, phase ^ 1, &s_abort)) {
             ok = false;
             break;
@@ -621,7 +662,6 @@ lmhead_accept_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_const
         }
       }
     }
-    __threadfence();
   }
 
   // ---- teardown: drain on abort, free TMEM --------------------------------
@@ -650,15 +690,26 @@ lmhead_accept_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_const
   if (aborted) return;
 
   // ---- last CTA: argmax decode (+ greedy acceptance) -------------------------
+  // the CTA's key publications (before the teardown barrier) are released with
+  // its ticket; the last CTA's ticket acquires every other CTA's
   if (threadIdx.x == 0) {
-    __threadfence();
-    const unsigned int ticket = atomicAdd(p.ticket, 1u);
+    const unsigned int ticket = atom_add_acq_rel(p.ticket, 1u);
     s_last = (ticket == gridDim.x - 1) ? 1 : 0;
   }
   __syncthreads();
   if (!s_last) return;
   __threadfence();
   int32_t* s_am = reinterpret_cast<int32_t*>(smem);   // pipeline buffers are idle now
+  int32_t* s_off = s_am + p.total_nodes;              // the sequences' node offsets (greedy acceptance)
+  // the node offsets are loaded beside the key exchange (one round trip for both)
+  int offv[(EE_MAX_LM_NODES + 1 + kThreads - 1) / kThreads];
+  if constexpr (!kVerify) {
+#pragma unroll
+    for (int k = 0; k < (EE_MAX_LM_NODES + 1 + kThreads - 1) / kThreads; ++k) {
+      const int i = threadIdx.x + k * kThreads;
+      offv[k] = i <= p.B ? p.node_off[i] : 0;
+    }
+  }
   for (int i = threadIdx.x; i < p.total_nodes; i += kThreads) {
     const unsigned long long k = atomicExch(&p.keys[i], 0ull);
     const int a = k ? (int)(0xFFFFFFFFu - (uint32_t)(k & 0xFFFFFFFFull)) : -1;
@@ -666,11 +717,17 @@ lmhead_accept_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_const
     p.argmax[i] = a;
   }
   if (threadIdx.x == 0) *p.ticket = 0u;
-  if (kVerify) return;   // the finalize kernel ranks, decides top_tau and accepts
-  __syncthreads();
-  AcceptArgs aa{p.B, p.max_T, p.total_nodes, EE_VERIFY_GREEDY, 1, p.node_off, p.parent, p.draft_tok,
-                p.depth, p.anc, nullptr, p.accept_len, p.path, p.bonus, p.err};
-  accept_sequences<false>(aa, s_am, nullptr, nullptr, warp, lane, kThreads / 32);
+  if constexpr (!kVerify) {   // (verification: the finalize kernel ranks, decides top_tau and accepts)
+#pragma unroll
+    for (int k = 0; k < (EE_MAX_LM_NODES + 1 + kThreads - 1) / kThreads; ++k) {
+      const int i = threadIdx.x + k * kThreads;
+      if (i <= p.B) s_off[i] = offv[k];
+    }
+    __syncthreads();
+    AcceptArgs aa{p.B, p.max_T, p.total_nodes, EE_VERIFY_GREEDY, 1, s_off, p.parent, p.draft_tok,
+                  p.depth, p.anc, nullptr, p.accept_len, p.path, p.bonus, p.err};
+    accept_sequences<false>(aa, s_am, nullptr, nullptr, warp, lane, kThreads / 32);
+  }
 }
 
 
@@ -989,7 +1046,8 @@ ee_status launch_lmhead(const ee_bf16* hidden, const ee_bf16* lm_w, int32_t hidd
 
   const size_t smem = 1024 + (size_t)p.stages * stage_bytes + 8 * (2 * p.stages + 5) + 8 + epi;
   // the last CTA reuses the pipeline buffers: argmax (+ ranked ids and top_tau) per node
-  const size_t last = 1024 + (size_t)(EE_MAX_LM_NODES + 4) * 4;   // the last CTA: argmax per node
+  // the last CTA: argmax per node and the node offsets
+  const size_t last = 1024 + (size_t)(2 * EE_MAX_LM_NODES + 5) * 4;
   const size_t smem_acc = std::max(smem, last);
   if (smem_acc > 227 * 1024) return EE_ERR_UNSUPPORTED;
   {
