@@ -11,10 +11,12 @@
 // tail, and a block-wide exclusive scan of the per-thread hit counts orders
 // the hits.  With G = 1 the CTA writes the outputs directly; otherwise it writes
 // its count and first max_matches hits to a workspace record, and the CTA that
-// finishes last (a ticket counter: nobody waits) concatenates the records in
+// finishes last (a ticket counter taken with one acquire-release add after the
+// CTA barrier: nobody waits, no separate fences) concatenates the records in
 // range order.  Integer compares only; bound by reading c once (4 bytes per
 // position) and, for short codes, by launch latency.
 #include "ee_common.cuh"
+#include "ee_ptx.cuh"
 
 namespace {
 
@@ -178,18 +180,17 @@ match_reuse_kernel(const int32_t* __restrict__ tok, const int64_t* off, const in
     if (tid == 0) n_matches[b] = total;
     return;
   }
-  // publish this range's hits and count; the last of the sequence's CTAs merges
-  __threadfence();
+  // publish this range's hits and count; the last of the sequence's CTAs
+  // merges.  The ticket is one acquire-release add after the CTA barrier: it
+  // releases every thread's record stores and acquires the other CTAs'.
   __syncthreads();
   if (tid == 0) {
     rec[0] = total;
-    __threadfence();
     uint32_t* ticket = reinterpret_cast<uint32_t*>(mws + (size_t)b * match_seq_bytes(Gl, max_matches));
-    s_last = atomicAdd(ticket, 1u) == (uint32_t)(G - 1);
+    s_last = ee::atom_add_acq_rel(ticket, 1u) == (uint32_t)(G - 1);
   }
   __syncthreads();
   if (!s_last) return;
-  __threadfence();
   const uint8_t* recs = mws + (size_t)b * match_seq_bytes(Gl, max_matches) + 16;
   // warp 0: the records' counts and their exclusive prefix (range order)
   if (warp == 0) {
