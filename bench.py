@@ -69,7 +69,7 @@ TRAFFIC = {
     ("tree_verify_attn", "7b"): 9063168,          # profiles/attn_tc_7b.md
     ("tree_verify_attn", "33b"): 160700928,       # profiles/attn_tc_33b.md
     ("tree_verify_attn", "batched"): 247678720,   # profiles/attn_tc_batched.md
-    ("lmhead_accept", "7b"): 1095581184,          # profiles/lmhead_accept_7b.md
+    ("lmhead_accept", "7b"): 1095706368,          # profiles/lmhead_accept_7b.md
     ("lmhead_accept", "long"): 1108085248,        # profiles/lmhead_accept_long.md
     ("chain_verify_attn", "long"): 30021120,      # profiles/attn_chain_long.md
 }

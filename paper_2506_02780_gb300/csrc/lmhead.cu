@@ -925,10 +925,7 @@ __global__ void __launch_bounds__(32 * kFinWarps, 1) lm_verify_finalize_kernel(c
   }
   // the last CTA to finish: acceptance, then zero the thresholds for the next call
   __syncthreads();
-  if (threadIdx.x == 0) {
-    __threadfence();
-    s_last = atomicAdd(p.ticket, 1u) == gridDim.x - 1 ? 1 : 0;
-  }
+  if (threadIdx.x == 0) s_last = atom_add_acq_rel(p.ticket, 1u) == gridDim.x - 1 ? 1 : 0;   // releases the CTA's writes
   __syncthreads();
   if (!s_last) return;
   __threadfence();
