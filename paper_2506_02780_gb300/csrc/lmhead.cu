@@ -4,7 +4,8 @@
 //
 // Design (sm_103a, one persistent CTA per SM):
 //   - Swap-AB GEMM on the 5th-generation tensor cores: the vocabulary is the
-//     MMA M side (128 rows of W per tile), the tree nodes are the N side
+//     MMA M side (up to 128 rows of W per tile, as many tiles for every CTA:
+//     126 rows at V = 152064 on 152 SMs), the tree nodes are the N side
 //     (BN = 16..256 columns), K = hidden in 64-element (128-byte) blocks.
 //     D[vocab_row][node] accumulates in fp32 in TMEM, never in registers and
 //     never in HBM (unless the caller asks for the logits).
@@ -59,6 +60,7 @@ constexpr int kABytes = BM * BK * 2;
 struct LmParams {
   int vocab, hidden, total_nodes, B, max_T;
   int BN, n_nt, n_vt, nkb, stages, tmem_cols;
+  int BMr;                    // vocabulary rows per tile (<= BM; the MMA's other rows are not used)
   const int32_t* draft_tok;
   const int32_t* parent;
   const int32_t* depth;
@@ -292,6 +294,7 @@ lmhead_accept_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_const
   ee::pdl_wait();   // no global access before the previous kernel's writes are visible
   const int S = p.stages, BN = p.BN;
   const uint32_t bBytes = (uint32_t)BN * BK * 2;
+  const uint32_t aBytes = (uint32_t)p.BMr * BK * 2;   // W rows a stage receives
   uint8_t* sA = smem;
   uint8_t* sB = smem + (size_t)S * kABytes;
   uint8_t* tail = sB + (size_t)S * bBytes;
@@ -340,8 +343,8 @@ lmhead_accept_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_const
       const int pre = min(S, p.nkb);
       for (int kb = 0; kb < pre; ++kb) {
         const uint32_t fb = full0 + 8 * kb;
-        mbar_expect_tx(fb, kABytes + bBytes);
-        tma_load_2d(smem_u32(sA + (size_t)kb * kABytes), &tmW, fb, kb * BK, vt * BM);
+        mbar_expect_tx(fb, aBytes + bBytes);
+        tma_load_2d(smem_u32(sA + (size_t)kb * kABytes), &tmW, fb, kb * BK, vt * p.BMr);
         tma_load_2d(smem_u32(sB + (size_t)kb * bBytes), &tmX, fb, kb * BK, nt * BN);
       }
       s_issued = pre;
@@ -388,8 +391,8 @@ lmhead_accept_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_const
             break;
           }
           const uint32_t fb = full0 + 8 * stage;
-          mbar_expect_tx(fb, kABytes + bBytes);
-          tma_load_2d(smem_u32(sA + (size_t)stage * kABytes), &tmW, fb, kb * BK, vt * BM);
+          mbar_expect_tx(fb, aBytes + bBytes);
+          tma_load_2d(smem_u32(sA + (size_t)stage * kABytes), &tmW, fb, kb * BK, vt * p.BMr);
           tma_load_2d(smem_u32(sB + (size_t)stage * bBytes), &tmX, fb, kb * BK, nt * BN);
           ++s_issued;
           if (++stage == S) {
@@ -454,8 +457,8 @@ lmhead_accept_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_const
         for (int c = threadIdx.x - 64; c < BN; c += kEpiThreads)
           if (nt * BN + c < p.total_nodes) atomicMax(&s_thr[c], __ldcg(p.gthr + nt * BN + c));
       }
-      const int row = vt * BM + q * 32 + lane;
-      const bool row_ok = row < p.vocab;
+      const int row = vt * p.BMr + q * 32 + lane;
+      const bool row_ok = q * 32 + lane < p.BMr && row < p.vocab;
       for (int c0 = 16 * half; c0 < BN; c0 += 32) {
         uint32_t r[16];
         tc_ld16(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN + c0), r);
@@ -537,7 +540,7 @@ lmhead_accept_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_const
           //     CTA's shared threshold; up to four candidates are inserted into
           //     the warp's sorted list by lane 0, more re-select the K best of
           //     list + candidates with K rounds of a warp argmax
-          const int row0 = vt * BM + q * 32;
+          const int row0 = vt * p.BMr + q * 32;
 #pragma unroll
           for (int j = 0; j < 16; ++j) {
             float* lv = s_lv + (size_t)(ew * BN + c0 + j) * K;
@@ -1000,7 +1003,18 @@ ee_status launch_lmhead(const ee_bf16* hidden, const ee_bf16* lm_w, int32_t hidd
   p.max_T = max_T;
   p.n_nt = (total_nodes + 255) / 256;
   p.BN = ((total_nodes + p.n_nt - 1) / p.n_nt + 15) / 16 * 16;
-  p.n_vt = (vocab + BM - 1) / BM;
+  // vocabulary tiles: as many per CTA for every CTA (the launch's end is the
+  // busiest CTA's), each of ceil(V / tiles) <= 128 rows; the MMA's remaining
+  // rows hold stale shared memory and are dropped by the epilogue.  Below 64
+  // rows a tile would waste most of its MMA: plain 128-row tiles then.
+  {
+    const int n_vt0 = (vocab + BM - 1) / BM;
+    const int per_group = std::max(1, ee::kNumSMs / p.n_nt);   // CTAs per node tile
+    const int k = (n_vt0 + per_group - 1) / per_group;
+    const int rows = (vocab + k * per_group - 1) / (k * per_group);
+    p.BMr = rows >= 64 ? rows : BM;
+    p.n_vt = (vocab + p.BMr - 1) / p.BMr;
+  }
   p.nkb = (hidden_dim + BK - 1) / BK;
   const size_t stage_bytes = (size_t)kABytes + (size_t)p.BN * BK * 2;
   const int K = va ? va->k : 1;
@@ -1037,7 +1051,7 @@ ee_status launch_lmhead(const ee_bf16* hidden, const ee_bf16* lm_w, int32_t hidd
   p.gthr = va ? reinterpret_cast<unsigned long long*>(va->part + ee::kLmGthrOff) : nullptr;
 
   CUtensorMap tmW, tmX;
-  if (!encode_2d(&tmW, lm_w, (uint64_t)hidden_dim, (uint64_t)vocab, BK, BM)) return EE_ERR_CUDA;
+  if (!encode_2d(&tmW, lm_w, (uint64_t)hidden_dim, (uint64_t)vocab, BK, (uint32_t)p.BMr)) return EE_ERR_CUDA;
   if (!encode_2d(&tmX, hidden, (uint64_t)hidden_dim, (uint64_t)total_nodes, BK, p.BN))
     return EE_ERR_CUDA;
 
