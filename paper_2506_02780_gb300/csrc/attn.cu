@@ -57,10 +57,12 @@
 //         barrier (release / acquire at cluster scope);
 //       cooperative: the launch is cooperative (every CTA resident at once);
 //         the row block's 64-bit count grows by 720720 = lcm(1..16) per
-//         launch: each of its S CTAs reads the count (a multiple of 720720)
-//         before arriving, stores its partial, and after a CTA barrier one
-//         thread adds 720720 / S with a release reduction and waits (acquire)
-//         for the next multiple.  One release per CTA orders all its threads'
+//         launch: each of its S CTAs reads the count at its start (a
+//         multiple of 720720 plus some of this launch's arrivals, never all:
+//         its own is missing; a relaxed load whose value is first used at the
+//         end), stores its partial, and after a CTA barrier one thread adds
+//         720720 / S with a release reduction and waits (acquire) for the next
+//         multiple.  One release per CTA orders all its threads'
 //         stores, and nothing resets the count at the end of the kernel.  No
 //         GPC packing constraint: S can be any value up to 16, so the grid can
 //         cover every SM.  Balanced launches count the pieces of each split
@@ -233,9 +235,10 @@ struct BalPiece {
 };
 // A split row block's pieces meet at a 64-bit count in the trailer of its first
 // partial slot: every launch raises it by kCountGen in all (kCountGen / K per
-// piece, a release reduction after the piece's partial is stored), so a piece
-// reads a multiple of kCountGen at any time before its own arrival and waits
-// (acquire) for the next multiple.  The count is never reset; ee_workspace_init
+// piece, a release reduction after the piece's partial is stored), so a count a
+// piece reads at any time before its own arrival is a multiple of kCountGen
+// plus fewer than K arrivals, and the piece waits (acquire) for the next
+// multiple.  The count is never reset; ee_workspace_init
 // zeroes it.
 constexpr unsigned long long kCountGen = 720720;   // lcm(1..16): K <= 16 divides it
 
@@ -445,7 +448,9 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
   // offset and rows for the merge
   const int split = kBal ? 0 : (int)(blockIdx.x % p.S);   // == cluster rank in the cluster mode
   int u_o = 0, u_R = 0;
-  unsigned long long u_target = 0;   // uniform cooperative mode: the row block's count target
+  // uniform cooperative mode, thread 0: the row block's count as read at the
+  // start (the target is the next multiple of kCountGen)
+  unsigned long long u_target = 0;
 
   for (;;) {
     // ---------------- the next segment of this CTA's work ----------------
@@ -565,6 +570,14 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
       b = blockIdx.z;
       hk = blockIdx.y;
       rb = blockIdx.x / p.S;                     // the S chunks of a row block are consecutive
+      // the row block's count, read now beside the node range (any time before
+      // this CTA's own arrival will do: it is a multiple of kCountGen plus the
+      // arrivals of this launch so far, never all of them)
+      if (p.coop && p.S > 1 && threadIdx.x == 0) {
+        const size_t cta0 = ((size_t)blockIdx.z * gridDim.y + blockIdx.y) * gridDim.x + (size_t)rb * p.S;
+        u_target = ld_relaxed64(
+            reinterpret_cast<const unsigned long long*>(p.part + cta0 * kAttnPartBytes + kAttnCntOff));
+      }
       // this chunk's page ids, issued now beside the sequence's node range and
       // context length so that the round trips overlap (validated below)
       const int pg_first = split * (p.chunk / EE_PAGE);
@@ -600,13 +613,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
       slot = ((size_t)blockIdx.z * gridDim.y + blockIdx.y) * gridDim.x + blockIdx.x;
       u_o = o;
       u_R = T * g;
-      if (p.coop && p.S > 1 && threadIdx.x == 0) {
-        // read now (before this CTA's own arrival): a multiple of kCountGen
-        const size_t cta0 = ((size_t)blockIdx.z * gridDim.y + blockIdx.y) * gridDim.x + (size_t)rb * p.S;
-        const unsigned long long c = ld_acquire64(
-            reinterpret_cast<const unsigned long long*>(p.part + cta0 * kAttnPartBytes + kAttnCntOff));
-        u_target = (c / kCountGen + 1) * kCountGen;
-      }
+
     }
     const int R = T * g;
     const int n_ctx_tiles = k_end > k_begin ? (k_end - k_begin + kKT - 1) / kKT : 0;
@@ -1089,7 +1096,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
       if (threadIdx.x == 0) {
         // this CTA's partial (every thread's stores precede the teardown barrier)
         red_add_release64(cnt, kCountGen / (unsigned)p.S);
-        const bool ready = wait_count64_geq(cnt, u_target);
+        const bool ready = wait_count64_geq(cnt, (u_target / kCountGen + 1) * kCountGen);
         if (!ready) flag_error(p.err, EE_DEVERR_TIMEOUT);
         s_ready[0] = ready;
       }

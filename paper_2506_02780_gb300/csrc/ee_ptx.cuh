@@ -259,6 +259,11 @@ __device__ __forceinline__ unsigned int atom_add_acq_rel(unsigned int* a, unsign
   asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], %2;" : "=r"(old) : "l"(a), "r"(v) : "memory");
   return old;
 }
+__device__ __forceinline__ unsigned long long ld_relaxed64(const unsigned long long* a) {
+  unsigned long long v;
+  asm volatile("ld.relaxed.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(a) : "memory");
+  return v;
+}
 __device__ __forceinline__ unsigned long long ld_acquire64(const unsigned long long* a) {
   unsigned long long v;
   asm volatile("ld.acquire.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(a) : "memory");
