@@ -158,3 +158,31 @@ def test_verify_7b_shapes():
     for k in (3, 5):
         r = _run(w, "entropy", k)
         _check(w, r, "entropy", k)
+
+
+@pytest.mark.parametrize("vocab", [30000, 152064 // 8 * 3])
+def test_vocab_tiles_drop_the_rows_of_the_next_tile(vocab):
+    """Every CTA takes as many vocabulary tiles; a tile of r < 128 rows still
+    runs a 128-row MMA whose last 128 - r rows are the next tile's first rows
+    and must be dropped.  The best and second-best rows of node 0 are planted
+    at first rows of tiles (each also inside the previous tile's MMA): argmax,
+    the top-k list (no id twice) and the acceptance agree with the oracle."""
+    w = W.build("tiny", seed=71, device="cuda", verify_plant=True, trees=[TREE], vocab=vocab)
+    per_group, n_vt0 = 152, (vocab + 127) // 128
+    k_tiles = (n_vt0 + per_group - 1) // per_group
+    rows = (vocab + k_tiles * per_group - 1) // (k_tiles * per_group)
+    assert 64 <= rows < 128, rows                     # the launch uses rows-high tiles
+    top, second = 5 * rows, 9 * rows
+    h0 = w.hidden_states[0].float()
+    w.lm_w[top] = (h0 / h0.norm() * 64.0).to(torch.bfloat16)
+    w.lm_w[second] = (h0 / h0.norm() * 48.0).to(torch.bfloat16)
+    for mode, k in (("topk", 4), ("entropy", 3)):
+        r = _run(w, mode, k)
+        assert r["argmax"][0] == top
+        assert list(r["topk"][0][:2]) == [top, second]
+        for a in range(w.total_nodes):
+            assert len(set(r["topk"][a].tolist())) == k, a
+        _check(w, r, mode, k)
+    g = _run(w, "greedy", 1, verify=False)            # ee_lmhead_accept
+    assert g["argmax"][0] == top
+    np.testing.assert_array_equal(g["argmax"], _run(w, "greedy", 1)["argmax"])
