@@ -623,6 +623,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
     // half-warp reads one 256-byte row; rows past R read row R - 1 and are
     // zeroed later) so that they leave before the K/V stream starts; the values
     // are consumed after the barrier below
+    bool pages_ok = true;
     uint4 qv[kRows / 16];
     if (warp >= kWarpSoft0) {
 #pragma unroll
@@ -647,11 +648,13 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
           const bool ok = pg >= 0 && pg < p.num_pages;
           if (!ok) flag_error(p.err, EE_DEVERR_PAGE);
           s_pages[i] = ok ? pg : -1;
+          pages_ok &= ok;
         }
       }
     }
     tc_fence_before();
-    __syncthreads();
+    // every page of the segment valid: whole context tiles need no mask
+    const bool seg_pages_ok = __syncthreads_and(pages_ok) != 0;
     tc_fence_after();
     tmem = s_tmem;
     // every thread has read the schedule position: advance it for the next segment
@@ -815,7 +818,9 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmKc, const __grid_constant__
           // visibility of this half's 64 keys as one 64-bit word
           uint64_t kw;
           const int i = tg + d < n_tiles ? tg + d : tg + d - n_tiles;
-          if (i < n_ctx_tiles) {
+          if (seg_pages_ok && k_begin + (i + 1) * kKT <= (kIP ? min(k_end, ctx) : k_end)) {
+            kw = ~0ull;   // a whole tile of context keys in valid pages: every row sees all of it
+          } else if (i < n_ctx_tiles) {
             const unsigned m = tile_mask(s_pages, i, k_begin, k_end);
             const int nv = min(max(k_end - (k_begin + i * kKT) - 64 * hf, 0), 64);
             uint64_t pgw = 0ull;
