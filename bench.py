@@ -134,24 +134,44 @@ def algorithmic(w):
 # ----------------------------------------------------------------------------
 
 class ClockSampler:
-    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+    """nvidia-smi samples of the SM clock and the throttle reasons every 20 ms,
+    each with its timestamp.  start() returns once the first sample is in (so
+    sampling is live before the region begins), mark_begin()/mark_end()
+    bracket the timed region on the host clock, and stop() summarises the
+    samples taken inside it (see summarize_clock_rows)."""
+    FIELDS = ("timestamp,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
               "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+    PERIOD_MS = 20
 
     def __init__(self, index):
         self.index = index
         self.proc = None
         self.file = None
+        self.t_begin = None
+        self.t_end = None
 
-    def start(self):
+    def start(self, wait_s=3.0):
         try:
             self.file = tempfile.NamedTemporaryFile("w+", delete=False, suffix=".csv")
             self.proc = subprocess.Popen(
                 ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}",
-                 "--format=csv,noheader,nounits", "-lms", "100"],
+                 "--format=csv,noheader,nounits", "-lms", str(self.PERIOD_MS)],
                 stdout=self.file, stderr=subprocess.DEVNULL)
         except (OSError, FileNotFoundError):
             self.proc = None
+            return
+        t0 = time.time()
+        while time.time() - t0 < wait_s and self.proc.poll() is None:
+            if os.path.getsize(self.file.name) > 0:
+                break
+            time.sleep(0.01)
+
+    def mark_begin(self):
+        self.t_begin = time.time()
+
+    def mark_end(self):
+        self.t_end = time.time()
 
     def stop(self):
         if self.proc is None:
@@ -166,21 +186,52 @@ class ClockSampler:
         rows = [r.split(",") for r in self.file.read().strip().splitlines() if r.strip()]
         self.file.close()
         os.unlink(self.file.name)
-        sm, mx, reasons = [], 0.0, set()
-        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        for r in rows:
-            try:
-                sm.append(float(r[0]))
-                mx = max(mx, float(r[1]))
-                for nm, v in zip(names, r[4:8]):
-                    if v.strip().lower() == "active":
-                        reasons.add(nm)
-            except (ValueError, IndexError):
-                continue
-        if not sm:
+        return summarize_clock_rows(rows, self.t_begin, self.t_end)
+
+
+def _clock_row_time(stamp):
+    """nvidia-smi's timestamp ("YYYY/MM/DD HH:MM:SS.mmm", local time) in seconds
+    since the epoch, or None."""
+    import datetime
+    try:
+        return datetime.datetime.strptime(stamp.strip(), "%Y/%m/%d %H:%M:%S.%f").timestamp()
+    except ValueError:
+        return None
+
+
+def summarize_clock_rows(rows, t_begin=None, t_end=None):
+    """Median SM clock, maximum clock, active throttle reasons and sample count
+    of the rows taken inside [t_begin, t_end] (host clock).  A region shorter
+    than the sampling period may hold none: then the nearest sample before and
+    the nearest after it stand in (``samples`` counts the rows used,
+    ``samples_in_region`` those inside).  Without marks every row counts."""
+    names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+    parsed = []
+    for r in rows:
+        try:
+            parsed.append((_clock_row_time(r[0]), float(r[1]), float(r[2]),
+                           {nm for nm, v in zip(names, r[5:9]) if v.strip().lower() == "active"}))
+        except (ValueError, IndexError):
+            continue
+    if not parsed:
+        return None
+    use, inside = parsed, None
+    if t_begin is not None and t_end is not None and all(p[0] is not None for p in parsed):
+        inside = [p for p in parsed if t_begin <= p[0] <= t_end]
+        use = inside
+        if not inside:
+            before = [p for p in parsed if p[0] < t_begin]
+            after = [p for p in parsed if p[0] > t_end]
+            use = ([max(before, key=lambda p: p[0])] if before else []) + \
+                  ([min(after, key=lambda p: p[0])] if after else [])
+        if not use:
             return None
-        return {"sm_mhz": float(np.median(sm)), "sm_max_mhz": mx, "reasons": sorted(reasons),
-                "samples": len(sm)}
+    out = {"sm_mhz": float(np.median([p[1] for p in use])), "sm_max_mhz": max(p[2] for p in use),
+           "reasons": sorted(set().union(*(p[3] for p in use))), "samples": len(use)}
+    if inside is not None:
+        out["samples_in_region"] = len(inside)
+        out["region_ms"] = round(1e3 * (t_end - t_begin), 2)
+    return out
 
 
 BAD_CLOCK_REASONS = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown")
@@ -566,8 +617,10 @@ def run_ours(args, rank, world, local_rank):
     if not args.no_clocks:
         clocks.start()
     torch.cuda.synchronize(dev)
+    clocks.mark_begin()
     ms_step = timed(plain, args.steps)
     torch.cuda.synchronize(dev)
+    clocks.mark_end()
     ms_step = reduce_max(ms_step, world, dev)
     ms_step_instr = timed(graphs, max(1, args.steps // 2), harvest) if phase_events else None
     torch.cuda.synchronize(dev)
@@ -583,8 +636,11 @@ def run_ours(args, rank, world, local_rank):
         clocks = ClockSampler(dev.index)
         clocks.start()
         torch.cuda.synchronize(dev)
-        ms_step = reduce_max(timed(plain, args.steps), world, dev)
+        clocks.mark_begin()
+        ms_step = timed(plain, args.steps)
         torch.cuda.synchronize(dev)
+        clocks.mark_end()
+        ms_step = reduce_max(ms_step, world, dev)
         if world > 1:
             torch.distributed.barrier()
         clk = clocks.stop() or {}
@@ -785,8 +841,10 @@ def time_config(name, args, rank, dev, stream, steps):
     if not args.no_clocks:
         clocks.start()
     torch.cuda.synchronize(dev)
+    clocks.mark_begin()
     ms = timed(plain, steps)
     torch.cuda.synchronize(dev)
+    clocks.mark_end()
     clk = None if args.no_clocks else clocks.stop()
     acc = np.zeros(2)
     n = max(2, steps // 4)

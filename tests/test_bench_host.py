@@ -70,15 +70,52 @@ def test_clock_record_rejects_slowdowns_and_stuck_clocks(clk, why):
 def test_clock_sampler_parses_nvidia_smi_rows():
     s = bench.ClockSampler(0)
     s.file = tempfile.NamedTemporaryFile("w+", delete=False, suffix=".csv")
-    s.file.write("2070, 2070, 812.4, 0x0000000000000000, Not Active, Not Active, Not Active, Not Active\n"
-                 "2070, 2070, 1190.0, 0x0000000000000004, Not Active, Not Active, Not Active, Active\n"
-                 "1980, 2070, 1375.2, 0x0000000000000004, Not Active, Not Active, Not Active, Active\n"
-                 "[N/A], 2070, [N/A], [N/A], [N/A], [N/A], [N/A], [N/A]\n")
+    s.file.write("2026/12/02 15:20:45.100, 2070, 2070, 812.4, 0x0000000000000000, Not Active, Not Active, Not Active, Not Active\n"
+                 "2026/12/02 15:20:45.120, 2070, 2070, 1190.0, 0x0000000000000004, Not Active, Not Active, Not Active, Active\n"
+                 "2026/12/02 15:20:45.140, 1980, 2070, 1375.2, 0x0000000000000004, Not Active, Not Active, Not Active, Active\n"
+                 "2026/12/02 15:20:45.160, [N/A], 2070, [N/A], [N/A], [N/A], [N/A], [N/A], [N/A]\n")
     s.proc = subprocess.Popen(["sleep", "30"])
-    clk = s.stop()
+    clk = s.stop()                                   # no region marks: every row counts
     assert clk["samples"] == 3 and clk["sm_mhz"] == 2070.0 and clk["sm_max_mhz"] == 2070.0
     assert clk["reasons"] == ["sw_power_cap"]
     assert bench.clocks_rejected(clk) is None
+
+
+def _rows(*spec):
+    """nvidia-smi rows at the given local times (seconds after 15:20:45) with the given SM clock and
+    hw_slowdown state."""
+    out = []
+    for t, mhz, slow in spec:
+        ms = int(round(t * 1000))
+        stamp = f"2026/12/02 15:20:{45 + ms // 1000:02d}.{ms % 1000:03d}"
+        out.append([stamp, str(mhz), "2070", "900", "0x0", "Active" if slow else "Not Active",
+                    "Not Active", "Not Active", "Not Active"])
+    return out
+
+
+def _t(sec):
+    import datetime
+    return datetime.datetime(2026, 12, 2, 15, 20, 45).timestamp() + sec
+
+
+def test_clock_record_keeps_only_samples_inside_the_timed_region():
+    """Samples before and after the timed region (here a slowdown during a
+    later, untimed pass) do not count."""
+    rows = _rows((0.00, 1500, False), (0.02, 2070, False), (0.04, 2070, False), (0.06, 2070, False),
+                 (0.08, 1200, True))
+    clk = bench.summarize_clock_rows(rows, _t(0.015), _t(0.065))
+    assert clk["samples"] == 3 and clk["samples_in_region"] == 3 and clk["sm_mhz"] == 2070.0
+    assert clk["reasons"] == [] and bench.clocks_rejected(clk) is None
+    assert clk["region_ms"] == 50.0
+
+
+def test_clock_record_of_a_region_shorter_than_the_sampling_period():
+    """A 12 ms region between two 20 ms samples: the nearest sample on each
+    side stands in, and the record says that none fell inside."""
+    rows = _rows((0.00, 1500, False), (0.02, 2070, False), (0.04, 2070, True), (0.06, 2070, False))
+    clk = bench.summarize_clock_rows(rows, _t(0.025), _t(0.037))
+    assert clk["samples_in_region"] == 0 and clk["samples"] == 2
+    assert clk["reasons"] == ["hw_slowdown"] and bench.clocks_rejected(clk) == "hw_slowdown"
 
 
 def test_clock_sampler_without_nvidia_smi_reports_nothing():
