@@ -22,6 +22,9 @@
  *   ee_chain_verify_attn causal attention of linear drafts of up to 2048
  *                        tokens verified in place (long reuse drafts; the LM
  *                        head takes them with anc NULL)
+ *   ee_lmhead_pack_weights / ee_lmhead_accept_packed
+ *                        the LM-head weights rearranged once into the
+ *                        kernel's tile order, and the LM head reading them
  *
  * Conventions shared by every entry point
  * ---------------------------------------
@@ -375,6 +378,40 @@ ee_status ee_lmhead_accept_static(const ee_bf16* hidden, const ee_bf16* lm_w, in
                                   int32_t B, int32_t total_nodes, int32_t max_T, int32_t* argmax,
                                   int32_t* accept_len, int32_t* path, int32_t* bonus,
                                   float* logits_or_null, ee_stream_t stream);
+
+/*
+ * ee_lmhead_pack_weights -- rearrange the LM-head weights once (at model load:
+ * a deployment layout, the paper has no counterpart) into the order the LM
+ * head streams them: W is cut into blocks of 128 vocabulary rows x 64 hidden
+ * columns, block (vt, kb) = rows 128 vt .. 128 vt + 127, columns 64 kb ..
+ * 64 kb + 63, stored row-major as one contiguous 16 KB run at element offset
+ * (vt * ceil(hidden_dim / 64) + kb) * 8192; rows past vocab and columns past
+ * hidden_dim are zero.  The LM head then reads whole 16 KB runs instead of
+ * 128-byte pieces 2 * hidden_dim bytes apart (measured: the 7B-shaped LM head
+ * 168 -> 161 us on one GB300).
+ *   lm_w   bf16 [vocab][hidden_dim] row-major, in
+ *   packed bf16, ee_lmhead_packed_bytes(vocab, hidden_dim) bytes, out
+ * hidden_dim a multiple of 8; both arrays 16-byte aligned; packed_bytes at
+ * least ee_lmhead_packed_bytes(...).  One kernel launch on `stream`.
+ * ee_lmhead_packed_bytes returns 0 for sizes the packing does not take.
+ */
+size_t ee_lmhead_packed_bytes(int32_t vocab, int32_t hidden_dim);
+ee_status ee_lmhead_pack_weights(const ee_bf16* lm_w, int32_t vocab, int32_t hidden_dim, ee_bf16* packed,
+                                 size_t packed_bytes, ee_stream_t stream);
+
+/*
+ * ee_lmhead_accept_packed -- ee_lmhead_accept (same arguments, results and
+ * errors) with the weights in the layout ee_lmhead_pack_weights writes:
+ * lm_w_packed is that array for the same vocab and hidden_dim.  The products
+ * are the same sums in the same order: argmax, path, accept_len, bonus and the
+ * optional logits are bit-identical to ee_lmhead_accept's.
+ */
+ee_status ee_lmhead_accept_packed(const ee_bf16* hidden, const ee_bf16* lm_w_packed, int32_t hidden_dim,
+                                  int32_t vocab, const int32_t* draft_tok, const int32_t* parent,
+                                  const int32_t* depth, const uint64_t* anc, const int32_t* node_off,
+                                  int32_t B, int32_t total_nodes, int32_t max_T, int32_t* argmax,
+                                  int32_t* accept_len, int32_t* path, int32_t* bonus,
+                                  float* logits_or_null, void* ws, size_t ws_bytes, ee_stream_t stream);
 
 /*
  * ee_kv_compact -- append the accepted path's K/V to the paged cache, every

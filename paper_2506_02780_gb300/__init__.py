@@ -33,7 +33,8 @@ EXPORTS = ("ee_version", "ee_status_string", "ee_workspace_size", "ee_workspace_
            "ee_read_errors", "ee_match_reuse", "ee_tree_prepare", "ee_tree_verify_attn", "ee_attn_plan",
            "ee_lmhead_accept", "ee_lmhead_verify", "ee_lmhead_accept_static", "ee_kv_compact",
            "ee_selftest_timeout", "ee_tree_verify_attn_inplace", "ee_kv_compact_inplace",
-           "ee_chain_verify_attn", "ee_build_reuse_tree", "ee_advance")
+           "ee_chain_verify_attn", "ee_build_reuse_tree", "ee_advance", "ee_lmhead_packed_bytes",
+           "ee_lmhead_pack_weights", "ee_lmhead_accept_packed")
 
 VERIFY_MODES = {"greedy": 0, "direct": 1, "topk": 2, "entropy": 3}
 
@@ -81,6 +82,10 @@ _SIGS = {
     "ee_lmhead_verify": ([_P, _P, _I, _I, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _P, _P, _P, _P, _P,
                           _P, _P, _P, _P, _SZ, _P], _I),
     "ee_lmhead_accept_static": ([_P, _P, _I, _I, _P, _P, _P, _P, _P, _I, _I, _I, _P, _P, _P, _P, _P,
+                                 _P], _I),
+    "ee_lmhead_packed_bytes": ([_I, _I], _SZ),
+    "ee_lmhead_pack_weights": ([_P, _I, _I, _P, _SZ, _P], _I),
+    "ee_lmhead_accept_packed": ([_P, _P, _I, _I, _P, _P, _P, _P, _P, _I, _I, _I, _P, _P, _P, _P, _P, _P, _SZ,
                                  _P], _I),
     "ee_kv_compact": ([_P, _P, _I64, _P, _P, _I64, _I, _I, _P, _I, _P, _P, _P, _P, _P, _I, _I, _I, _I,
                        _P, _P, _SZ, _P], _I),
@@ -257,6 +262,36 @@ def ee_lmhead_accept(hidden, lm_w, draft_tok, parent, depth, anc, node_off, max_
                                 _p(anc), _p(node_off), B, total, max_T, _p(argmax), _p(accept_len),
                                 _p(path), _p(bonus), _p(logits), _p(ws), ws.numel(), _stream(stream))
     _ok("ee_lmhead_accept", st)
+
+
+def ee_lmhead_packed_bytes(vocab, hidden_dim):
+    """Bytes of the tile-ordered LM-head weights for these sizes (0: not supported)."""
+    return int(lib().ee_lmhead_packed_bytes(int(vocab), int(hidden_dim)))
+
+
+def ee_lmhead_pack_weights(lm_w, packed, stream=None):
+    """Write `lm_w` ([vocab][hidden] bf16) into `packed` (a bf16 tensor of at least
+    ee_lmhead_packed_bytes(vocab, hidden) bytes) in the LM head's tile order."""
+    _check(lm_w, torch.bfloat16, "lm_w")
+    _check(packed, torch.bfloat16, "packed")
+    V, H = lm_w.shape
+    st = lib().ee_lmhead_pack_weights(_p(lm_w), V, H, _p(packed), packed.numel() * 2, _stream(stream))
+    _ok("ee_lmhead_pack_weights", st)
+
+
+def ee_lmhead_accept_packed(hidden, lm_w_packed, vocab, draft_tok, parent, depth, anc, node_off, max_T, argmax,
+                            accept_len, path, bonus, ws, logits=None, stream=None):
+    """ee_lmhead_accept with the weights packed by ee_lmhead_pack_weights (the
+    vocabulary size is an argument: the packed array is padded)."""
+    _check(hidden, torch.bfloat16, "hidden")
+    _check(lm_w_packed, torch.bfloat16, "lm_w_packed")
+    total, H = hidden.shape
+    B = node_off.numel() - 1
+    st = lib().ee_lmhead_accept_packed(_p(hidden), _p(lm_w_packed), H, int(vocab), _p(draft_tok), _p(parent),
+                                       _p(depth), _p(anc), _p(node_off), B, total, max_T, _p(argmax),
+                                       _p(accept_len), _p(path), _p(bonus), _p(logits), _p(ws), ws.numel(),
+                                       _stream(stream))
+    _ok("ee_lmhead_accept_packed", st)
 
 
 def ee_lmhead_verify(hidden, lm_w, draft_tok, parent, depth, anc, node_off, max_T, mode, k, argmax,

@@ -61,6 +61,7 @@ struct LmParams {
   int vocab, hidden, total_nodes, B, max_T;
   int BN, n_nt, n_vt, nkb, stages, tmem_cols;
   int BMr;                    // vocabulary rows per tile (<= BM; the MMA's other rows are not used)
+  int packed;                 // W in tile order ([V/128][H/64][128][64], ee_lmhead_pack_weights): BMr = BM
   const int32_t* draft_tok;
   const int32_t* parent;
   const int32_t* depth;
@@ -344,7 +345,10 @@ lmhead_accept_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_const
       for (int kb = 0; kb < pre; ++kb) {
         const uint32_t fb = full0 + 8 * kb;
         mbar_expect_tx(fb, aBytes + bBytes);
-        tma_load_2d(smem_u32(sA + (size_t)kb * kABytes), &tmW, fb, kb * BK, vt * p.BMr);
+        if (p.packed)
+          tma_load_2d(smem_u32(sA + (size_t)kb * kABytes), &tmW, fb, 0, (vt * p.nkb + kb) * BM);
+        else
+          tma_load_2d(smem_u32(sA + (size_t)kb * kABytes), &tmW, fb, kb * BK, vt * p.BMr);
         tma_load_2d(smem_u32(sB + (size_t)kb * bBytes), &tmX, fb, kb * BK, nt * BN);
       }
       s_issued = pre;
@@ -392,7 +396,10 @@ lmhead_accept_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_const
           }
           const uint32_t fb = full0 + 8 * stage;
           mbar_expect_tx(fb, aBytes + bBytes);
-          tma_load_2d(smem_u32(sA + (size_t)stage * kABytes), &tmW, fb, kb * BK, vt * p.BMr);
+          if (p.packed)   // one contiguous 16 KB block of W
+            tma_load_2d(smem_u32(sA + (size_t)stage * kABytes), &tmW, fb, 0, (vt * p.nkb + kb) * BM);
+          else
+            tma_load_2d(smem_u32(sA + (size_t)stage * kABytes), &tmW, fb, kb * BK, vt * p.BMr);
           tma_load_2d(smem_u32(sB + (size_t)stage * bBytes), &tmX, fb, kb * BK, nt * BN);
           ++s_issued;
           if (++stage == S) {
@@ -994,8 +1001,9 @@ ee_status launch_lmhead(const ee_bf16* hidden, const ee_bf16* lm_w, int32_t hidd
                         int32_t total_nodes, int32_t max_T, int32_t* argmax, int32_t* accept_len,
                         int32_t* path, int32_t* bonus, float* logits_or_null,
                         unsigned long long* keys, unsigned int* ticket, int32_t* err,
-                        ee_stream_t stream, bool pdl, const VerifyArgs* va = nullptr) {
+                        ee_stream_t stream, bool pdl, const VerifyArgs* va = nullptr, bool packed = false) {
   LmParams p;
+  p.packed = packed ? 1 : 0;
   p.vocab = vocab;
   p.hidden = hidden_dim;
   p.total_nodes = total_nodes;
@@ -1012,7 +1020,7 @@ ee_status launch_lmhead(const ee_bf16* hidden, const ee_bf16* lm_w, int32_t hidd
     const int per_group = std::max(1, ee::kNumSMs / p.n_nt);   // CTAs per node tile
     const int k = (n_vt0 + per_group - 1) / per_group;
     const int rows = (vocab + k * per_group - 1) / (k * per_group);
-    p.BMr = rows >= 64 ? rows : BM;
+    p.BMr = rows >= 64 && !packed ? rows : BM;
     p.n_vt = (vocab + p.BMr - 1) / p.BMr;
   }
   p.nkb = (hidden_dim + BK - 1) / BK;
@@ -1051,7 +1059,12 @@ ee_status launch_lmhead(const ee_bf16* hidden, const ee_bf16* lm_w, int32_t hidd
   p.gthr = va ? reinterpret_cast<unsigned long long*>(va->part + ee::kLmGthrOff) : nullptr;
 
   CUtensorMap tmW, tmX;
-  if (!encode_2d(&tmW, lm_w, (uint64_t)hidden_dim, (uint64_t)vocab, BK, (uint32_t)p.BMr)) return EE_ERR_CUDA;
+  if (packed) {
+    // the packed W as rows of 64 elements: block (vt, kb) is rows (vt * nkb + kb) * 128 ..
+    if (!encode_2d(&tmW, lm_w, (uint64_t)BK, (uint64_t)p.n_vt * p.nkb * BM, BK, (uint32_t)BM)) return EE_ERR_CUDA;
+  } else if (!encode_2d(&tmW, lm_w, (uint64_t)hidden_dim, (uint64_t)vocab, BK, (uint32_t)p.BMr)) {
+    return EE_ERR_CUDA;
+  }
   if (!encode_2d(&tmX, hidden, (uint64_t)hidden_dim, (uint64_t)total_nodes, BK, p.BN))
     return EE_ERR_CUDA;
 
@@ -1153,6 +1166,81 @@ extern "C" ee_status ee_lmhead_accept(const ee_bf16* hidden, const ee_bf16* lm_w
                        reinterpret_cast<unsigned long long*>(wsb + ee::kArgmaxOff),
                        reinterpret_cast<unsigned int*>(wsb + ee::kTicketOff), ee::err_word(ws),
                        stream, true);
+}
+
+namespace {
+
+// ---------------------------------------------------------------------------
+// Tile-ordered LM-head weights (ee_lmhead_pack_weights): the 128-row x
+// 64-column blocks of W that the kernel loads one per ring stage, each stored
+// as one contiguous 16 KB run, so that the weight stream reads whole DRAM
+// pages instead of 128-byte pieces 2*H bytes apart.  Block (vt, kb) = rows
+// [128 vt, 128 vt + 128) x columns [64 kb, 64 kb + 64) of W, row-major inside
+// the block, at element ((vt * nkb + kb) * 128) * 64; rows past V and columns
+// past H are zero.
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(256) pack_w_kernel(const uint4* __restrict__ w, int vocab, int hidden,
+                                                     int n_vt, int nkb, uint4* __restrict__ out) {
+  const size_t total = (size_t)n_vt * nkb * BM * (BK / 8);   // 16-byte words
+  for (size_t q = (size_t)blockIdx.x * blockDim.x + threadIdx.x; q < total; q += (size_t)gridDim.x * blockDim.x) {
+    const int c8 = (int)(q & 7);
+    const size_t rest = q >> 3;
+    const int r = (int)(rest & (BM - 1));
+    const size_t blk = rest / BM;
+    const int kb = (int)(blk % (size_t)nkb), vt = (int)(blk / (size_t)nkb);
+    const int row = vt * BM + r, col = kb * BK + c8 * 8;
+    uint4 v = make_uint4(0u, 0u, 0u, 0u);
+    if (row < vocab && col < hidden) v = w[((size_t)row * hidden + col) / 8];
+    out[q] = v;
+  }
+}
+
+size_t packed_w_bytes(int32_t vocab, int32_t hidden_dim) {
+  if (vocab < 1 || hidden_dim < 8 || hidden_dim % 8 != 0) return 0;
+  return (size_t)((vocab + BM - 1) / BM) * BM * (size_t)((hidden_dim + BK - 1) / BK) * BK * 2;
+}
+
+}  // namespace
+
+extern "C" size_t ee_lmhead_packed_bytes(int32_t vocab, int32_t hidden_dim) {
+  return packed_w_bytes(vocab, hidden_dim);
+}
+
+extern "C" ee_status ee_lmhead_pack_weights(const ee_bf16* lm_w, int32_t vocab, int32_t hidden_dim, ee_bf16* packed,
+                                            size_t packed_bytes, ee_stream_t stream) {
+  const size_t need = packed_w_bytes(vocab, hidden_dim);
+  if (need == 0) return vocab < 1 || hidden_dim < 8 ? EE_ERR_INVALID_ARG : EE_ERR_UNSUPPORTED;
+  if (!lm_w || !packed || !ee::aligned(lm_w, 16) || !ee::aligned(packed, 16)) return EE_ERR_INVALID_ARG;
+  if (packed_bytes < need) return EE_ERR_INVALID_ARG;
+  const int n_vt = (vocab + BM - 1) / BM, nkb = (hidden_dim + BK - 1) / BK;
+  const size_t words = need / 16;
+  const int grid = (int)std::min<size_t>((words + 255) / 256, (size_t)ee::kNumSMs * 16);
+  pack_w_kernel<<<grid, 256, 0, (cudaStream_t)stream>>>(reinterpret_cast<const uint4*>(lm_w), vocab, hidden_dim,
+                                                        n_vt, nkb, reinterpret_cast<uint4*>(packed));
+  EE_CUDA_OK(cudaGetLastError());
+  return EE_OK;
+}
+
+extern "C" ee_status ee_lmhead_accept_packed(const ee_bf16* hidden, const ee_bf16* lm_w_packed,
+                                             int32_t hidden_dim, int32_t vocab, const int32_t* draft_tok,
+                                             const int32_t* parent, const int32_t* depth, const uint64_t* anc,
+                                             const int32_t* node_off, int32_t B, int32_t total_nodes,
+                                             int32_t max_T, int32_t* argmax, int32_t* accept_len,
+                                             int32_t* path, int32_t* bonus, float* logits_or_null,
+                                             void* ws, size_t ws_bytes, ee_stream_t stream) {
+  bool empty = false;
+  const ee_status st = check_lm_args(hidden, lm_w_packed, hidden_dim, vocab, draft_tok, parent, depth, anc,
+                                     node_off, B, total_nodes, max_T, argmax, accept_len, path,
+                                     bonus, &empty, true);
+  if (st != EE_OK || empty) return st;
+  if (!ws || !ee::aligned(ws, 256)) return EE_ERR_INVALID_ARG;
+  if (ws_bytes < ee::kWorkspaceBytes) return EE_ERR_WORKSPACE;
+  char* wsb = static_cast<char*>(ws);
+  return launch_lmhead(hidden, lm_w_packed, hidden_dim, vocab, draft_tok, parent, depth, anc, node_off, B,
+                       total_nodes, max_T, argmax, accept_len, path, bonus, logits_or_null,
+                       reinterpret_cast<unsigned long long*>(wsb + ee::kArgmaxOff),
+                       reinterpret_cast<unsigned int*>(wsb + ee::kTicketOff), ee::err_word(ws),
+                       stream, true, nullptr, true);
 }
 
 extern "C" ee_status ee_lmhead_verify(const ee_bf16* hidden, const ee_bf16* lm_w, int32_t hidden_dim,

@@ -24,8 +24,8 @@ import math
 import torch
 
 from . import (EE_HEAD_DIM, ee_chain_verify_attn, ee_kv_compact, ee_kv_compact_inplace, ee_lmhead_accept,
-               ee_lmhead_verify, ee_match_reuse, ee_tree_prepare, ee_tree_verify_attn,
-               ee_tree_verify_attn_inplace, new_workspace)
+               ee_lmhead_accept_packed, ee_lmhead_pack_weights, ee_lmhead_packed_bytes, ee_lmhead_verify,
+               ee_match_reuse, ee_tree_prepare, ee_tree_verify_attn, ee_tree_verify_attn_inplace, new_workspace)
 
 
 class VerifyStep:
@@ -41,13 +41,16 @@ class VerifyStep:
     K/V in the cache at positions ctx + i (in-place speculative K/V): at set-up
     they are copied there from k_tree / v_tree, where a K/V projection would
     have written them, and the block table gets the columns max_ctx + max_T
-    positions need (-1 padded).
+    positions need (-1 padded).  ``packed_lm`` (default) rearranges lm_w once,
+    at set-up, into the LM head's tile order (ee_lmhead_pack_weights, a model-
+    load step, not part of a verification step) and runs the greedy LM head on
+    that copy (ee_lmhead_accept_packed: bit-identical results).
     """
 
     def __init__(self, *, orig_tokens, orig_off, tail, cursor, parent, node_off, draft_tok, ctx_len,
                  block_table, q, k_tree, v_tree, k_cache, v_cache, hidden, lm_w, max_ctx, max_T,
                  max_matches=8, scale=None, keep_layers=True, verify=None, gen_mask=None, inplace_kv=False,
-                 chain=False):
+                 chain=False, packed_lm=True):
         self.inp = dict(orig_tokens=orig_tokens, orig_off=orig_off, tail=tail, cursor=cursor,
                         parent=parent, node_off=node_off, draft_tok=draft_tok, ctx_len=ctx_len,
                         block_table=block_table, q=q, k_tree=k_tree, v_tree=v_tree, k_cache=k_cache,
@@ -88,6 +91,14 @@ class VerifyStep:
         self.inplace_kv = bool(inplace_kv) or self.chain
         if self.inplace_kv:
             self._place_tree_kv()
+        self.lm_packed = None
+        if packed_lm and lm_w is not None:
+            V, H = lm_w.shape
+            n = ee_lmhead_packed_bytes(V, H)
+            if n:
+                self.lm_packed = torch.empty(n // 2, dtype=torch.bfloat16, device=dev)
+                ee_lmhead_pack_weights(lm_w, self.lm_packed)
+                torch.cuda.synchronize(dev)
         self.graph = None
 
     def _place_tree_kv(self):
@@ -134,7 +145,13 @@ class VerifyStep:
                                     x["v_cache"][l], x["block_table"], x["ctx_len"], self.max_ctx,
                                     x["node_off"], self.anc, self.max_T, self.scale, out, self.ws, stream)
         mark(1)
-        if self.chain:
+        if self.verify is None and self.lm_packed is not None:
+            chain = self.chain
+            ee_lmhead_accept_packed(x["hidden"], self.lm_packed, x["lm_w"].shape[0], x["draft_tok"],
+                                    None if chain else x["parent"], None if chain else self.depth,
+                                    None if chain else self.anc, x["node_off"], self.max_T, self.argmax,
+                                    self.accept_len, self.path, self.bonus, self.ws, logits=logits, stream=stream)
+        elif self.chain:
             ee_lmhead_accept(x["hidden"], x["lm_w"], x["draft_tok"], None, None, None, x["node_off"], self.max_T,
                              self.argmax, self.accept_len, self.path, self.bonus, self.ws, logits=logits,
                              stream=stream)
@@ -175,7 +192,7 @@ class VerifyStep:
         return (1 if self.chain else 2) + self.L + 2 + (0 if self.verify is None else 1)
 
 
-def from_workload(w, device="cuda", keep_layers=True, verify=None, inplace_kv=False, chain=None):
+def from_workload(w, device="cuda", keep_layers=True, verify=None, inplace_kv=False, chain=None, packed_lm=True):
     """VerifyStep over a workloads.Workload (its float tensors already on ``device``);
     ``verify`` = (mode, k) uses that rule on the workload's generated branches;
     ``inplace_kv`` verifies with the tree's K/V placed in the cache; ``chain``
@@ -193,4 +210,4 @@ def from_workload(w, device="cuda", keep_layers=True, verify=None, inplace_kv=Fa
         hidden=w.hidden_states, lm_w=w.lm_w, max_ctx=int(w.ctx_len.max()), max_T=w.max_T,
         max_matches=w.max_matches, keep_layers=keep_layers, verify=verify,
         gen_mask=torch.as_tensor(w.gen_mask).to(device) if verify is not None else None,
-        inplace_kv=inplace_kv, chain=chain)
+        inplace_kv=inplace_kv, chain=chain, packed_lm=packed_lm)

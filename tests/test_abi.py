@@ -230,3 +230,26 @@ def test_controller_rejects_bad_args(L):
     assert a(*bad) == 1
     bad = list(abase); bad[13] = None
     assert a(*bad) == 1
+
+
+def test_lmhead_packing_sizes_and_checks(L):
+    """The tile-ordered weights take ceil(V / 128) * 128 rows of ceil(H / 64) * 64
+    columns; bad sizes, pointers and short buffers are rejected before a launch."""
+    assert L.ee_lmhead_packed_bytes(152064, 3584) == 152064 * 3584 * 2
+    assert L.ee_lmhead_packed_bytes(1000, 512) == 1024 * 512 * 2
+    assert L.ee_lmhead_packed_bytes(1000, 520) == 1024 * 576 * 2
+    assert L.ee_lmhead_packed_bytes(1000, 12) == 0 and L.ee_lmhead_packed_bytes(0, 512) == 0
+    f = L.ee_lmhead_pack_weights
+    n = L.ee_lmhead_packed_bytes(1000, 512)
+    assert f(None, 1000, 512, FAKE, n, None) == 1
+    assert f(FAKE, 1000, 512, None, n, None) == 1
+    assert f(FAKE, 1000, 512, FAKE, n - 16, None) == 1            # buffer too small
+    assert f(ctypes.c_void_p(0x10002), 1000, 512, FAKE, n, None) == 1
+    assert f(FAKE, 1000, 12, FAKE, n, None) == 2                  # hidden not a multiple of 8
+    assert f(FAKE, 0, 512, FAKE, n, None) == 1
+    g = L.ee_lmhead_accept_packed
+    base = [FAKE, FAKE, 3584, 152064] + [FAKE] * 5 + [1, 64, 64] + [FAKE] * 4 + [None, FAKE, 1 << 20, None]
+    h7 = list(base); h7[2] = 3583
+    assert g(*h7) == 2                                            # as ee_lmhead_accept
+    small = list(base); small[18] = 64
+    assert g(*small) == 5
