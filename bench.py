@@ -69,8 +69,8 @@ TRAFFIC = {
     ("tree_verify_attn", "7b"): 9062144,          # profiles/attn_tc_7b.md
     ("tree_verify_attn", "33b"): 161879296,       # profiles/attn_tc_33b.md
     ("tree_verify_attn", "batched"): 246827008,   # profiles/attn_tc_batched.md
-    ("lmhead_accept", "7b"): 1095706368,          # profiles/lmhead_accept_7b.md
-    ("lmhead_accept", "long"): 1107766528,        # profiles/lmhead_accept_long.md
+    ("lmhead_accept", "7b"): 1096552192,          # profiles/lmhead_accept_7b.md
+    ("lmhead_accept", "long"): 1107782912,        # profiles/lmhead_accept_long.md
     ("chain_verify_attn", "long"): 30021120,      # profiles/attn_chain_long.md
 }
 
