@@ -994,7 +994,7 @@ def _clone_step(st):
                         q=c["q"], k_tree=c["k_tree"], v_tree=c["v_tree"], k_cache=x["k_cache"],
                         v_cache=x["v_cache"], hidden=c["hidden"], lm_w=x["lm_w"], max_ctx=st.max_ctx,
                         max_T=st.max_T, max_matches=st.max_matches, keep_layers=False,
-                        inplace_kv=st.inplace_kv, chain=st.chain)
+                        inplace_kv=st.inplace_kv, chain=st.chain, lm_packed=st.lm_packed)
 
 
 def run_e2e(st, graph, stream, steps, dev, world):
@@ -1011,7 +1011,9 @@ def run_e2e(st, graph, stream, steps, dev, world):
     host_in = {n: st.inp[n].detach().cpu().pin_memory() for n in names_in}
 
     def outs_of(s):
-        return [s.accept_len, s.path, s.bonus, s.argmax, s.match_pos, s.n_matches, s.ctx_out]
+        # accept_len, path, bonus, argmax, match_pos, n_matches, ctx_out: views of one buffer
+        return [s.outputs]
+    acc0 = st.out_layout["accept_len"][0]    # where accept_len[0] sits in it
     h2d = sum(t.numel() * t.element_size() for t in host_in.values())
 
     # serial: one buffer set
@@ -1073,9 +1075,9 @@ def run_e2e(st, graph, stream, steps, dev, world):
             if i >= 1:                                     # the previous step's results, on the host
                 k = (i - 1) % 2
                 done[k].synchronize()
-                seen.append(int(sets[k][3][0][0]))
+                seen.append(int(sets[k][3][0][acc0]))
         done[(n - 1) % 2].synchronize()
-        seen.append(int(sets[(n - 1) % 2][3][0][0]))
+        seen.append(int(sets[(n - 1) % 2][3][0][acc0]))
         torch.cuda.synchronize(dev)
 
     pipelined(6)

@@ -44,13 +44,14 @@ class VerifyStep:
     positions need (-1 padded).  ``packed_lm`` (default) rearranges lm_w once,
     at set-up, into the LM head's tile order (ee_lmhead_pack_weights, a model-
     load step, not part of a verification step) and runs the greedy LM head on
-    that copy (ee_lmhead_accept_packed: bit-identical results).
+    that copy (ee_lmhead_accept_packed: bit-identical results); ``lm_packed``
+    passes an already packed copy instead.
     """
 
     def __init__(self, *, orig_tokens, orig_off, tail, cursor, parent, node_off, draft_tok, ctx_len,
                  block_table, q, k_tree, v_tree, k_cache, v_cache, hidden, lm_w, max_ctx, max_T,
                  max_matches=8, scale=None, keep_layers=True, verify=None, gen_mask=None, inplace_kv=False,
-                 chain=False, packed_lm=True):
+                 chain=False, packed_lm=True, lm_packed=None):
         self.inp = dict(orig_tokens=orig_tokens, orig_off=orig_off, tail=tail, cursor=cursor,
                         parent=parent, node_off=node_off, draft_tok=draft_tok, ctx_len=ctx_len,
                         block_table=block_table, q=q, k_tree=k_tree, v_tree=v_tree, k_cache=k_cache,
@@ -65,17 +66,24 @@ class VerifyStep:
         self.max_matches = int(max_matches)
         self.scale = 1.0 / math.sqrt(d) if scale is None else float(scale)
         i32 = dict(dtype=torch.int32, device=dev)
-        self.match_pos = torch.empty((self.B, self.max_matches), **i32)
-        self.n_matches = torch.empty(self.B, **i32)
+        # the step's results are views of one int32 buffer (``outputs``; each view
+        # starts on a 64-byte boundary, ``out_layout`` = name -> (offset, shape)),
+        # so one device-to-host copy returns all of them
+        specs = (("match_pos", (self.B, self.max_matches)), ("n_matches", (self.B,)), ("argmax", (self.total,)),
+                 ("accept_len", (self.B,)), ("path", (self.B, self.max_T)), ("bonus", (self.B,)),
+                 ("ctx_out", (self.B,)))
+        sizes = [math.prod(sh) for _, sh in specs]
+        self.outputs = torch.empty(sum(-(-n // 16) * 16 for n in sizes), **i32)
+        self.out_layout = {}
+        off = 0
+        for (name, sh), n in zip(specs, sizes):
+            setattr(self, name, self.outputs[off:off + n].view(sh))
+            self.out_layout[name] = (off, sh)
+            off += -(-n // 16) * 16
         self.depth = torch.empty(self.total, **i32)
         self.anc = torch.empty((self.total, 2), dtype=torch.int64, device=dev)
         n_out = self.L if keep_layers else 1
         self.attn_out = torch.empty((n_out, self.total, self.n_q, d), dtype=torch.float32, device=dev)
-        self.argmax = torch.empty(self.total, **i32)
-        self.accept_len = torch.empty(self.B, **i32)
-        self.path = torch.empty((self.B, self.max_T), **i32)
-        self.bonus = torch.empty(self.B, **i32)
-        self.ctx_out = torch.empty(self.B, **i32)
         self.dst_slot = torch.empty((self.B, self.max_T), **i32)
         self.ws = new_workspace(self.B, self.total, self.n_q, self.max_ctx, device=dev)
         self.verify = None if verify is None else (verify[0], int(verify[1]))
@@ -91,8 +99,8 @@ class VerifyStep:
         self.inplace_kv = bool(inplace_kv) or self.chain
         if self.inplace_kv:
             self._place_tree_kv()
-        self.lm_packed = None
-        if packed_lm and lm_w is not None:
+        self.lm_packed = lm_packed   # tile-ordered weights to share with another step, or None
+        if self.lm_packed is None and packed_lm and lm_w is not None:
             V, H = lm_w.shape
             n = ee_lmhead_packed_bytes(V, H)
             if n:
